@@ -1,0 +1,303 @@
+/*
+ * awsrc.h — C ABI of the GB300 (sm_103a) implementation of the hot path of
+ * Activation-Weighted Seeded Residual Coding (AWSRC, arXiv 2608.23144):
+ * per-(tile, seed) search over the residual R = W - W0 of a fixed backbone,
+ * byte-aware record selection, and decode-apply.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every array argument documented as "device" is caller-owned device memory
+ *    on the current CUDA device; "host" arguments are caller-owned host memory.
+ *    The library never allocates device memory: scratch space is the caller's
+ *    `workspace`, whose size is queried with the matching *_workspace_bytes call.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Every launch is asynchronous on that stream; no entry point synchronises
+ *    unless its comment says so.
+ *  - Errors are returned as awsrc_status, never thrown. Arguments are validated
+ *    on the host before any launch; on error nothing is launched and no output
+ *    is written. A CUDA runtime failure returns AWSRC_ERR_CUDA, and
+ *    awsrc_last_error_message() gives the runtime's text (thread-local).
+ *  - Inputs are never modified; the only exception is W_hat aliasing W0 in
+ *    AWSRC_DECODE_INPLACE mode.
+ *  - Matrices are row-major: element (i, j) of a rows x cols module is at
+ *    i*cols + j (output row i, input channel j). Tiles are C contiguous input
+ *    channels of one output row (Sec. 3.1): tile t = i*(cols/C) + cb covers
+ *    columns [cb*C, cb*C + C). Global tile indices concatenate modules in the
+ *    order given: module m's tiles start at sum_{m'<m} rows*cols/C.
+ *
+ * Numeric convention
+ * ------------------
+ * Encoder and decoder share the generator and the numeric convention (Sec. 3.1);
+ * basis generation and tie breaking are fixed (Sec. 4). The convention is IEEE
+ * binary32, round-to-nearest-even, in exactly this order (fma = one rounding,
+ * every other operation rounds once; sums run j = 0..C-1 ascending):
+ *
+ *  GenBasis(s) (Eq. 2). SplitMix64 (Steele, Lea & Flood 2014): the n-th output
+ *   (n >= 1) of the stream started at state x is mix64(x + n*0x9E3779B97F4A7C15).
+ *   key_s = output s+1 of the stream at gen_seed; draws are outputs 1, 2, ... of
+ *   the stream at key_s, consumed in this order: ceil(C/64) sign words (bit j%64
+ *   of word j/64 is sigma_j, 1 = negative); if permute, for i = C-1 down to 1 one
+ *   draw, k = ((draw >> 32) * (i+1)) >> 32, swap(pi[i], pi[k]) starting from the
+ *   identity; then for p = 0..P-1 one draw, k = p + (((draw >> 32) * (C-p)) >> 32),
+ *   swap(col[p], col[k]) on the identity array, c_p = col[p]. Entry (j, p) of
+ *   B_s is C^-1/2 * (-1)^(sigma_j + popcount(pi[j] & c_p)) (Sylvester Hadamard).
+ *   m_p(j) denotes the sign (+-1) of that entry.
+ *  Weights. r_j = W - W0 (after exact widening to f32); U: d_j = a_j; PF:
+ *   d_j = w_act*a_j + w_fisher*F_ij; y_j = d_j * r_j. A tile is invalid (gain
+ *   -inf) unless every r_j is finite with |r_j| <= 2^16 and every d_j is in [0, 2^32].
+ *  Fit (Eq. 3). c = RN(C^-1/2), c2 = 1/C. u_p = sum_j m_p(j)*y_j (u = fma(m, y, u));
+ *   b_p = c*u_p. gd = c2 * sum_j d_j; G_pp = gd; G_pq = c2 * sum_j m_p(j)m_q(j) d_j.
+ *   eps = ridge_rel*gd; A = G + eps*I. LDL^T, k = 0..P-1: for j < k:
+ *   v = A_kj, v = fma(-L_ki, E_ji, v) for i < j, E_kj = v, L_kj = v*invD_j;
+ *   D_k = A_kk, D_k = fma(-L_ki, E_ki, D_k) for i < k; the candidate is invalid
+ *   unless 0 < D_k <= FLT_MAX; invD_k = 1/D_k. Solve: z_k = b_k then
+ *   z_k = fma(-L_ki, z_i, z_k) for i < k; w_k = z_k*invD_k; for k = P-1 down to 0:
+ *   alpha_k = w_k then alpha_k = fma(-L_ik, alpha_i, alpha_k) for i = k+1..P-1.
+ *  Quantisation (Sec. 3.2). amax = max_p |alpha_p| (NaN propagates); invalid
+ *   unless 2^-100 <= amax <= 2^32. POW2: e = smallest integer with
+ *   amax <= qmax*2^e, clamped to the exponent range; code_p =
+ *   clamp(rint(alpha_p*2^-e), -qmax, qmax); sc = 2^e. FP16: sc = binary16_RN(
+ *   amax/qmax) (invalid if 0 or inf), code_p = clamp(rint(alpha_p/sc), -qmax, qmax).
+ *  Gain (Eq. 4, unregularised G). Aq = fma(code_p, b_p, Aq) over p; Qq over p
+ *   ascending: Qq = fma(code_p^2, G_pp, Qq), then for q > p
+ *   Qq = fma(2*code_p*code_q, G_pq, Qq); gain = sc * (2*Aq - sc*Qq).
+ *  Selection. s* = argmax_s gain (strictly greater replaces: ties keep the
+ *   smallest s); a tile whose every candidate is invalid has gain -inf.
+ * Integer outputs (seed selectors, exponents, codes, record order, byte counts)
+ * are therefore reproducible bit for bit by any implementation of this recipe.
+ */
+#ifndef AWSRC_H
+#define AWSRC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum awsrc_status {
+  AWSRC_OK = 0,
+  AWSRC_ERR_INVALID_ARG = 1,  /* null pointer, bad enum, n_mod < 1, K out of range */
+  AWSRC_ERR_SHAPE = 2,        /* cols % C != 0, rows/cols < 1, C not a power of two */
+  AWSRC_ERR_UNSUPPORTED = 3,  /* parameter outside the supported ranges below */
+  AWSRC_ERR_BUDGET = 4,       /* a byte budget is smaller than the stream header */
+  AWSRC_ERR_CUDA = 5,         /* CUDA runtime error; see awsrc_last_error_message() */
+  AWSRC_ERR_WORKSPACE = 6,    /* workspace NULL or smaller than the queried size */
+  AWSRC_ERR_CAPACITY = 7,     /* output stream buffer smaller than awsrc_stream_capacity() */
+  AWSRC_ERR_DEVICE = 8        /* a kernel reported a fault in its inputs (corrupt stream) */
+} awsrc_status;
+
+enum { AWSRC_VARIANT_U = 0, AWSRC_VARIANT_PF = 1 };
+enum { AWSRC_SCALE_POW2 = 0, AWSRC_SCALE_FP16 = 1 };
+enum { AWSRC_DTYPE_F32 = 0, AWSRC_DTYPE_BF16 = 1 };
+enum { AWSRC_DECODE_DENSE = 0, AWSRC_DECODE_INPLACE = 1 };
+
+/*
+ * Codec parameters (Sec. 3.1: C locality, P subspace dimension, b coefficient
+ * precision, S basis diversity; Eq. 5: b_e scale-exponent width).
+ *   C          tile length; power of two in [4, 256] (Sylvester Hadamard order).
+ *   P          atoms (basis columns) per tile, 1 <= P <= min(8, C).
+ *   b          coefficient bits, 2 <= b <= 8. Codes are symmetric round-to-
+ *              nearest-even integers in [-qmax, qmax], qmax = 2^(b-1) - 1 (Sec. 3.2).
+ *   S          seeds searched per tile, 1 <= S <= 65536; selector s in [0, S).
+ *   b_e        scale field width. POW2: 1..8 bits holding e - e_bias in two's
+ *              complement (the paper's power-of-two scale exponent, Sec. 3.2);
+ *              FP16: must be 16 (binary16 scale, the small synthetic workload's option).
+ *   e_bias     POW2 only: exponents are clamped to
+ *              [max(e_bias - 2^(b_e-1), -126), min(e_bias + 2^(b_e-1) - 1, 126)],
+ *              which must be non-empty.
+ *   scale_mode AWSRC_SCALE_POW2 or AWSRC_SCALE_FP16.
+ *   permute    1: each seed draws a coordinate permutation (Sec. 3.1); 0: identity.
+ *   variant    AWSRC_VARIANT_U (activation weights, per-module quotas) or
+ *              AWSRC_VARIANT_PF (blended activation/Fisher weights, global
+ *              progressive prefixes) (Sec. 3.3).
+ *   ridge_rel  ridge of Eq. 3 relative to the tile's mean weight:
+ *              eps = ridge_rel * (1/C) * sum_j d_{t,j}; finite, >= 0.
+ *   gen_seed   key of the shared deterministic basis generator (Sec. 3.1).
+ */
+typedef struct awsrc_params {
+  int32_t C, P, b, S;
+  int32_t b_e, e_bias;
+  int32_t scale_mode, permute, variant;
+  float ridge_rel;
+  uint64_t gen_seed;
+} awsrc_params;
+
+/*
+ * One linear module (a weight matrix W with backbone reconstruction W0 = Q(W),
+ * Eq. 1) and its per-input-channel statistics (Sec. 3.2).
+ *   rows, cols  output and input dimensions; cols % C == 0.
+ *   W, W0       device, rows*cols elements of w_dtype / w0_dtype (F32 or BF16).
+ *               The encoder reads both; the decoder reads W0 only (W may be NULL).
+ *   act         device, cols floats: activation second moments a_j = E[x_j^2].
+ *   fisher      device, rows*cols floats: Fisher diagonal (PF only; NULL for U).
+ *   w_act, w_fisher  PF blend weights including their normalisers: the element
+ *               weight is d_ij = w_act*a_j + w_fisher*F_ij (Sec. 3.3). Ignored by U,
+ *               where d_ij = a_j (the activation diagonal is shared by rows, Sec. 3.2).
+ */
+typedef struct awsrc_module {
+  int64_t rows, cols;
+  int32_t w_dtype, w0_dtype;
+  const void* W;
+  const void* W0;
+  const float* act;
+  const float* fisher;
+  float w_act, w_fisher;
+} awsrc_module;
+
+/*
+ * Best candidate of one tile (Sec. 3.2: the seed with the lowest post-quantisation
+ * weighted error, i.e. the largest gain). 16 bytes, device arrays of these are
+ * indexed by global tile.
+ *   gain   weighted error reduction of Eq. 4 (numerator), computed from the
+ *          quantised coefficients; -inf when no seed yields a valid fit.
+ *   seed   selector s_t* in [0, S) (0 when gain is -inf).
+ *   scale  POW2: exponent e (scale 2^e); FP16: raw binary16 bits of the scale.
+ *   code   the P signed b-bit codes; entries p >= P are 0.
+ */
+typedef struct awsrc_candidate {
+  float gain;
+  uint16_t seed;
+  int16_t scale;
+  int8_t code[8];
+} awsrc_candidate;
+
+/* ---------------------------------------------------------------- encoder -- */
+
+/*
+ * awsrc_encode_workspace_bytes — device scratch needed by awsrc_encode_tiles for
+ * these parameters and modules (basis masks, per-(seed, column block) Gram
+ * factors for U, per-split partial results). Host-only; launches nothing.
+ */
+awsrc_status awsrc_encode_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, size_t* bytes);
+
+/*
+ * awsrc_encode_tiles — the seed search of Sec. 3.2 for every tile of every
+ * module. For each tile t and each seed s it regenerates B_s = GenBasis(s, C, P)
+ * (Eq. 2), fits alpha*_{t,s} by the weighted ridge least squares of Eq. 3,
+ * quantises it coefficient-wise with one scale per tile, scores the quantised
+ * reconstruction by the weighted error reduction of Eq. 4, and keeps the best
+ * seed (ties: smallest s).
+ *   out        device, sum_m rows_m*cols_m/C candidates, indexed by global tile.
+ *   workspace  device, >= awsrc_encode_workspace_bytes(); contents are scratch.
+ * Errors: INVALID_ARG, SHAPE, UNSUPPORTED, WORKSPACE, CUDA.
+ */
+awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod,
+                                const awsrc_module* mods, awsrc_candidate* out,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * awsrc_gen_basis — writes the sign masks of GenBasis (Eq. 2) for seeds [0, S):
+ * masks[(s*P + p)*W + w], W = ceil(C/64) words, bit j%64 of word j/64 set when
+ * entry (j, p) of B_s is negative. Device array of S*P*W uint64. Used by the
+ * decoder and exposed for tests.
+ */
+awsrc_status awsrc_gen_basis(const awsrc_params* prm, uint64_t* masks, void* stream);
+
+/* ------------------------------------------------------------- selection -- */
+
+/* Serialized record size L of Eq. 5 in bytes for T candidate tiles:
+ * ceil((ceil(log2 T) + ceil(log2 S) + b_e + P*b) / 8). Host-only. Returns -1 on
+ * invalid parameters. */
+int64_t awsrc_record_bytes(const awsrc_params* prm, int64_t T);
+
+/* Stream header size h of Eq. 5: 40 bytes + 8 bytes per module. Host-only. */
+int64_t awsrc_header_bytes(int32_t n_mod);
+
+/*
+ * awsrc_stream_capacity — bytes the stream buffer of awsrc_select_records must
+ * hold: h + K_max*L, K_max the largest record count any of the rates allows.
+ * Host-only.
+ */
+awsrc_status awsrc_stream_capacity(const awsrc_params* prm, int32_t n_mod,
+                                   const awsrc_module* mods, const double* rates_bpw,
+                                   int32_t n_rates, size_t* bytes);
+
+awsrc_status awsrc_select_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, size_t* bytes);
+
+/*
+ * awsrc_select_records — byte-aware allocation (Sec. 3.3) and serialisation
+ * (Sec. 3.4, Eq. 5). Candidates with gain <= 0 (or non-finite) are discarded.
+ * Records are ranked by rho_t = gain_t / L (Eq. 4); L is the same for every
+ * record, so the order is gain descending, ties by global tile ascending.
+ * Budgets are B = floor(rate * N_scope / 8) bytes including the header, with
+ * N_scope = sum_m rows*cols.
+ *   U  (n_rates == 1): module m receives quota_m = floor((B - h) * N_m / N_scope)
+ *      bytes and keeps K_m = min(#positive_m, floor(quota_m / L)) records; the
+ *      stream holds module 0's records, then module 1's, ..., each block in
+ *      rank order. d_counts[m] = K_m (n_mod entries), d_bytes[0] = stream bytes.
+ *   PF (n_rates >= 1): one global ranking; rate r keeps the longest prefix
+ *      K_r = min(#positive, floor((B_r - h) / L)); the stream holds the longest
+ *      prefix and every shorter one decodes as it stands. d_counts[r] = K_r,
+ *      d_bytes[r] = h + K_r*L.
+ *   stream_out  device, >= awsrc_stream_capacity() bytes: header + records.
+ *   d_counts, d_bytes  device int64 arrays as above.
+ * Stream layout (little-endian): header of 40 + 8*n_mod bytes, then fixed-width
+ * records of L bytes. Record bits are LSB-first from bit 0: tile (ceil(log2 T)
+ * bits), seed (ceil(log2 S)), scale field (b_e), codes 0..P-1 (b bits each, two's
+ * complement); remaining bits zero. Header: u32 magic 0x52535741, u16 version 1,
+ * u8 variant, u8 scale_mode, u16 C, u8 P, u8 b, u8 b_e, i8 e_bias, u8 permute,
+ * u8 0, u32 S, u32 n_mod, u64 gen_seed, u64 K (records in this stream), then per
+ * module u32 tiles, u32 records.
+ * Errors: INVALID_ARG, UNSUPPORTED (U with n_rates != 1), BUDGET, CAPACITY,
+ * WORKSPACE, CUDA.
+ */
+awsrc_status awsrc_select_records(const awsrc_params* prm, int32_t n_mod,
+                                  const awsrc_module* mods, const awsrc_candidate* cands,
+                                  const double* rates_bpw, int32_t n_rates,
+                                  uint8_t* stream_out, size_t stream_capacity,
+                                  int64_t* d_counts, int64_t* d_bytes,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------- decoder -- */
+
+awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, int32_t mode,
+                                          size_t* bytes);
+
+/*
+ * awsrc_decode_apply — the decoder of Sec. 3.2: for each of the first K records
+ * it regenerates B_s (Eq. 2) and adds r_hat = B_s * alpha_hat to W0 (Eq. 1);
+ * tiles without a record keep W0 unchanged, so K == 0 returns W0 exactly.
+ * Any prefix of a progressive stream decodes against the same W0 (Sec. 3.3).
+ *   stream   device, header + records as written by awsrc_select_records.
+ *   K        records to apply (0 <= K <= header's K). K < 0 applies all the
+ *            header's records (read on the device; no synchronisation).
+ *   W_hat    host array of n_mod device pointers, rows*cols elements of out_dtype.
+ *   mode     DENSE: every element of W_hat is written (W0 copied, corrected where
+ *            a record exists). INPLACE: only the tiles named by records are
+ *            written; W_hat must already hold W0 (it may be W0 itself when
+ *            out_dtype == w0_dtype).
+ * Each corrected element is fl(W0 + fl(fl(k_j * C^-1/2) * scale)) with the exact
+ * integer k_j = sum_p sign_{j,p} * code_p, rounded once more to BF16 when
+ * out_dtype is BF16. Records naming a tile >= T or a seed >= S are skipped and
+ * reported through awsrc_workspace_status(). Requires the same params as the encoder.
+ */
+awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
+                                const awsrc_module* mods, const uint8_t* stream,
+                                int64_t K, void* const* W_hat, int32_t out_dtype,
+                                int32_t mode, void* workspace, size_t workspace_bytes,
+                                void* stream_handle);
+
+/* ------------------------------------------------------------------ misc -- */
+
+/*
+ * awsrc_workspace_status — synchronises `stream`, then reads and clears the
+ * device fault word kept at the start of an encode/select/decode workspace.
+ * *flags == 0 means no kernel reported a fault since the last call.
+ * Bit 1: a record named a tile or seed out of range (decoder);
+ * bit 2: encoder self-check mismatch between search and finalisation.
+ */
+awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags);
+
+const char* awsrc_status_string(awsrc_status st);
+const char* awsrc_last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AWSRC_H */

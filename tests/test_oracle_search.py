@@ -1,0 +1,140 @@
+"""Pins of the oracle's seed search (Sec. 3.2) and its Eq. 4 gain: the FP32 gain
+against the direct double-precision definition, the chosen seed against brute
+force over seeds, selection by the quantised (not the float) fit, tie breaking
+to the smallest selector, and the degenerate cases (zero residual, zero weights,
+out-of-domain values)."""
+import numpy as np
+import pytest
+
+
+def _module(rng, rows, cols, scale_r=1e-3):
+    W0 = rng.normal(0, 0.02, (rows, cols)).astype(np.float32)
+    W = (W0 + rng.normal(0, scale_r, (rows, cols))).astype(np.float32)
+    act = rng.lognormal(0, 1.5, cols).astype(np.float32)
+    return W, W0, act
+
+
+def _tile_rd(W, W0, act, C, t):
+    n_cb = W.shape[1] // C
+    i, cb = divmod(t, n_cb)
+    r = (W[i, cb * C:(cb + 1) * C] - W0[i, cb * C:(cb + 1) * C]).astype(np.float32)
+    return r, act[cb * C:(cb + 1) * C]
+
+
+@pytest.mark.parametrize("C,P,b,smode", [(8, 2, 3, 0), (16, 4, 4, 0), (64, 4, 4, 1), (32, 3, 2, 0)])
+def test_gain_matches_direct_definition(orc, C, P, b, smode):
+    rng = np.random.default_rng(11)
+    prm = orc.params(C=C, P=P, b=b, S=1, scale_mode=smode, b_e=16 if smode else 8, ridge_rel=1e-5)
+    for s in range(80):
+        r = rng.normal(0, 1e-3, C).astype(np.float32)
+        d = rng.lognormal(0, 1, C).astype(np.float32)
+        neg = orc.gen_basis(3, s, C, P, 1)[3]
+        out = orc.score_candidate(prm, r, d, neg)
+        energy = float(np.sum(d.astype(np.float64) * r.astype(np.float64) ** 2))
+        g_def = orc.def_gain(C, P, r, d, neg, out["codes"], orc.scale_value(prm, out["scale"]))
+        assert abs(out["gain"] - g_def) <= 1e-5 * energy
+
+
+def test_chosen_seed_is_brute_force_argmax(orc):
+    """Every seed re-scored in double from its own stored codes; the oracle's
+    choice must be the best, up to near-ties of 1e-6 relative."""
+    rng = np.random.default_rng(12)
+    C, P, b, S = 8, 2, 3, 16
+    prm = orc.params(C=C, P=P, b=b, S=S, ridge_rel=1e-5)
+    W, W0, act = _module(rng, 16, 16)
+    masks = orc.basis_masks(prm)
+    cand = orc.encode_tiles(prm, W, W0, act, masks=masks)
+    for t in range(len(cand)):
+        r, d = _tile_rd(W, W0, act, C, t)
+        g = []
+        for s in range(S):
+            out = orc.score_candidate(prm, r, d, masks[s])
+            g.append(-np.inf if out is None else
+                     orc.def_gain(C, P, r, d, masks[s], out["codes"], orc.scale_value(prm, out["scale"])))
+        g = np.array(g)
+        best = g.max()
+        chosen = g[cand[t]["seed"]]
+        assert chosen >= best - 1e-6 * abs(best)
+        # the stored fields are the chosen seed's own quantised fit
+        out = orc.score_candidate(prm, r, d, masks[cand[t]["seed"]])
+        assert out["gain"] == cand[t]["gain"]
+        assert np.array_equal(out["codes"], cand[t]["code"][:P])
+
+
+def test_selection_uses_quantised_coefficients(orc):
+    """Sec. 3.2: the seed is chosen by post-quantisation error. With 2-bit codes
+    the float-fit ranking and the quantised ranking often disagree; the oracle
+    must follow the quantised one in every such tile."""
+    rng = np.random.default_rng(13)
+    C, P, b, S = 16, 4, 2, 16
+    prm = orc.params(C=C, P=P, b=b, S=S, ridge_rel=1e-6)
+    W, W0, act = _module(rng, 32, 32)
+    masks = orc.basis_masks(prm)
+    cand = orc.encode_tiles(prm, W, W0, act, masks=masks)
+    disagreements = 0
+    for t in range(len(cand)):
+        r, d = _tile_rd(W, W0, act, C, t)
+        gq, gf = [], []
+        for s in range(S):
+            B = np.where(masks[s].T == 1, -1.0, 1.0) / np.sqrt(C)
+            bv = B.T @ (d.astype(np.float64) * r)
+            G = B.T @ (d.astype(np.float64)[:, None] * B)
+            gf.append(bv @ np.linalg.solve(G, bv))
+            gq.append(orc.score_candidate(prm, r, d, masks[s])["gain"])
+        if int(np.argmax(gf)) != int(np.argmax(gq)):
+            disagreements += 1
+        assert cand[t]["seed"] == int(np.argmax(gq))
+    assert disagreements > 0
+
+
+def test_ties_go_to_the_smallest_selector(orc):
+    rng = np.random.default_rng(14)
+    C, P, S = 16, 2, 12
+    prm = orc.params(C=C, P=P, b=4, S=S, ridge_rel=1e-6)
+    W, W0, act = _module(rng, 1, 16)
+    masks = orc.basis_masks(prm)
+    first = orc.encode_tiles(prm, W, W0, act, masks=masks)[0]
+    s_best = int(first["seed"])
+    tied = masks.copy()
+    tied[9] = masks[s_best]
+    tied[4] = masks[s_best]
+    got = orc.encode_tiles(prm, W, W0, act, masks=tied)[0]
+    assert got["gain"] == first["gain"]
+    assert got["seed"] == min(4, s_best)
+
+
+def test_degenerate_tiles_have_no_candidate(orc):
+    C = 16
+    prm = orc.params(C=C, P=2, b=4, S=8)
+    rng = np.random.default_rng(15)
+    W, W0, act = _module(rng, 4, 32)
+    W[0, :16] = W0[0, :16]          # zero residual tile
+    act2 = act.copy()
+    act2[16:] = 0.0                 # all-zero weights in the second column block
+    W[2, 3] = 1e6                   # residual outside the supported domain
+    cand = orc.encode_tiles(prm, W, W0, act2)
+    assert cand[0]["gain"] == -np.inf          # tile (row 0, cb 0)
+    assert all(cand[t]["gain"] == -np.inf for t in (1, 3, 5, 7))   # cb 1 has d = 0
+    assert cand[4]["gain"] == -np.inf          # row 2, cb 0 holds the huge residual
+    assert cand[2]["gain"] > 0 and cand[6]["gain"] > 0
+    for t in (0, 1, 3, 4, 5, 7):
+        assert cand[t]["seed"] == 0 and cand[t]["scale"] == 0 and not cand[t]["code"].any()
+
+
+def test_pf_weights_blend_activation_and_fisher(orc):
+    """PF: d_ij = w_act*a_j + w_fisher*F_ij (Sec. 3.3). With w_fisher = 0 the PF
+    search equals U; with a row-constant Fisher it equals U on the blended diagonal."""
+    rng = np.random.default_rng(16)
+    C = 16
+    W, W0, act = _module(rng, 8, 32)
+    F = rng.lognormal(0, 1.5, (8, 32)).astype(np.float32)
+    pu = orc.params(C=C, P=4, b=4, S=8, variant=0)
+    pf = orc.params(C=C, P=4, b=4, S=8, variant=1)
+    u = orc.encode_tiles(pu, W, W0, act)
+    f0 = orc.encode_tiles(pf, W, W0, act, fisher=F, w_act=1.0, w_fisher=0.0)
+    assert np.array_equal(u, f0)
+    Frow = np.tile(rng.lognormal(0, 1, 32).astype(np.float32), (8, 1))
+    blend = (np.float32(0.5) * act + np.float32(0.25) * Frow[0]).astype(np.float32)
+    f1 = orc.encode_tiles(pf, W, W0, act, fisher=Frow, w_act=0.5, w_fisher=0.25)
+    u1 = orc.encode_tiles(pu, W, W0, blend)
+    assert np.array_equal(f1, u1)

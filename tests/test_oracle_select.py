@@ -1,0 +1,127 @@
+"""Pins of the oracle's allocation (Sec. 3.3) and stream (Sec. 3.4) by their
+invariants: positivity, rank order, quota and budget feasibility and
+maximality, nested progressive prefixes, and a header/records round trip."""
+import struct
+
+import numpy as np
+import pytest
+
+
+def _cands(orc, rng, prm, shapes):
+    out = []
+    for rows, cols in shapes:
+        W0 = rng.normal(0, 0.02, (rows, cols)).astype(np.float32)
+        W = (W0 + rng.normal(0, 1e-3, (rows, cols))).astype(np.float32)
+        act = rng.lognormal(0, 1.5, cols).astype(np.float32)
+        F = rng.lognormal(0, 1.5, (rows, cols)).astype(np.float32)
+        out.append(orc.encode_tiles(prm, W, W0, act, fisher=F, w_act=0.5, w_fisher=0.5))
+    c = np.concatenate(out)
+    # a few non-positive / invalid gains to exercise eligibility
+    kill = rng.choice(len(c), len(c) // 20, replace=False)
+    c["gain"][kill[: len(kill) // 2]] = -np.inf
+    c["gain"][kill[len(kill) // 2:]] = -np.abs(c["gain"][kill[len(kill) // 2:]])
+    return c
+
+
+def _parse(orc, prm, stream, shapes):
+    n_mod = len(shapes)
+    h = orc.header_bytes(n_mod)
+    magic, ver, var, smode, C, P, b, b_e, e_bias, perm, _, S, nm, gseed, K = struct.unpack_from(
+        "<IHBBHBBBbBBIIQQ", stream, 0)
+    assert (magic, ver, var, smode, C, P, b, b_e, e_bias, perm, S, nm, gseed) == (
+        0x52535741, 1, prm.variant, prm.scale_mode, prm.C, prm.P, prm.b, prm.b_e, prm.e_bias,
+        prm.permute, prm.S, n_mod, prm.gen_seed)
+    mods = [struct.unpack_from("<II", stream, 40 + 8 * m) for m in range(n_mod)]
+    T = sum(r * c // prm.C for r, c in shapes)
+    L = orc.record_bytes(prm, T)
+    assert len(stream) == h + K * L
+    recs = [orc.unpack_record(prm, T, stream[h + k * L: h + (k + 1) * L]) for k in range(K)]
+    return K, mods, recs
+
+
+def test_u_per_module_quotas(orc):
+    rng = np.random.default_rng(21)
+    prm = orc.params(C=16, P=2, b=4, S=8, variant=0)
+    shapes = [(32, 64), (8, 32), (64, 48)]
+    cands = _cands(orc, rng, prm, shapes)
+    rate = 0.9
+    stream, counts, nbytes = orc.select_records(prm, shapes, cands, [rate])
+    K, mods, recs = _parse(orc, prm, stream, shapes)
+    N = sum(r * c for r, c in shapes)
+    h = orc.header_bytes(len(shapes))
+    T_m = [r * c // 16 for r, c in shapes]
+    L = orc.record_bytes(prm, sum(T_m))
+    B = orc.budget_bytes(rate, N)
+    assert nbytes[0] == len(stream) <= B
+    assert [m[0] for m in mods] == T_m and [m[1] for m in mods] == list(counts)
+    off = np.cumsum([0] + T_m)
+    k = 0
+    for m, (rows, cols) in enumerate(shapes):
+        mine = recs[k:k + counts[m]]
+        k += counts[m]
+        tiles = [t for t, _ in mine]
+        assert all(off[m] <= t < off[m + 1] for t in tiles)
+        gains = [float(cands[t]["gain"]) for t in tiles]
+        assert all(g > 0 for g in gains)
+        assert all(gains[i] > gains[i + 1] or (gains[i] == gains[i + 1] and tiles[i] < tiles[i + 1])
+                   for i in range(len(tiles) - 1))
+        pos = [t for t in range(off[m], off[m + 1]) if cands[t]["gain"] > 0]
+        dropped = sorted(set(pos) - set(tiles))
+        if dropped:
+            assert max(cands["gain"][dropped]) <= min(gains) if gains else True
+        # quota feasibility and maximality: proportional share of the byte budget
+        share = (B - h) * rows * cols / N
+        assert counts[m] * L <= share + 1e-9
+        assert counts[m] == len(pos) or (counts[m] + 1) * L > share
+        for t, c in mine:
+            assert c["seed"] == cands[t]["seed"] and c["scale"] == cands[t]["scale"]
+            assert np.array_equal(c["code"], cands[t]["code"])
+
+
+def test_pf_progressive_prefixes_nest(orc):
+    rng = np.random.default_rng(22)
+    prm = orc.params(C=16, P=4, b=4, S=8, variant=1)
+    shapes = [(16, 64), (32, 32)]
+    cands = _cands(orc, rng, prm, shapes)
+    rates = [0.5, 1.0, 2.0, 4.0]
+    stream, counts, nbytes = orc.select_records(prm, shapes, cands, rates)
+    K, mods, recs = _parse(orc, prm, stream, shapes)
+    N = sum(r * c for r, c in shapes)
+    T = sum(r * c // 16 for r, c in shapes)
+    L = orc.record_bytes(prm, T)
+    h = orc.header_bytes(2)
+    npos = int((cands["gain"] > 0).sum())
+    assert K == max(counts) and list(counts) == sorted(counts)
+    for r, k, nb in zip(rates, counts, nbytes):
+        B = orc.budget_bytes(r, N)
+        assert nb == h + k * L <= B
+        assert k == npos or nb + L > B
+        # the single-rate stream is the same ranked prefix
+        s1, c1, _ = orc.select_records(prm, shapes, cands, [r])
+        assert c1[0] == k and s1[h:] == stream[h:h + k * L]
+    gains = np.array([cands[t]["gain"] for t, _ in recs], np.float64)
+    assert np.all(gains > 0) and np.all(np.diff(gains) <= 0)
+    assert len({t for t, _ in recs}) == len(recs)
+    # tiles disjoint: cumulative gain over nested prefixes is non-decreasing
+    assert np.all(np.diff(np.cumsum(gains)) >= 0)
+    # every eligible tile not in the stream ranks below the last one kept
+    kept = {t for t, _ in recs}
+    rest = [cands[t]["gain"] for t in range(T) if cands[t]["gain"] > 0 and t not in kept]
+    if rest and recs:
+        assert max(rest) <= gains[-1]
+    assert sum(m[1] for m in mods) == K
+
+
+def test_budget_below_header_is_an_error(orc):
+    prm = orc.params(C=16, P=2, b=4, S=4)
+    cands = np.zeros(4, orc.CANDIDATE_DTYPE)
+    with pytest.raises(ValueError):
+        orc.select_records(prm, [(4, 16)], cands, [1.0])   # 64 weights -> 8 B < 48 B header
+
+
+def test_no_positive_gain_gives_empty_stream(orc):
+    prm = orc.params(C=16, P=2, b=4, S=4)
+    cands = np.zeros(64, orc.CANDIDATE_DTYPE)
+    cands["gain"] = -np.inf
+    stream, counts, nbytes = orc.select_records(prm, [(64, 16)], cands, [8.0])
+    assert counts[0] == 0 and len(stream) == orc.header_bytes(1)
