@@ -1,0 +1,382 @@
+#!/usr/bin/env python
+"""Throughput of the AWSRC hot path on GB300.
+
+One step = one pass of the whole path over one synthetic Qwen2.5-3B-shaped
+layer (7 modules, 77,070,336 BF16 weights, 1,204,224 tiles of C = 64):
+seed search over S = 4096 seeds (P = 4 atoms, INT4 codes, power-of-two scale),
+AWSRC-U selection at 0.162 bits/weight with the stream written, and a dense
+decode-apply of every module. Inputs are resident in HBM (308 MB of W and W0,
+larger than the 129 MB L2) when the timed region starts.
+
+Reported: (tile, seed) candidates/s for the whole step (`value`), layers/s,
+decode-apply GB/s, the search kernel against the FP32 pipe (`roofline`), the
+end-to-end figure through the public API with host buffers (`e2e`), and the
+CPU oracle on a bounded sample (`cpu_baseline`). `--impl reference` times the
+oracle alone (the baseline arm). Under torchrun each rank encodes its own layer
+(weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "qwen2.5-3b_layer"
+RATE = 0.162
+METRIC = "AWSRC encode (tile,seed) candidates/s + layers/s; decode-apply HBM GB/s"
+UNIT = "candidates/s"
+# FP32-pipe operations per (tile, seed) candidate of the C=64, P=4, U search:
+# C*P = 256 correlation FFMAs plus the 80-operation epilogue of the numeric
+# convention (solve 20, quantise 25, gain 34, compare 1).
+OPS_PER_CANDIDATE = 256 + 80
+# DRAM traffic of one search launch from an ncu capture (profiles/), valid only
+# for the kernel source it was measured on.
+SEARCH_TRAFFIC = {"source_sha256": None, "bytes_per_launch": None}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+# ------------------------------------------------------------------ clocks --
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.gpu_id:
+            cmd += ["-i", self.gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        pw = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def gpu_id_for(dev) -> str:
+    import torch
+    try:
+        p = torch.cuda.get_device_properties(dev)
+        return "%08X:%02X:%02X.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+        return vis.split(",")[dev.index or 0] if vis else str(dev.index or 0)
+
+
+# ----------------------------------------------------------- cpu baseline --
+def oracle_sample(wl, mods_host, target_s: float, seed: int = 0):
+    """Time the oracle (as it stands, all host cores) on whole rows sampled from
+    every module of the layer; returns (candidates/s, cores, description)."""
+    import numpy as np
+    from oracle import oracle as orc
+    oprm = orc.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
+    masks = orc.basis_masks(oprm)
+    rng = np.random.default_rng(seed)
+
+    def run(rows_per_module):
+        n = 0
+        t0 = time.perf_counter()
+        for m in mods_host:
+            rows = rng.choice(m["W"].shape[0], rows_per_module, replace=False)
+            orc.encode_tiles(oprm, m["W"][rows], m["W0"][rows], m["act"], masks=masks)
+            n += rows_per_module * m["W"].shape[1] // wl.C
+        return n, time.perf_counter() - t0
+
+    n1, t1 = run(1)                       # calibration: one row of every module
+    per_tile = t1 / n1
+    rows = max(1, int(target_s / (per_tile * sum(m["W"].shape[1] // wl.C for m in mods_host))))
+    n, t = run(rows)
+    cands = n * wl.S
+    desc = (f"{rows} random whole rows of each of the 7 modules ({n} tiles x {wl.S} seeds = "
+            f"{cands:,} candidates) in {t:.1f} s")
+    return cands / t, orc.num_threads(), desc
+
+
+def host_modules(mods):
+    return [{"W": m["W"].float().cpu().numpy(), "W0": m["W0"].float().cpu().numpy(),
+             "act": m["act"].cpu().numpy()} for m in mods]
+
+
+# ------------------------------------------------------------- reference --
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+    from oracle import oracle as orc
+    from synth import WORKLOADS, make_layer
+    wl = WORKLOADS[WORKLOAD]
+    orc.build()
+    mods = host_modules(make_layer(wl, layer=0, device="cpu"))
+    oprm = orc.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
+    masks = orc.basis_masks(oprm)
+    rng = np.random.default_rng(1)
+    # one step = one whole row of every module (1 row x n_cb tiles each)
+    def step():
+        n = 0
+        for m in mods:
+            r = int(rng.integers(m["W"].shape[0]))
+            orc.encode_tiles(oprm, m["W"][r:r + 1], m["W0"][r:r + 1], m["act"], masks=masks)
+            n += m["W"].shape[1] // wl.C
+        return n * wl.S
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    cands = sum(step() for _ in range(args.steps))
+    dt = time.perf_counter() - t0
+    v = cands / dt
+    sample = (f"per step one random whole row of each of the 7 modules "
+              f"({cands // args.steps:,} candidates, S = {wl.S})")
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": {"workload": wl.description},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": orc.num_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ ours --
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_23144_gb300 as aw
+    from synth import WORKLOADS, make_layer
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    wl = WORKLOADS[WORKLOAD]
+    mods = make_layer(wl, layer=rank, device=dev)
+    prm = aw.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
+    T = wl.tiles_per_layer
+    cands_per_step = T * wl.S
+    enc_ws = torch.empty(aw.awsrc_encode_workspace_bytes(prm, mods), dtype=torch.uint8, device=dev)
+    cands = torch.empty((T, 16), dtype=torch.uint8, device=dev)
+    outs = [torch.empty_like(m["W0"]) for m in mods]
+    cap = aw.awsrc_stream_capacity(prm, mods, [RATE])
+    sel_out = torch.zeros(cap, dtype=torch.uint8, device=dev)
+    sel_counts = torch.empty(len(mods), dtype=torch.int64, device=dev)
+    sel_bytes = torch.empty(1, dtype=torch.int64, device=dev)
+    stream_dev = [None]
+    sel_ws = [None]
+    dec_ws = [None]
+
+    def step(ev_dec=None):
+        aw.awsrc_encode_tiles(prm, mods, out=cands, workspace=enc_ws)
+        s, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, [RATE], workspace=sel_ws[0],
+                                                    out=sel_out, counts=sel_counts, nbytes=sel_bytes)
+        sel_ws[0] = s._awsrc_workspace
+        stream_dev[0] = (s, counts, nbytes)
+        if ev_dec is not None:
+            ev_dec[0].record()
+        aw.awsrc_decode_apply(prm, mods, s, -1, outs=outs, workspace=dec_ws[0])
+        dec_ws[0] = outs[0]._awsrc_workspace
+        if ev_dec is not None:
+            ev_dec[1].record()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    assert aw.awsrc_workspace_status(enc_ws) == 0, "encoder self-check fault"
+
+    # timed region: K steps, events on the launching stream
+    ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev_d = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    l0 = aw.awsrc_kernel_launches()
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_id_for(dev)) as clk:
+        start.record()
+        for k in range(args.steps):
+            aw.awsrc_set_timing_events(ev_s[k], ev_e[k])
+            step(ev_d[k])
+        end.record()
+        torch.cuda.synchronize()
+    barrier()
+    aw.awsrc_set_timing_events(None, None)
+    launches = aw.awsrc_kernel_launches() - l0
+    ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    search_ms = statistics.mean(a.elapsed_time(b) for a, b in zip(ev_s, ev_e))
+    dec_ms = statistics.mean(a.elapsed_time(b) for a, b in zip(ev_d))
+    s, counts, nbytes = stream_dev[0]
+    stream_bytes = int(nbytes[0].item())
+    w0_bytes = sum(m["W0"].numel() * m["W0"].element_size() for m in mods)
+    out_bytes = sum(o.numel() * o.element_size() for o in outs)
+    dec_gbs = (w0_bytes + out_bytes + stream_bytes) / (dec_ms * 1e-3) / 1e9
+
+    peaks, peak_kind = measured_peaks()
+    nsm = torch.cuda.get_device_properties(dev).multi_processor_count
+    fp32_peak = nsm * 128 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
+    achieved = cands_per_step * OPS_PER_CANDIDATE / (search_ms * 1e-3)
+    src = open(os.path.join(ROOT, "paper_2608_23144_gb300", "csrc", "search_c64p4.cu"), "rb").read()
+    traffic = (SEARCH_TRAFFIC["bytes_per_launch"]
+               if SEARCH_TRAFFIC["source_sha256"] == hashlib.sha256(src).hexdigest() else None)
+    roofline = {"bound": "alu", "kernel": "search_c64p4", "achieved": achieved / 1e9,
+                "peak": fp32_peak / 1e9, "unit": "Gop/s", "frac": achieved / fp32_peak,
+                "traffic": traffic, "peak_kind": f"{peak_kind}: {nsm} SMs x 128 FP32 lanes x "
+                f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
+                "ops_per_candidate": OPS_PER_CANDIDATE, "search_ms": search_ms}
+    decode = {"gbs": dec_gbs, "ms": dec_ms, "frac_of_hbm": dec_gbs / float(peaks.get("hbm_gbs", 6800.0)),
+              "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0))}
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        host = [{k: (v.cpu().pin_memory() if torch.is_tensor(v) else v) for k, v in m.items()} for m in mods]
+        h2d = sum(v.numel() * v.element_size() for m in host for k, v in m.items()
+                  if k in ("W", "W0", "act") and torch.is_tensor(v))
+        host_stream = torch.empty(s.numel(), dtype=torch.uint8).pin_memory()
+        host_counts = torch.empty(counts.numel() + nbytes.numel(), dtype=torch.int64).pin_memory()
+        d2h = host_stream.numel() + host_counts.numel() * 8
+
+        def e2e_step():
+            for m, hm in zip(mods, host):
+                for k in ("W", "W0", "act"):
+                    m[k].copy_(hm[k], non_blocking=True)
+            step()
+            s2, c2, n2 = stream_dev[0]
+            host_stream.copy_(s2, non_blocking=True)
+            host_counts[: c2.numel()].copy_(c2, non_blocking=True)
+            host_counts[c2.numel():].copy_(n2, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            e2e_step()
+            torch.cuda.synchronize()   # the result is read back on the host every step
+        dt = time.perf_counter() - t0
+        barrier()
+        if world > 1:
+            t = torch.tensor([dt], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            dt = float(t.item())
+        e2e = {"value": world * cands_per_step * args.steps / dt, "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": 1e3 * dt / args.steps}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, cores, desc = oracle_sample(wl, host_modules(mods), args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
+
+    if rank == 0:
+        value = world * cands_per_step * args.steps / (ms * 1e-3)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": wl.description, "tiles_per_gpu": T, "seeds": wl.S, "C": wl.C,
+                       "P": wl.P, "b": wl.b, "rate_bpw": RATE, "variant": "U",
+                       "parallelism": f"{world} independent layers" if world > 1 else "single GPU",
+                       "l2": "inputs larger than L2 (W and W0 of the layer: 308 MB per step)"},
+            "layers_per_s": world * args.steps / (ms * 1e-3),
+            "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
+            "decode_apply": decode,
+            "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

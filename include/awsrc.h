@@ -264,8 +264,10 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  * tiles without a record keep W0 unchanged, so K == 0 returns W0 exactly.
  * Any prefix of a progressive stream decodes against the same W0 (Sec. 3.3).
  *   stream   device, header + records as written by awsrc_select_records.
+ *   stream_len  bytes readable at `stream`; records beyond it are never read.
  *   K        records to apply (0 <= K <= header's K). K < 0 applies all the
- *            header's records (read on the device; no synchronisation).
+ *            header's records (read on the device; no synchronisation). Either
+ *            way at most (stream_len - h) / L records are applied.
  *   W_hat    host array of n_mod device pointers, rows*cols elements of out_dtype.
  *   mode     DENSE: every element of W_hat is written (W0 copied, corrected where
  *            a record exists). INPLACE: only the tiles named by records are
@@ -278,7 +280,7 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  */
 awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 const awsrc_module* mods, const uint8_t* stream,
-                                int64_t K, void* const* W_hat, int32_t out_dtype,
+                                size_t stream_len, int64_t K, void* const* W_hat, int32_t out_dtype,
                                 int32_t mode, void* workspace, size_t workspace_bytes,
                                 void* stream_handle);
 
@@ -286,15 +288,33 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
 
 /*
  * awsrc_workspace_status — synchronises `stream`, then reads and clears the
- * device fault word kept at the start of an encode/select/decode workspace.
- * *flags == 0 means no kernel reported a fault since the last call.
- * Bit 1: a record named a tile or seed out of range (decoder);
- * bit 2: encoder self-check mismatch between search and finalisation.
+ * device fault word kept in the first bytes of an encode/select/decode
+ * workspace. Each of those entry points clears the word when it starts, so the
+ * flags describe the last call made with this workspace; 0 means no fault.
+ * Bit 0 (1): a record named a tile or seed out of range (decoder; skipped).
+ * Bit 1 (2): encoder self-check — the finalisation recomputed a different gain
+ *            than the search found (never expected).
+ * Bit 2 (4): a bounded wait inside a kernel gave up (never expected).
  */
 awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags);
 
 const char* awsrc_status_string(awsrc_status st);
 const char* awsrc_last_error_message(void);
+
+/* -------------------------------------------------------------- diagnostics --
+ * Measurement hooks with no counterpart in the paper. */
+
+/*
+ * awsrc_set_timing_events — for the calling host thread, makes every later
+ * awsrc_encode_tiles record `before_search` (a cudaEvent_t) on its stream
+ * immediately before its first seed-search kernel and `after_search`
+ * immediately after its last one. NULL, NULL switches it off. The events are
+ * owned by the caller and must outlive the calls that record them.
+ */
+void awsrc_set_timing_events(void* before_search, void* after_search);
+
+/* Number of kernels this library has launched in the process so far. */
+uint64_t awsrc_kernel_launches(void);
 
 #ifdef __cplusplus
 }

@@ -63,6 +63,8 @@ def lib():
             L = ct.CDLL(_LIB_PATH)
             P = ct.POINTER
             vp = ct.c_void_p
+            L.orc_num_threads.restype = ct.c_int
+            L.orc_num_threads.argtypes = []
             L.orc_splitmix64_output.restype = ct.c_uint64
             L.orc_splitmix64_output.argtypes = [ct.c_uint64, ct.c_uint64]
             L.orc_gen_basis.argtypes = [ct.c_uint64, ct.c_uint32, ct.c_int, ct.c_int, ct.c_int, vp, vp, vp, vp]
@@ -109,6 +111,10 @@ def params(C=64, P=4, b=4, S=256, b_e=8, e_bias=0, scale_mode=0, permute=1, vari
 
 def _ptr(a: np.ndarray):
     return a.ctypes.data_as(ct.c_void_p)
+
+
+def num_threads() -> int:
+    return int(lib().orc_num_threads())
 
 
 def splitmix64_output(x: int, n: int) -> int:

@@ -1,0 +1,284 @@
+"""ctypes binding of libawsrc.so (include/awsrc.h): argument marshalling only.
+
+Every entry point takes torch tensors that already live on the current CUDA
+device, passes their data pointers and the current stream to the C ABI and
+returns the output tensors. Workspaces are allocated here, on the caller's
+side of the ABI, with torch's allocator; the library itself allocates nothing.
+If the shared library is missing the import of this module fails loudly: there
+is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes as ct
+import os
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libawsrc.so")
+
+VARIANT_U, VARIANT_PF = 0, 1
+SCALE_POW2, SCALE_FP16 = 0, 1
+DTYPE_F32, DTYPE_BF16 = 0, 1
+DECODE_DENSE, DECODE_INPLACE = 0, 1
+
+STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "unsupported", 4: "budget",
+          5: "cuda", 6: "workspace", 7: "capacity", 8: "device fault"}
+
+CANDIDATE_DTYPE = np.dtype([("gain", "<f4"), ("seed", "<u2"), ("scale", "<i2"), ("code", "i1", (8,))])
+
+
+class AwsrcError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str = ""):
+        super().__init__(f"{where}: awsrc status {status} ({STATUS.get(status, '?')}) {msg}".strip())
+        self.status = status
+
+
+class Params(ct.Structure):
+    _fields_ = [
+        ("C", ct.c_int32), ("P", ct.c_int32), ("b", ct.c_int32), ("S", ct.c_int32),
+        ("b_e", ct.c_int32), ("e_bias", ct.c_int32),
+        ("scale_mode", ct.c_int32), ("permute", ct.c_int32), ("variant", ct.c_int32),
+        ("ridge_rel", ct.c_float), ("gen_seed", ct.c_uint64),
+    ]
+
+
+class Module(ct.Structure):
+    _fields_ = [
+        ("rows", ct.c_int64), ("cols", ct.c_int64),
+        ("w_dtype", ct.c_int32), ("w0_dtype", ct.c_int32),
+        ("W", ct.c_void_p), ("W0", ct.c_void_p),
+        ("act", ct.c_void_p), ("fisher", ct.c_void_p),
+        ("w_act", ct.c_float), ("w_fisher", ct.c_float),
+    ]
+
+
+def params(C=64, P=4, b=4, S=4096, b_e=8, e_bias=0, scale_mode=SCALE_POW2, permute=1,
+           variant=VARIANT_U, ridge_rel=1e-6, gen_seed=0) -> Params:
+    return Params(C, P, b, S, b_e, e_bias, scale_mode, permute, variant,
+                  ct.c_float(ridge_rel).value, gen_seed)
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(
+            f"AWSRC CUDA library not built ({LIB_PATH} missing): run "
+            "`python -c 'import __graft_entry__ as g; g.build()'` first")
+    L = ct.CDLL(LIB_PATH)
+    P = ct.POINTER
+    vp, sz = ct.c_void_p, ct.c_size_t
+    st = ct.c_int
+    L.awsrc_status_string.restype = ct.c_char_p
+    L.awsrc_status_string.argtypes = [st]
+    L.awsrc_last_error_message.restype = ct.c_char_p
+    L.awsrc_last_error_message.argtypes = []
+    L.awsrc_record_bytes.restype = ct.c_int64
+    L.awsrc_record_bytes.argtypes = [P(Params), ct.c_int64]
+    L.awsrc_header_bytes.restype = ct.c_int64
+    L.awsrc_header_bytes.argtypes = [ct.c_int32]
+    L.awsrc_encode_workspace_bytes.restype = st
+    L.awsrc_encode_workspace_bytes.argtypes = [P(Params), ct.c_int32, P(Module), P(sz)]
+    L.awsrc_encode_tiles.restype = st
+    L.awsrc_encode_tiles.argtypes = [P(Params), ct.c_int32, P(Module), vp, vp, sz, vp]
+    L.awsrc_gen_basis.restype = st
+    L.awsrc_gen_basis.argtypes = [P(Params), vp, vp]
+    L.awsrc_stream_capacity.restype = st
+    L.awsrc_stream_capacity.argtypes = [P(Params), ct.c_int32, P(Module), P(ct.c_double), ct.c_int32, P(sz)]
+    L.awsrc_select_workspace_bytes.restype = st
+    L.awsrc_select_workspace_bytes.argtypes = [P(Params), ct.c_int32, P(Module), P(sz)]
+    L.awsrc_select_records.restype = st
+    L.awsrc_select_records.argtypes = [P(Params), ct.c_int32, P(Module), vp, P(ct.c_double), ct.c_int32,
+                                       vp, sz, vp, vp, vp, sz, vp]
+    L.awsrc_decode_workspace_bytes.restype = st
+    L.awsrc_decode_workspace_bytes.argtypes = [P(Params), ct.c_int32, P(Module), ct.c_int32, P(sz)]
+    L.awsrc_decode_apply.restype = st
+    L.awsrc_decode_apply.argtypes = [P(Params), ct.c_int32, P(Module), vp, sz, ct.c_int64, P(vp), ct.c_int32,
+                                     ct.c_int32, vp, sz, vp]
+    L.awsrc_set_timing_events.restype = None
+    L.awsrc_set_timing_events.argtypes = [vp, vp]
+    L.awsrc_kernel_launches.restype = ct.c_uint64
+    L.awsrc_kernel_launches.argtypes = []
+    L.awsrc_workspace_status.restype = st
+    L.awsrc_workspace_status.argtypes = [vp, vp, P(ct.c_uint32)]
+    return L
+
+
+lib = _load()
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        msg = lib.awsrc_last_error_message().decode() if status == 5 else ""
+        raise AwsrcError(status, where, msg)
+
+
+def _stream(stream=None) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return DTYPE_F32
+    if t.dtype == torch.bfloat16:
+        return DTYPE_BF16
+    raise TypeError(f"unsupported weight dtype {t.dtype} (float32 or bfloat16)")
+
+
+def _dev_ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("tensors passed to the AWSRC library must be contiguous CUDA tensors")
+    return t.data_ptr()
+
+
+def module_array(modules: Sequence[Dict[str, object]], decoder: bool = False):
+    """awsrc_module[] from dicts with W, W0, act (and fisher, w_act, w_fisher)."""
+    arr = (Module * len(modules))()
+    for i, m in enumerate(modules):
+        W0 = m["W0"]
+        W = m.get("W")
+        rows, cols = W0.shape
+        arr[i].rows, arr[i].cols = rows, cols
+        arr[i].w0_dtype = _dtype_code(W0)
+        arr[i].W0 = _dev_ptr(W0)
+        if W is not None and not decoder:
+            arr[i].w_dtype = _dtype_code(W)
+            arr[i].W = _dev_ptr(W)
+        if m.get("act") is not None and not decoder:
+            arr[i].act = _dev_ptr(m["act"])
+        if m.get("fisher") is not None and not decoder:
+            arr[i].fisher = _dev_ptr(m["fisher"])
+        arr[i].w_act = float(m.get("w_act", 1.0))
+        arr[i].w_fisher = float(m.get("w_fisher", 0.0))
+    return arr
+
+
+def _tiles(prm: Params, modules) -> int:
+    return sum(int(m["W0"].shape[0]) * int(m["W0"].shape[1]) // prm.C for m in modules)
+
+
+def awsrc_record_bytes(prm: Params, T: int) -> int:
+    return int(lib.awsrc_record_bytes(ct.byref(prm), T))
+
+
+def awsrc_header_bytes(n_mod: int) -> int:
+    return int(lib.awsrc_header_bytes(n_mod))
+
+
+def awsrc_encode_workspace_bytes(prm: Params, modules) -> int:
+    mods = module_array(modules)
+    n = ct.c_size_t()
+    _check(lib.awsrc_encode_workspace_bytes(ct.byref(prm), len(modules), mods, ct.byref(n)), "encode_workspace_bytes")
+    return n.value
+
+
+def awsrc_encode_tiles(prm: Params, modules, out: Optional[torch.Tensor] = None,
+                       workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Seed search (Sec. 3.2): one best candidate per tile, uint8 [T, 16] on the device."""
+    mods = module_array(modules)
+    T = _tiles(prm, modules)
+    dev = modules[0]["W0"].device
+    if out is None:
+        out = torch.empty((T, 16), dtype=torch.uint8, device=dev)
+    need = awsrc_encode_workspace_bytes(prm, modules)
+    if workspace is None or workspace.numel() < need:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(lib.awsrc_encode_tiles(ct.byref(prm), len(modules), mods, _dev_ptr(out), _dev_ptr(workspace),
+                                  workspace.numel(), _stream(stream)), "encode_tiles")
+    out._awsrc_workspace = workspace  # keep alive for awsrc_workspace_status
+    return out
+
+
+def awsrc_gen_basis(prm: Params, stream=None, device="cuda") -> torch.Tensor:
+    W = (prm.C + 63) // 64
+    masks = torch.empty(prm.S * prm.P * W, dtype=torch.int64, device=device)
+    _check(lib.awsrc_gen_basis(ct.byref(prm), _dev_ptr(masks), _stream(stream)), "gen_basis")
+    return masks
+
+
+def awsrc_stream_capacity(prm: Params, modules, rates: Sequence[float]) -> int:
+    mods = module_array(modules, decoder=True)
+    r = (ct.c_double * len(rates))(*rates)
+    n = ct.c_size_t()
+    _check(lib.awsrc_stream_capacity(ct.byref(prm), len(modules), mods, r, len(rates), ct.byref(n)), "stream_capacity")
+    return n.value
+
+
+def awsrc_select_records(prm: Params, modules, cands: torch.Tensor, rates: Sequence[float],
+                         workspace: Optional[torch.Tensor] = None, stream=None,
+                         out: Optional[torch.Tensor] = None, counts: Optional[torch.Tensor] = None,
+                         nbytes: Optional[torch.Tensor] = None):
+    """Sec. 3.3 allocation + Eq. 5 serialisation. Returns (stream bytes [capacity] uint8,
+    counts int64 (U: per module, PF: per rate), bytes int64 (per rate)), all on the device.
+    Only the first bytes[r] bytes of the stream are written."""
+    mods = module_array(modules, decoder=True)
+    dev = cands.device
+    r = (ct.c_double * len(rates))(*rates)
+    cap = awsrc_stream_capacity(prm, modules, rates)
+    n = ct.c_size_t()
+    _check(lib.awsrc_select_workspace_bytes(ct.byref(prm), len(modules), mods, ct.byref(n)), "select_workspace_bytes")
+    if workspace is None or workspace.numel() < n.value:
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=dev)
+    if out is None or out.numel() < cap:
+        out = torch.zeros(cap, dtype=torch.uint8, device=dev)
+    ncount = len(modules) if prm.variant == VARIANT_U else len(rates)
+    if counts is None or counts.numel() < ncount:
+        counts = torch.empty(ncount, dtype=torch.int64, device=dev)
+    if nbytes is None or nbytes.numel() < len(rates):
+        nbytes = torch.empty(len(rates), dtype=torch.int64, device=dev)
+    _check(lib.awsrc_select_records(ct.byref(prm), len(modules), mods, _dev_ptr(cands), r, len(rates),
+                                    _dev_ptr(out), out.numel(), _dev_ptr(counts), _dev_ptr(nbytes),
+                                    _dev_ptr(workspace), workspace.numel(), _stream(stream)), "select_records")
+    out._awsrc_workspace = workspace
+    return out, counts, nbytes
+
+
+def awsrc_decode_apply(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
+                       outs: Optional[List[torch.Tensor]] = None, out_dtype=None,
+                       mode: int = DECODE_DENSE, workspace: Optional[torch.Tensor] = None,
+                       stream=None) -> List[torch.Tensor]:
+    """Decoder (Sec. 3.2): W_hat = W0 + B_s alpha_hat for the first K records (K < 0: all)."""
+    mods = module_array(modules, decoder=True)
+    dev = stream_bytes.device
+    if out_dtype is None:
+        out_dtype = modules[0]["W0"].dtype
+    code = DTYPE_F32 if out_dtype == torch.float32 else DTYPE_BF16
+    if outs is None:
+        outs = [torch.empty_like(m["W0"], dtype=out_dtype) for m in modules]
+    ptrs = (ct.c_void_p * len(outs))(*[_dev_ptr(o) for o in outs])
+    n = ct.c_size_t()
+    _check(lib.awsrc_decode_workspace_bytes(ct.byref(prm), len(modules), mods, mode, ct.byref(n)), "decode_workspace_bytes")
+    if workspace is None or workspace.numel() < n.value:
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=dev)
+    _check(lib.awsrc_decode_apply(ct.byref(prm), len(modules), mods, _dev_ptr(stream_bytes),
+                                  stream_bytes.numel(), int(K), ptrs,
+                                  code, mode, _dev_ptr(workspace), workspace.numel(), _stream(stream)),
+           "decode_apply")
+    outs[0]._awsrc_workspace = workspace
+    return outs
+
+
+def awsrc_workspace_status(workspace: torch.Tensor, stream=None) -> int:
+    flags = ct.c_uint32()
+    _check(lib.awsrc_workspace_status(_dev_ptr(workspace), _stream(stream), ct.byref(flags)), "workspace_status")
+    return flags.value
+
+
+def awsrc_set_timing_events(before: Optional[torch.cuda.Event], after: Optional[torch.cuda.Event]):
+    """Record `before`/`after` around the seed-search launches of later encode calls."""
+    b = before.cuda_event if before is not None else None
+    a = after.cuda_event if after is not None else None
+    lib.awsrc_set_timing_events(b, a)
+
+
+def awsrc_kernel_launches() -> int:
+    return int(lib.awsrc_kernel_launches())
+
+
+def candidates_to_numpy(cands: torch.Tensor) -> np.ndarray:
+    """Device candidate bytes -> host structured array (gain, seed, scale, code[8])."""
+    return cands.cpu().numpy().reshape(-1).view(CANDIDATE_DTYPE)

@@ -1,0 +1,450 @@
+// api.cu — the extern "C" entry points declared in include/awsrc.h: argument
+// validation, workspace layout and the launch sequence of each step.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+#include "internal.h"
+
+namespace awsrc {
+
+namespace {
+thread_local char g_err[512] = "";
+thread_local cudaEvent_t g_ev_before = nullptr, g_ev_after = nullptr;
+std::atomic<uint64_t> g_launches{0};
+constexpr int64_t kTargetBlocks = 1216;  // enough blocks to fill a GB300 (152 SMs) several times
+
+int ceil_log2_host(uint64_t x) {
+  int n = 0;
+  while (n < 64 && (1ull << n) < x) ++n;
+  return n;
+}
+
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+bool use_c64p4(const Prm& pr) {
+  return pr.C == 64 && pr.P == 4 && pr.variant == AWSRC_VARIANT_U;
+}
+
+awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mods, bool encoder,
+                           int64_t* T_out) {
+  if (n_mod < 1 || mods == nullptr) return AWSRC_ERR_INVALID_ARG;
+  int64_t T = 0;
+  for (int m = 0; m < n_mod; ++m) {
+    const awsrc_module& md = mods[m];
+    if (md.rows < 1 || md.cols < 1) return AWSRC_ERR_SHAPE;
+    if (md.cols % pr.C != 0) return AWSRC_ERR_SHAPE;
+    if (md.w0_dtype != AWSRC_DTYPE_F32 && md.w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+    if (encoder) {
+      if (md.w_dtype != AWSRC_DTYPE_F32 && md.w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+      if (!md.W || !md.W0 || !md.act) return AWSRC_ERR_INVALID_ARG;
+      if (pr.variant == AWSRC_VARIANT_PF && !md.fisher) return AWSRC_ERR_INVALID_ARG;
+    }
+    T += md.rows * (md.cols / pr.C);
+  }
+  if (T >= (1ll << 32)) return AWSRC_ERR_UNSUPPORTED;
+  *T_out = T;
+  return AWSRC_OK;
+}
+
+struct EncodeLayout {
+  size_t masks, gram, mexp, partials, total;
+  int nsplit;
+  bool spec;
+};
+
+EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mods, int64_t T) {
+  EncodeLayout L{};
+  L.spec = use_c64p4(pr);
+  const int rb = L.spec ? search_c64p4_rows() : generic_rows();
+  int64_t base_blocks = 0, ncb = 0;
+  for (int m = 0; m < n_mod; ++m) {
+    const int64_t n_cb = mods[m].cols / pr.C;
+    ncb += n_cb;
+    base_blocks += n_cb * ((mods[m].rows + rb - 1) / rb);
+  }
+  const int64_t units = L.spec ? pr.S_pad / search_c64p4_chunk()
+                               : (pr.S + generic_chunk() - 1) / generic_chunk();
+  int64_t ns = (kTargetBlocks + base_blocks - 1) / base_blocks;
+  ns = std::max<int64_t>(1, std::min<int64_t>(ns, units));
+  L.nsplit = (int)ns;
+  size_t off = kStatusBytes;
+  L.masks = off;
+  off += align_up((size_t)pr.S_pad * pr.P * pr.W * 8, 256);
+  L.gram = off;
+  if (pr.variant == AWSRC_VARIANT_U) off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
+  L.mexp = off;
+  if (L.spec) off += align_up((size_t)pr.S_pad * 64 * 4 * 4, 256);
+  L.partials = off;
+  off += align_up((size_t)L.nsplit * T * 8, 256);
+  L.total = off;
+  return L;
+}
+
+}  // namespace
+
+void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+awsrc_status cuda_fail(cudaError_t e, const char* where) {
+  snprintf(g_err, sizeof g_err, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
+  return AWSRC_ERR_CUDA;
+}
+
+awsrc_status check_launch(const char* where) {
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, where);
+  return AWSRC_OK;
+}
+
+awsrc_status make_prm(const awsrc_params* p, Prm* out) {
+  if (!p) return AWSRC_ERR_INVALID_ARG;
+  if (!is_pow2(p->C) || p->C < 4 || p->C > kMaxC) return AWSRC_ERR_SHAPE;
+  if (p->P < 1 || p->P > kMaxP || p->P > p->C) return AWSRC_ERR_UNSUPPORTED;
+  if (p->b < 2 || p->b > 8) return AWSRC_ERR_UNSUPPORTED;
+  if (p->S < 1 || p->S > 65536) return AWSRC_ERR_UNSUPPORTED;
+  if (p->variant != AWSRC_VARIANT_U && p->variant != AWSRC_VARIANT_PF) return AWSRC_ERR_INVALID_ARG;
+  if (p->permute != 0 && p->permute != 1) return AWSRC_ERR_INVALID_ARG;
+  if (!(p->ridge_rel >= 0.0f) || !std::isfinite(p->ridge_rel)) return AWSRC_ERR_INVALID_ARG;
+  Prm r{};
+  r.C = p->C; r.P = p->P; r.b = p->b; r.S = p->S; r.b_e = p->b_e; r.e_bias = p->e_bias;
+  r.scale_mode = p->scale_mode; r.permute = p->permute; r.variant = p->variant;
+  r.ridge_rel = p->ridge_rel; r.gen_seed = p->gen_seed;
+  if (p->scale_mode == AWSRC_SCALE_POW2) {
+    if (p->b_e < 1 || p->b_e > 8) return AWSRC_ERR_UNSUPPORTED;
+    r.e_lo = std::max(p->e_bias - (1 << (p->b_e - 1)), -126);
+    r.e_hi = std::min(p->e_bias + (1 << (p->b_e - 1)) - 1, 126);
+    if (r.e_lo > r.e_hi) return AWSRC_ERR_UNSUPPORTED;
+  } else if (p->scale_mode == AWSRC_SCALE_FP16) {
+    if (p->b_e != 16) return AWSRC_ERR_UNSUPPORTED;
+    r.e_lo = r.e_hi = 0;
+  } else {
+    return AWSRC_ERR_INVALID_ARG;
+  }
+  r.qmax = (1 << (p->b - 1)) - 1;
+  r.qmaxf = (float)r.qmax;
+  r.c = (float)(1.0 / std::sqrt((double)p->C));
+  r.c2 = 1.0f / (float)p->C;
+  r.W = (p->C + 63) / 64;
+  r.S_pad = (p->S + 31) / 32 * 32;
+  r.logC = ceil_log2_host((uint64_t)p->C);
+  *out = r;
+  return AWSRC_OK;
+}
+
+}  // namespace awsrc
+
+using namespace awsrc;
+
+extern "C" {
+
+const char* awsrc_status_string(awsrc_status st) {
+  switch (st) {
+    case AWSRC_OK: return "ok";
+    case AWSRC_ERR_INVALID_ARG: return "invalid argument";
+    case AWSRC_ERR_SHAPE: return "unsupported shape (C must be a power of two in [4, 256] dividing cols)";
+    case AWSRC_ERR_UNSUPPORTED: return "parameter outside the supported range";
+    case AWSRC_ERR_BUDGET: return "byte budget smaller than the stream header";
+    case AWSRC_ERR_CUDA: return "CUDA runtime error";
+    case AWSRC_ERR_WORKSPACE: return "workspace missing or too small";
+    case AWSRC_ERR_CAPACITY: return "output stream buffer too small";
+    case AWSRC_ERR_DEVICE: return "a kernel reported a fault in its inputs";
+  }
+  return "unknown status";
+}
+
+const char* awsrc_last_error_message(void) { return g_err; }
+
+void awsrc_set_timing_events(void* before_search, void* after_search) {
+  g_ev_before = (cudaEvent_t)before_search;
+  g_ev_after = (cudaEvent_t)after_search;
+}
+
+uint64_t awsrc_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+int64_t awsrc_header_bytes(int32_t n_mod) { return n_mod < 0 ? -1 : 40 + 8 * (int64_t)n_mod; }
+
+int64_t awsrc_record_bytes(const awsrc_params* prm, int64_t T) {
+  Prm pr;
+  if (make_prm(prm, &pr) != AWSRC_OK || T < 1) return -1;
+  const int64_t bits = ceil_log2_host((uint64_t)T) + ceil_log2_host((uint64_t)pr.S) + pr.b_e +
+                       (int64_t)pr.P * pr.b;
+  return (bits + 7) / 8;
+}
+
+awsrc_status awsrc_encode_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, size_t* bytes) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  if (!bytes) return AWSRC_ERR_INVALID_ARG;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  *bytes = encode_layout(pr, n_mod, mods, T).total;
+  return AWSRC_OK;
+}
+
+awsrc_status awsrc_gen_basis(const awsrc_params* prm, uint64_t* masks, void* stream) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  if (!masks) return AWSRC_ERR_INVALID_ARG;
+  const cudaError_t e = launch_gen_basis(pr, masks, pr.S, (cudaStream_t)stream);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "gen_basis");
+}
+
+awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                awsrc_candidate* out, void* workspace, size_t workspace_bytes,
+                                void* stream) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, true, &T)) != AWSRC_OK) return s;
+  if (!out) return AWSRC_ERR_INVALID_ARG;
+  const EncodeLayout lay = encode_layout(pr, n_mod, mods, T);
+  if (!workspace || workspace_bytes < lay.total) return AWSRC_ERR_WORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ws);
+  uint64_t* masks = reinterpret_cast<uint64_t*>(ws + lay.masks);
+  float* gram = reinterpret_cast<float*>(ws + lay.gram);
+  float* mexp = reinterpret_cast<float*>(ws + lay.mexp);
+  float2* partials = reinterpret_cast<float2*>(ws + lay.partials);
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return cuda_fail(e, "encode: clear status");
+  e = launch_gen_basis(pr, masks, pr.S_pad, st);
+  if (e != cudaSuccess) return cuda_fail(e, "encode: gen_basis");
+  if (lay.spec && (e = launch_expand_masks_c64p4(pr, masks, mexp, st)) != cudaSuccess)
+    return cuda_fail(e, "encode: expand masks");
+  const int rb = lay.spec ? search_c64p4_rows() : generic_rows();
+  int64_t tile_off = 0, gram_off = 0;
+  for (int g0 = 0; g0 < n_mod; g0 += kMaxModsPerLaunch) {
+    LaunchDesc ld;
+    std::memset(&ld, 0, sizeof ld);
+    ld.n = std::min(kMaxModsPerLaunch, n_mod - g0);
+    ld.T = T;
+    int64_t blocks = 0;
+    for (int i = 0; i < ld.n; ++i) {
+      const awsrc_module& md = mods[g0 + i];
+      ModDesc& d = ld.m[i];
+      d.W = md.W; d.W0 = md.W0; d.act = md.act; d.fisher = md.fisher;
+      d.rows = md.rows; d.cols = md.cols; d.n_cb = md.cols / pr.C;
+      d.n_rb = (md.rows + rb - 1) / rb;
+      d.tile_off = tile_off;
+      d.gram_off = gram_off;
+      d.block_off = blocks;
+      d.w_dtype = md.w_dtype; d.w0_dtype = md.w0_dtype;
+      d.nsplit = lay.nsplit;
+      d.w_act = md.w_act; d.w_fisher = md.w_fisher;
+      blocks += d.n_cb * d.n_rb * d.nsplit;
+      tile_off += d.rows * d.n_cb;
+      gram_off += d.n_cb * pr.S_pad;
+    }
+    if (pr.variant == AWSRC_VARIANT_U && (e = launch_gram_u(pr, ld, masks, gram, st)) != cudaSuccess)
+      return cuda_fail(e, "encode: gram");
+    if (g0 == 0 && g_ev_before && (e = cudaEventRecord(g_ev_before, st)) != cudaSuccess)
+      return cuda_fail(e, "encode: timing event");
+    if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, gram, blocks, partials, status, st);
+    else e = launch_search_generic(pr, ld, masks, gram, blocks, partials, st);
+    if (e != cudaSuccess) return cuda_fail(e, "encode: search");
+    if (g0 + kMaxModsPerLaunch >= n_mod && g_ev_after && (e = cudaEventRecord(g_ev_after, st)) != cudaSuccess)
+      return cuda_fail(e, "encode: timing event");
+    if ((e = launch_finalize(pr, ld, masks, gram, partials, lay.nsplit, out, status, st)) != cudaSuccess)
+      return cuda_fail(e, "encode: finalize");
+  }
+  return AWSRC_OK;
+}
+
+// ------------------------------------------------------------------ select --
+
+static awsrc_status select_plan(const Prm& pr, int32_t n_mod, const awsrc_module* mods,
+                                const double* rates, int32_t n_rates, SelectPlan* sp,
+                                std::vector<int64_t>* tile_off, std::vector<int64_t>* kcap) {
+  int64_t T;
+  awsrc_status s = check_modules(pr, n_mod, mods, false, &T);
+  if (s != AWSRC_OK) return s;
+  if (!rates || n_rates < 1) return AWSRC_ERR_INVALID_ARG;
+  if (pr.variant == AWSRC_VARIANT_U && n_rates != 1) return AWSRC_ERR_UNSUPPORTED;
+  if (n_rates > 64 || n_mod > 1024) return AWSRC_ERR_UNSUPPORTED;
+  sp->n_mod = n_mod;
+  sp->n_rates = n_rates;
+  sp->T = T;
+  sp->h = 40 + 8 * (int64_t)n_mod;
+  sp->L = (ceil_log2_host((uint64_t)T) + ceil_log2_host((uint64_t)pr.S) + pr.b_e +
+           (int64_t)pr.P * pr.b + 7) / 8;
+  int64_t N = 0;
+  tile_off->assign(n_mod + 1, 0);
+  int64_t maxTm = 1;
+  for (int m = 0; m < n_mod; ++m) {
+    const int64_t Tm = mods[m].rows * (mods[m].cols / pr.C);
+    (*tile_off)[m + 1] = (*tile_off)[m] + Tm;
+    maxTm = std::max(maxTm, Tm);
+    N += mods[m].rows * mods[m].cols;
+  }
+  for (int r = 0; r < n_rates; ++r)
+    if (!(rates[r] >= 0.0) || !std::isfinite(rates[r])) return AWSRC_ERR_INVALID_ARG;
+  kcap->clear();
+  if (pr.variant == AWSRC_VARIANT_U) {
+    const int64_t B = (int64_t)std::floor(rates[0] * (double)N / 8.0);
+    if (B < sp->h) return AWSRC_ERR_BUDGET;
+    int64_t cap = 0;
+    for (int m = 0; m < n_mod; ++m) {
+      const unsigned __int128 q = (unsigned __int128)(uint64_t)(B - sp->h) *
+                                  (uint64_t)(mods[m].rows * mods[m].cols);
+      const int64_t quota = (int64_t)(q / (uint64_t)N);
+      const int64_t k = std::min(quota / sp->L, (*tile_off)[m + 1] - (*tile_off)[m]);
+      kcap->push_back(k);
+      cap += k;
+    }
+    sp->cap_records = cap;
+    sp->tile_bits_local = ceil_log2_host((uint64_t)maxTm);
+    sp->mod_shift = 31 + sp->tile_bits_local;
+    sp->key_bits = sp->mod_shift + ceil_log2_host((uint64_t)n_mod);
+  } else {
+    int64_t cap = 0;
+    for (int r = 0; r < n_rates; ++r) {
+      const int64_t B = (int64_t)std::floor(rates[r] * (double)N / 8.0);
+      if (B < sp->h) return AWSRC_ERR_BUDGET;
+      const int64_t k = std::min((B - sp->h) / sp->L, T);
+      kcap->push_back(k);
+      cap = std::max(cap, k);
+    }
+    sp->cap_records = cap;
+    sp->tile_bits_local = ceil_log2_host((uint64_t)T);
+    sp->mod_shift = 0;
+    sp->key_bits = 31 + sp->tile_bits_local;
+  }
+  if (sp->key_bits > 64) return AWSRC_ERR_UNSUPPORTED;
+  sp->nblocks = (T + 2047) / 2048;
+  return AWSRC_OK;
+}
+
+awsrc_status awsrc_stream_capacity(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                   const double* rates_bpw, int32_t n_rates, size_t* bytes) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  if (!bytes) return AWSRC_ERR_INVALID_ARG;
+  SelectPlan sp;
+  std::vector<int64_t> to, kc;
+  if ((s = select_plan(pr, n_mod, mods, rates_bpw, n_rates, &sp, &to, &kc)) != AWSRC_OK) return s;
+  *bytes = (size_t)(sp.h + sp.cap_records * sp.L);
+  return AWSRC_OK;
+}
+
+awsrc_status awsrc_select_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, size_t* bytes) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  if (!bytes) return AWSRC_ERR_INVALID_ARG;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  SelectPlan sp{};
+  sp.T = T;
+  sp.nblocks = (T + 2047) / 2048;
+  *bytes = select_ws_bytes(sp);
+  return AWSRC_OK;
+}
+
+awsrc_status awsrc_select_records(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                  const awsrc_candidate* cands, const double* rates_bpw,
+                                  int32_t n_rates, uint8_t* stream_out, size_t stream_capacity,
+                                  int64_t* d_counts, int64_t* d_bytes, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  SelectPlan sp;
+  std::vector<int64_t> to, kc;
+  if ((s = select_plan(pr, n_mod, mods, rates_bpw, n_rates, &sp, &to, &kc)) != AWSRC_OK) return s;
+  if (!cands || !stream_out || !d_counts || !d_bytes) return AWSRC_ERR_INVALID_ARG;
+  if (stream_capacity < (size_t)(sp.h + sp.cap_records * sp.L)) return AWSRC_ERR_CAPACITY;
+  if (!workspace || workspace_bytes < select_ws_bytes(sp)) return AWSRC_ERR_WORKSPACE;
+  std::vector<int64_t> mt(n_mod);
+  for (int m = 0; m < n_mod; ++m) mt[m] = to[m + 1] - to[m];
+  const cudaError_t e = cudaMemsetAsync(workspace, 0, sizeof(uint32_t), (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "select: clear status");
+  return select_run(pr, sp, to.data(), mt.data(), kc.data(), cands, stream_out, d_counts, d_bytes,
+                    workspace, workspace_bytes, (cudaStream_t)stream);
+}
+
+// ------------------------------------------------------------------ decode --
+
+awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod,
+                                          const awsrc_module* mods, int32_t mode, size_t* bytes) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  if (!bytes) return AWSRC_ERR_INVALID_ARG;
+  if (mode != AWSRC_DECODE_DENSE && mode != AWSRC_DECODE_INPLACE) return AWSRC_ERR_INVALID_ARG;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  *bytes = kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256) + decode_scratch_bytes(T, mode);
+  return AWSRC_OK;
+}
+
+awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                const uint8_t* stream, size_t stream_len, int64_t K, void* const* W_hat,
+                                int32_t out_dtype, int32_t mode, void* workspace,
+                                size_t workspace_bytes, void* stream_handle) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  if (!stream || !W_hat) return AWSRC_ERR_INVALID_ARG;
+  if (out_dtype != AWSRC_DTYPE_F32 && out_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+  if (mode != AWSRC_DECODE_DENSE && mode != AWSRC_DECODE_INPLACE) return AWSRC_ERR_INVALID_ARG;
+  std::vector<DecodeMod> dm(n_mod);
+  int64_t off = 0;
+  for (int m = 0; m < n_mod; ++m) {
+    if (!W_hat[m]) return AWSRC_ERR_INVALID_ARG;
+    if (mode == AWSRC_DECODE_DENSE && !mods[m].W0) return AWSRC_ERR_INVALID_ARG;
+    if (mode == AWSRC_DECODE_INPLACE && mods[m].w0_dtype != out_dtype) return AWSRC_ERR_INVALID_ARG;
+    dm[m].W0 = mods[m].W0;
+    dm[m].out = W_hat[m];
+    dm[m].rows = mods[m].rows;
+    dm[m].cols = mods[m].cols;
+    dm[m].tile_off = off;
+    dm[m].w0_dtype = mods[m].w0_dtype;
+    dm[m].pad_ = 0;
+    off += mods[m].rows * (mods[m].cols / pr.C);
+  }
+  size_t need;
+  if ((s = awsrc_decode_workspace_bytes(prm, n_mod, mods, mode, &need)) != AWSRC_OK) return s;
+  if (!workspace || workspace_bytes < need) return AWSRC_ERR_WORKSPACE;
+  const int64_t L = awsrc_record_bytes(prm, T), h = awsrc_header_bytes(n_mod);
+  if (stream_len < (size_t)h) return AWSRC_ERR_INVALID_ARG;
+  const int64_t kmax = std::min<int64_t>(((int64_t)stream_len - h) / L, T);
+  if (K > kmax) return AWSRC_ERR_INVALID_ARG;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ws);
+  uint64_t* masks = reinterpret_cast<uint64_t*>(ws + kStatusBytes);
+  int32_t* map = reinterpret_cast<int32_t*>(ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256));
+  cudaStream_t st = (cudaStream_t)stream_handle;
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return cuda_fail(e, "decode: clear status");
+  e = launch_gen_basis(pr, masks, pr.S, st);
+  if (e != cudaSuccess) return cuda_fail(e, "decode: gen_basis");
+  e = launch_decode(pr, n_mod, dm.data(), T, L, h, stream, K, kmax, out_dtype, mode, masks, map, status, st);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "decode");
+}
+
+awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags) {
+  if (!workspace || !flags) return AWSRC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "workspace_status: sync");
+  uint32_t v = 0;
+  if ((e = cudaMemcpy(&v, workspace, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "workspace_status: read");
+  if ((e = cudaMemset(workspace, 0, sizeof v)) != cudaSuccess) return cuda_fail(e, "workspace_status: clear");
+  *flags = v;
+  return AWSRC_OK;
+}
+
+}  // extern "C"

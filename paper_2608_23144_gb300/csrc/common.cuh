@@ -1,0 +1,221 @@
+// common.cuh — device-side building blocks shared by the AWSRC kernels:
+// the shared basis generator (Sec. 3.1, Eq. 2), the binary32 fit / quantise /
+// gain epilogue (Eq. 3, Sec. 3.2, Eq. 4) and small launch descriptors.
+//
+// Every floating-point operation that decides an integer output is written
+// with an explicit round-to-nearest intrinsic (__fmaf_rn, __fmul_rn, ...), and
+// the library is compiled with --fmad=false, so the compiler cannot fuse or
+// reorder them: the order is the one the public header fixes.
+#pragma once
+
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "awsrc.h"
+
+namespace awsrc {
+
+constexpr int kMaxP = 8;
+constexpr int kMaxC = 256;
+constexpr int kMaxModsPerLaunch = 16;
+
+// Fault bits of the device status word kept at the start of every workspace.
+constexpr uint32_t kFaultRecord = 1u;     // decoder: record names a tile/seed out of range
+constexpr uint32_t kFaultSelfCheck = 2u;  // encoder: finalisation disagrees with the search
+constexpr uint32_t kFaultTimeout = 4u;    // a bounded wait gave up
+constexpr size_t kStatusBytes = 256;
+
+// Host-validated parameters plus derived constants, passed by value.
+struct Prm {
+  int C, P, b, S, b_e, e_bias, scale_mode, permute, variant;
+  float ridge_rel;
+  uint64_t gen_seed;
+  int qmax;       // 2^(b-1) - 1
+  float qmaxf;
+  int e_lo, e_hi; // POW2 exponent range, within [-126, 126]
+  float c;        // RN(C^-1/2)
+  float c2;       // 1/C (exact)
+  int W;          // 64-bit mask words per (seed, atom)
+  int S_pad;      // seeds rounded up to the search chunk
+  int logC;       // log2(C)
+};
+
+// ---------------------------------------------------------------- generator --
+// SplitMix64 (Steele, Lea & Flood 2014): n-th output of the stream at state x.
+__host__ __device__ __forceinline__ uint64_t sm64_output(uint64_t x, uint64_t n) {
+  uint64_t z = x + n * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// --------------------------------------------------------------- numerics --
+__device__ __forceinline__ float sign_f(uint64_t bit) {  // bit 1 -> -1.0f, 0 -> +1.0f
+  return __int_as_float(0x3f800000u | ((uint32_t)(bit & 1u) << 31));
+}
+
+// max with NaN propagation (PTX max.NaN.f32)
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+
+__device__ __forceinline__ float load_elem(const void* p, int64_t i, int dtype) {
+  if (dtype == AWSRC_DTYPE_F32) return static_cast<const float*>(p)[i];
+  return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
+}
+
+// Tile-domain check: |r| <= 2^16 and 0 <= d <= 2^32 (NaN fails both).
+__device__ __forceinline__ bool in_domain(float r, float d) {
+  return (fabsf(r) <= 65536.0f) && (d >= 0.0f) && (d <= 4294967296.0f);
+}
+
+// Packed strict-lower-triangle index of (k, i), k > i.
+__host__ __device__ constexpr int tri(int k, int i) { return k * (k - 1) / 2 + i; }
+
+// Floats per (column block, seed) entry of the U Gram table:
+// L (P(P-1)/2), invD (P), G off-diagonal (P(P-1)/2), gd (1), padded to 4.
+__host__ __device__ constexpr int gram_stride(int P) {
+  return ((P * (P - 1) + P + 1) + 3) / 4 * 4;
+}
+
+// LDL^T of A = G + eps I with G_pp = gd, G_pq = Goff[tri(q, p)]. Writes L and
+// invD; returns false if some pivot is not in (0, FLT_MAX].
+template <int P>
+__device__ __forceinline__ bool ldl_factor(float gd, float eps, const float* Goff, float* L,
+                                           float* invD) {
+  float E[P * (P - 1) / 2 + 1];
+  bool ok = true;
+  const float diag = __fadd_rn(gd, eps);
+#pragma unroll
+  for (int k = 0; k < P; ++k) {
+#pragma unroll
+    for (int j = 0; j < k; ++j) {
+      float v = Goff[tri(k, j)];
+#pragma unroll
+      for (int i = 0; i < j; ++i) v = __fmaf_rn(-L[tri(k, i)], E[tri(j, i)], v);
+      E[tri(k, j)] = v;
+      L[tri(k, j)] = __fmul_rn(v, invD[j]);
+    }
+    float dk = diag;
+#pragma unroll
+    for (int i = 0; i < k; ++i) dk = __fmaf_rn(-L[tri(k, i)], E[tri(k, i)], dk);
+    ok = ok && (dk > 0.0f) && (dk <= 3.402823466e38f);
+    invD[k] = __frcp_rn(dk);
+  }
+  return ok;
+}
+
+// Solve (L D L^T) alpha = b.
+template <int P>
+__device__ __forceinline__ void ldl_solve(const float* L, const float* invD, const float* bv,
+                                          float* alpha) {
+  float z[P];
+#pragma unroll
+  for (int k = 0; k < P; ++k) {
+    float v = bv[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) v = __fmaf_rn(-L[tri(k, i)], z[i], v);
+    z[k] = v;
+  }
+#pragma unroll
+  for (int k = P - 1; k >= 0; --k) {
+    float v = __fmul_rn(z[k], invD[k]);
+#pragma unroll
+    for (int i = k + 1; i < P; ++i) v = __fmaf_rn(-L[tri(i, k)], alpha[i], v);
+    alpha[k] = v;
+  }
+}
+
+// Quantise alpha (Sec. 3.2) and return the Eq. 4 gain with the unregularised
+// Gram; -inf when the candidate is invalid. q receives the codes as floats and
+// *sf the scale field (exponent or binary16 bits).
+template <int P>
+__device__ __forceinline__ float quant_gain(const Prm& pr, const float* alpha, const float* bv,
+                                            float gd, const float* Goff, float* q, int* sf) {
+  float amax = fabsf(alpha[0]);
+#pragma unroll
+  for (int p = 1; p < P; ++p) amax = fmax_nan(amax, fabsf(alpha[p]));
+  bool ok = (amax >= 0x1p-100f) && (amax <= 4294967296.0f);
+  float sc;
+  if (pr.scale_mode == AWSRC_SCALE_POW2) {
+    const int E = (int)((__float_as_uint(amax) >> 23) & 0xffu) - 127;
+    const int e0 = E - (pr.b - 2);  // ilogb(qmax) = b - 2
+    const int e0c = min(max(e0, -126), 126);
+    const float thr = __fmul_rn(pr.qmaxf, __int_as_float((e0c + 127) << 23));
+    int e = e0 + (amax > thr ? 1 : 0);
+    e = min(max(e, pr.e_lo), pr.e_hi);
+    sc = __int_as_float((e + 127) << 23);
+    const float inv = __int_as_float((127 - e) << 23);
+#pragma unroll
+    for (int p = 0; p < P; ++p) {
+      float x = __fmul_rn(alpha[p], inv);
+      x = fminf(fmaxf(x, -pr.qmaxf), pr.qmaxf);
+      q[p] = __fsub_rn(__fadd_rn(x, 12582912.0f), 12582912.0f);  // RNE to integer
+    }
+    *sf = e;
+  } else {
+    const __half h = __float2half_rn(__fdiv_rn(amax, pr.qmaxf));
+    sc = __half2float(h);
+    ok = ok && (sc > 0.0f) && (sc <= 3.402823466e38f);
+#pragma unroll
+    for (int p = 0; p < P; ++p) {
+      float x = __fdiv_rn(alpha[p], sc);
+      x = fminf(fmaxf(x, -pr.qmaxf), pr.qmaxf);
+      q[p] = __fsub_rn(__fadd_rn(x, 12582912.0f), 12582912.0f);
+    }
+    *sf = (int)(int16_t)__half_as_ushort(h);
+  }
+  float Aq = 0.0f;
+#pragma unroll
+  for (int p = 0; p < P; ++p) Aq = __fmaf_rn(q[p], bv[p], Aq);
+  float Qq = 0.0f;
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    Qq = __fmaf_rn(__fmul_rn(q[p], q[p]), gd, Qq);
+#pragma unroll
+    for (int r = p + 1; r < P; ++r)
+      Qq = __fmaf_rn(__fmul_rn(__fmul_rn(2.0f, q[p]), q[r]), Goff[tri(r, p)], Qq);
+  }
+  const float t = __fmul_rn(sc, Qq);
+  const float g = __fmul_rn(sc, __fsub_rn(__fmul_rn(2.0f, Aq), t));
+  return ok ? g : -__int_as_float(0x7f800000);
+}
+
+// Candidate comparison of the seed argmax: larger gain wins, equal gains keep
+// the smaller selector.
+__device__ __forceinline__ bool better(float g, uint32_t s, float bg, uint32_t bs) {
+  return g > bg || (g == bg && s < bs);
+}
+
+// ------------------------------------------------------------- descriptors --
+struct ModDesc {
+  const void* W;
+  const void* W0;
+  const float* act;
+  const float* fisher;
+  int64_t rows, cols, n_cb, n_rb;
+  int64_t tile_off;   // first global tile of the module
+  int64_t gram_off;   // U: first Gram-table entry of the module ([cb][S_pad])
+  int64_t block_off;  // first block of the module in the launch
+  int32_t w_dtype, w0_dtype, nsplit, pad_;
+  float w_act, w_fisher;
+};
+
+struct LaunchDesc {
+  int n;
+  int64_t T;          // tiles in the whole call (partials stride)
+  ModDesc m[kMaxModsPerLaunch];
+};
+
+__device__ __forceinline__ int find_mod(const LaunchDesc& ld, int64_t block) {
+  int mi = 0;
+  for (int i = 1; i < ld.n; ++i)
+    if (block >= ld.m[i].block_off) mi = i;
+  return mi;
+}
+
+}  // namespace awsrc

@@ -1,0 +1,378 @@
+// encode.cu — the seed search of Sec. 3.2 for any supported (C, P) and both
+// variants, plus the two kernels around every search:
+//
+//  gram_u      U only. The activation diagonal is shared by all rows of a module
+//              (Sec. 3.2), so the Gram matrix B_s^T D B_s of Eq. 3 and its LDL^T
+//              depend on (column block, seed) only. They are computed once per
+//              (cb, s) and reused by every row.
+//  search      per (tile, seed): correlation b = B_s^T D r, solve, quantise,
+//              gain; running argmax over the seeds of one split.
+//  finalize    per tile: argmax over splits, then recomputation of the winning
+//              seed's codes and scale with the same operations; the recomputed
+//              gain must equal the searched one bit for bit (self-check bit).
+#include <cfloat>
+
+#include "internal.h"
+
+namespace awsrc {
+
+namespace {
+
+constexpr int kGenRows = 32;      // rows per block of the generic search
+constexpr int kGenLanes = 8;      // seed lanes per row
+constexpr int kGenThreads = kGenRows * kGenLanes;
+
+__device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
+
+// ----------------------------------------------------------------- gram_u --
+template <int P>
+__global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
+                                                     const uint64_t* __restrict__ masks,
+                                                     float* __restrict__ gram) {
+  // blockIdx.y enumerates the column blocks of all modules of the launch
+  int mi = 0;
+  int64_t cb = blockIdx.y;
+  while (mi < ld.n - 1 && cb >= ld.m[mi].n_cb) { cb -= ld.m[mi].n_cb; ++mi; }
+  const ModDesc& md = ld.m[mi];
+  const int C = pr.C;
+  __shared__ float d[kMaxC];
+  __shared__ int dok;
+  if (threadIdx.x == 0) dok = 1;
+  __syncthreads();
+  for (int j = threadIdx.x; j < C; j += blockDim.x) {
+    const float v = md.act[cb * C + j];
+    d[j] = v;
+    if (!(v >= 0.0f && v <= 4294967296.0f)) dok = 0;
+  }
+  __syncthreads();
+  const int s = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s >= pr.S_pad) return;
+  constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
+  float w = 0.0f;
+  for (int j = 0; j < C; ++j) w = __fadd_rn(w, d[j]);
+  const float gd = __fmul_rn(pr.c2, w);
+  float Goff[NL], L[NL], invD[P];
+  const uint64_t* mk = masks + (size_t)s * P * pr.W;
+#pragma unroll
+  for (int q = 1; q < P; ++q) {
+#pragma unroll
+    for (int p = 0; p < q; ++p) {
+      float v = 0.0f;
+      for (int wd = 0; wd < pr.W; ++wd) {
+        const uint64_t x = mk[p * pr.W + wd] ^ mk[q * pr.W + wd];
+        const int jn = min(64, C - 64 * wd);
+        for (int jj = 0; jj < jn; ++jj) v = __fmaf_rn(sign_f(x >> jj), d[64 * wd + jj], v);
+      }
+      Goff[tri(q, p)] = __fmul_rn(pr.c2, v);
+    }
+  }
+  const float eps = __fmul_rn(pr.ridge_rel, gd);
+  bool ok = ldl_factor<P>(gd, eps, Goff, L, invD);
+  ok = ok && dok && (s < pr.S);
+  float* out = gram + (size_t)(md.gram_off + cb * pr.S_pad + s) * gram_stride(P);
+  const float qnan = __int_as_float(0x7fc00000);
+#pragma unroll
+  for (int i = 0; i < P * (P - 1) / 2; ++i) out[i] = L[i];
+#pragma unroll
+  for (int k = 0; k < P; ++k) out[P * (P - 1) / 2 + k] = ok ? invD[k] : qnan;
+#pragma unroll
+  for (int i = 0; i < P * (P - 1) / 2; ++i) out[P * (P - 1) / 2 + P + i] = Goff[i];
+  out[P * (P - 1) + P] = gd;
+}
+
+// Tile staging shared by search and finalisation: r = W - W0, d, y = d*r.
+__device__ __forceinline__ void tile_elem(const Prm& pr, const ModDesc& md, int64_t row,
+                                          int64_t cb, int j, float* y, float* d, bool* ok) {
+  const int64_t idx = row * md.cols + cb * pr.C + j;
+  const float r = __fsub_rn(load_elem(md.W, idx, md.w_dtype), load_elem(md.W0, idx, md.w0_dtype));
+  const float a = md.act[cb * pr.C + j];
+  float dv;
+  if (pr.variant == AWSRC_VARIANT_U) dv = a;
+  else dv = __fadd_rn(__fmul_rn(md.w_act, a), __fmul_rn(md.w_fisher, md.fisher[idx]));
+  *ok = in_domain(r, dv);
+  *d = dv;
+  *y = __fmul_rn(dv, r);
+}
+
+// Score of seed s for one tile given its staged y (and d, gd for PF).
+template <int P, int VAR>
+__device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const float* d,
+                                            float gd_row, const uint64_t* __restrict__ masks,
+                                            const float* __restrict__ gram_cb, uint32_t s,
+                                            float* q, int* sf) {
+  constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
+  const uint64_t* mk = masks + (size_t)s * P * pr.W;
+  float u[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) u[p] = 0.0f;
+  float v[NL];
+#pragma unroll
+  for (int i = 0; i < NL; ++i) v[i] = 0.0f;
+  for (int wd = 0; wd < pr.W; ++wd) {
+    uint64_t m[P];
+#pragma unroll
+    for (int p = 0; p < P; ++p) m[p] = mk[p * pr.W + wd];
+    const int jn = min(64, pr.C - 64 * wd);
+    for (int jj = 0; jj < jn; ++jj) {
+      const float yj = y[64 * wd + jj];
+#pragma unroll
+      for (int p = 0; p < P; ++p) u[p] = __fmaf_rn(sign_f(m[p] >> jj), yj, u[p]);
+      if (VAR == AWSRC_VARIANT_PF) {
+        const float dj = d[64 * wd + jj];
+#pragma unroll
+        for (int qq = 1; qq < P; ++qq)
+#pragma unroll
+          for (int p = 0; p < qq; ++p)
+            v[tri(qq, p)] = __fmaf_rn(sign_f((m[p] ^ m[qq]) >> jj), dj, v[tri(qq, p)]);
+      }
+    }
+  }
+  float bv[P], alpha[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) bv[p] = __fmul_rn(pr.c, u[p]);
+  if (VAR == AWSRC_VARIANT_U) {
+    const float* gt = gram_cb + (size_t)s * gram_stride(P);
+    float L[NL], invD[P], Goff[NL];
+#pragma unroll
+    for (int i = 0; i < P * (P - 1) / 2; ++i) L[i] = gt[i];
+#pragma unroll
+    for (int k = 0; k < P; ++k) invD[k] = gt[P * (P - 1) / 2 + k];
+#pragma unroll
+    for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = gt[P * (P - 1) / 2 + P + i];
+    const float gd = gt[P * (P - 1) + P];
+    ldl_solve<P>(L, invD, bv, alpha);
+    return quant_gain<P>(pr, alpha, bv, gd, Goff, q, sf);
+  } else {
+    float Goff[NL], L[NL], invD[P];
+#pragma unroll
+    for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(pr.c2, v[i]);
+    const float eps = __fmul_rn(pr.ridge_rel, gd_row);
+    const bool ok = ldl_factor<P>(gd_row, eps, Goff, L, invD);
+    ldl_solve<P>(L, invD, bv, alpha);
+    const float g = quant_gain<P>(pr, alpha, bv, gd_row, Goff, q, sf);
+    return ok ? g : neg_inf();
+  }
+}
+
+// Seed range of split z in units of `chunk` seeds.
+__device__ __forceinline__ void split_range(int S, int chunk, int nsplit, int z, int* s0, int* s1) {
+  const int nck = (S + chunk - 1) / chunk;
+  const int per = (nck + nsplit - 1) / nsplit;
+  *s0 = min(S, z * per * chunk);
+  *s1 = min(S, (z + 1) * per * chunk);
+}
+
+// ---------------------------------------------------------- generic search --
+template <int P, int VAR>
+__global__ void __launch_bounds__(kGenThreads) search_generic_kernel(
+    Prm pr, LaunchDesc ld, const uint64_t* __restrict__ masks, const float* __restrict__ gram,
+    float2* __restrict__ partials) {
+  extern __shared__ float smem[];
+  const int mi = find_mod(ld, blockIdx.x);
+  const ModDesc& md = ld.m[mi];
+  const int64_t b = blockIdx.x - md.block_off;
+  const int z = (int)(b % md.nsplit);
+  const int64_t rest = b / md.nsplit;
+  const int64_t rb = rest % md.n_rb;
+  const int64_t cb = rest / md.n_rb;
+  const int C = pr.C, ldc = C + 1;
+  float* ys = smem;
+  float* ds = smem + kGenRows * ldc;
+  __shared__ int rowok[kGenRows];
+  __shared__ float gds[kGenRows];
+  const int tid = threadIdx.x;
+  if (tid < kGenRows) rowok[tid] = 1;
+  __syncthreads();
+  for (int e = tid; e < kGenRows * C; e += kGenThreads) {
+    const int r = e / C, j = e % C;
+    const int64_t row = rb * kGenRows + r;
+    float y = 0.0f, d = 0.0f;
+    if (row < md.rows) {
+      bool ok;
+      tile_elem(pr, md, row, cb, j, &y, &d, &ok);
+      if (!ok) rowok[r] = 0;
+    }
+    ys[r * ldc + j] = y;
+    if (VAR == AWSRC_VARIANT_PF) ds[r * ldc + j] = d;
+  }
+  __syncthreads();
+  if (VAR == AWSRC_VARIANT_PF && tid < kGenRows) {
+    float w = 0.0f;
+    for (int j = 0; j < C; ++j) w = __fadd_rn(w, ds[tid * ldc + j]);
+    gds[tid] = __fmul_rn(pr.c2, w);
+  }
+  __syncthreads();
+  const int r = tid / kGenLanes, sl = tid % kGenLanes;
+  const int64_t row = rb * kGenRows + r;
+  int s0, s1;
+  split_range(pr.S, kGenLanes, md.nsplit, z, &s0, &s1);
+  float bg = neg_inf();
+  uint32_t bs = 0xffffffffu;
+  const float* gram_cb = (VAR == AWSRC_VARIANT_U)
+                             ? gram + (size_t)(md.gram_off + cb * pr.S_pad) * gram_stride(P)
+                             : nullptr;
+  if (row < md.rows && rowok[r]) {
+    for (int s = s0 + sl; s < s1; s += kGenLanes) {
+      float q[P];
+      int sf;
+      const float g = score_seed<P, VAR>(pr, ys + r * ldc, ds + r * ldc,
+                                         VAR == AWSRC_VARIANT_PF ? gds[r] : 0.0f, masks, gram_cb,
+                                         (uint32_t)s, q, &sf);
+      if (better(g, (uint32_t)s, bg, bs)) { bg = g; bs = (uint32_t)s; }
+    }
+  }
+#pragma unroll
+  for (int off = 1; off < kGenLanes; off <<= 1) {
+    const float og = __shfl_xor_sync(0xffffffffu, bg, off);
+    const uint32_t os = __shfl_xor_sync(0xffffffffu, bs, off);
+    if (better(og, os, bg, bs)) { bg = og; bs = os; }
+  }
+  if (sl == 0 && row < md.rows) {
+    const int64_t t = md.tile_off + row * md.n_cb + cb;
+    partials[(size_t)z * ld.T + t] = make_float2(rowok[r] ? bg : neg_inf(), __uint_as_float(bs));
+  }
+}
+
+// --------------------------------------------------------------- finalize --
+template <int P, int VAR>
+__global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
+                                                       const uint64_t* __restrict__ masks,
+                                                       const float* __restrict__ gram,
+                                                       const float2* __restrict__ partials,
+                                                       awsrc_candidate* __restrict__ out,
+                                                       uint32_t* __restrict__ status) {
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t first = ld.m[0].tile_off;
+  const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
+  if (t < first || t >= last) return;
+  int mi = 0;
+  for (int i = 1; i < ld.n; ++i)
+    if (t >= ld.m[i].tile_off) mi = i;
+  const ModDesc& md = ld.m[mi];
+  const int64_t lt = t - md.tile_off;
+  const int64_t row = lt / md.n_cb, cb = lt % md.n_cb;
+  float bg = neg_inf();
+  uint32_t bs = 0xffffffffu;
+  for (int z = 0; z < md.nsplit; ++z) {
+    const float2 pz = partials[(size_t)z * ld.T + t];
+    const float g = pz.x;
+    const uint32_t s = __float_as_uint(pz.y);
+    if (better(g, s, bg, bs)) { bg = g; bs = s; }
+  }
+  awsrc_candidate cd;
+  cd.gain = neg_inf();
+  cd.seed = 0;
+  cd.scale = 0;
+#pragma unroll
+  for (int p = 0; p < 8; ++p) cd.code[p] = 0;
+  if (bg > neg_inf() && bs < (uint32_t)pr.S) {
+    float y[kMaxC], d[kMaxC];
+    bool ok = true;
+    for (int j = 0; j < pr.C; ++j) {
+      bool okj;
+      tile_elem(pr, md, row, cb, j, &y[j], &d[j], &okj);
+      ok = ok && okj;
+    }
+    float gd_row = 0.0f;
+    if (VAR == AWSRC_VARIANT_PF) {
+      float w = 0.0f;
+      for (int j = 0; j < pr.C; ++j) w = __fadd_rn(w, d[j]);
+      gd_row = __fmul_rn(pr.c2, w);
+    }
+    const float* gram_cb = (VAR == AWSRC_VARIANT_U)
+                               ? gram + (size_t)(md.gram_off + cb * pr.S_pad) * gram_stride(P)
+                               : nullptr;
+    float q[P];
+    int sf = 0;
+    const float g = score_seed<P, VAR>(pr, y, d, gd_row, masks, gram_cb, bs, q, &sf);
+    if (!ok || __float_as_uint(g) != __float_as_uint(bg)) atomicOr(status, kFaultSelfCheck);
+    if (ok && g > neg_inf()) {
+      cd.gain = g;
+      cd.seed = (uint16_t)bs;
+      cd.scale = (int16_t)sf;
+#pragma unroll
+      for (int p = 0; p < P; ++p) cd.code[p] = (int8_t)(int)q[p];
+    }
+  }
+  out[t] = cd;
+}
+
+template <int P>
+cudaError_t launch_gram_p(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, float* gram,
+                          cudaStream_t st) {
+  int64_t ncb = 0;
+  for (int i = 0; i < ld.n; ++i) ncb += ld.m[i].n_cb;
+  dim3 grid((pr.S_pad + 127) / 128, (unsigned)ncb);
+  gram_u_kernel<P><<<grid, 128, 0, st>>>(pr, ld, masks, gram);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+template <int P, int VAR>
+cudaError_t launch_search_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                             const float* gram, int64_t n_blocks, float2* partials,
+                             cudaStream_t st) {
+  const size_t smem = (size_t)kGenRows * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
+  auto k = search_generic_kernel<P, VAR>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k<<<(unsigned)n_blocks, kGenThreads, smem, st>>>(pr, ld, masks, gram, partials);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+template <int P, int VAR>
+cudaError_t launch_finalize_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                               const float* gram, const float2* partials, awsrc_candidate* out,
+                               uint32_t* status, cudaStream_t st) {
+  const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
+  const int tpb = 128;
+  finalize_kernel<P, VAR><<<(unsigned)((last + tpb - 1) / tpb), tpb, 0, st>>>(
+      pr, ld, masks, gram, partials, out, status);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+#define AWSRC_DISPATCH_P(P_, EXPR) \
+  switch (P_) {                    \
+    case 1: { constexpr int PP = 1; return EXPR; } \
+    case 2: { constexpr int PP = 2; return EXPR; } \
+    case 3: { constexpr int PP = 3; return EXPR; } \
+    case 4: { constexpr int PP = 4; return EXPR; } \
+    case 5: { constexpr int PP = 5; return EXPR; } \
+    case 6: { constexpr int PP = 6; return EXPR; } \
+    case 7: { constexpr int PP = 7; return EXPR; } \
+    case 8: { constexpr int PP = 8; return EXPR; } \
+    default: return cudaErrorInvalidValue;          \
+  }
+
+cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, float* gram,
+                          cudaStream_t st) {
+  AWSRC_DISPATCH_P(pr.P, (launch_gram_p<PP>(pr, ld, masks, gram, st)));
+}
+
+cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                                  const float* gram, int64_t n_blocks, float2* partials,
+                                  cudaStream_t st) {
+  if (pr.variant == AWSRC_VARIANT_U) {
+    AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_U>(pr, ld, masks, gram, n_blocks, partials, st)));
+  }
+  AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_PF>(pr, ld, masks, gram, n_blocks, partials, st)));
+}
+
+cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                            const float* gram, const float2* partials, int nsplit_max,
+                            awsrc_candidate* out, uint32_t* status, cudaStream_t st) {
+  (void)nsplit_max;
+  if (pr.variant == AWSRC_VARIANT_U) {
+    AWSRC_DISPATCH_P(pr.P, (launch_finalize_pv<PP, AWSRC_VARIANT_U>(pr, ld, masks, gram, partials, out, status, st)));
+  }
+  AWSRC_DISPATCH_P(pr.P, (launch_finalize_pv<PP, AWSRC_VARIANT_PF>(pr, ld, masks, gram, partials, out, status, st)));
+}
+
+int generic_rows() { return kGenRows; }
+int generic_chunk() { return kGenLanes; }
+
+}  // namespace awsrc

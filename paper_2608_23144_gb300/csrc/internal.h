@@ -1,0 +1,74 @@
+// internal.h — host-side declarations shared by the library's translation units.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace awsrc {
+
+// Validated parameters -> Prm (derived constants). Returns AWSRC_OK or an error.
+awsrc_status make_prm(const awsrc_params* prm, Prm* out);
+
+// Records the CUDA error text for awsrc_last_error_message() and maps it.
+awsrc_status cuda_fail(cudaError_t e, const char* where);
+awsrc_status check_launch(const char* where);
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Launch counter behind awsrc_kernel_launches(): every launch site adds its kernels.
+void note_launches(int n);
+
+// basis.cu: masks[(s*P + p)*W + w] for s in [0, S_pad); seeds >= S get zero masks.
+cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st);
+// Expanded +-1.0f masks for the C=64, P=4 search: [chunk][j][seed_in_chunk][p].
+cudaError_t launch_expand_masks_c64p4(const Prm& pr, const uint64_t* masks, float* out,
+                                      cudaStream_t st);
+
+// encode.cu
+cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                          float* gram, cudaStream_t st);
+cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                                  const float* gram, int64_t n_blocks, float2* partials,
+                                  cudaStream_t st);
+cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
+                            const float* gram, const float2* partials, int nsplit_max,
+                            awsrc_candidate* out, uint32_t* status, cudaStream_t st);
+// search_c64p4.cu
+cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const float* mexp,
+                                const float* gram, int64_t n_blocks, float2* partials,
+                                uint32_t* status, cudaStream_t st);
+int search_c64p4_rows();   // rows per block of the specialised kernel
+int search_c64p4_chunk();  // seeds per chunk of the specialised kernel
+
+// select.cu
+struct SelectPlan {
+  int n_mod, n_rates;
+  int64_t T, L, h;
+  int key_bits, tile_bits_local, mod_shift;
+  int64_t cap_records;      // upper bound on records written
+  int64_t nblocks;          // radix blocks
+};
+awsrc_status select_run(const Prm& pr, const SelectPlan& sp, const int64_t* tile_off,
+                        const int64_t* mod_tiles, const int64_t* kcap /* U: per module; PF: per rate */,
+                        const awsrc_candidate* cands, uint8_t* stream_out, int64_t* d_counts,
+                        int64_t* d_bytes, void* ws, size_t ws_bytes, cudaStream_t st);
+size_t select_ws_bytes(const SelectPlan& sp);
+
+// decode.cu
+struct DecodeMod {
+  const void* W0;
+  void* out;
+  int64_t rows, cols, tile_off;
+  int32_t w0_dtype, pad_;
+};
+cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
+                          int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
+                          const uint64_t* masks, int32_t* map, uint32_t* status, cudaStream_t st);
+size_t decode_scratch_bytes(int64_t T, int mode);
+int generic_rows();
+int generic_chunk();
+
+}  // namespace awsrc

@@ -1,0 +1,105 @@
+"""CPU checks of the C ABI library: it loads without a GPU, exports every entry
+point declared in include/awsrc.h, and its host-only helpers (byte accounting,
+argument validation) agree with the oracle. No compute call is made."""
+import ctypes as ct
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "awsrc.h")
+
+
+@pytest.fixture(scope="module")
+def libpath():
+    from paper_2608_23144_gb300 import build as b
+    return b.build()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(awsrc_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_three_steps():
+    syms = declared_symbols()
+    for s in ("awsrc_encode_tiles", "awsrc_select_records", "awsrc_decode_apply"):
+        assert s in syms
+
+
+def test_library_exports_every_declared_symbol(libpath):
+    out = subprocess.run(["nm", "-D", "--defined-only", libpath], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\bT (awsrc_\w+)", out))
+    missing = [s for s in declared_symbols() if s not in exported]
+    assert not missing, f"declared but not exported: {missing}"
+    lib = ct.CDLL(libpath)
+    for s in declared_symbols():
+        assert hasattr(lib, s)
+
+
+def test_host_byte_accounting_matches_oracle(libpath, orc):
+    import paper_2608_23144_gb300 as aw
+    for C, P, b, S, b_e, smode in [(64, 4, 4, 256, 8, 0), (64, 4, 4, 256, 16, 1), (16, 4, 4, 16, 8, 0),
+                                   (128, 2, 4, 2, 8, 0), (8, 8, 8, 65536, 3, 0)]:
+        for T in (1, 2, 2048, 1_204_224, 152_174_592, 487_587_840):
+            p = aw.params(C=C, P=P, b=b, S=S, b_e=b_e, scale_mode=smode)
+            q = orc.params(C=C, P=P, b=b, S=S, b_e=b_e, scale_mode=smode)
+            assert aw.awsrc_record_bytes(p, T) == orc.record_bytes(q, T)
+    for n in (1, 7, 108, 252):
+        assert aw.awsrc_header_bytes(n) == orc.header_bytes(n)
+
+
+def test_host_validation_rejects_bad_arguments(libpath):
+    import paper_2608_23144_gb300 as aw
+    lib = aw.lib
+    n = ct.c_size_t()
+    mods = (aw.Module * 1)()
+    mods[0].rows, mods[0].cols = 8, 96   # 96 is not a multiple of C = 64
+    p = aw.params(C=64)
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(p), 1, mods, ct.byref(n)) == 2     # SHAPE
+    mods[0].cols = 128
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(p), 1, mods, ct.byref(n)) == 0
+    assert n.value > 0
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(C=48)), 1, mods, ct.byref(n)) == 2
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(P=9)), 1, mods, ct.byref(n)) == 3
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(b=1)), 1, mods, ct.byref(n)) == 3
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(S=70000)), 1, mods, ct.byref(n)) == 3
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(scale_mode=1, b_e=8)), 1, mods, ct.byref(n)) == 3
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(aw.params(ridge_rel=-1.0)), 1, mods, ct.byref(n)) == 1
+    assert lib.awsrc_encode_workspace_bytes(ct.byref(p), 0, mods, ct.byref(n)) == 1
+    # encode with NULL tensors is refused before any launch
+    assert lib.awsrc_encode_tiles(ct.byref(p), 1, mods, None, None, 0, None) == 1
+    # a budget below the header: 8x128 weights at 0.01 bpw -> 1 byte < 48
+    r = (ct.c_double * 1)(0.01)
+    assert lib.awsrc_stream_capacity(ct.byref(p), 1, mods, r, 1, ct.byref(n)) == 4
+    r = (ct.c_double * 1)(8.0)
+    assert lib.awsrc_stream_capacity(ct.byref(p), 1, mods, r, 1, ct.byref(n)) == 0
+    # U takes exactly one rate
+    r2 = (ct.c_double * 2)(4.0, 8.0)
+    assert lib.awsrc_stream_capacity(ct.byref(p), 1, mods, r2, 2, ct.byref(n)) == 3
+    assert lib.awsrc_status_string(4) == b"byte budget smaller than the stream header"
+
+
+def test_stream_capacity_matches_oracle_budget(libpath, orc):
+    import paper_2608_23144_gb300 as aw
+    lib = aw.lib
+    shapes = [(2048, 2048), (256, 2048), (256, 2048), (2048, 2048), (11008, 2048), (11008, 2048), (2048, 11008)]
+    mods = (aw.Module * len(shapes))()
+    for i, (r, c) in enumerate(shapes):
+        mods[i].rows, mods[i].cols = r, c
+    p = aw.params(C=64, S=4096)
+    q = orc.params(C=64, S=4096)
+    n = ct.c_size_t()
+    rates = (ct.c_double * 1)(0.162)
+    assert lib.awsrc_stream_capacity(ct.byref(p), len(shapes), mods, rates, 1, ct.byref(n)) == 0
+    N = sum(r * c for r, c in shapes)
+    T = N // 64
+    B = orc.budget_bytes(0.162, N)
+    h, L = orc.header_bytes(len(shapes)), orc.record_bytes(q, T)
+    quotas = [((B - h) * r * c) // N for r, c in shapes]
+    assert n.value == h + sum(qm // L for qm in quotas) * L
+    assert n.value <= B
