@@ -14,8 +14,8 @@ HEADER = os.path.join(ROOT, "include", "awsrc.h")
 
 @pytest.fixture(scope="module")
 def libpath():
-    from paper_2608_23144_gb300 import build as b
-    return b.build()
+    import __graft_entry__
+    return __graft_entry__._cuda_build_module().build()
 
 
 def declared_symbols():
