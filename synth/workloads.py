@@ -114,17 +114,20 @@ def module_seed(base: int, layer: int, module: int) -> int:
 
 
 def rtn_int4_g128(W: torch.Tensor, group: int = 128) -> torch.Tensor:
-    """RTN-INT4 symmetric backbone of Eq. 1, per (row, group of 128 inputs).
-    Returns the float32 reconstruction q*s (exact in float32)."""
+    """RTN-INT4 symmetric backbone of Eq. 1, per (row, group of 128 inputs; the
+    last group of a row may be shorter). Returns the float32 reconstruction q*s
+    (exact in float32)."""
     rows, cols = W.shape
-    assert cols % group == 0
-    w = W.float().reshape(rows, cols // group, group)
+    ng = (cols + group - 1) // group
+    w = torch.zeros(rows, ng * group, dtype=torch.float32, device=W.device)
+    w[:, :cols] = W.float()
+    w = w.reshape(rows, ng, group)
     amax = w.abs().amax(dim=-1, keepdim=True)
     s = (amax / 7.0).to(torch.float16).float()
     safe = torch.where(s > 0, s, torch.ones_like(s))
     q = torch.clamp(torch.round(w / safe), -8, 7)
     q = torch.where(s > 0, q, torch.zeros_like(q))
-    return (q * s).reshape(rows, cols)
+    return (q * s).reshape(rows, ng * group)[:, :cols].contiguous()
 
 
 def activation_moments(cols: int, gen: torch.Generator, device, tokens: int = 1024,

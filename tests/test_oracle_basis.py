@@ -110,3 +110,19 @@ def test_generator_follows_the_documented_draw_schedule(orc, C, P, permute):
             cols.append(pool[p])
         o_sign, o_perm, o_cols, _ = orc.gen_basis(gen_seed, s, C, P, permute)
         assert list(o_sign) == sign and list(o_perm) == perm and list(o_cols) == cols
+
+
+def test_rtn_backbone_is_round_to_nearest_int4():
+    """The synthetic backbone generator: per group of 128, codes in [-8, 7] times an
+    fp16 scale max|w|/7; ragged last groups included."""
+    import torch
+    from synth import rtn_int4_g128
+    g = torch.Generator().manual_seed(0)
+    W = torch.randn(5, 320, generator=g) * 0.02
+    W0 = rtn_int4_g128(W)
+    for gi in range(3):
+        sl = slice(128 * gi, min(320, 128 * gi + 128))
+        s = (W[:, sl].abs().amax(1, keepdim=True) / 7.0).half().float()
+        q = W0[:, sl] / s
+        assert torch.equal(q, torch.round(q)) and q.abs().max() <= 8
+        assert torch.equal(q, torch.clamp(torch.round(W[:, sl] / s), -8, 7))
