@@ -264,6 +264,9 @@ def run_ours(args):
     ev_d = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
             for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for ev in ev_s + ev_e:   # torch creates the CUDA event on first record
+        ev.record()
+    torch.cuda.synchronize()
     l0 = aw.awsrc_kernel_launches()
     barrier()
     torch.cuda.synchronize()

@@ -269,9 +269,12 @@ def awsrc_workspace_status(workspace: torch.Tensor, stream=None) -> int:
 
 
 def awsrc_set_timing_events(before: Optional[torch.cuda.Event], after: Optional[torch.cuda.Event]):
-    """Record `before`/`after` around the seed-search launches of later encode calls."""
+    """Record `before`/`after` around the seed-search launches of later encode calls.
+    The events must already exist (torch creates them on their first record())."""
     b = before.cuda_event if before is not None else None
     a = after.cuda_event if after is not None else None
+    if (before is not None and not b) or (after is not None and not a):
+        raise ValueError("record the events once before handing them to the library")
     lib.awsrc_set_timing_events(b, a)
 
 
