@@ -286,7 +286,7 @@ def run_ours(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     search_ms = statistics.mean(a.elapsed_time(b) for a, b in zip(ev_s, ev_e))
-    dec_ms = statistics.mean(a.elapsed_time(b) for a, b in zip(ev_d))
+    dec_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_d)
     s, counts, nbytes = stream_dev[0]
     stream_bytes = int(nbytes[0].item())
     w0_bytes = sum(m["W0"].numel() * m["W0"].element_size() for m in mods)
