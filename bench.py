@@ -53,6 +53,8 @@ def parse():
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--modules", default="",
+                    help="comma-separated subset of the layer's modules (profiling runs only)")
     return ap.parse_args()
 
 
@@ -156,7 +158,7 @@ def oracle_sample(wl, mods_host, target_s: float, seed: int = 0):
     rows = max(1, int(target_s / (per_tile * sum(m["W"].shape[1] // wl.C for m in mods_host))))
     n, t = run(rows)
     cands = n * wl.S
-    desc = (f"{rows} random whole rows of each of the 7 modules ({n} tiles x {wl.S} seeds = "
+    desc = (f"{rows} random whole rows of each of the {len(mods_host)} modules ({n} tiles x {wl.S} seeds = "
             f"{cands:,} candidates) in {t:.1f} s")
     return cands / t, orc.num_threads(), desc
 
@@ -221,9 +223,15 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     wl = WORKLOADS[WORKLOAD]
-    mods = make_layer(wl, layer=rank, device=dev)
+    if args.modules:
+        keep = args.modules.split(",")
+        idx = [i for i, (name, _, _) in enumerate(wl.shapes) if name in keep]
+        assert idx, f"no module of {wl.name} in {keep}"
+        mods = make_layer(wl, layer=rank, device=dev, modules=idx)
+    else:
+        mods = make_layer(wl, layer=rank, device=dev)
     prm = aw.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
-    T = wl.tiles_per_layer
+    T = sum(m["rows"] * m["cols"] // wl.C for m in mods)
     cands_per_step = T * wl.S
     enc_ws = torch.empty(aw.awsrc_encode_workspace_bytes(prm, mods), dtype=torch.uint8, device=dev)
     cands = torch.empty((T, 16), dtype=torch.uint8, device=dev)
@@ -357,11 +365,12 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": wl.description, "tiles_per_gpu": T, "seeds": wl.S, "C": wl.C,
+            "config": {"workload": wl.description if not args.modules else
+                       f"{wl.name} modules {args.modules} (profiling subset)", "tiles_per_gpu": T, "seeds": wl.S, "C": wl.C,
                        "P": wl.P, "b": wl.b, "rate_bpw": RATE, "variant": "U",
                        "parallelism": f"{world} independent layers" if world > 1 else "single GPU",
                        "l2": "inputs larger than L2 (W and W0 of the layer: 308 MB per step)"},
-            "layers_per_s": world * args.steps / (ms * 1e-3),
+            "layers_per_s": world * args.steps / (ms * 1e-3) if not args.modules else None,
             "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
