@@ -284,6 +284,34 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 int32_t mode, void* workspace, size_t workspace_bytes,
                                 void* stream_handle);
 
+/*
+ * awsrc_decode_apply_inplace_noalloc — the in-place decode of awsrc_decode_apply
+ * (mode AWSRC_DECODE_INPLACE) for callers that may not allocate device memory:
+ * a model loader inside an engine that has handed all device memory to its own
+ * pool, a plain C program without an allocator, a recovery path that must not
+ * allocate. The paper has no counterpart; this is an interface convenience.
+ * It takes no workspace: its scratch (the basis mask table and a fault word)
+ * is a static device array of this library, about 1 MiB that every GPU which
+ * loads the library keeps until the process exits. It allocates nothing (no
+ * cudaMalloc, cudaFree or allocating library call).
+ *   W_hat   host array of n_mod device pointers; each must already hold that
+ *           module's W0 (dtype mods[m].w0_dtype, the same for all modules) and
+ *           receives W0 + r_hat on the tiles the first K records name.
+ *   mods    rows, cols and w0_dtype are read; W, W0 and the statistics are not.
+ *   stream, stream_len, K  as in awsrc_decode_apply.
+ * Limits: S * P * ceil(C/64) <= 131072 (else AWSRC_ERR_UNSUPPORTED, with the
+ * numbers in awsrc_last_error_message()); at most 16 modules per call.
+ * All calls share the one array per device and leave their contents in it;
+ * calls whose kernels overlap on the GPU race on it, so the caller serialises
+ * them. The first call on a device looks up the array's address with that
+ * device current and should come before any stream capture. Records naming a
+ * tile or seed out of range are skipped; this entry point does not report them.
+ */
+awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t n_mod,
+                                                const awsrc_module* mods, const uint8_t* stream,
+                                                size_t stream_len, int64_t K, void* const* W_hat,
+                                                void* stream_handle);
+
 /* ------------------------------------------------------------------ misc -- */
 
 /*

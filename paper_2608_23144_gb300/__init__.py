@@ -24,6 +24,7 @@ from ._binding import (  # noqa: F401
     Module,
     Params,
     awsrc_decode_apply,
+    awsrc_decode_apply_inplace_noalloc,
     awsrc_encode_tiles,
     awsrc_encode_workspace_bytes,
     awsrc_gen_basis,

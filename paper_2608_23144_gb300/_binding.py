@@ -96,6 +96,9 @@ def _load():
     L.awsrc_decode_apply.restype = st
     L.awsrc_decode_apply.argtypes = [P(Params), ct.c_int32, P(Module), vp, sz, ct.c_int64, P(vp), ct.c_int32,
                                      ct.c_int32, vp, sz, vp]
+    L.awsrc_decode_apply_inplace_noalloc.restype = st
+    L.awsrc_decode_apply_inplace_noalloc.argtypes = [P(Params), ct.c_int32, P(Module), vp, sz, ct.c_int64,
+                                                     P(vp), vp]
     L.awsrc_set_timing_events.restype = None
     L.awsrc_set_timing_events.argtypes = [vp, vp]
     L.awsrc_kernel_launches.restype = ct.c_uint64
@@ -259,6 +262,18 @@ def awsrc_decode_apply(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
                                   code, mode, _dev_ptr(workspace), workspace.numel(), _stream(stream)),
            "decode_apply")
     outs[0]._awsrc_workspace = workspace
+    return outs
+
+
+def awsrc_decode_apply_inplace_noalloc(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
+                                       outs: List[torch.Tensor], stream=None) -> List[torch.Tensor]:
+    """In-place decode that allocates nothing on either side of the ABI: `outs`
+    must already hold W0; their tiles named by the first K records get W0 + r_hat."""
+    mods = module_array(modules, decoder=True)
+    ptrs = (ct.c_void_p * len(outs))(*[_dev_ptr(o) for o in outs])
+    _check(lib.awsrc_decode_apply_inplace_noalloc(ct.byref(prm), len(modules), mods, _dev_ptr(stream_bytes),
+                                                  stream_bytes.numel(), int(K), ptrs, _stream(stream)),
+           "decode_apply_inplace_noalloc")
     return outs
 
 

@@ -3,6 +3,7 @@
 #include <algorithm>
 #include <atomic>
 #include <cmath>
+#include <cstdarg>
 #include <cstdio>
 #include <cstring>
 #include <vector>
@@ -91,6 +92,13 @@ void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_
 awsrc_status cuda_fail(cudaError_t e, const char* where) {
   snprintf(g_err, sizeof g_err, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
   return AWSRC_ERR_CUDA;
+}
+
+void set_error_message(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof g_err, fmt, ap);
+  va_end(ap);
 }
 
 awsrc_status check_launch(const char* where) {

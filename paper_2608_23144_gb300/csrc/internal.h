@@ -15,6 +15,8 @@ awsrc_status make_prm(const awsrc_params* prm, Prm* out);
 // Records the CUDA error text for awsrc_last_error_message() and maps it.
 awsrc_status cuda_fail(cudaError_t e, const char* where);
 awsrc_status check_launch(const char* where);
+// Sets the text awsrc_last_error_message() returns (printf-style).
+void set_error_message(const char* fmt, ...);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
