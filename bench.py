@@ -38,9 +38,10 @@ UNIT = "candidates/s"
 # C*P = 256 correlation FFMAs plus the 80-operation epilogue of the numeric
 # convention (solve 20, quantise 25, gain 34, compare 1).
 OPS_PER_CANDIDATE = 256 + 80
-# DRAM traffic of one search launch from an ncu capture (profiles/), valid only
-# for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": None, "bytes_per_launch": None}
+# DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
+# list of this workload; valid only for the kernel source it was measured on.
+SEARCH_TRAFFIC = {"source_sha256": "b7550f8142e968b87e5cc09cd18cbf0704837c7c70751c8111b4f570691bdd1e",
+                  "bytes_per_launch": 447428352}
 
 
 def parse():

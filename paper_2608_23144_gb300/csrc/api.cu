@@ -138,6 +138,16 @@ awsrc_status make_prm(const awsrc_params* p, Prm* out) {
   r.W = (p->C + 63) / 64;
   r.S_pad = (p->S + 31) / 32 * 32;
   r.logC = ceil_log2_host((uint64_t)p->C);
+  {
+    const float qf = r.qmaxf;
+    uint32_t qb;
+    std::memcpy(&qb, &qf, 4);
+    r.mant_q = qb & 0x007FFFFFu;
+  }
+  // valid candidates have 2^-100 <= amax <= 2^32, so e lies in
+  // [-100 - (b-2), 33 - (b-2)]; if the range covers that, it never binds
+  r.fast_pow2 = (p->scale_mode == AWSRC_SCALE_POW2) && r.e_lo <= -100 - (p->b - 2) &&
+                r.e_hi >= 33 - (p->b - 2);
   *out = r;
   return AWSRC_OK;
 }
@@ -432,13 +442,11 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const aw
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   uint32_t* status = reinterpret_cast<uint32_t*>(ws);
   uint64_t* masks = reinterpret_cast<uint64_t*>(ws + kStatusBytes);
-  int32_t* map = reinterpret_cast<int32_t*>(ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256));
+  void* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
   cudaStream_t st = (cudaStream_t)stream_handle;
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
   if (e != cudaSuccess) return cuda_fail(e, "decode: clear status");
-  e = launch_gen_basis(pr, masks, pr.S, st);
-  if (e != cudaSuccess) return cuda_fail(e, "decode: gen_basis");
-  e = launch_decode(pr, n_mod, dm.data(), T, L, h, stream, K, kmax, out_dtype, mode, masks, map, status, st);
+  e = launch_decode(pr, n_mod, dm.data(), T, L, h, stream, K, kmax, out_dtype, mode, masks, scratch, status, st);
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "decode");
 }
 

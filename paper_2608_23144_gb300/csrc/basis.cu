@@ -6,62 +6,27 @@
 // of B_s as bits (bit j set when entry (j, p) is negative). The draw schedule is
 // the one the public header documents; it is integer-only, so every device and
 // host reproduces it exactly.
+#include "basis.cuh"
 #include "internal.h"
 
 namespace awsrc {
 
-__global__ void gen_basis_kernel(Prm pr, uint64_t* __restrict__ masks, int S_out) {
-  const int s = blockIdx.x * blockDim.x + threadIdx.x;
-  if (s >= S_out) return;
-  const int C = pr.C, P = pr.P, W = pr.W;
-  if (s >= pr.S) {  // padding seeds of the last search chunk: never selected
-    for (int i = 0; i < P * W; ++i) masks[(size_t)s * P * W + i] = 0ull;
-    return;
-  }
-  const uint64_t key = sm64_output(pr.gen_seed, (uint64_t)s + 1);
-  uint64_t n = 1;
-  uint64_t sign[kMaxC / 64];
-  for (int w = 0; w < W; ++w) sign[w] = sm64_output(key, n++);
-  if (C < 64) sign[0] &= (1ull << C) - 1ull;
-  uint8_t perm[kMaxC];
-  for (int j = 0; j < C; ++j) perm[j] = (uint8_t)j;
-  if (pr.permute) {
-    for (int i = C - 1; i >= 1; --i) {
-      const uint64_t x = sm64_output(key, n++) >> 32;
-      const int k = (int)((x * (uint64_t)(i + 1)) >> 32);
-      const uint8_t t = perm[i];
-      perm[i] = perm[k];
-      perm[k] = t;
-    }
-  }
-  uint8_t pool[kMaxC];
-  for (int j = 0; j < C; ++j) pool[j] = (uint8_t)j;
-  int cols[kMaxP];
-  for (int p = 0; p < P; ++p) {
-    const uint64_t x = sm64_output(key, n++) >> 32;
-    const int k = p + (int)((x * (uint64_t)(C - p)) >> 32);
-    const uint8_t t = pool[p];
-    pool[p] = pool[k];
-    pool[k] = t;
-    cols[p] = pool[p];
-  }
-  for (int p = 0; p < P; ++p) {
-    for (int w = 0; w < W; ++w) {
-      uint64_t m = 0;
-      const int jn = min(64, C - 64 * w);
-      for (int jj = 0; jj < jn; ++jj) {
-        const int j = 64 * w + jj;
-        const uint64_t h = (uint64_t)(__popc((unsigned)(perm[j] & cols[p])) & 1);
-        m |= (((sign[w] >> jj) & 1ull) ^ h) << jj;
-      }
-      masks[((size_t)s * P + p) * W + w] = m;
-    }
-  }
+constexpr int kBasisWarps = 4;  // seeds per block of the stand-alone kernel
+
+__global__ void __launch_bounds__(32 * kBasisWarps) gen_basis_kernel(Prm pr, uint64_t* __restrict__ masks,
+                                                                     int S_out) {
+  __shared__ uint8_t perm_s[kBasisWarps][kMaxC];
+  __shared__ uint8_t kidx_s[kBasisWarps][kMaxC];
+  __shared__ uint8_t pool_s[kBasisWarps][kMaxC];
+  __shared__ int cols_s[kBasisWarps][kMaxP];
+  const int warp = threadIdx.x >> 5;
+  const int s = blockIdx.x * kBasisWarps + warp;
+  if (s >= S_out) return;  // whole warp leaves together
+  basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
 }
 
 cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st) {
-  const int tpb = 128;
-  gen_basis_kernel<<<(S_out + tpb - 1) / tpb, tpb, 0, st>>>(pr, masks, S_out);
+  gen_basis_kernel<<<(S_out + kBasisWarps - 1) / kBasisWarps, 32 * kBasisWarps, 0, st>>>(pr, masks, S_out);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -40,6 +40,8 @@ struct Prm {
   int W;          // 64-bit mask words per (seed, atom)
   int S_pad;      // seeds rounded up to the search chunk
   int logC;       // log2(C)
+  int fast_pow2;  // POW2 scale whose exponent range can never bind for a valid candidate
+  uint32_t mant_q;  // mantissa field of (float)qmax
 };
 
 // ---------------------------------------------------------------- generator --
@@ -182,6 +184,45 @@ __device__ __forceinline__ float quant_gain(const Prm& pr, const float* alpha, c
   }
   const float t = __fmul_rn(sc, Qq);
   const float g = __fmul_rn(sc, __fsub_rn(__fmul_rn(2.0f, Aq), t));
+  return ok ? g : -__int_as_float(0x7f800000);
+}
+
+// The POW2 branch of quant_gain when the exponent range never binds (fast_pow2):
+// the same results with integer work on the bit pattern of amax. For a valid
+// candidate amax = f_a*2^E is normal and the smallest e with amax <= qmax*2^e is
+// E - ilogb(qmax) + [f_a > f_qmax] (compare mantissa fields); |alpha_p|*2^-e then
+// never exceeds qmax, so the code clamps are no-ops and are left out. Goff2
+// holds 2*G_pq (exact), which gives the same fma as (2*code_p*code_q)*G_pq
+// because the fused product is exact.
+template <int P>
+__device__ __forceinline__ float quant_gain_fast(const Prm& pr, const float* alpha, const float* bv,
+                                                 float gd, const float* Goff2, float* q, int* e_out) {
+  float amax = fabsf(alpha[0]);
+#pragma unroll
+  for (int p = 1; p < P; ++p) amax = fmax_nan(amax, fabsf(alpha[p]));
+  const uint32_t ab = __float_as_uint(amax);
+  // 2^-100 <= amax <= 2^32 (NaN and inf fail: their bit patterns lie above)
+  const bool ok = (ab - 0x0D800000u) <= (0x4F800000u - 0x0D800000u);
+  const uint32_t sc_bits = (ab & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23) +
+                           (((ab & 0x007FFFFFu) > pr.mant_q) ? 0x00800000u : 0u);
+  const float sc = __uint_as_float(sc_bits);
+  const float inv = __uint_as_float(0x7F000000u - sc_bits);
+#pragma unroll
+  for (int p = 0; p < P; ++p)
+    q[p] = __fsub_rn(__fadd_rn(__fmul_rn(alpha[p], inv), 12582912.0f), 12582912.0f);
+  *e_out = (int)(sc_bits >> 23) - 127;
+  float Aq = 0.0f;
+#pragma unroll
+  for (int p = 0; p < P; ++p) Aq = __fmaf_rn(q[p], bv[p], Aq);
+  float Qq = 0.0f;
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    Qq = __fmaf_rn(__fmul_rn(q[p], q[p]), gd, Qq);
+#pragma unroll
+    for (int r = p + 1; r < P; ++r) Qq = __fmaf_rn(__fmul_rn(q[p], q[r]), Goff2[tri(r, p)], Qq);
+  }
+  const float t = __fmul_rn(sc, Qq);
+  const float g = __fmul_rn(sc, __fmaf_rn(2.0f, Aq, -t));
   return ok ? g : -__int_as_float(0x7f800000);
 }
 

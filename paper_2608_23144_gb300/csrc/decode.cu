@@ -2,28 +2,34 @@
 // named by records, W0 elsewhere (Eq. 1); any prefix of a progressive stream
 // decodes the same way (Sec. 3.3).
 //
-//  scatter   one thread per record: unpack tile, seed, scale, codes; bounds-
-//            check tile < T and seed < S (a bad record is skipped and flagged);
-//            map[tile] = k and a 16-byte decoded record dec[k].
-//  dense     streams every element of W0 to W_hat with 16-byte vector loads and
-//            stores (two groups in flight per thread); a group whose tile has a
-//            record adds r_hat_j = fl(fl(k_j * C^-1/2) * scale), k_j = sum_p
-//            sign * code_p computed exactly in integers.
-//  inplace   one warp per record touches only that tile of W_hat.
+//  copy      (dense mode) W_hat = W0 converted to the output dtype, a pure
+//            stream of 16-byte vectors, four in flight per thread.
+//  patch     one warp per record: unpack tile, seed, scale, codes; bounds-check
+//            tile < T and seed < S (a bad record is skipped and flagged); write
+//            W_hat_j = fl(W0_j + fl(fl(k_j * C^-1/2) * scale)) on the tile, with
+//            k_j = sum_p sign * code_p exact in integers. It reads W0, so W_hat
+//            may alias W0 (in-place mode).
+// Keeping the record lookup out of the streaming pass keeps dependent loads
+// (record -> masks) off the bandwidth-critical path; the patch re-touches only
+// the recorded tiles (about 16% of a layer at 0.162 bits/weight).
 #include <algorithm>
 
+#include "basis.cuh"
 #include "internal.h"
 
 namespace awsrc {
 
 namespace {
 
-struct DecRec {   // 16 bytes
+struct DecRec {   // an unpacked record; codes packed as signed bytes, code p in byte p
   uint16_t seed;
   int16_t scale;
-  int32_t pad;
-  int8_t code[8];
+  uint32_t cw[2];
 };
+
+__device__ __forceinline__ int code_of(const DecRec& d, int p) {
+  return (int)(int8_t)((p < 4 ? d.cw[0] : d.cw[1]) >> (8 * (p & 3)));
+}
 
 struct DecArgs {
   int n_mod;
@@ -36,11 +42,26 @@ __device__ __forceinline__ int ceil_log2_dev(uint64_t x) {
   return x <= 1 ? 0 : 64 - __clzll((long long)(x - 1));
 }
 
-__device__ __forceinline__ uint64_t get_bits(const uint8_t* rec, int* pos, int nbits) {
-  uint64_t v = 0;
-  for (int k = 0; k < nbits; ++k, ++*pos)
-    if ((rec[*pos >> 3] >> (*pos & 7)) & 1u) v |= 1ull << k;
-  return v;
+// A record is at most 128 bits (tile < 2^32, seed < 2^16, scale <= 16 bits,
+// codes <= 64 bits): read its L bytes little-endian into two words.
+__device__ __forceinline__ void load_record(const uint8_t* rec, int L, uint64_t* w0, uint64_t* w1) {
+  uint64_t a = 0, b = 0;
+  for (int i = 0; i < L; ++i) {
+    const uint64_t v = rec[i];
+    if (i < 8) a |= v << (8 * i);
+    else b |= v << (8 * (i - 8));
+  }
+  *w0 = a;
+  *w1 = b;
+}
+
+// Bits [pos, pos + n) of the 128-bit value (w1:w0), n <= 64.
+__device__ __forceinline__ uint64_t field(uint64_t w0, uint64_t w1, int pos, int n) {
+  uint64_t v;
+  if (pos >= 64) v = w1 >> (pos - 64);
+  else if (pos == 0) v = w0;
+  else v = (w0 >> pos) | (w1 << (64 - pos));
+  return n >= 64 ? v : (v & ((1ull << n) - 1ull));
 }
 
 __device__ __forceinline__ int64_t sign_extend(uint64_t v, int bits) {
@@ -59,35 +80,48 @@ __device__ __forceinline__ int64_t stream_K(const uint8_t* stream, int64_t K, in
 }
 
 // Unpack record k; returns the tile or -1 when it names a tile/seed out of range.
+// `end` bounds the bytes that may be read (h + kmax*L); when the three 8-byte
+// words around the record lie inside it and the stream is 8-byte aligned, the
+// record is read with word loads and a funnel shift, else byte by byte.
 __device__ __forceinline__ int64_t unpack(const Prm& pr, const uint8_t* stream, int64_t T, int64_t L,
-                                          int64_t h, int64_t k, DecRec* d) {
-  const uint8_t* rec = stream + h + k * L;
+                                          int64_t h, int64_t k, DecRec* d, int64_t end = -1) {
+  uint64_t w0, w1;
+  const int64_t off = h + k * L;
+  const int64_t a0 = off & ~7ll;
+  if (end >= 0 && a0 + 24 <= end && (reinterpret_cast<uintptr_t>(stream) & 7) == 0) {
+    const uint64_t* q = reinterpret_cast<const uint64_t*>(stream + a0);
+    const uint64_t x0 = __ldg(q), x1 = __ldg(q + 1), x2 = __ldg(q + 2);
+    const int sh = (int)(off - a0) * 8;
+    w0 = sh ? (x0 >> sh) | (x1 << (64 - sh)) : x0;
+    w1 = sh ? (x1 >> sh) | (x2 << (64 - sh)) : x1;
+  } else {
+    load_record(stream + off, (int)L, &w0, &w1);
+  }
+  const int tb = ceil_log2_dev((uint64_t)T), sb = ceil_log2_dev((uint64_t)pr.S);
   int pos = 0;
-  const int64_t tile = (int64_t)get_bits(rec, &pos, ceil_log2_dev((uint64_t)T));
-  const uint32_t seed = (uint32_t)get_bits(rec, &pos, ceil_log2_dev((uint64_t)pr.S));
-  const uint64_t sf = get_bits(rec, &pos, pr.b_e);
+  const int64_t tile = (int64_t)field(w0, w1, pos, tb);
+  pos += tb;
+  const uint32_t seed = (uint32_t)field(w0, w1, pos, sb);
+  pos += sb;
+  const uint64_t sf = field(w0, w1, pos, pr.b_e);
+  pos += pr.b_e;
   d->seed = (uint16_t)seed;
   d->scale = pr.scale_mode == AWSRC_SCALE_POW2 ? (int16_t)(sign_extend(sf, pr.b_e) + pr.e_bias)
                                                : (int16_t)(uint16_t)sf;
-  d->pad = 0;
-  for (int p = 0; p < 8; ++p)
-    d->code[p] = p < pr.P ? (int8_t)sign_extend(get_bits(rec, &pos, pr.b), pr.b) : (int8_t)0;
+  uint32_t c0 = 0u, c1 = 0u;
+#pragma unroll
+  for (int p = 0; p < 8; ++p) {
+    if (p < pr.P) {
+      const uint32_t c = (uint32_t)(uint8_t)(int8_t)sign_extend(field(w0, w1, pos, pr.b), pr.b);
+      if (p < 4) c0 |= c << (8 * p);
+      else c1 |= c << (8 * (p - 4));
+      pos += pr.b;
+    }
+  }
+  d->cw[0] = c0;
+  d->cw[1] = c1;
   if (tile >= T || seed >= (uint32_t)pr.S) return -1;
   return tile;
-}
-
-__global__ void scatter_kernel(Prm pr, const uint8_t* __restrict__ stream, int64_t T, int64_t L,
-                               int64_t h, int64_t K, int64_t kmax, int32_t* __restrict__ map,
-                               DecRec* __restrict__ dec, uint32_t* __restrict__ status) {
-  const int64_t Kd = stream_K(stream, K, kmax);
-  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < Kd;
-       k += (int64_t)gridDim.x * blockDim.x) {
-    DecRec d;
-    const int64_t tile = unpack(pr, stream, T, L, h, k, &d);
-    if (tile < 0) { atomicOr(status, kFaultRecord); continue; }
-    dec[k] = d;
-    if (map) map[tile] = (int32_t)k;
-  }
 }
 
 __device__ __forceinline__ float scale_of(const Prm& pr, int16_t s) {
@@ -109,83 +143,97 @@ template <> struct Io<__nv_bfloat16> {
 template <typename TI, int G>
 struct alignas(sizeof(TI) * G) Vec { TI v[G]; };
 
-template <typename TI, typename TO, int G>
-__device__ __forceinline__ void apply_group(const Prm& pr, const Vec<TI, G>& in, int j0,
-                                            const DecRec* dr, const uint64_t* __restrict__ masks,
-                                            Vec<TO, G>* out) {
-  float w[G];
+// Raw vector type of the same width, for the streaming load/store intrinsics.
+template <int BYTES> struct RawVec;
+template <> struct RawVec<16> { using T = uint4; };
+template <> struct RawVec<8> { using T = uint2; };
+
+template <typename V>
+__device__ __forceinline__ V ld_stream(const V* p) {
+  constexpr int B = sizeof(V) >= 16 ? 16 : (int)sizeof(V);
+  using R = typename RawVec<B>::T;
+  V v;
 #pragma unroll
-  for (int g = 0; g < G; ++g) w[g] = Io<TI>::ld(in.v, g);
-  if (dr) {
-    const uint64_t* mk = masks + (size_t)dr->seed * pr.P * pr.W + (j0 >> 6);
-    int kj[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) kj[g] = 0;
-    for (int p = 0; p < pr.P; ++p) {
-      const uint64_t bits = mk[(size_t)p * pr.W] >> (j0 & 63);
-      const int cp = dr->code[p];
-#pragma unroll
-      for (int g = 0; g < G; ++g) kj[g] += ((bits >> g) & 1ull) ? -cp : cp;
-    }
-    const float sc = scale_of(pr, dr->scale);
-#pragma unroll
-    for (int g = 0; g < G; ++g)
-      w[g] = __fadd_rn(w[g], __fmul_rn(__fmul_rn((float)kj[g], pr.c), sc));
+  for (int i = 0; i < (int)sizeof(V) / B; ++i) {
+    const R r = __ldcs(reinterpret_cast<const R*>(p) + i);
+    memcpy(reinterpret_cast<char*>(&v) + i * B, &r, B);
   }
-#pragma unroll
-  for (int g = 0; g < G; ++g) out->v[g] = Io<TO>::cvt(w[g]);
+  return v;
 }
 
+template <typename V>
+__device__ __forceinline__ void st_stream(V* p, const V& v) {
+  constexpr int B = sizeof(V) >= 16 ? 16 : (int)sizeof(V);
+  using R = typename RawVec<B>::T;
+#pragma unroll
+  for (int i = 0; i < (int)sizeof(V) / B; ++i) {
+    R r;
+    memcpy(&r, reinterpret_cast<const char*>(&v) + i * B, B);
+    __stcs(reinterpret_cast<R*>(p) + i, r);
+  }
+}
+
+// Dense pass: W_hat = convert(W0) for every element, a pure stream with U
+// independent 16-byte vectors in flight per thread and no dependent loads.
+// With `basis`, the blocks of grid slice y = 0 (dispatched first) generate the
+// basis masks, one warp per selector, overlapping GenBasis with the
+// memory-bound stream of the other slices.
 template <typename TI, typename TO, int G>
-__global__ void __launch_bounds__(256) dense_kernel(Prm pr, const __grid_constant__ DecArgs a,
-                                                    const int32_t* __restrict__ map,
-                                                    const DecRec* __restrict__ dec,
-                                                    const uint64_t* __restrict__ masks) {
-  const DecodeMod& md = a.m[blockIdx.y];
+__global__ void __launch_bounds__(256) copy_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                   uint64_t* __restrict__ masks, int basis) {
+  constexpr int U = 4;
+  if (basis && blockIdx.y == 0) {
+    __shared__ uint8_t perm_s[8][kMaxC], kidx_s[8][kMaxC], pool_s[8][kMaxC];
+    __shared__ int cols_s[8][kMaxP];
+    const int warp = threadIdx.x >> 5;
+    const int s = blockIdx.x * 8 + warp;
+    if (s < pr.S) basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
+    return;
+  }
+  const DecodeMod& md = a.m[blockIdx.y - (basis ? 1 : 0)];
   const int64_t ngroups = md.rows * md.cols / G;
-  const TI* __restrict__ src = static_cast<const TI*>(md.W0);
-  TO* __restrict__ dst = static_cast<TO*>(md.out);
+  const Vec<TI, G>* __restrict__ src = static_cast<const Vec<TI, G>*>(md.W0);
+  Vec<TO, G>* __restrict__ dst = static_cast<Vec<TO, G>*>(md.out);
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  for (; gi + stride < ngroups; gi += 2 * stride) {
-    const int64_t g1 = gi + stride;
-    const Vec<TI, G> v0 = *reinterpret_cast<const Vec<TI, G>*>(src + gi * G);
-    const Vec<TI, G> v1 = *reinterpret_cast<const Vec<TI, G>*>(src + g1 * G);
-    const int32_t r0 = __ldg(map + md.tile_off + ((gi * G) >> pr.logC));
-    const int32_t r1 = __ldg(map + md.tile_off + ((g1 * G) >> pr.logC));
-    DecRec d0, d1;
-    if (r0 >= 0) d0 = dec[r0];
-    if (r1 >= 0) d1 = dec[r1];
-    Vec<TO, G> o0, o1;
-    apply_group<TI, TO, G>(pr, v0, (int)((gi * G) & (pr.C - 1)), r0 >= 0 ? &d0 : nullptr, masks, &o0);
-    apply_group<TI, TO, G>(pr, v1, (int)((g1 * G) & (pr.C - 1)), r1 >= 0 ? &d1 : nullptr, masks, &o1);
-    *reinterpret_cast<Vec<TO, G>*>(dst + gi * G) = o0;
-    *reinterpret_cast<Vec<TO, G>*>(dst + g1 * G) = o1;
-  }
-  if (gi < ngroups) {
-    const Vec<TI, G> v0 = *reinterpret_cast<const Vec<TI, G>*>(src + gi * G);
-    const int32_t r0 = map[md.tile_off + ((gi * G) >> pr.logC)];
-    DecRec d0;
-    if (r0 >= 0) d0 = dec[r0];
-    Vec<TO, G> o0;
-    apply_group<TI, TO, G>(pr, v0, (int)((gi * G) & (pr.C - 1)), r0 >= 0 ? &d0 : nullptr, masks, &o0);
-    *reinterpret_cast<Vec<TO, G>*>(dst + gi * G) = o0;
+  for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g0 < ngroups; g0 += U * stride) {
+    Vec<TI, G> v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (g0 + u * stride < ngroups) v[u] = ld_stream(src + g0 + u * stride);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (g0 + u * stride >= ngroups) break;
+      Vec<TO, G> o;
+#pragma unroll
+      for (int g = 0; g < G; ++g) o.v[g] = Io<TO>::cvt(Io<TI>::ld(v[u].v, g));
+      st_stream(dst + g0 + u * stride, o);
+    }
   }
 }
 
-// One warp per record; W_hat already holds W0 (same dtype).
-template <typename TO>
-__global__ void inplace_kernel(Prm pr, const __grid_constant__ DecArgs a,
-                               const uint8_t* __restrict__ stream, const uint64_t* __restrict__ masks,
-                               uint32_t* __restrict__ status) {
+// Patch pass: G-element groups of the recorded tiles, one thread per group
+// (C/G threads per record, adjacent threads on the same record), so each
+// record's tile moves as whole 16-byte vectors and many records are in flight.
+// W_hat = fl(W0 + r_hat) is computed from W0, which may be W_hat itself.
+// One thread per G-element group of a recorded tile (C/G adjacent threads per
+// record), so each record's tile moves as coalesced 16-byte vectors.
+template <typename TI, typename TO, int G>
+__global__ void __launch_bounds__(256) patch_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                    const uint8_t* __restrict__ stream,
+                                                    const uint64_t* __restrict__ masks,
+                                                    uint32_t* __restrict__ status) {
   const int64_t Kd = stream_K(stream, a.K, a.kmax);
-  const int lane = threadIdx.x & 31;
-  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t k = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < Kd; k += warps) {
+  const int gshift = pr.logC - (G == 8 ? 3 : 2);  // log2 of the groups per tile
+  const int64_t total = Kd << gshift;
+  const int64_t end = a.h + a.kmax * a.L;
+  for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total;
+       x += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t k = x >> gshift;
+    const int gj = (int)(x & ((1 << gshift) - 1));
     DecRec d;
-    const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d);
+    const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d, end);
     if (tile < 0) {
-      if (lane == 0) atomicOr(status, kFaultRecord);
+      if (gj == 0) atomicOr(status, kFaultRecord);
       continue;
     }
     const DecodeMod& mlast = a.m[a.n_mod - 1];
@@ -194,104 +242,151 @@ __global__ void inplace_kernel(Prm pr, const __grid_constant__ DecArgs a,
     for (int i = 1; i < a.n_mod; ++i)
       if (tile >= a.m[i].tile_off) mi = i;
     const DecodeMod& md = a.m[mi];
-    TO* dst = static_cast<TO*>(md.out) + (tile - md.tile_off) * pr.C;
-    const float sc = scale_of(pr, d.scale);
-    const uint64_t* mk = masks + (size_t)d.seed * pr.P * pr.W;
-    for (int j = lane; j < pr.C; j += 32) {
-      int kj = 0;
-      for (int p = 0; p < pr.P; ++p) {
-        const uint64_t bit = (mk[(size_t)p * pr.W + (j >> 6)] >> (j & 63)) & 1ull;
-        kj += bit ? -d.code[p] : d.code[p];
-      }
-      const float w = Io<TO>::ld(dst, j);
-      dst[j] = Io<TO>::cvt(__fadd_rn(w, __fmul_rn(__fmul_rn((float)kj, pr.c), sc)));
+    const int j0 = gj * G;
+    const int64_t e0 = (tile - md.tile_off) * pr.C + j0;
+    const Vec<TI, G> v = *reinterpret_cast<const Vec<TI, G>*>(static_cast<const TI*>(md.W0) + e0);
+    const uint64_t* mk = masks + (size_t)d.seed * pr.P * pr.W + (j0 >> 6);
+    // k_j = sum_p (1 - 2 bit_pj) c_p = (sum_p c_p) - 2 sum_p bit_pj c_p, exact in integers
+    int tot = 0, acc[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) acc[g] = 0;
+    for (int p = 0; p < pr.P; ++p) {
+      const uint32_t bits = (uint32_t)(__ldg(mk + (size_t)p * pr.W) >> (j0 & 63));
+      const int cp = code_of(d, p);
+      tot += cp;
+#pragma unroll
+      for (int g = 0; g < G; ++g) acc[g] += (int)((bits >> g) & 1u) * cp;
     }
+    const float sc = scale_of(pr, d.scale);
+    Vec<TO, G> o;
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+      o.v[g] = Io<TO>::cvt(__fadd_rn(Io<TI>::ld(v.v, g),
+                                     __fmul_rn(__fmul_rn((float)(tot - 2 * acc[g]), pr.c), sc)));
+    *reinterpret_cast<Vec<TO, G>*>(static_cast<TO*>(md.out) + e0) = o;
   }
 }
 
+// Tiles smaller than one vector take one thread per element.
+template <typename TI, typename TO>
+__global__ void __launch_bounds__(256) patch_small_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                          const uint8_t* __restrict__ stream,
+                                                          const uint64_t* __restrict__ masks,
+                                                          uint32_t* __restrict__ status) {
+  const int64_t Kd = stream_K(stream, a.K, a.kmax);
+  const int64_t total = Kd * pr.C;
+  for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total;
+       x += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t k = x >> pr.logC;
+    const int j = (int)(x & (pr.C - 1));
+    DecRec d;
+    const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d);
+    if (tile < 0) {
+      if (j == 0) atomicOr(status, kFaultRecord);
+      continue;
+    }
+    const DecodeMod& mlast = a.m[a.n_mod - 1];
+    if (tile < a.m[0].tile_off || tile >= mlast.tile_off + mlast.rows * mlast.cols / pr.C) continue;
+    int mi = 0;
+    for (int i = 1; i < a.n_mod; ++i)
+      if (tile >= a.m[i].tile_off) mi = i;
+    const DecodeMod& md = a.m[mi];
+    const int64_t e = (tile - md.tile_off) * pr.C + j;
+    const uint64_t* mk = masks + (size_t)d.seed * pr.P * pr.W;
+    int kj = 0;
+    for (int p = 0; p < pr.P; ++p) kj += ((mk[(size_t)p * pr.W + (j >> 6)] >> (j & 63)) & 1ull) ? -code_of(d, p) : code_of(d, p);
+    const float w = Io<TI>::ld(static_cast<const TI*>(md.W0) + e, 0);
+    static_cast<TO*>(md.out)[e] = Io<TO>::cvt(__fadd_rn(w, __fmul_rn(__fmul_rn((float)kj, pr.c), scale_of(pr, d.scale))));
+  }
+}
+
+// copy: stream the modules of `a`; basis: also generate the masks (an extra
+// grid slice). With copy false only the basis slice runs.
 template <typename TI, typename TO, int G>
-cudaError_t launch_dense_t(const Prm& pr, const DecArgs& a, const int32_t* map, const DecRec* dec,
-                           const uint64_t* masks, cudaStream_t st) {
+cudaError_t launch_copy_t(const Prm& pr, DecArgs a, bool copy, bool basis, uint64_t* masks,
+                          cudaStream_t st) {
   int64_t maxg = 0;
+  if (!copy) a.n_mod = 0;
   for (int i = 0; i < a.n_mod; ++i) maxg = std::max<int64_t>(maxg, a.m[i].rows * a.m[i].cols / G);
   int dev = 0, nsm = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t want = (maxg + 2 * 256 - 1) / (2 * 256);
-  const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)nsm * 8));
-  dense_kernel<TI, TO, G><<<dim3(gx, a.n_mod), 256, 0, st>>>(pr, a, map, dec, masks);
+  const int64_t want = (maxg + 4 * 256 - 1) / (4 * 256);
+  int64_t gx = std::min<int64_t>(want, (int64_t)nsm * 8);
+  if (basis) gx = std::max<int64_t>(gx, (pr.S + 7) / 8);
+  gx = std::max<int64_t>(gx, 1);
+  copy_kernel<TI, TO, G><<<dim3((unsigned)gx, a.n_mod + (basis ? 1 : 0)), 256, 0, st>>>(pr, a, masks,
+                                                                                      basis ? 1 : 0);
   note_launches(1);
   return cudaGetLastError();
 }
 
-}  // namespace
-
-cudaError_t launch_dense_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype,
-                               const int32_t* map, const DecRec* dec, const uint64_t* masks,
-                               cudaStream_t st) {
-  const bool f32in = (w0_dtype == AWSRC_DTYPE_F32), f32out = (out_dtype == AWSRC_DTYPE_F32);
-  if (f32in && f32out) return launch_dense_t<float, float, 4>(pr, a, map, dec, masks, st);
-  if (f32in) return launch_dense_t<float, __nv_bfloat16, 4>(pr, a, map, dec, masks, st);
-  if (pr.C >= 8) {
-    if (f32out) return launch_dense_t<__nv_bfloat16, float, 8>(pr, a, map, dec, masks, st);
-    return launch_dense_t<__nv_bfloat16, __nv_bfloat16, 8>(pr, a, map, dec, masks, st);
+template <typename TI, typename TO>
+cudaError_t launch_patch_t(const Prm& pr, const DecArgs& a, const uint8_t* stream, const uint64_t* masks,
+                           uint32_t* status, cudaStream_t st) {
+  const int64_t work = a.K >= 0 ? std::min(a.K, a.kmax) : a.kmax;
+  if (work <= 0) return cudaSuccess;
+  constexpr int G = 16 / sizeof(TI) < 16 / sizeof(TO) ? 16 / sizeof(TI) : 16 / sizeof(TO);
+  if (pr.C >= G) {
+    const int64_t threads = work * (pr.C / G);
+    const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>((threads + 255) / 256, 1 << 20));
+    patch_kernel<TI, TO, G><<<gx, 256, 0, st>>>(pr, a, stream, masks, status);
+  } else {
+    const int64_t threads = work * pr.C;
+    const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>((threads + 255) / 256, 1 << 20));
+    patch_small_kernel<TI, TO><<<gx, 256, 0, st>>>(pr, a, stream, masks, status);
   }
-  if (f32out) return launch_dense_t<__nv_bfloat16, float, 4>(pr, a, map, dec, masks, st);
-  return launch_dense_t<__nv_bfloat16, __nv_bfloat16, 4>(pr, a, map, dec, masks, st);
+  note_launches(1);
+  return cudaGetLastError();
 }
+
+cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype, bool copy,
+                         bool basis, const uint8_t* stream, uint64_t* masks, uint32_t* status,
+                         cudaStream_t st) {
+  const bool f32in = (w0_dtype == AWSRC_DTYPE_F32), f32out = (out_dtype == AWSRC_DTYPE_F32);
+  cudaError_t e = cudaSuccess;
+  if (copy || basis) {
+    if (f32in && f32out) e = launch_copy_t<float, float, 4>(pr, a, copy, basis, masks, st);
+    else if (f32in) e = launch_copy_t<float, __nv_bfloat16, 4>(pr, a, copy, basis, masks, st);
+    else if (f32out) e = launch_copy_t<__nv_bfloat16, float, 8>(pr, a, copy, basis, masks, st);
+    else e = launch_copy_t<__nv_bfloat16, __nv_bfloat16, 8>(pr, a, copy, basis, masks, st);
+    if (e != cudaSuccess) return e;
+  }
+  if (f32in && f32out) return launch_patch_t<float, float>(pr, a, stream, masks, status, st);
+  if (f32in) return launch_patch_t<float, __nv_bfloat16>(pr, a, stream, masks, status, st);
+  if (f32out) return launch_patch_t<__nv_bfloat16, float>(pr, a, stream, masks, status, st);
+  return launch_patch_t<__nv_bfloat16, __nv_bfloat16>(pr, a, stream, masks, status, st);
+}
+
+}  // namespace
 
 cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
-                          const uint64_t* masks, int32_t* map, uint32_t* status, cudaStream_t st) {
-  cudaError_t e;
-  if (mode == AWSRC_DECODE_DENSE) {
-    // map[T] then decoded records dec[T]
-    DecRec* dec = reinterpret_cast<DecRec*>(map + align_up((size_t)T, 64));
-    e = cudaMemsetAsync(map, 0xff, (size_t)T * sizeof(int32_t), st);
-    if (e != cudaSuccess) return e;
-    const int64_t work = (K >= 0 ? std::min(K, kmax) : kmax);
-    if (work > 0) {
-      const unsigned gx = (unsigned)std::min<int64_t>((work + 255) / 256, 65535);
-      scatter_kernel<<<gx, 256, 0, st>>>(pr, stream, T, L, h, K, kmax, map, dec, status);
-      note_launches(1);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    // launches over runs of at most 16 modules sharing the input dtype
-    int i0 = 0;
-    while (i0 < n_mod) {
-      int i1 = i0 + 1;
-      while (i1 < n_mod && i1 - i0 < kMaxModsPerLaunch && mods[i1].w0_dtype == mods[i0].w0_dtype) ++i1;
-      DecArgs a;
-      a.n_mod = i1 - i0;
-      a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
-      for (int i = 0; i < a.n_mod; ++i) a.m[i] = mods[i0 + i];
-      if ((e = launch_dense_group(pr, a, mods[i0].w0_dtype, out_dtype, map, dec, masks, st)) != cudaSuccess)
-        return e;
-      i0 = i1;
-    }
-    return cudaSuccess;
-  }
-  // in place: every launch walks the record list and applies the records that
-  // fall in its group of modules
-  for (int i0 = 0; i0 < n_mod; i0 += kMaxModsPerLaunch) {
+                          uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
+  (void)scratch;
+  // launches over runs of at most 16 modules sharing the input dtype: DENSE
+  // copies every element (the first launch also generates the basis masks),
+  // then both modes patch the tiles named by records
+  int i0 = 0;
+  while (i0 < n_mod) {
+    int i1 = i0 + 1;
+    while (i1 < n_mod && i1 - i0 < kMaxModsPerLaunch && mods[i1].w0_dtype == mods[i0].w0_dtype) ++i1;
     DecArgs a;
-    a.n_mod = std::min(kMaxModsPerLaunch, n_mod - i0);
+    a.n_mod = i1 - i0;
     a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
     for (int i = 0; i < a.n_mod; ++i) a.m[i] = mods[i0 + i];
-    const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
-    if (work == 0) continue;
-    const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>((work + 7) / 8, 65535));
-    if (out_dtype == AWSRC_DTYPE_F32) inplace_kernel<float><<<gx, 256, 0, st>>>(pr, a, stream, masks, status);
-    else inplace_kernel<__nv_bfloat16><<<gx, 256, 0, st>>>(pr, a, stream, masks, status);
-    note_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const cudaError_t e = launch_group(pr, a, mods[i0].w0_dtype, out_dtype, mode == AWSRC_DECODE_DENSE,
+                                       i0 == 0, stream, masks, status, st);
+    if (e != cudaSuccess) return e;
+    i0 = i1;
   }
   return cudaSuccess;
 }
 
 size_t decode_scratch_bytes(int64_t T, int mode) {
-  if (mode != AWSRC_DECODE_DENSE) return 0;
-  return align_up((size_t)T, 64) * sizeof(int32_t) + (size_t)T * sizeof(DecRec);
+  (void)T;
+  (void)mode;
+  return 0;
 }
 
 }  // namespace awsrc

@@ -115,8 +115,6 @@ extern "C" awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* p
   cudaStream_t st = (cudaStream_t)stream_handle;
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);  // the fault word starts at 0
   if (e != cudaSuccess) return cuda_fail(e, "decode_noalloc: clear");
-  e = launch_gen_basis(pr, masks, pr.S, st);
-  if (e != cudaSuccess) return cuda_fail(e, "decode_noalloc: gen_basis");
   e = launch_decode(pr, n_mod, dm, T, L, h, stream, K, kmax, mods[0].w0_dtype, AWSRC_DECODE_INPLACE,
                     masks, nullptr, status, st);
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "decode_noalloc");

@@ -95,7 +95,7 @@ __device__ __forceinline__ void tile_elem(const Prm& pr, const ModDesc& md, int6
 }
 
 // Score of seed s for one tile given its staged y (and d, gd for PF).
-template <int P, int VAR>
+template <int P, int VAR, bool ALLOW_FAST = true>
 __device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const float* d,
                                             float gd_row, const uint64_t* __restrict__ masks,
                                             const float* __restrict__ gram_cb, uint32_t s,
@@ -141,6 +141,11 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const
     for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = gt[P * (P - 1) / 2 + P + i];
     const float gd = gt[P * (P - 1) + P];
     ldl_solve<P>(L, invD, bv, alpha);
+    if (ALLOW_FAST && pr.fast_pow2) {
+#pragma unroll
+      for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(2.0f, Goff[i]);
+      return quant_gain_fast<P>(pr, alpha, bv, gd, Goff, q, sf);
+    }
     return quant_gain<P>(pr, alpha, bv, gd, Goff, q, sf);
   } else {
     float Goff[NL], L[NL], invD[P];
@@ -149,7 +154,14 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const
     const float eps = __fmul_rn(pr.ridge_rel, gd_row);
     const bool ok = ldl_factor<P>(gd_row, eps, Goff, L, invD);
     ldl_solve<P>(L, invD, bv, alpha);
-    const float g = quant_gain<P>(pr, alpha, bv, gd_row, Goff, q, sf);
+    float g;
+    if (ALLOW_FAST && pr.fast_pow2) {
+#pragma unroll
+      for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(2.0f, Goff[i]);
+      g = quant_gain_fast<P>(pr, alpha, bv, gd_row, Goff, q, sf);
+    } else {
+      g = quant_gain<P>(pr, alpha, bv, gd_row, Goff, q, sf);
+    }
     return ok ? g : neg_inf();
   }
 }
@@ -233,7 +245,85 @@ __global__ void __launch_bounds__(kGenThreads) search_generic_kernel(
   }
 }
 
+// V consecutive elements (V = 4 or 8) of a weight array as floats; idx is a
+// multiple of V. Vector loads when the array is 16-byte aligned.
+template <int V>
+__device__ __forceinline__ void load_run(const void* p, int64_t idx, int dtype, bool aligned, float* out) {
+  if (aligned && dtype == AWSRC_DTYPE_F32) {
+#pragma unroll
+    for (int i = 0; i < V; i += 4) {
+      const float4 f = *reinterpret_cast<const float4*>(static_cast<const float*>(p) + idx + i);
+      out[i] = f.x; out[i + 1] = f.y; out[i + 2] = f.z; out[i + 3] = f.w;
+    }
+  } else if (aligned && V == 8) {
+    const uint4 u = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p) + idx);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = __uint_as_float(w[i] << 16);
+      out[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < V; ++i) out[i] = load_elem(p, idx + i, dtype);
+  }
+}
+
 // --------------------------------------------------------------- finalize --
+// One thread per tile; a block stages its tiles' y (and d) in shared memory with
+// coalesced loads: tiles are numbered row-major, so consecutive tiles of a
+// module are consecutive C-element runs of its weight arrays.
+__host__ __device__ inline int fin_tiles(int C) { return C <= 64 ? 128 : 16384 / C; }
+
+// Stage y = d*(W - W0) (and d) of tiles [t0, t0 + TB) in shared memory, V
+// elements per load, loads of four runs issued before any is used.
+template <int V, int VAR>
+__device__ __forceinline__ void stage_tiles(const Prm& pr, const LaunchDesc& ld, int64_t t0, int64_t last,
+                                            int TB, const int* tmod, int* tok, float* ys, float* ds) {
+  const int C = pr.C, ldc = C + 1;
+  const int nrun = TB * C / V;
+#pragma unroll 4
+  for (int g = threadIdx.x; g < nrun; g += blockDim.x) {
+    const int lt = (g * V) >> pr.logC, j0 = (g * V) & (C - 1);
+    const int64_t t = t0 + lt;
+    float y[V], d[V];
+    if (t < last) {
+      const ModDesc& md = ld.m[tmod[lt]];
+      const int64_t ltm = t - md.tile_off;
+      const int64_t idx = ltm * C + j0;  // a module's tiles are consecutive runs of C elements
+      const int64_t cb = ltm % md.n_cb;
+      const bool alW = ((reinterpret_cast<uintptr_t>(md.W) | reinterpret_cast<uintptr_t>(md.W0)) & 15) == 0;
+      float w[V], w0[V], a[V];
+      load_run<V>(md.W, idx, md.w_dtype, alW, w);
+      load_run<V>(md.W0, idx, md.w0_dtype, alW, w0);
+      load_run<V>(md.act, cb * C + j0, AWSRC_DTYPE_F32, (reinterpret_cast<uintptr_t>(md.act) & 15) == 0, a);
+      float f[V];
+      if (VAR == AWSRC_VARIANT_PF)
+        load_run<V>(md.fisher, idx, AWSRC_DTYPE_F32, (reinterpret_cast<uintptr_t>(md.fisher) & 15) == 0, f);
+      bool ok = true;
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        const float r = __fsub_rn(w[i], w0[i]);
+        const float dv = VAR == AWSRC_VARIANT_U
+                             ? a[i]
+                             : __fadd_rn(__fmul_rn(md.w_act, a[i]), __fmul_rn(md.w_fisher, f[i]));
+        ok = ok && in_domain(r, dv);
+        d[i] = dv;
+        y[i] = __fmul_rn(dv, r);
+      }
+      if (!ok) tok[lt] = 0;
+    } else {
+#pragma unroll
+      for (int i = 0; i < V; ++i) { y[i] = 0.0f; d[i] = 0.0f; }
+    }
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      ys[lt * ldc + j0 + i] = y[i];
+      if (VAR == AWSRC_VARIANT_PF) ds[lt * ldc + j0 + i] = d[i];
+    }
+  }
+}
+
 template <int P, int VAR>
 __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
                                                        const uint64_t* __restrict__ masks,
@@ -241,16 +331,33 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
                                                        const float2* __restrict__ partials,
                                                        awsrc_candidate* __restrict__ out,
                                                        uint32_t* __restrict__ status) {
-  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  extern __shared__ float fsm[];
+  const int C = pr.C, ldc = C + 1, TB = fin_tiles(C);
+  float* ys = fsm;
+  float* ds = fsm + TB * ldc;
+  __shared__ int tmod[128];
+  __shared__ int tok[128];
   const int64_t first = ld.m[0].tile_off;
   const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
-  if (t < first || t >= last) return;
-  int mi = 0;
-  for (int i = 1; i < ld.n; ++i)
-    if (t >= ld.m[i].tile_off) mi = i;
-  const ModDesc& md = ld.m[mi];
-  const int64_t lt = t - md.tile_off;
-  const int64_t row = lt / md.n_cb, cb = lt % md.n_cb;
+  const int64_t t0 = first + (int64_t)blockIdx.x * TB;
+  const int tid = threadIdx.x;
+  if (tid < TB) {
+    const int64_t t = t0 + tid;
+    int mi = 0;
+    for (int i = 1; i < ld.n; ++i)
+      if (t >= ld.m[i].tile_off) mi = i;
+    tmod[tid] = mi;
+    tok[tid] = 1;
+  }
+  __syncthreads();
+  if (C >= 8) stage_tiles<8, VAR>(pr, ld, t0, last, TB, tmod, tok, ys, ds);
+  else stage_tiles<4, VAR>(pr, ld, t0, last, TB, tmod, tok, ys, ds);
+  __syncthreads();
+  if (tid >= TB) return;
+  const int64_t t = t0 + tid;
+  if (t >= last) return;
+  const ModDesc& md = ld.m[tmod[tid]];
+  const int64_t cb = (t - md.tile_off) % md.n_cb;
   float bg = neg_inf();
   uint32_t bs = 0xffffffffu;
   for (int z = 0; z < md.nsplit; ++z) {
@@ -266,17 +373,11 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
 #pragma unroll
   for (int p = 0; p < 8; ++p) cd.code[p] = 0;
   if (bg > neg_inf() && bs < (uint32_t)pr.S) {
-    float y[kMaxC], d[kMaxC];
-    bool ok = true;
-    for (int j = 0; j < pr.C; ++j) {
-      bool okj;
-      tile_elem(pr, md, row, cb, j, &y[j], &d[j], &okj);
-      ok = ok && okj;
-    }
+    const bool ok = tok[tid] != 0;
     float gd_row = 0.0f;
     if (VAR == AWSRC_VARIANT_PF) {
       float w = 0.0f;
-      for (int j = 0; j < pr.C; ++j) w = __fadd_rn(w, d[j]);
+      for (int j = 0; j < C; ++j) w = __fadd_rn(w, ds[tid * ldc + j]);
       gd_row = __fmul_rn(pr.c2, w);
     }
     const float* gram_cb = (VAR == AWSRC_VARIANT_U)
@@ -284,7 +385,10 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
                                : nullptr;
     float q[P];
     int sf = 0;
-    const float g = score_seed<P, VAR>(pr, y, d, gd_row, masks, gram_cb, bs, q, &sf);
+    // the general quantiser here, so the self-check also compares it with the
+    // fast path the search used
+    const float g = score_seed<P, VAR, false>(pr, ys + tid * ldc, ds + tid * ldc, gd_row, masks,
+                                              gram_cb, bs, q, &sf);
     if (!ok || __float_as_uint(g) != __float_as_uint(bg)) atomicOr(status, kFaultSelfCheck);
     if (ok && g > neg_inf()) {
       cd.gain = g;
@@ -325,10 +429,14 @@ template <int P, int VAR>
 cudaError_t launch_finalize_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
                                const float* gram, const float2* partials, awsrc_candidate* out,
                                uint32_t* status, cudaStream_t st) {
+  const int64_t first = ld.m[0].tile_off;
   const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
-  const int tpb = 128;
-  finalize_kernel<P, VAR><<<(unsigned)((last + tpb - 1) / tpb), tpb, 0, st>>>(
-      pr, ld, masks, gram, partials, out, status);
+  const int TB = fin_tiles(pr.C);
+  const size_t smem = (size_t)TB * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
+  auto k = finalize_kernel<P, VAR>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k<<<(unsigned)((last - first + TB - 1) / TB), 128, smem, st>>>(pr, ld, masks, gram, partials, out, status);
   note_launches(1);
   return cudaGetLastError();
 }

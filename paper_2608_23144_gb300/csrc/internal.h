@@ -23,7 +23,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Launch counter behind awsrc_kernel_launches(): every launch site adds its kernels.
 void note_launches(int n);
 
-// basis.cu: masks[(s*P + p)*W + w] for s in [0, S_pad); seeds >= S get zero masks.
+// masks[(s*P + p)*W + w] for s in [0, S_pad); seeds >= S get zero masks.
 cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st);
 // Expanded +-1.0f masks for the C=64, P=4 search: [chunk][j][seed_in_chunk][p].
 cudaError_t launch_expand_masks_c64p4(const Prm& pr, const uint64_t* masks, float* out,
@@ -68,7 +68,7 @@ struct DecodeMod {
 };
 cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
-                          const uint64_t* masks, int32_t* map, uint32_t* status, cudaStream_t st);
+                          uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
 size_t decode_scratch_bytes(int64_t T, int mode);
 int generic_rows();
 int generic_chunk();

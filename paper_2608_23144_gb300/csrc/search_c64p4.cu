@@ -91,6 +91,7 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
+template <bool FAST>
 __global__ void __launch_bounds__(NT, 2)
     search_c64p4_kernel(Prm pr, LaunchDesc ld, const float* __restrict__ mexp,
                         const float* __restrict__ gram, float2* __restrict__ partials,
@@ -153,58 +154,68 @@ __global__ void __launch_bounds__(NT, 2)
 #pragma unroll
   for (int i = 0; i < 8; ++i) { bg[i] = neg_inf(); bs[i] = 0xffffffffu; }
 
+  // Seeds reach a thread in increasing order (chunk by chunk, tx before tx+16),
+  // so within a thread a strictly greater gain is the whole tie rule.
   bool timed_out = false;
   for (int k = 0; k < nck; ++k) {
     const int buf = k & 1;
     const bool ok = mbar_wait(&sm.mbar[buf], (uint32_t)((k >> 1) & 1));
-    if (__syncthreads_or(!ok)) { timed_out = true; break; }
+    if (!ok) timed_out = true;
 
-    float acc[8][8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int q = 0; q < 8; ++q) acc[i][q] = 0.0f;
-    const float* ysb = &sm.Ys[0][ty * 8];
-    const float* msb = &sm.Ms[buf][0][0];
-#pragma unroll 4
-    for (int j = 0; j < 64; ++j) {
-      const float4 ya = *reinterpret_cast<const float4*>(ysb + j * BM);
-      const float4 yb = *reinterpret_cast<const float4*>(ysb + j * BM + 4);
-      const float4 ma = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + tx * 4);
-      const float4 mb = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + (tx + 16) * 4);
-      const float yv[8] = {ya.x, ya.y, ya.z, ya.w, yb.x, yb.y, yb.z, yb.w};
-      const float mv[8] = {ma.x, ma.y, ma.z, ma.w, mb.x, mb.y, mb.z, mb.w};
+    if (!timed_out) {
+      float acc[8][8];
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[i][q] = __fmaf_rn(mv[q], yv[i], acc[i][q]);
-    }
-    // fused epilogue: solve, quantise, score, running argmax
+        for (int q = 0; q < 8; ++q) acc[i][q] = 0.0f;
+      const float* ysb = &sm.Ys[0][ty * 8];
+      const float* msb = &sm.Ms[buf][0][0];
+#pragma unroll 4
+      for (int j = 0; j < 64; ++j) {
+        const float4 ya = *reinterpret_cast<const float4*>(ysb + j * BM);
+        const float4 yb = *reinterpret_cast<const float4*>(ysb + j * BM + 4);
+        const float4 ma = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + tx * 4);
+        const float4 mb = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + (tx + 16) * 4);
+        const float yv[8] = {ya.x, ya.y, ya.z, ya.w, yb.x, yb.y, yb.z, yb.w};
+        const float mv[8] = {ma.x, ma.y, ma.z, ma.w, mb.x, mb.y, mb.z, mb.w};
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int sl = tx + 16 * h;
-      const uint32_t s = (uint32_t)((c0 + k) * CH + sl);
-      const float* gt = &sm.Gs[buf][sl * GS];
-      const float4 g0 = *reinterpret_cast<const float4*>(gt);
-      const float4 g1 = *reinterpret_cast<const float4*>(gt + 4);
-      const float4 g2 = *reinterpret_cast<const float4*>(gt + 8);
-      const float4 g3 = *reinterpret_cast<const float4*>(gt + 12);
-      const float gd = gt[16];
-      const float L[6] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y};
-      const float invD[4] = {g1.z, g1.w, g2.x, g2.y};
-      const float Goff[6] = {g2.z, g2.w, g3.x, g3.y, g3.z, g3.w};
+        for (int i = 0; i < 8; ++i)
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        float bv[4], alpha[4], q[4];
+          for (int q = 0; q < 8; ++q) acc[i][q] = __fmaf_rn(mv[q], yv[i], acc[i][q]);
+      }
+      // fused epilogue: solve, quantise, score, running argmax
 #pragma unroll
-        for (int p = 0; p < 4; ++p) bv[p] = __fmul_rn(c, acc[i][h * 4 + p]);
-        ldl_solve<4>(L, invD, bv, alpha);
-        int sf;
-        const float g = quant_gain<4>(pr, alpha, bv, gd, Goff, q, &sf);
-        if (better(g, s, bg[i], bs[i])) { bg[i] = g; bs[i] = s; }
+      for (int h = 0; h < 2; ++h) {
+        const int sl = tx + 16 * h;
+        const uint32_t s = (uint32_t)((c0 + k) * CH + sl);
+        const float* gt = &sm.Gs[buf][sl * GS];
+        const float4 g0 = *reinterpret_cast<const float4*>(gt);
+        const float4 g1 = *reinterpret_cast<const float4*>(gt + 4);
+        const float4 g2 = *reinterpret_cast<const float4*>(gt + 8);
+        const float4 g3 = *reinterpret_cast<const float4*>(gt + 12);
+        const float gd = gt[16];
+        const float L[6] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y};
+        const float invD[4] = {g1.z, g1.w, g2.x, g2.y};
+        float Gq[6] = {g2.z, g2.w, g3.x, g3.y, g3.z, g3.w};
+        if (FAST) {
+#pragma unroll
+          for (int i = 0; i < 6; ++i) Gq[i] = __fmul_rn(2.0f, Gq[i]);  // exact
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float bv[4], alpha[4], q[4];
+#pragma unroll
+          for (int p = 0; p < 4; ++p) bv[p] = __fmul_rn(c, acc[i][h * 4 + p]);
+          ldl_solve<4>(L, invD, bv, alpha);
+          int sf;
+          const float g = FAST ? quant_gain_fast<4>(pr, alpha, bv, gd, Gq, q, &sf)
+                               : quant_gain<4>(pr, alpha, bv, gd, Gq, q, &sf);
+          if (g > bg[i]) { bg[i] = g; bs[i] = s; }
+        }
       }
     }
-    __syncthreads();  // every thread is done with buffer `buf`
+    // every thread is done with buffer `buf`; a timeout anywhere ends the block
+    if (__syncthreads_or(timed_out)) { timed_out = true; break; }
     if (tid == 0 && k + 2 < nck) {
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_expect_tx(&sm.mbar[buf], kMsBytes + kGsBytes);
@@ -254,10 +265,10 @@ cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const float
                                 const float* gram, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st) {
   const size_t smem = sizeof(Smem);
-  cudaError_t e = cudaFuncSetAttribute(search_c64p4_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  search_c64p4_kernel<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, mexp, gram, partials, status);
+  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, mexp, gram, partials, status);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -171,46 +171,70 @@ __global__ void __launch_bounds__(RT) radix_scatter_kernel(const uint64_t* __res
   }
 }
 
-// Count eligible keys and cut: U per module, PF per rate.
-__global__ void cut_kernel(const uint64_t* __restrict__ keys, const __grid_constant__ SelArgs a,
-                           SelWs* __restrict__ sw, int64_t* __restrict__ d_counts,
-                           int64_t* __restrict__ d_bytes) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
-  auto invalid = [&](uint64_t k) { return ((k >> a.tbl) & 0x7FFFFFFFull) == 0x7FFFFFFFull; };
+// First index in [lo, hi) whose key is ineligible (eligible keys form a prefix
+// of the range), by one warp: each round the lanes test 32 evenly spaced
+// positions and the range shrinks to the gap where eligibility ends.
+__device__ __forceinline__ int64_t first_ineligible(const uint64_t* __restrict__ keys, int64_t lo,
+                                                    int64_t hi, int tbl) {
+  const int lane = threadIdx.x & 31;
+  while (hi - lo > 1) {
+    const int64_t span = (hi - lo + 31) / 32;
+    const int64_t pos = lo + lane * span;
+    bool valid = false;
+    if (pos < hi) valid = ((keys[pos] >> tbl) & 0x7FFFFFFFull) != 0x7FFFFFFFull;
+    const int cnt = __popc(__ballot_sync(0xffffffffu, valid));  // valid starts form a prefix of lanes
+    if (cnt == 0) return lo;                                      // keys[lo] already ineligible
+    const int64_t last_valid = lo + (int64_t)(cnt - 1) * span;
+    lo = last_valid + 1;
+    hi = min(hi, lo - 1 + span);
+  }
+  if (lo < hi) {
+    const bool v = ((keys[lo] >> tbl) & 0x7FFFFFFFull) != 0x7FFFFFFFull;
+    return v ? hi : lo;
+  }
+  return lo;
+}
+
+// Count eligible keys and cut: U per module (one warp per module), PF per rate.
+__global__ void __launch_bounds__(256) cut_kernel(const uint64_t* __restrict__ keys,
+                                                  const __grid_constant__ SelArgs a,
+                                                  SelWs* __restrict__ sw, int64_t* __restrict__ d_counts,
+                                                  int64_t* __restrict__ d_bytes) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (a.variant == AWSRC_VARIANT_U) {
-    int64_t off = 0;
-    for (int m = 0; m < a.n_mod; ++m) {
+    for (int m = warp; m < a.n_mod; m += blockDim.x >> 5) {
       const int64_t beg = a.tile_off[m], end = a.tile_off[m + 1];
-      int64_t lo = beg, hi = end;  // first invalid key in [beg, end)
-      while (lo < hi) {
-        const int64_t mid = (lo + hi) / 2;
-        if (invalid(keys[mid])) hi = mid; else lo = mid + 1;
+      const int64_t f = first_ineligible(keys, beg, end, a.tbl);
+      if (lane == 0) sw->K[m] = min(f - beg, a.kcap[m]);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int64_t off = 0;
+      for (int m = 0; m < a.n_mod; ++m) {
+        sw->rec_off[m] = off;
+        d_counts[m] = sw->K[m];
+        off += sw->K[m];
       }
-      const int64_t K = min(lo - beg, a.kcap[m]);
-      sw->K[m] = K;
-      sw->rec_off[m] = off;
-      d_counts[m] = K;
-      off += K;
+      sw->rec_off[a.n_mod] = off;
+      sw->kstream = off;
+      d_bytes[0] = a.h + off * a.L;
     }
-    sw->rec_off[a.n_mod] = off;
-    sw->kstream = off;
-    d_bytes[0] = a.h + off * a.L;
   } else {
-    int64_t lo = 0, hi = a.T;
-    while (lo < hi) {
-      const int64_t mid = (lo + hi) / 2;
-      if (invalid(keys[mid])) hi = mid; else lo = mid + 1;
+    if (warp == 0) {
+      const int64_t npos = first_ineligible(keys, 0, a.T, a.tbl);
+      if (lane == 0) {
+        sw->npos = npos;
+        int64_t kmax = 0;
+        for (int r = 0; r < a.n_rates; ++r) {
+          const int64_t K = min(npos, a.kcap[r]);
+          d_counts[r] = K;
+          d_bytes[r] = a.h + K * a.L;
+          kmax = max(kmax, K);
+        }
+        sw->kstream = kmax;
+      }
     }
-    sw->npos = lo;
-    int64_t kmax = 0;
-    for (int r = 0; r < a.n_rates; ++r) {
-      const int64_t K = min(lo, a.kcap[r]);
-      d_counts[r] = K;
-      d_bytes[r] = a.h + K * a.L;
-      kmax = max(kmax, K);
-    }
-    sw->kstream = kmax;
-    for (int m = 0; m < a.n_mod; ++m) sw->K[m] = 0;
+    for (int m = threadIdx.x; m < a.n_mod; m += blockDim.x) sw->K[m] = 0;
   }
 }
 
@@ -218,9 +242,18 @@ __device__ __forceinline__ int ceil_log2_dev(uint64_t x) {
   return x <= 1 ? 0 : 64 - __clzll((long long)(x - 1));
 }
 
-__device__ __forceinline__ void put_bits(uint8_t* rec, int* pos, uint64_t v, int nbits) {
-  for (int k = 0; k < nbits; ++k, ++*pos)
-    if ((v >> k) & 1ull) rec[*pos >> 3] |= (uint8_t)(1u << (*pos & 7));
+// Append the low nbits (<= 64) of v at bit *pos of the 128-bit record (w1:w0).
+__device__ __forceinline__ void put_bits(uint64_t* w0, uint64_t* w1, int* pos, uint64_t v, int nbits) {
+  if (nbits == 0) return;
+  v &= nbits >= 64 ? ~0ull : ((1ull << nbits) - 1ull);
+  const int p = *pos;
+  if (p >= 64) {
+    *w1 |= v << (p - 64);
+  } else {
+    *w0 |= v << p;
+    if (p + nbits > 64) *w1 |= v >> (64 - p);
+  }
+  *pos += nbits;
 }
 
 __global__ void pack_kernel(const uint64_t* __restrict__ keys, const awsrc_candidate* __restrict__ cands,
@@ -248,20 +281,17 @@ __global__ void pack_kernel(const uint64_t* __restrict__ keys, const awsrc_candi
     atomicAdd(reinterpret_cast<unsigned long long*>(&sw->K[lo]), 1ull);
   }
   const awsrc_candidate cd = cands[tile];
-  uint8_t rec[32];
-#pragma unroll
-  for (int k = 0; k < 32; ++k) rec[k] = 0;
+  uint64_t w0 = 0, w1 = 0;
   int pos = 0;
-  put_bits(rec, &pos, (uint64_t)tile, ceil_log2_dev((uint64_t)a.T));
-  put_bits(rec, &pos, cd.seed, ceil_log2_dev((uint64_t)pr.S));
+  put_bits(&w0, &w1, &pos, (uint64_t)tile, ceil_log2_dev((uint64_t)a.T));
+  put_bits(&w0, &w1, &pos, cd.seed, ceil_log2_dev((uint64_t)pr.S));
   uint64_t sf;
   if (pr.scale_mode == AWSRC_SCALE_POW2) sf = (uint64_t)(int64_t)(cd.scale - pr.e_bias);
   else sf = (uint16_t)cd.scale;
-  put_bits(rec, &pos, sf & ((1ull << pr.b_e) - 1ull), pr.b_e);
-  for (int p = 0; p < pr.P; ++p)
-    put_bits(rec, &pos, (uint64_t)(int64_t)cd.code[p] & ((1ull << pr.b) - 1ull), pr.b);
+  put_bits(&w0, &w1, &pos, sf, pr.b_e);
+  for (int p = 0; p < pr.P; ++p) put_bits(&w0, &w1, &pos, (uint64_t)(int64_t)cd.code[p], pr.b);
   uint8_t* dst = stream + a.h + i * a.L;
-  for (int k = 0; k < a.L; ++k) dst[k] = rec[k];
+  for (int k = 0; k < a.L; ++k) dst[k] = (uint8_t)(k < 8 ? (w0 >> (8 * k)) : (w1 >> (8 * (k - 8))));
 }
 
 __device__ __forceinline__ void put_le(uint8_t* p, uint64_t v, int n) {
@@ -354,7 +384,7 @@ awsrc_status select_run(const Prm& pr, const SelectPlan& sp, const int64_t* tile
     }
     if (cudaGetLastError() != cudaSuccess) return check_launch("select: sort");
   }
-  cut_kernel<<<1, 32, 0, st>>>(ka, a, sw, d_counts, d_bytes);
+  cut_kernel<<<1, 256, 0, st>>>(ka, a, sw, d_counts, d_bytes);
   note_launches(1);
   if (sp.cap_records > 0)
     pack_kernel<<<(unsigned)((sp.cap_records + 127) / 128), 128, 0, st>>>(ka, cands, a, pr, sw,
