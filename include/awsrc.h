@@ -45,8 +45,12 @@
  *  Weights. r_j = W - W0 (after exact widening to f32); U: d_j = a_j; PF:
  *   d_j = w_act*a_j + w_fisher*F_ij; y_j = d_j * r_j. A tile is invalid (gain
  *   -inf) unless every r_j is finite with |r_j| <= 2^16 and every d_j is in [0, 2^32].
- *  Fit (Eq. 3). c = RN(C^-1/2), c2 = 1/C. u_p = sum_j m_p(j)*y_j (u = fma(m, y, u));
- *   b_p = c*u_p. gd = c2 * sum_j d_j; G_pp = gd; G_pq = c2 * sum_j m_p(j)m_q(j) d_j.
+ *  Fit (Eq. 3). c = RN(C^-1/2), c2 = 1/C. The +-1 correlations are exact
+ *   integer sums on a per-tile fixed-point grid: for a vector x (y or d) let
+ *   q = ilogb(max_j |x_j|) - 20 and X_j = rint(x_j*2^-q), so |X_j| <= 2^21 (x is
+ *   all zero, q = 0, when max |x| < 2^-100). Then u_p = 2^qy * RN(sum_j m_p(j) Y_j)
+ *   and b_p = c*u_p; gd = c2 * 2^qd * RN(sum_j D_j); G_pp = gd;
+ *   G_pq = c2 * 2^qd * RN(sum_j m_p(j)m_q(j) D_j) (each sum exact, rounded once).
  *   eps = ridge_rel*gd; A = G + eps*I. LDL^T, k = 0..P-1: for j < k:
  *   v = A_kj, v = fma(-L_ki, E_ji, v) for i < j, E_kj = v, L_kj = v*invD_j;
  *   D_k = A_kk, D_k = fma(-L_ki, E_ki, D_k) for i < k; the candidate is invalid

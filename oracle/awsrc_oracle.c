@@ -183,6 +183,23 @@ static void orc_exp_range(const orc_params* prm, int* lo, int* hi) {
   if (*hi > 126) *hi = 126;
 }
 
+/* Per-tile fixed point: q = ilogb(max |x_j|) - 20 so that max |x| 2^-q lies in
+ * [2^20, 2^21), and X_j = rint(x_j 2^-q) (exact scaling, one rounding), so
+ * |X_j| <= 2^21. A vector whose largest magnitude is below 2^-100 is all zero
+ * (q = 0). Returns q. */
+int orc_fixed_point(int C, const float* x, int32_t* X) {
+  float m = 0.0f;
+  for (int j = 0; j < C; ++j)
+    if (fabsf(x[j]) > m) m = fabsf(x[j]);
+  if (!(m >= 0x1p-100f)) {
+    for (int j = 0; j < C; ++j) X[j] = 0;
+    return 0;
+  }
+  int q = ilogbf(m) - 20;
+  for (int j = 0; j < C; ++j) X[j] = (int32_t)rintf(ldexpf(x[j], -q));
+  return q;
+}
+
 int orc_tile_valid(int C, const float* r, const float* d) {
   for (int j = 0; j < C; ++j) {
     if (!(fabsf(r[j]) <= 65536.0f)) return 0;                  /* also rejects NaN */
@@ -201,24 +218,33 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
   float y[256];
   for (int j = 0; j < C; ++j) y[j] = d[j] * r[j];
 
+  /* Correlations of Eq. 3 on a per-tile fixed-point grid: y and d become
+   * integers Y = rint(y 2^-qy), D = rint(d 2^-qd) with at most 21 bits, their
+   * +-1 correlations are summed exactly (integers) and rounded once. */
+  int32_t Y[256], Dq[256];
+  int qy = orc_fixed_point(C, y, Y);
+  int qd = orc_fixed_point(C, d, Dq);
+
   /* right-hand side b = B_s^T D r  (Eq. 3 normal equations) */
   float bvec[ORC_MAXP];
   for (int p = 0; p < P; ++p) {
-    float u = 0.0f;
-    for (int j = 0; j < C; ++j) u = u + (negmask[p * C + j] ? -y[j] : y[j]);
+    int64_t su = 0;
+    for (int j = 0; j < C; ++j) su += negmask[p * C + j] ? -(int64_t)Y[j] : (int64_t)Y[j];
+    float u = ldexpf((float)su, qy);
     bvec[p] = c * u;
   }
   /* Gram G = B_s^T D B_s */
   float G[ORC_MAXP][ORC_MAXP];
-  float wsum = 0.0f;
-  for (int j = 0; j < C; ++j) wsum = wsum + d[j];
-  float gd = c2 * wsum;
+  int64_t sd = 0;
+  for (int j = 0; j < C; ++j) sd += Dq[j];
+  float gd = c2 * ldexpf((float)sd, qd);
   for (int p = 0; p < P; ++p) {
     G[p][p] = gd;
     for (int q = p + 1; q < P; ++q) {
-      float v = 0.0f;
-      for (int j = 0; j < C; ++j) v = v + ((negmask[p * C + j] ^ negmask[q * C + j]) ? -d[j] : d[j]);
-      G[p][q] = G[q][p] = c2 * v;
+      int64_t sv = 0;
+      for (int j = 0; j < C; ++j)
+        sv += (negmask[p * C + j] ^ negmask[q * C + j]) ? -(int64_t)Dq[j] : (int64_t)Dq[j];
+      G[p][q] = G[q][p] = c2 * ldexpf((float)sv, qd);
     }
   }
   /* ridge (Eq. 3): A = G + eps I */

@@ -74,6 +74,8 @@ def lib():
             L.orc_f16_to_f32.argtypes = [ct.c_uint16]
             L.orc_f32_to_bf16.restype = ct.c_uint16
             L.orc_f32_to_bf16.argtypes = [ct.c_float]
+            L.orc_fixed_point.restype = ct.c_int
+            L.orc_fixed_point.argtypes = [ct.c_int, vp, vp]
             L.orc_tile_valid.restype = ct.c_int
             L.orc_tile_valid.argtypes = [ct.c_int, vp, vp]
             L.orc_score_candidate.restype = ct.c_int
@@ -172,6 +174,14 @@ def score_candidate(prm: Params, r, d, negmask):
         return None
     return {"gain": float(g[0]), "scale": int(sf[0]), "codes": codes[: prm.P].astype(np.int64),
             "alpha": alpha[: prm.P].copy()}
+
+
+def fixed_point(x):
+    """Per-tile fixed point of the correlations: returns (q, X) with X = rint(x 2^-q)."""
+    x = np.ascontiguousarray(x, np.float32)
+    X = np.zeros(len(x), np.int32)
+    q = lib().orc_fixed_point(len(x), _ptr(x), _ptr(X))
+    return int(q), X
 
 
 def tile_valid(r, d) -> bool:

@@ -78,7 +78,7 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   L.gram = off;
   if (pr.variant == AWSRC_VARIANT_U) off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
   L.mexp = off;
-  if (L.spec) off += align_up((size_t)pr.S_pad * 64 * 4 * 4, 256);
+  if (L.spec) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
   L.partials = off;
   off += align_up((size_t)L.nsplit * T * 8, 256);
   L.total = off;
@@ -229,14 +229,14 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   uint32_t* status = reinterpret_cast<uint32_t*>(ws);
   uint64_t* masks = reinterpret_cast<uint64_t*>(ws + lay.masks);
   float* gram = reinterpret_cast<float*>(ws + lay.gram);
-  float* mexp = reinterpret_cast<float*>(ws + lay.mexp);
+  void* mexp = ws + lay.mexp;
   float2* partials = reinterpret_cast<float2*>(ws + lay.partials);
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
   if (e != cudaSuccess) return cuda_fail(e, "encode: clear status");
   e = launch_gen_basis(pr, masks, pr.S_pad, st);
   if (e != cudaSuccess) return cuda_fail(e, "encode: gen_basis");
-  if (lay.spec && (e = launch_expand_masks_c64p4(pr, masks, mexp, st)) != cudaSuccess)
-    return cuda_fail(e, "encode: expand masks");
+  if (lay.spec && (e = launch_bfrag_c64p4(pr, masks, mexp, st)) != cudaSuccess)
+    return cuda_fail(e, "encode: atom fragments");
   const int rb = lay.spec ? search_c64p4_rows() : generic_rows();
   int64_t tile_off = 0, gram_off = 0;
   for (int g0 = 0; g0 < n_mod; g0 += kMaxModsPerLaunch) {

@@ -31,34 +31,4 @@ cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStre
   return cudaGetLastError();
 }
 
-// Expand the bit masks of C = 64, P = 4 into +-1.0f in the layout the
-// specialised search streams into shared memory with one bulk copy per chunk:
-// out[((chunk*64 + j)*CH + sl)*4 + p], seed = chunk*CH + sl.
-__global__ void expand_masks_c64p4_kernel(const uint64_t* __restrict__ masks, float* __restrict__ out,
-                                          int S_pad, int CH) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;  // one float4 (4 atoms)
-  const int64_t n = (int64_t)S_pad * 64;
-  if (i >= n) return;
-  const int sl = (int)(i % CH);
-  const int j = (int)((i / CH) % 64);
-  const int chunk = (int)(i / (CH * 64));
-  const int s = chunk * CH + sl;
-  float4 v;
-  v.x = sign_f(masks[(size_t)s * 4 + 0] >> j);
-  v.y = sign_f(masks[(size_t)s * 4 + 1] >> j);
-  v.z = sign_f(masks[(size_t)s * 4 + 2] >> j);
-  v.w = sign_f(masks[(size_t)s * 4 + 3] >> j);
-  reinterpret_cast<float4*>(out)[i] = v;
-}
-
-cudaError_t launch_expand_masks_c64p4(const Prm& pr, const uint64_t* masks, float* out,
-                                      cudaStream_t st) {
-  const int64_t n = (int64_t)pr.S_pad * 64;
-  const int tpb = 256;
-  expand_masks_c64p4_kernel<<<(unsigned)((n + tpb - 1) / tpb), tpb, 0, st>>>(
-      masks, out, pr.S_pad, search_c64p4_chunk());
-  note_launches(1);
-  return cudaGetLastError();
-}
-
 }  // namespace awsrc

@@ -70,6 +70,28 @@ __device__ __forceinline__ float load_elem(const void* p, int64_t i, int dtype) 
   return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
 }
 
+// Per-tile fixed point of the correlations: for m = max_j |x_j| >= 2^-100,
+// q = ilogb(m) - 20, and x_j is represented by X_j = rint(x_j * 2^-q), |X_j| <= 2^21.
+// Smaller (or NaN) m: the vector counts as zero (q = 0). Returns 2^-q, or 0 for a
+// zero vector; *q receives q.
+__device__ __forceinline__ float fixed_point_inv(float m, int* q) {
+  if (!(m >= 0x1p-100f)) {
+    *q = 0;
+    return 0.0f;
+  }
+  const int e = (int)((__float_as_uint(m) >> 23) & 0xffu) - 127;  // m is normal here
+  const int qq = min(e, 126) - 20;
+  *q = qq;
+  return __int_as_float((127 - qq) << 23);
+}
+
+__device__ __forceinline__ float pow2f(int q) { return __int_as_float((127 + q) << 23); }
+
+// X = rint(x * inv), exact scaling then round half to even.
+__device__ __forceinline__ int fixed_point_int(float x, float inv) {
+  return __float2int_rn(__fmul_rn(x, inv));
+}
+
 // Tile-domain check: |r| <= 2^16 and 0 <= d <= 2^32 (NaN fails both).
 __device__ __forceinline__ bool in_domain(float r, float d) {
   return (fabsf(r) <= 65536.0f) && (d >= 0.0f) && (d <= 4294967296.0f);

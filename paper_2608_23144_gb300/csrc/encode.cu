@@ -36,7 +36,10 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   const ModDesc& md = ld.m[mi];
   const int C = pr.C;
   __shared__ float d[kMaxC];
+  __shared__ int Dq[kMaxC];
   __shared__ int dok;
+  __shared__ float dmax;
+  __shared__ float two_qd;
   if (threadIdx.x == 0) dok = 1;
   __syncthreads();
   for (int j = threadIdx.x; j < C; j += blockDim.x) {
@@ -45,25 +48,39 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     if (!(v >= 0.0f && v <= 4294967296.0f)) dok = 0;
   }
   __syncthreads();
+  if (threadIdx.x == 0) {
+    float m = 0.0f;
+    for (int j = 0; j < C; ++j) m = fmaxf(m, fabsf(d[j]));
+    dmax = m;
+  }
+  __syncthreads();
+  int qd;
+  const float inv = fixed_point_inv(dmax, &qd);
+  for (int j = threadIdx.x; j < C; j += blockDim.x) Dq[j] = inv == 0.0f ? 0 : fixed_point_int(d[j], inv);
+  if (threadIdx.x == 0) two_qd = pow2f(qd);
+  __syncthreads();
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s >= pr.S_pad) return;
   constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
-  float w = 0.0f;
-  for (int j = 0; j < C; ++j) w = __fadd_rn(w, d[j]);
-  const float gd = __fmul_rn(pr.c2, w);
+  int sd = 0;
+  for (int j = 0; j < C; ++j) sd += Dq[j];
+  const float gd = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(sd), two_qd));
   float Goff[NL], L[NL], invD[P];
   const uint64_t* mk = masks + (size_t)s * P * pr.W;
 #pragma unroll
   for (int q = 1; q < P; ++q) {
 #pragma unroll
     for (int p = 0; p < q; ++p) {
-      float v = 0.0f;
+      int v = 0;
       for (int wd = 0; wd < pr.W; ++wd) {
         const uint64_t x = mk[p * pr.W + wd] ^ mk[q * pr.W + wd];
         const int jn = min(64, C - 64 * wd);
-        for (int jj = 0; jj < jn; ++jj) v = __fmaf_rn(sign_f(x >> jj), d[64 * wd + jj], v);
+        for (int jj = 0; jj < jn; ++jj) {
+          const int dj = Dq[64 * wd + jj];
+          v += ((x >> jj) & 1ull) ? -dj : dj;
+        }
       }
-      Goff[tri(q, p)] = __fmul_rn(pr.c2, v);
+      Goff[tri(q, p)] = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(v), two_qd));
     }
   }
   const float eps = __fmul_rn(pr.ridge_rel, gd);
@@ -94,42 +111,42 @@ __device__ __forceinline__ void tile_elem(const Prm& pr, const ModDesc& md, int6
   *y = __fmul_rn(dv, r);
 }
 
-// Score of seed s for one tile given its staged y (and d, gd for PF).
+// Score of seed s for one tile from its fixed-point Y (and D for PF): the +-1
+// correlations are exact integer sums, rounded once and scaled by 2^q.
 template <int P, int VAR, bool ALLOW_FAST = true>
-__device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const float* d,
-                                            float gd_row, const uint64_t* __restrict__ masks,
-                                            const float* __restrict__ gram_cb, uint32_t s,
-                                            float* q, int* sf) {
+__device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const int* Di, float two_qy,
+                                            float two_qd, float gd_row, const uint64_t* __restrict__ masks,
+                                            const float* __restrict__ gram_cb, uint32_t s, float* q,
+                                            int* sf) {
   constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
   const uint64_t* mk = masks + (size_t)s * P * pr.W;
-  float u[P];
+  int u[P];
 #pragma unroll
-  for (int p = 0; p < P; ++p) u[p] = 0.0f;
-  float v[NL];
+  for (int p = 0; p < P; ++p) u[p] = 0;
+  int v[NL];
 #pragma unroll
-  for (int i = 0; i < NL; ++i) v[i] = 0.0f;
+  for (int i = 0; i < NL; ++i) v[i] = 0;
   for (int wd = 0; wd < pr.W; ++wd) {
     uint64_t m[P];
 #pragma unroll
     for (int p = 0; p < P; ++p) m[p] = mk[p * pr.W + wd];
     const int jn = min(64, pr.C - 64 * wd);
     for (int jj = 0; jj < jn; ++jj) {
-      const float yj = y[64 * wd + jj];
+      const int yj = Yi[64 * wd + jj];
 #pragma unroll
-      for (int p = 0; p < P; ++p) u[p] = __fmaf_rn(sign_f(m[p] >> jj), yj, u[p]);
+      for (int p = 0; p < P; ++p) u[p] += ((m[p] >> jj) & 1ull) ? -yj : yj;
       if (VAR == AWSRC_VARIANT_PF) {
-        const float dj = d[64 * wd + jj];
+        const int dj = Di[64 * wd + jj];
 #pragma unroll
         for (int qq = 1; qq < P; ++qq)
 #pragma unroll
-          for (int p = 0; p < qq; ++p)
-            v[tri(qq, p)] = __fmaf_rn(sign_f((m[p] ^ m[qq]) >> jj), dj, v[tri(qq, p)]);
+          for (int p = 0; p < qq; ++p) v[tri(qq, p)] += (((m[p] ^ m[qq]) >> jj) & 1ull) ? -dj : dj;
       }
     }
   }
   float bv[P], alpha[P];
 #pragma unroll
-  for (int p = 0; p < P; ++p) bv[p] = __fmul_rn(pr.c, u[p]);
+  for (int p = 0; p < P; ++p) bv[p] = __fmul_rn(pr.c, __fmul_rn(__int2float_rn(u[p]), two_qy));
   if (VAR == AWSRC_VARIANT_U) {
     const float* gt = gram_cb + (size_t)s * gram_stride(P);
     float L[NL], invD[P], Goff[NL];
@@ -150,7 +167,7 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const
   } else {
     float Goff[NL], L[NL], invD[P];
 #pragma unroll
-    for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(pr.c2, v[i]);
+    for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(v[i]), two_qd));
     const float eps = __fmul_rn(pr.ridge_rel, gd_row);
     const bool ok = ldl_factor<P>(gd_row, eps, Goff, L, invD);
     ldl_solve<P>(L, invD, bv, alpha);
@@ -164,6 +181,25 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const float* y, const
     }
     return ok ? g : neg_inf();
   }
+}
+
+// Turn a staged row of C floats (y or d) into its fixed-point integers in place
+// (one thread per row); returns 2^q. The integer array aliases the floats.
+__device__ __forceinline__ float row_to_fixed(float* x, int C) {
+  float m = 0.0f;
+  for (int j = 0; j < C; ++j) m = fmaxf(m, fabsf(x[j]));
+  int q;
+  const float inv = fixed_point_inv(m, &q);
+  int* X = reinterpret_cast<int*>(x);
+  for (int j = 0; j < C; ++j) X[j] = inv == 0.0f ? 0 : fixed_point_int(x[j], inv);
+  return pow2f(q);
+}
+
+// gd = c2 * 2^qd * RN(sum_j D_j) for a row of fixed-point D.
+__device__ __forceinline__ float row_gd(const Prm& pr, const int* D, float two_qd) {
+  int sd = 0;
+  for (int j = 0; j < pr.C; ++j) sd += D[j];
+  return __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(sd), two_qd));
 }
 
 // Seed range of split z in units of `chunk` seeds.
@@ -208,10 +244,13 @@ __global__ void __launch_bounds__(kGenThreads) search_generic_kernel(
     if (VAR == AWSRC_VARIANT_PF) ds[r * ldc + j] = d;
   }
   __syncthreads();
-  if (VAR == AWSRC_VARIANT_PF && tid < kGenRows) {
-    float w = 0.0f;
-    for (int j = 0; j < C; ++j) w = __fadd_rn(w, ds[tid * ldc + j]);
-    gds[tid] = __fmul_rn(pr.c2, w);
+  __shared__ float tqy[kGenRows], tqd[kGenRows];
+  if (tid < kGenRows) {
+    tqy[tid] = row_to_fixed(ys + tid * ldc, C);
+    if (VAR == AWSRC_VARIANT_PF) {
+      tqd[tid] = row_to_fixed(ds + tid * ldc, C);
+      gds[tid] = row_gd(pr, reinterpret_cast<const int*>(ds + tid * ldc), tqd[tid]);
+    }
   }
   __syncthreads();
   const int r = tid / kGenLanes, sl = tid % kGenLanes;
@@ -227,7 +266,9 @@ __global__ void __launch_bounds__(kGenThreads) search_generic_kernel(
     for (int s = s0 + sl; s < s1; s += kGenLanes) {
       float q[P];
       int sf;
-      const float g = score_seed<P, VAR>(pr, ys + r * ldc, ds + r * ldc,
+      const float g = score_seed<P, VAR>(pr, reinterpret_cast<const int*>(ys + r * ldc),
+                                         reinterpret_cast<const int*>(ds + r * ldc), tqy[r],
+                                         VAR == AWSRC_VARIANT_PF ? tqd[r] : 0.0f,
                                          VAR == AWSRC_VARIANT_PF ? gds[r] : 0.0f, masks, gram_cb,
                                          (uint32_t)s, q, &sf);
       if (better(g, (uint32_t)s, bg, bs)) { bg = g; bs = (uint32_t)s; }
@@ -374,11 +415,11 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
   for (int p = 0; p < 8; ++p) cd.code[p] = 0;
   if (bg > neg_inf() && bs < (uint32_t)pr.S) {
     const bool ok = tok[tid] != 0;
-    float gd_row = 0.0f;
+    const float two_qy = row_to_fixed(ys + tid * ldc, C);
+    float two_qd = 0.0f, gd_row = 0.0f;
     if (VAR == AWSRC_VARIANT_PF) {
-      float w = 0.0f;
-      for (int j = 0; j < C; ++j) w = __fadd_rn(w, ds[tid * ldc + j]);
-      gd_row = __fmul_rn(pr.c2, w);
+      two_qd = row_to_fixed(ds + tid * ldc, C);
+      gd_row = row_gd(pr, reinterpret_cast<const int*>(ds + tid * ldc), two_qd);
     }
     const float* gram_cb = (VAR == AWSRC_VARIANT_U)
                                ? gram + (size_t)(md.gram_off + cb * pr.S_pad) * gram_stride(P)
@@ -387,8 +428,9 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
     int sf = 0;
     // the general quantiser here, so the self-check also compares it with the
     // fast path the search used
-    const float g = score_seed<P, VAR, false>(pr, ys + tid * ldc, ds + tid * ldc, gd_row, masks,
-                                              gram_cb, bs, q, &sf);
+    const float g = score_seed<P, VAR, false>(pr, reinterpret_cast<const int*>(ys + tid * ldc),
+                                              reinterpret_cast<const int*>(ds + tid * ldc), two_qy, two_qd,
+                                              gd_row, masks, gram_cb, bs, q, &sf);
     if (!ok || __float_as_uint(g) != __float_as_uint(bg)) atomicOr(status, kFaultSelfCheck);
     if (ok && g > neg_inf()) {
       cd.gain = g;

@@ -25,9 +25,7 @@ void note_launches(int n);
 
 // masks[(s*P + p)*W + w] for s in [0, S_pad); seeds >= S get zero masks.
 cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st);
-// Expanded +-1.0f masks for the C=64, P=4 search: [chunk][j][seed_in_chunk][p].
-cudaError_t launch_expand_masks_c64p4(const Prm& pr, const uint64_t* masks, float* out,
-                                      cudaStream_t st);
+
 
 // encode.cu
 cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
@@ -39,7 +37,10 @@ cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t*
                             const float* gram, const float2* partials, int nsplit_max,
                             awsrc_candidate* out, uint32_t* status, cudaStream_t st);
 // search_c64p4.cu
-cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const float* mexp,
+// FP16 B-fragment table of the +-1 atoms, then the tensor-core search.
+size_t search_c64p4_table_bytes(int S_pad);
+cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
+cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
                                 const float* gram, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st);
 int search_c64p4_rows();   // rows per block of the specialised kernel

@@ -1,21 +1,26 @@
-// search_c64p4.cu — seed search (Sec. 3.2) specialised for C = 64, P = 4, AWSRC-U.
+// search_c64p4.cu — seed search (Sec. 3.2) specialised for C = 64, P = 4, AWSRC-U,
+// with the correlation on the tensor cores.
 //
-// The correlation b = B_s^T D r of Eq. 3 for a block of 128 rows (tiles of one
-// column block) and a chunk of 32 seeds is a 128 x 64 by 64 x 128 product whose
-// right operand is +-1. It runs on the FP32 pipe: each thread owns an 8-row x
-// 2-seed x 4-atom register tile and accumulates over j = 0..63 in ascending
-// order with one FFMA per term (m*y is exact, so FFMA rounds like the canonical
-// sum). The fused epilogue solves with the precomputed LDL^T of the (cb, s)
-// Gram matrix, quantises and scores every candidate in registers and keeps a
-// running argmax per row; a 16-lane shuffle reduction finishes the seeds.
+// The correlation u = B_s^T (D r) of Eq. 3 is an exact integer sum on the
+// tile's fixed-point grid: Y_j = rint(y_j 2^-q) with |Y_j| <= 2^21, split as
+// Y = 2048*Y_hi + Y_lo with Y_hi in [-1024, 1024] and Y_lo in [0, 2047]. Both
+// halves and the +-1 atoms are exact in FP16, every product is exact, and every
+// partial sum of 64 terms is an integer below 2^17, so FP32 accumulation on the
+// tensor cores (mma.sync m16n8k16) is exact in any order. The epilogue forms
+// u = 2^q * RN(2048*S_hi + S_lo) — the correctly rounded exact sum, one rounding.
 //
-// Data movement: the residual tile block is staged once per block (plain loads,
-// y = d*r written j-major to shared memory). The +-1.0f atoms (32 KB per chunk)
-// and the chunk's 32 Gram entries (2.5 KB) are streamed by bulk TMA copies
-// (cp.async.bulk) into two shared-memory buffers completed by mbarrier
-// transaction counts, so the next chunk lands while the current one computes.
-// Every mbarrier wait is bounded in time; on expiry the block records a
-// timeout fault, drains its own copies (again bounded) and returns.
+// Block: 128 rows (tiles of one column block) x 32 seeds per chunk, 8 warps;
+// warp w owns rows 16w..16w+15 and keeps their A fragments (both halves, K = 64)
+// in registers for the whole seed loop. Per group of 4 seeds the warp issues 16
+// MMAs (2 halves x 4 k-steps x 2 column tiles); the column order puts atoms
+// p0,p1 of seed t in tile 0 and p2,p3 in tile 1, so lane (g, t) holds all four
+// correlations of candidates (row g, seed t) and (row g+8, seed t) and runs the
+// fused epilogue (solve with the (cb, s) LDL^T, quantise, score, running argmax)
+// on them directly. B fragments (16 KB per chunk, pre-arranged in fragment order)
+// and the chunk's Gram entries (2.5 KB) are streamed by bulk TMA copies into two
+// shared-memory buffers completed by mbarrier transaction counts. Every mbarrier
+// wait is bounded in time; on expiry the block records a timeout fault, drains its
+// own copies (again bounded) and returns.
 #include "internal.h"
 
 namespace awsrc {
@@ -26,16 +31,18 @@ constexpr int BM = 128;   // rows (tiles) per block
 constexpr int CH = 32;    // seeds per chunk
 constexpr int NT = 256;   // threads
 constexpr int GS = gram_stride(4);  // 20 floats per (cb, s) entry
-constexpr uint32_t kMsBytes = 64u * CH * 4u * 4u;  // 32 KB
-constexpr uint32_t kGsBytes = CH * GS * 4u;        // 2560 B
-constexpr uint64_t kWaitNs = 2000000000ull;        // 2 s per wait
+constexpr uint32_t kBBytes = (CH / 4) * 4 * 32 * 16;  // 16 KB of B fragments per chunk
+constexpr uint32_t kGsBytes = CH * GS * 4u;            // 2560 B
+constexpr uint64_t kWaitNs = 2000000000ull;            // 2 s per wait
 
 struct Smem {
-  float Ys[64][BM];
-  float Ms[2][64][CH * 4];
+  float Yst[BM][65];
+  float two_q[BM];
+  float inv_q[BM];
+  int rowok[BM];
+  uint4 Bf[2][CH / 4][4][32];
   float Gs[2][CH * GS];
   unsigned long long mbar[2];
-  int rowok[BM];
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -89,16 +96,29 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+__device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Two FP16 halves (exact small integers) packed low-first.
+__device__ __forceinline__ uint32_t pack_h2(int lo, int hi) {
+  return (uint32_t)__half_as_ushort(__int2half_rn(lo)) | ((uint32_t)__half_as_ushort(__int2half_rn(hi)) << 16);
+}
+
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
 template <bool FAST>
 __global__ void __launch_bounds__(NT, 2)
-    search_c64p4_kernel(Prm pr, LaunchDesc ld, const float* __restrict__ mexp,
+    search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ bfrag,
                         const float* __restrict__ gram, float2* __restrict__ partials,
                         uint32_t* __restrict__ status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int mi = find_mod(ld, blockIdx.x);
   const ModDesc& md = ld.m[mi];
   const int64_t b = blockIdx.x - md.block_off;
@@ -113,7 +133,7 @@ __global__ void __launch_bounds__(NT, 2)
   const int c0 = min(nchunks, z * per);
   const int c1 = min(nchunks, c0 + per);
   const int nck = c1 - c0;
-  const float* ms_src = mexp + (size_t)c0 * (64 * CH * 4);
+  const uint4* bf_src = bfrag + (size_t)c0 * (kBBytes / 16);
   const float* gs_src = gram + (size_t)(md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) * GS;
 
   if (tid == 0) {
@@ -125,14 +145,14 @@ __global__ void __launch_bounds__(NT, 2)
   __syncthreads();
   if (tid == 0) {
     for (int k = 0; k < 2 && k < nck; ++k) {
-      mbar_expect_tx(&sm.mbar[k], kMsBytes + kGsBytes);
-      bulk_g2s(&sm.Ms[k][0][0], ms_src + (size_t)k * (64 * CH * 4), kMsBytes, &sm.mbar[k]);
+      mbar_expect_tx(&sm.mbar[k], kBBytes + kGsBytes);
+      bulk_g2s(&sm.Bf[k][0][0][0], bf_src + (size_t)k * (kBBytes / 16), kBBytes, &sm.mbar[k]);
       bulk_g2s(&sm.Gs[k][0], gs_src + (size_t)k * CH * GS, kGsBytes, &sm.mbar[k]);
     }
   }
-  // stage y = d * (W - W0), j-major; consecutive threads take consecutive rows
+  // stage y = d * (W - W0): consecutive threads take consecutive columns of a row
   for (int e = tid; e < BM * 64; e += NT) {
-    const int r = e % BM, j = e / BM;
+    const int r = e >> 6, j = e & 63;
     const int64_t row = rb * BM + r;
     float y = 0.0f;
     if (row < md.rows) {
@@ -142,51 +162,76 @@ __global__ void __launch_bounds__(NT, 2)
       if (!in_domain(rr, d)) sm.rowok[r] = 0;
       y = __fmul_rn(d, rr);
     }
-    sm.Ys[j][r] = y;
+    sm.Yst[r][j] = y;
+  }
+  __syncthreads();
+  if (tid < BM) {  // the row's fixed-point exponent
+    float m = 0.0f;
+    for (int j = 0; j < 64; ++j) m = fmaxf(m, fabsf(sm.Yst[tid][j]));
+    int q;
+    const float inv = fixed_point_inv(m, &q);
+    sm.inv_q[tid] = sm.rowok[tid] ? inv : 0.0f;
+    sm.two_q[tid] = pow2f(q);
   }
   __syncthreads();
 
-  const int ty = tid >> 4;  // rows ty*8 .. ty*8+7
-  const int tx = tid & 15;  // seeds tx and tx+16 of the chunk
-  const float c = pr.c;
-  float bg[8];
-  uint32_t bs[8];
+  // A fragments of the warp's 16 rows: Y split into hi (a_h) and lo (a_l) halves
+  const int g = lane >> 2, t = lane & 3;
+  const int R0 = warp * 16 + g, R1 = R0 + 8;
+  uint32_t a_h[4][4], a_l[4][4];
+  {
+    const float i0 = sm.inv_q[R0], i1 = sm.inv_q[R1];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) { bg[i] = neg_inf(); bs[i] = 0xffffffffu; }
+    for (int ks = 0; ks < 4; ++ks) {
+#pragma unroll
+      for (int reg = 0; reg < 4; ++reg) {
+        const int row = (reg & 1) ? R1 : R0;
+        const float inv = (reg & 1) ? i1 : i0;
+        const int k = 16 * ks + 2 * t + ((reg & 2) ? 8 : 0);
+        const int y0 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[row][k], inv);
+        const int y1 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[row][k + 1], inv);
+        a_h[ks][reg] = pack_h2(y0 >> 11, y1 >> 11);
+        a_l[ks][reg] = pack_h2(y0 & 2047, y1 & 2047);
+      }
+    }
+  }
+  const float tq0 = sm.two_q[R0], tq1 = sm.two_q[R1];
+  const float c = pr.c;
+  float bg[2] = {neg_inf(), neg_inf()};
+  uint32_t bs[2] = {0xffffffffu, 0xffffffffu};
 
-  // Seeds reach a thread in increasing order (chunk by chunk, tx before tx+16),
-  // so within a thread a strictly greater gain is the whole tie rule.
+  // Seeds reach a lane in increasing order (chunk by chunk, group by group), so
+  // within a lane a strictly greater gain is the whole tie rule.
   bool timed_out = false;
   for (int k = 0; k < nck; ++k) {
     const int buf = k & 1;
     const bool ok = mbar_wait(&sm.mbar[buf], (uint32_t)((k >> 1) & 1));
     if (!ok) timed_out = true;
-
     if (!timed_out) {
-      float acc[8][8];
+#pragma unroll 1
+      for (int grp = 0; grp < CH / 4; ++grp) {
+        uint32_t bb[4][4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
+        for (int ks = 0; ks < 4; ++ks) {
+          const uint4 v = sm.Bf[buf][grp][ks][lane];
+          bb[ks][0] = v.x; bb[ks][1] = v.y; bb[ks][2] = v.z; bb[ks][3] = v.w;
+        }
+        float acc[2][2][4];  // [half][column tile][fragment]
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[i][q] = 0.0f;
-      const float* ysb = &sm.Ys[0][ty * 8];
-      const float* msb = &sm.Ms[buf][0][0];
-#pragma unroll 4
-      for (int j = 0; j < 64; ++j) {
-        const float4 ya = *reinterpret_cast<const float4*>(ysb + j * BM);
-        const float4 yb = *reinterpret_cast<const float4*>(ysb + j * BM + 4);
-        const float4 ma = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + tx * 4);
-        const float4 mb = *reinterpret_cast<const float4*>(msb + j * (CH * 4) + (tx + 16) * 4);
-        const float yv[8] = {ya.x, ya.y, ya.z, ya.w, yb.x, yb.y, yb.z, yb.w};
-        const float mv[8] = {ma.x, ma.y, ma.z, ma.w, mb.x, mb.y, mb.z, mb.w};
+        for (int h = 0; h < 2; ++h)
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
+          for (int n = 0; n < 2; ++n)
 #pragma unroll
-          for (int q = 0; q < 8; ++q) acc[i][q] = __fmaf_rn(mv[q], yv[i], acc[i][q]);
-      }
-      // fused epilogue: solve, quantise, score, running argmax
+            for (int i = 0; i < 4; ++i) acc[h][n][i] = 0.0f;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int sl = tx + 16 * h;
+        for (int ks = 0; ks < 4; ++ks) {
+          mma16816(acc[0][0], a_h[ks], bb[ks][0], bb[ks][1]);
+          mma16816(acc[0][1], a_h[ks], bb[ks][2], bb[ks][3]);
+          mma16816(acc[1][0], a_l[ks], bb[ks][0], bb[ks][1]);
+          mma16816(acc[1][1], a_l[ks], bb[ks][2], bb[ks][3]);
+        }
+        // epilogue: candidates (R0, seed t) and (R1, seed t) of this group
+        const int sl = 4 * grp + t;
         const uint32_t s = (uint32_t)((c0 + k) * CH + sl);
         const float* gt = &sm.Gs[buf][sl * GS];
         const float4 g0 = *reinterpret_cast<const float4*>(gt);
@@ -202,15 +247,22 @@ __global__ void __launch_bounds__(NT, 2)
           for (int i = 0; i < 6; ++i) Gq[i] = __fmul_rn(2.0f, Gq[i]);  // exact
         }
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int rr = 0; rr < 2; ++rr) {
+          const float tq = rr ? tq1 : tq0;
           float bv[4], alpha[4], q[4];
 #pragma unroll
-          for (int p = 0; p < 4; ++p) bv[p] = __fmul_rn(c, acc[i][h * 4 + p]);
+          for (int p = 0; p < 4; ++p) {
+            // atoms p0, p1 sit in column tile 0, p2, p3 in tile 1; fragment
+            // elements 0,1 are row R0 and 2,3 row R1
+            const int n = p >> 1, e = 2 * rr + (p & 1);
+            const float u = __fmul_rn(__fadd_rn(__fmul_rn(2048.0f, acc[0][n][e]), acc[1][n][e]), tq);
+            bv[p] = __fmul_rn(c, u);
+          }
           ldl_solve<4>(L, invD, bv, alpha);
           int sf;
-          const float g = FAST ? quant_gain_fast<4>(pr, alpha, bv, gd, Gq, q, &sf)
-                               : quant_gain<4>(pr, alpha, bv, gd, Gq, q, &sf);
-          if (g > bg[i]) { bg[i] = g; bs[i] = s; }
+          const float gn = FAST ? quant_gain_fast<4>(pr, alpha, bv, gd, Gq, q, &sf)
+                                : quant_gain<4>(pr, alpha, bv, gd, Gq, q, &sf);
+          if (gn > bg[rr]) { bg[rr] = gn; bs[rr] = s; }
         }
       }
     }
@@ -218,8 +270,8 @@ __global__ void __launch_bounds__(NT, 2)
     if (__syncthreads_or(timed_out)) { timed_out = true; break; }
     if (tid == 0 && k + 2 < nck) {
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_expect_tx(&sm.mbar[buf], kMsBytes + kGsBytes);
-      bulk_g2s(&sm.Ms[buf][0][0], ms_src + (size_t)(k + 2) * (64 * CH * 4), kMsBytes, &sm.mbar[buf]);
+      mbar_expect_tx(&sm.mbar[buf], kBBytes + kGsBytes);
+      bulk_g2s(&sm.Bf[buf][0][0][0], bf_src + (size_t)(k + 2) * (kBBytes / 16), kBBytes, &sm.mbar[buf]);
       bulk_g2s(&sm.Gs[buf][0], gs_src + (size_t)(k + 2) * CH * GS, kGsBytes, &sm.mbar[buf]);
     }
   }
@@ -232,43 +284,77 @@ __global__ void __launch_bounds__(NT, 2)
     __syncthreads();
     return;
   }
-  // reduce the running argmax over the 16 threads (tx) that share rows
+  // reduce the running argmax over the 4 lanes (t) that share rows R0, R1
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
+  for (int rr = 0; rr < 2; ++rr) {
 #pragma unroll
-    for (int off = 1; off < 16; off <<= 1) {
-      const float og = __shfl_xor_sync(0xffffffffu, bg[i], off);
-      const uint32_t os = __shfl_xor_sync(0xffffffffu, bs[i], off);
-      if (better(og, os, bg[i], bs[i])) { bg[i] = og; bs[i] = os; }
+    for (int off = 1; off < 4; off <<= 1) {
+      const float og = __shfl_xor_sync(0xffffffffu, bg[rr], off);
+      const uint32_t os = __shfl_xor_sync(0xffffffffu, bs[rr], off);
+      if (better(og, os, bg[rr], bs[rr])) { bg[rr] = og; bs[rr] = os; }
     }
   }
-  if (tx == 0) {
+  if (t == 0) {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int r = ty * 8 + i;
+    for (int rr = 0; rr < 2; ++rr) {
+      const int r = rr ? R1 : R0;
       const int64_t row = rb * BM + r;
       if (row < md.rows) {
-        const int64_t t = md.tile_off + row * md.n_cb + cb;
-        partials[(size_t)z * ld.T + t] =
-            make_float2(sm.rowok[r] ? bg[i] : neg_inf(), __uint_as_float(bs[i]));
+        const int64_t tt = md.tile_off + row * md.n_cb + cb;
+        partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[r] ? bg[rr] : neg_inf(), __uint_as_float(bs[rr]));
       }
     }
   }
+}
+
+// B fragments of the +-1 atoms in the order the kernel reads them:
+// out[((chunk*8 + grp)*4 + ks)*32 + lane] = {b0, b1 of column tile 0, b0, b1 of
+// tile 1} for k-step ks, where lane = 4g + t holds column g (seed 4*grp + g/2,
+// atom 2*tile + g%2) at rows k = 16ks + 2t (+1) and 16ks + 2t + 8 (+9).
+__global__ void bfrag_kernel(const uint64_t* __restrict__ masks, uint4* __restrict__ out, int S_pad) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t n = (int64_t)S_pad / 4 * 4 * 32;
+  if (i >= n) return;
+  const int ln = (int)(i & 31), ks = (int)((i >> 5) & 3);
+  const int64_t grp = i >> 7;  // global group of 4 seeds
+  const int g = ln >> 2, t = ln & 3;
+  const int64_t seed = grp * 4 + (g >> 1);
+  uint32_t w[4];
+#pragma unroll
+  for (int tile = 0; tile < 2; ++tile) {
+    const uint64_t m = masks[(size_t)seed * 4 + 2 * tile + (g & 1)];
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int k = 16 * ks + 2 * t + 8 * half;
+      const uint32_t lo = ((m >> k) & 1ull) ? 0xBC00u : 0x3C00u;       // -1 : +1 in FP16
+      const uint32_t hi = ((m >> (k + 1)) & 1ull) ? 0xBC00u : 0x3C00u;
+      w[2 * tile + half] = lo | (hi << 16);
+    }
+  }
+  out[i] = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 }  // namespace
 
 int search_c64p4_rows() { return BM; }
 int search_c64p4_chunk() { return CH; }
+size_t search_c64p4_table_bytes(int S_pad) { return (size_t)S_pad * 4 * 32 * 16 / 4; }
 
-cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const float* mexp,
+cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st) {
+  const int64_t n = (int64_t)pr.S_pad / 4 * 4 * 32;
+  bfrag_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(masks, static_cast<uint4*>(out), pr.S_pad);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
                                 const float* gram, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st) {
   const size_t smem = sizeof(Smem);
   auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, mexp, gram, partials, status);
+  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), gram, partials, status);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -139,3 +139,42 @@ def test_quantised_gain_never_exceeds_ls_optimum(orc):
         g_ls = bv @ np.linalg.solve(G, bv)
         g_q = orc.def_gain(C, P, r, d, neg, out["codes"], orc.scale_value(prm, out["scale"]))
         assert g_q <= g_ls * (1 + 1e-9)
+
+
+def test_fixed_point_grid(orc):
+    """q = ilogb(max|x|) - 20 and X = rint(x 2^-q) (numpy: frexp/ldexp/rint, half to even)."""
+    rng = np.random.default_rng(8)
+    for trial in range(200):
+        scale = 10.0 ** rng.uniform(-30, 10)
+        x = (rng.normal(0, 1, 64) * scale).astype(np.float32)
+        if trial % 7 == 0:
+            x[rng.integers(64)] = 0.0
+        q, X = orc.fixed_point(x)
+        m = np.abs(x).max()
+        e = np.frexp(np.float64(m))[1] - 1          # ilogb
+        assert q == e - 20
+        want = np.rint(np.ldexp(x.astype(np.float64), -q))
+        assert np.array_equal(X, want.astype(np.int32))
+        assert np.abs(X).max() <= 2 ** 21 and np.abs(X).max() >= 2 ** 20
+    assert orc.fixed_point(np.zeros(16, np.float32))[0] == 0
+    q, X = orc.fixed_point(np.full(16, 1e-35, np.float32))      # below 2^-100: all zero
+    assert q == 0 and not X.any()
+
+
+def test_correlation_is_the_rounded_exact_sum(orc):
+    """u_p = 2^q * RN(sum_j m_p(j) Y_j): recomputed here with exact Python integers,
+    and within (C/2 + 1) 2^q of the real correlation sum_j m_p(j) y_j."""
+    rng = np.random.default_rng(9)
+    C, P = 64, 4
+    prm = orc.params(C=C, P=P, ridge_rel=0.0)
+    for s in range(30):
+        r = rng.normal(0, 1e-3, C).astype(np.float32)
+        neg = orc.gen_basis(0, s, C, P, 1)[3]
+        out = orc.score_candidate(prm, r, np.ones(C, np.float32), neg)  # d = 1: G = I, alpha = b
+        q, Y = orc.fixed_point(r)
+        for p in range(P):
+            exact = sum(int(-Y[j]) if neg[p, j] else int(Y[j]) for j in range(C))
+            u = np.float32(np.ldexp(np.float32(exact), q))             # float32() rounds once
+            assert out["alpha"][p] == np.float32(np.float32(1 / 8) * u)
+            real = float(np.sum(np.where(neg[p] == 1, -1.0, 1.0) * r.astype(np.float64)))
+            assert abs(float(u) - real) <= (C / 2 + 1) * 2.0 ** q
