@@ -52,7 +52,7 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
 }
 
 struct EncodeLayout {
-  size_t masks, gram, mexp, partials, total;
+  size_t masks, gram, pairs, mexp, partials, total;
   int nsplit;
   bool spec;
 };
@@ -77,6 +77,8 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   off += align_up((size_t)pr.S_pad * pr.P * pr.W * 8, 256);
   L.gram = off;
   if (pr.variant == AWSRC_VARIANT_U) off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
+  L.pairs = off;
+  if (L.spec) off += align_up((size_t)ncb * pr.S_pad * pair_stride(pr.P) * 8, 256);
   L.mexp = off;
   if (L.spec) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
   L.partials = off;
@@ -229,6 +231,7 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   uint32_t* status = reinterpret_cast<uint32_t*>(ws);
   uint64_t* masks = reinterpret_cast<uint64_t*>(ws + lay.masks);
   float* gram = reinterpret_cast<float*>(ws + lay.gram);
+  float2* pairs = lay.spec ? reinterpret_cast<float2*>(ws + lay.pairs) : nullptr;
   void* mexp = ws + lay.mexp;
   float2* partials = reinterpret_cast<float2*>(ws + lay.partials);
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
@@ -261,11 +264,11 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
       tile_off += d.rows * d.n_cb;
       gram_off += d.n_cb * pr.S_pad;
     }
-    if (pr.variant == AWSRC_VARIANT_U && (e = launch_gram_u(pr, ld, masks, gram, st)) != cudaSuccess)
+    if (pr.variant == AWSRC_VARIANT_U && (e = launch_gram_u(pr, ld, masks, gram, pairs, st)) != cudaSuccess)
       return cuda_fail(e, "encode: gram");
     if (g0 == 0 && g_ev_before && (e = cudaEventRecord(g_ev_before, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
-    if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, gram, blocks, partials, status, st);
+    if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, pairs, blocks, partials, status, st);
     else e = launch_search_generic(pr, ld, masks, gram, blocks, partials, st);
     if (e != cudaSuccess) return cuda_fail(e, "encode: search");
     if (g0 + kMaxModsPerLaunch >= n_mod && g_ev_after && (e = cudaEventRecord(g_ev_after, st)) != cudaSuccess)

@@ -106,6 +106,13 @@ __host__ __device__ constexpr int gram_stride(int P) {
   return ((P * (P - 1) + P + 1) + 3) / 4 * 4;
 }
 
+// float2 entries per (column block, seed) of the paired table the C = 64, P = 4
+// search streams: -L, invD, G off-diagonal (2*G_pq on the fast power-of-two
+// path), gd, each duplicated into both components, padded to an even count.
+__host__ __device__ constexpr int pair_stride(int P) {
+  return ((P * (P - 1) + P + 1) + 1) / 2 * 2;
+}
+
 // LDL^T of A = G + eps I with G_pp = gd, G_pq = Goff[tri(q, p)]. Writes L and
 // invD; returns false if some pivot is not in (0, FLT_MAX].
 template <int P>
@@ -246,6 +253,80 @@ __device__ __forceinline__ float quant_gain_fast(const Prm& pr, const float* alp
   const float t = __fmul_rn(sc, Qq);
   const float g = __fmul_rn(sc, __fmaf_rn(2.0f, Aq, -t));
   return ok ? g : -__int_as_float(0x7f800000);
+}
+
+// ------------------------------------------------------- paired epilogue --
+// The same solve and power-of-two quantiser for two candidates at once, one per
+// component of a float2, on the packed binary32 instructions of sm_100-class
+// GPUs (__ffma2_rn, __fmul2_rn, __fadd2_rn round each component exactly like
+// their scalar forms). nL holds -L (exact), so every step is one packed fma.
+template <int P>
+__device__ __forceinline__ void ldl_solve2(const float2* nL, const float2* invD, const float2* bv,
+                                           float2* alpha) {
+  float2 z[P];
+#pragma unroll
+  for (int k = 0; k < P; ++k) {
+    float2 v = bv[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) v = __ffma2_rn(nL[tri(k, i)], z[i], v);
+    z[k] = v;
+  }
+#pragma unroll
+  for (int k = P - 1; k >= 0; --k) {
+    float2 v = __fmul2_rn(z[k], invD[k]);
+#pragma unroll
+    for (int i = k + 1; i < P; ++i) v = __ffma2_rn(nL[tri(i, k)], alpha[i], v);
+    alpha[k] = v;
+  }
+}
+
+// Exponent of one candidate for quant_gain_fast2: scale bits, or 0 when amax is
+// outside [2^-100, 2^32] (NaN and inf included).
+__device__ __forceinline__ uint32_t fast_scale_bits(const Prm& pr, float amax) {
+  const uint32_t ab = __float_as_uint(amax);
+  const bool ok = (ab - 0x0D800000u) <= (0x4F800000u - 0x0D800000u);
+  const uint32_t sc_bits = (ab & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23) +
+                           (((ab & 0x007FFFFFu) > pr.mant_q) ? 0x00800000u : 0u);
+  return ok ? sc_bits : 0u;
+}
+
+// quant_gain_fast on two candidates. Each code is RN(alpha*2^-e + 1.5*2^23) -
+// 1.5*2^23 with the product fused: alpha*2^-e is exact whenever it can reach
+// a rounding boundary, so this is the code of the scalar form. -t is formed as
+// (-sc)*Qq, the exact negation of sc*Qq.
+template <int P>
+__device__ __forceinline__ float2 quant_gain_fast2(const Prm& pr, const float2* alpha, const float2* bv,
+                                                   float2 gd, const float2* Goff2) {
+  float m0 = fabsf(alpha[0].x), m1 = fabsf(alpha[0].y);
+#pragma unroll
+  for (int p = 1; p < P; ++p) {
+    m0 = fmax_nan(m0, fabsf(alpha[p].x));
+    m1 = fmax_nan(m1, fabsf(alpha[p].y));
+  }
+  const uint32_t s0 = fast_scale_bits(pr, m0), s1 = fast_scale_bits(pr, m1);
+  const float2 sc = make_float2(__uint_as_float(s0), __uint_as_float(s1));
+  const float2 nsc = make_float2(__uint_as_float(s0 | 0x80000000u), __uint_as_float(s1 | 0x80000000u));
+  const float2 inv = make_float2(__uint_as_float(0x7F000000u - s0), __uint_as_float(0x7F000000u - s1));
+  const float2 magic = make_float2(12582912.0f, 12582912.0f);
+  const float2 nmagic = make_float2(-12582912.0f, -12582912.0f);
+  float2 q[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) q[p] = __fadd2_rn(__ffma2_rn(alpha[p], inv, magic), nmagic);
+  float2 Aq = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int p = 0; p < P; ++p) Aq = __ffma2_rn(q[p], bv[p], Aq);
+  float2 Qq = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    Qq = __ffma2_rn(__fmul2_rn(q[p], q[p]), gd, Qq);
+#pragma unroll
+    for (int r = p + 1; r < P; ++r) Qq = __ffma2_rn(__fmul2_rn(q[p], q[r]), Goff2[tri(r, p)], Qq);
+  }
+  const float2 tn = __fmul2_rn(nsc, Qq);
+  float2 g = __fmul2_rn(sc, __ffma2_rn(make_float2(2.0f, 2.0f), Aq, tn));
+  if (s0 == 0u) g.x = -__int_as_float(0x7f800000);
+  if (s1 == 0u) g.y = -__int_as_float(0x7f800000);
+  return g;
 }
 
 // Candidate comparison of the seed argmax: larger gain wins, equal gains keep

@@ -28,7 +28,8 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 template <int P>
 __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
                                                      const uint64_t* __restrict__ masks,
-                                                     float* __restrict__ gram) {
+                                                     float* __restrict__ gram,
+                                                     float2* __restrict__ pairs) {
   // blockIdx.y enumerates the column blocks of all modules of the launch
   int mi = 0;
   int64_t cb = blockIdx.y;
@@ -95,6 +96,24 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
 #pragma unroll
   for (int i = 0; i < P * (P - 1) / 2; ++i) out[P * (P - 1) / 2 + P + i] = Goff[i];
   out[P * (P - 1) + P] = gd;
+  if (pairs) {
+    float2* po = pairs + (size_t)(md.gram_off + cb * pr.S_pad + s) * pair_stride(P);
+    constexpr int nl = P * (P - 1) / 2;
+#pragma unroll
+    for (int i = 0; i < nl; ++i) po[i] = make_float2(-L[i], -L[i]);
+#pragma unroll
+    for (int k = 0; k < P; ++k) {
+      const float v = ok ? invD[k] : qnan;
+      po[nl + k] = make_float2(v, v);
+    }
+#pragma unroll
+    for (int i = 0; i < nl; ++i) {
+      const float v = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];  // exact
+      po[nl + P + i] = make_float2(v, v);
+    }
+    po[2 * nl + P] = make_float2(gd, gd);
+    for (int i = 2 * nl + P + 1; i < pair_stride(P); ++i) po[i] = make_float2(0.0f, 0.0f);
+  }
 }
 
 // Tile staging shared by search and finalisation: r = W - W0, d, y = d*r.
@@ -445,11 +464,11 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
 
 template <int P>
 cudaError_t launch_gram_p(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, float* gram,
-                          cudaStream_t st) {
+                          float2* pairs, cudaStream_t st) {
   int64_t ncb = 0;
   for (int i = 0; i < ld.n; ++i) ncb += ld.m[i].n_cb;
   dim3 grid((pr.S_pad + 127) / 128, (unsigned)ncb);
-  gram_u_kernel<P><<<grid, 128, 0, st>>>(pr, ld, masks, gram);
+  gram_u_kernel<P><<<grid, 128, 0, st>>>(pr, ld, masks, gram, pairs);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -499,8 +518,8 @@ cudaError_t launch_finalize_pv(const Prm& pr, const LaunchDesc& ld, const uint64
   }
 
 cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, float* gram,
-                          cudaStream_t st) {
-  AWSRC_DISPATCH_P(pr.P, (launch_gram_p<PP>(pr, ld, masks, gram, st)));
+                          float2* pairs, cudaStream_t st) {
+  AWSRC_DISPATCH_P(pr.P, (launch_gram_p<PP>(pr, ld, masks, gram, pairs, st)));
 }
 
 cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,

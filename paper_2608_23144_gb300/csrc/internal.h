@@ -28,8 +28,10 @@ cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStre
 
 
 // encode.cu
+// Writes the Gram table and, when `pairs` is not null, the paired table
+// (pair_stride(P) float2 per entry) the C = 64, P = 4 search reads.
 cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                          float* gram, cudaStream_t st);
+                          float* gram, float2* pairs, cudaStream_t st);
 cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
                                   const float* gram, int64_t n_blocks, float2* partials,
                                   cudaStream_t st);
@@ -41,7 +43,7 @@ cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t*
 size_t search_c64p4_table_bytes(int S_pad);
 cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
-                                const float* gram, int64_t n_blocks, float2* partials,
+                                const float2* pairs, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st);
 int search_c64p4_rows();   // rows per block of the specialised kernel
 int search_c64p4_chunk();  // seeds per chunk of the specialised kernel

@@ -30,9 +30,9 @@ namespace {
 constexpr int BM = 128;   // rows (tiles) per block
 constexpr int CH = 32;    // seeds per chunk
 constexpr int NT = 256;   // threads
-constexpr int GS = gram_stride(4);  // 20 floats per (cb, s) entry
+constexpr int PS = pair_stride(4);  // 18 float2 per (cb, s) entry of the paired table
 constexpr uint32_t kBBytes = (CH / 4) * 4 * 32 * 16;  // 16 KB of B fragments per chunk
-constexpr uint32_t kGsBytes = CH * GS * 4u;            // 2560 B
+constexpr uint32_t kGsBytes = CH * PS * 8u;            // 4608 B
 constexpr uint64_t kWaitNs = 2000000000ull;            // 2 s per wait
 
 struct Smem {
@@ -41,7 +41,7 @@ struct Smem {
   float inv_q[BM];
   int rowok[BM];
   uint4 Bf[2][CH / 4][4][32];
-  float Gs[2][CH * GS];
+  float2 Gp[2][CH * PS];
   unsigned long long mbar[2];
 };
 
@@ -97,7 +97,7 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 }
 
 __device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
@@ -114,7 +114,7 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 template <bool FAST>
 __global__ void __launch_bounds__(NT, 2)
     search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ bfrag,
-                        const float* __restrict__ gram, float2* __restrict__ partials,
+                        const float2* __restrict__ pairs, float2* __restrict__ partials,
                         uint32_t* __restrict__ status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(NT, 2)
   const int c1 = min(nchunks, c0 + per);
   const int nck = c1 - c0;
   const uint4* bf_src = bfrag + (size_t)c0 * (kBBytes / 16);
-  const float* gs_src = gram + (size_t)(md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) * GS;
+  const float2* gs_src = pairs + (size_t)(md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) * PS;
 
   if (tid == 0) {
     mbar_init(&sm.mbar[0], 1);
@@ -147,7 +147,7 @@ __global__ void __launch_bounds__(NT, 2)
     for (int k = 0; k < 2 && k < nck; ++k) {
       mbar_expect_tx(&sm.mbar[k], kBBytes + kGsBytes);
       bulk_g2s(&sm.Bf[k][0][0][0], bf_src + (size_t)k * (kBBytes / 16), kBBytes, &sm.mbar[k]);
-      bulk_g2s(&sm.Gs[k][0], gs_src + (size_t)k * CH * GS, kGsBytes, &sm.mbar[k]);
+      bulk_g2s(&sm.Gp[k][0], gs_src + (size_t)k * CH * PS, kGsBytes, &sm.mbar[k]);
     }
   }
   // stage y = d * (W - W0): consecutive threads take consecutive columns of a row
@@ -195,8 +195,9 @@ __global__ void __launch_bounds__(NT, 2)
       }
     }
   }
-  const float tq0 = sm.two_q[R0], tq1 = sm.two_q[R1];
-  const float c = pr.c;
+  // b = c * 2^q * RN(S) = RN(S) * (2^q c): c = 1/8 and 2^q >= 2^-120 keep every
+  // product exact (normal range), so one multiply per atom gives b.
+  const float2 tqc = make_float2(__fmul_rn(sm.two_q[R0], pr.c), __fmul_rn(sm.two_q[R1], pr.c));
   float bg[2] = {neg_inf(), neg_inf()};
   uint32_t bs[2] = {0xffffffffu, 0xffffffffu};
 
@@ -208,15 +209,14 @@ __global__ void __launch_bounds__(NT, 2)
     const bool ok = mbar_wait(&sm.mbar[buf], (uint32_t)((k >> 1) & 1));
     if (!ok) timed_out = true;
     if (!timed_out) {
-#pragma unroll 1
-      for (int grp = 0; grp < CH / 4; ++grp) {
+      // 16 MMAs of one group of 4 seeds into acc[half][column tile][fragment]
+      auto mma_group = [&](int grp, float (&acc)[2][2][4]) {
         uint32_t bb[4][4];
 #pragma unroll
         for (int ks = 0; ks < 4; ++ks) {
           const uint4 v = sm.Bf[buf][grp][ks][lane];
           bb[ks][0] = v.x; bb[ks][1] = v.y; bb[ks][2] = v.z; bb[ks][3] = v.w;
         }
-        float acc[2][2][4];  // [half][column tile][fragment]
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -230,40 +230,63 @@ __global__ void __launch_bounds__(NT, 2)
           mma16816(acc[1][0], a_l[ks], bb[ks][0], bb[ks][1]);
           mma16816(acc[1][1], a_l[ks], bb[ks][2], bb[ks][3]);
         }
-        // epilogue: candidates (R0, seed t) and (R1, seed t) of this group
+      };
+      auto epilogue = [&](int grp, const float (&acc)[2][2][4]) {
+        // epilogue: candidates (R0, seed t) and (R1, seed t) of this group, one
+        // per float2 component
         const int sl = 4 * grp + t;
         const uint32_t s = (uint32_t)((c0 + k) * CH + sl);
-        const float* gt = &sm.Gs[buf][sl * GS];
-        const float4 g0 = *reinterpret_cast<const float4*>(gt);
-        const float4 g1 = *reinterpret_cast<const float4*>(gt + 4);
-        const float4 g2 = *reinterpret_cast<const float4*>(gt + 8);
-        const float4 g3 = *reinterpret_cast<const float4*>(gt + 12);
-        const float gd = gt[16];
-        const float L[6] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y};
-        const float invD[4] = {g1.z, g1.w, g2.x, g2.y};
-        float Gq[6] = {g2.z, g2.w, g3.x, g3.y, g3.z, g3.w};
+        const float4* pe = reinterpret_cast<const float4*>(&sm.Gp[buf][sl * PS]);
+        float2 pv[PS];
+#pragma unroll
+        for (int i = 0; i < PS / 2; ++i) {
+          const float4 v = pe[i];
+          pv[2 * i] = make_float2(v.x, v.y);
+          pv[2 * i + 1] = make_float2(v.z, v.w);
+        }
+        const float2* nL = pv;          // -L
+        const float2* invD = pv + 6;
+        const float2* Go = pv + 10;     // G off-diagonal (doubled on the fast path)
+        const float2 gd = pv[16];
+        float2 bv[4], alpha[4];
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          // atoms p0, p1 sit in column tile 0, p2, p3 in tile 1; fragment
+          // elements 0,1 are row R0 and 2,3 row R1
+          const int n = p >> 1, e = p & 1;
+          const float2 u = make_float2(__fmaf_rn(2048.0f, acc[0][n][e], acc[1][n][e]),
+                                       __fmaf_rn(2048.0f, acc[0][n][2 + e], acc[1][n][2 + e]));
+          bv[p] = __fmul2_rn(u, tqc);
+        }
+        ldl_solve2<4>(nL, invD, bv, alpha);
+        float2 gn;
         if (FAST) {
+          gn = quant_gain_fast2<4>(pr, alpha, bv, gd, Go);
+        } else {
+          float Gx[6], q[4];
 #pragma unroll
-          for (int i = 0; i < 6; ++i) Gq[i] = __fmul_rn(2.0f, Gq[i]);  // exact
-        }
-#pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          const float tq = rr ? tq1 : tq0;
-          float bv[4], alpha[4], q[4];
-#pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            // atoms p0, p1 sit in column tile 0, p2, p3 in tile 1; fragment
-            // elements 0,1 are row R0 and 2,3 row R1
-            const int n = p >> 1, e = 2 * rr + (p & 1);
-            const float u = __fmul_rn(__fadd_rn(__fmul_rn(2048.0f, acc[0][n][e]), acc[1][n][e]), tq);
-            bv[p] = __fmul_rn(c, u);
-          }
-          ldl_solve<4>(L, invD, bv, alpha);
+          for (int i = 0; i < 6; ++i) Gx[i] = Go[i].x;
           int sf;
-          const float gn = FAST ? quant_gain_fast<4>(pr, alpha, bv, gd, Gq, q, &sf)
-                                : quant_gain<4>(pr, alpha, bv, gd, Gq, q, &sf);
-          if (gn > bg[rr]) { bg[rr] = gn; bs[rr] = s; }
+          float a0[4] = {alpha[0].x, alpha[1].x, alpha[2].x, alpha[3].x};
+          float b0[4] = {bv[0].x, bv[1].x, bv[2].x, bv[3].x};
+          float a1[4] = {alpha[0].y, alpha[1].y, alpha[2].y, alpha[3].y};
+          float b1[4] = {bv[0].y, bv[1].y, bv[2].y, bv[3].y};
+          gn.x = quant_gain<4>(pr, a0, b0, gd.x, Gx, q, &sf);
+          gn.y = quant_gain<4>(pr, a1, b1, gd.x, Gx, q, &sf);
         }
+        if (gn.x > bg[0]) { bg[0] = gn.x; bs[0] = s; }
+        if (gn.y > bg[1]) { bg[1] = gn.y; bs[1] = s; }
+      };
+      // the MMAs of the next group are issued before the epilogue of the current
+      // one, so the tensor pipe and the FP32 pipe overlap within each warp
+      float accA[2][2][4], accB[2][2][4];
+      mma_group(0, accA);
+#pragma unroll 1
+      for (int grp = 0; grp < CH / 4; grp += 2) {
+        mma_group(grp + 1, accB);
+        epilogue(grp, accA);
+        if (grp + 2 < CH / 4) mma_group(grp + 2, accA);
+        epilogue(grp + 1, accB);
       }
     }
     // every thread is done with buffer `buf`; a timeout anywhere ends the block
@@ -272,7 +295,7 @@ __global__ void __launch_bounds__(NT, 2)
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_expect_tx(&sm.mbar[buf], kBBytes + kGsBytes);
       bulk_g2s(&sm.Bf[buf][0][0][0], bf_src + (size_t)(k + 2) * (kBBytes / 16), kBBytes, &sm.mbar[buf]);
-      bulk_g2s(&sm.Gs[buf][0], gs_src + (size_t)(k + 2) * CH * GS, kGsBytes, &sm.mbar[buf]);
+      bulk_g2s(&sm.Gp[buf][0], gs_src + (size_t)(k + 2) * CH * PS, kGsBytes, &sm.mbar[buf]);
     }
   }
   if (timed_out) {
@@ -348,13 +371,13 @@ cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, 
 }
 
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
-                                const float* gram, int64_t n_blocks, float2* partials,
+                                const float2* pairs, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st) {
   const size_t smem = sizeof(Smem);
   auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), gram, partials, status);
+  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), pairs, partials, status);
   note_launches(1);
   return cudaGetLastError();
 }
