@@ -78,7 +78,7 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   L.gram = off;
   if (pr.variant == AWSRC_VARIANT_U) off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
   L.pairs = off;
-  if (L.spec) off += align_up((size_t)ncb * pr.S_pad * pair_stride(pr.P) * 8, 256);
+  if (L.spec) off += align_up((size_t)ncb * (pr.S_pad / 2) * pair_stride(pr.P) * 8, 256);
   L.mexp = off;
   if (L.spec) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
   L.partials = off;

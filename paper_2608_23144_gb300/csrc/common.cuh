@@ -106,9 +106,10 @@ __host__ __device__ constexpr int gram_stride(int P) {
   return ((P * (P - 1) + P + 1) + 3) / 4 * 4;
 }
 
-// float2 entries per (column block, seed) of the paired table the C = 64, P = 4
-// search streams: -L, invD, G off-diagonal (2*G_pq on the fast power-of-two
-// path), gd, each duplicated into both components, padded to an even count.
+// float2 entries per (column block, seed pair) of the paired table the C = 64,
+// P = 4 search streams: -L, invD, G off-diagonal (2*G_pq on the fast
+// power-of-two path), gd, with seed 2i in component x and seed 2i+1 in y,
+// padded to an even count.
 __host__ __device__ constexpr int pair_stride(int P) {
   return ((P * (P - 1) + P + 1) + 1) / 2 * 2;
 }

@@ -97,22 +97,18 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   for (int i = 0; i < P * (P - 1) / 2; ++i) out[P * (P - 1) / 2 + P + i] = Goff[i];
   out[P * (P - 1) + P] = gd;
   if (pairs) {
-    float2* po = pairs + (size_t)(md.gram_off + cb * pr.S_pad + s) * pair_stride(P);
+    // seed s is component s & 1 of seed pair s >> 1 (entries start on even seeds)
+    float* po = reinterpret_cast<float*>(pairs) +
+                (size_t)((md.gram_off + cb * pr.S_pad + s) >> 1) * pair_stride(P) * 2 + (s & 1);
     constexpr int nl = P * (P - 1) / 2;
 #pragma unroll
-    for (int i = 0; i < nl; ++i) po[i] = make_float2(-L[i], -L[i]);
+    for (int i = 0; i < nl; ++i) po[2 * i] = -L[i];
 #pragma unroll
-    for (int k = 0; k < P; ++k) {
-      const float v = ok ? invD[k] : qnan;
-      po[nl + k] = make_float2(v, v);
-    }
+    for (int k = 0; k < P; ++k) po[2 * (nl + k)] = ok ? invD[k] : qnan;
 #pragma unroll
-    for (int i = 0; i < nl; ++i) {
-      const float v = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];  // exact
-      po[nl + P + i] = make_float2(v, v);
-    }
-    po[2 * nl + P] = make_float2(gd, gd);
-    for (int i = 2 * nl + P + 1; i < pair_stride(P); ++i) po[i] = make_float2(0.0f, 0.0f);
+    for (int i = 0; i < nl; ++i) po[2 * (nl + P + i)] = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];
+    po[2 * (2 * nl + P)] = gd;
+    for (int i = 2 * nl + P + 1; i < pair_stride(P); ++i) po[2 * i] = 0.0f;
   }
 }
 

@@ -29,7 +29,7 @@ cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStre
 
 // encode.cu
 // Writes the Gram table and, when `pairs` is not null, the paired table
-// (pair_stride(P) float2 per entry) the C = 64, P = 4 search reads.
+// (pair_stride(P) float2 per seed pair) the C = 64, P = 4 search reads.
 cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
                           float* gram, float2* pairs, cudaStream_t st);
 cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
@@ -39,7 +39,7 @@ cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t*
                             const float* gram, const float2* partials, int nsplit_max,
                             awsrc_candidate* out, uint32_t* status, cudaStream_t st);
 // search_c64p4.cu
-// FP16 B-fragment table of the +-1 atoms, then the tensor-core search.
+// FP16 table of the +-1 atoms in MMA operand order, then the tcgen05 search.
 size_t search_c64p4_table_bytes(int S_pad);
 cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,

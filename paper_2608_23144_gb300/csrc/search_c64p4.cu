@@ -1,48 +1,69 @@
 // search_c64p4.cu — seed search (Sec. 3.2) specialised for C = 64, P = 4, AWSRC-U,
-// with the correlation on the tensor cores.
+// with the correlation on the fifth-generation tensor cores (tcgen05, TMEM).
 //
 // The correlation u = B_s^T (D r) of Eq. 3 is an exact integer sum on the
 // tile's fixed-point grid: Y_j = rint(y_j 2^-q) with |Y_j| <= 2^21, split as
 // Y = 2048*Y_hi + Y_lo with Y_hi in [-1024, 1024] and Y_lo in [0, 2047]. Both
 // halves and the +-1 atoms are exact in FP16, every product is exact, and every
 // partial sum of 64 terms is an integer below 2^17, so FP32 accumulation on the
-// tensor cores (mma.sync m16n8k16) is exact in any order. The epilogue forms
-// u = 2^q * RN(2048*S_hi + S_lo) — the correctly rounded exact sum, one rounding.
+// tensor cores is exact in any order. The epilogue forms
+// b = RN(2048*S_hi + S_lo) * (2^q c) — the correctly rounded exact sum, one
+// rounding, scaled exactly (c = 1/8 and 2^q >= 2^-120 keep the product normal).
 //
-// Block: 128 rows (tiles of one column block) x 32 seeds per chunk, 8 warps;
-// warp w owns rows 16w..16w+15 and keeps their A fragments (both halves, K = 64)
-// in registers for the whole seed loop. Per group of 4 seeds the warp issues 16
-// MMAs (2 halves x 4 k-steps x 2 column tiles); the column order puts atoms
-// p0,p1 of seed t in tile 0 and p2,p3 in tile 1, so lane (g, t) holds all four
-// correlations of candidates (row g, seed t) and (row g+8, seed t) and runs the
-// fused epilogue (solve with the (cb, s) LDL^T, quantise, score, running argmax)
-// on them directly. B fragments (16 KB per chunk, pre-arranged in fragment order)
-// and the chunk's Gram entries (2.5 KB) are streamed by bulk TMA copies into two
-// shared-memory buffers completed by mbarrier transaction counts. Every mbarrier
-// wait is bounded in time; on expiry the block records a timeout fault, drains its
-// own copies (again bounded) and returns.
+// Block: 128 rows (tiles of one column block; row m = TMEM lane m) and 17 warps.
+//  * Warp 16 (producer): one thread streams each chunk of 32 seeds — FP16 atoms
+//    in the canonical K-major layout (16 KB) and the chunk's paired Gram factors
+//    (2.3 KB) — by bulk copies into a 4-stage shared-memory ring, and issues the
+//    chunk's 8 MMAs (M = 128, N = 128, K = 16; halves hi and lo, 4 k-steps) into
+//    one of two 256-column TMEM accumulators, committed to an mbarrier.
+//  * Warps 0..15 (epilogue): warp w reads TMEM lanes 32(w%4).. (its threads'
+//    rows) and the columns of seeds 8(w/4)..8(w/4)+7 of each chunk, and runs the
+//    fit / quantise / score epilogue on seed pairs as float2 streams, keeping a
+//    running argmax per row. The four warps of a row merge at the end.
+// Columns of a chunk are seed-pair major: column 8i + 2p + e holds atom p of
+// seed 2i + e, so one 32x32b.x16 TMEM load gives a thread two seed pairs with
+// each atom's two seeds in adjacent registers.
+// Every mbarrier wait is bounded in time; on expiry the block records a timeout
+// fault, waits (bounded) for its own copies and MMAs in flight, frees its TMEM
+// and returns.
 #include "internal.h"
 
 namespace awsrc {
 
 namespace {
 
-constexpr int BM = 128;   // rows (tiles) per block
-constexpr int CH = 32;    // seeds per chunk
-constexpr int NT = 256;   // threads
-constexpr int PS = pair_stride(4);  // 18 float2 per (cb, s) entry of the paired table
-constexpr uint32_t kBBytes = (CH / 4) * 4 * 32 * 16;  // 16 KB of B fragments per chunk
-constexpr uint32_t kGsBytes = CH * PS * 8u;            // 4608 B
-constexpr uint64_t kWaitNs = 2000000000ull;            // 2 s per wait
+constexpr int BM = 128;             // rows (tiles) per block = TMEM lanes
+constexpr int CH = 32;              // seeds per chunk
+constexpr int NCOL = 4 * CH;        // MMA N: 128 columns per half
+constexpr int EW = 16;              // epilogue warps
+constexpr int NT = 32 * (EW + 1);   // + the producer warp
+constexpr int STAGES = 4;
+constexpr int PS = pair_stride(4);  // 18 float2 per seed pair
+constexpr uint32_t kBBytes = NCOL * 64 * 2;        // 16 KB of FP16 atoms per chunk
+constexpr uint32_t kPBytes = (CH / 2) * PS * 8u;   // 2304 B of paired factors per chunk
+constexpr uint32_t kStageBytes = 19456;            // B at 0, factors at kBBytes (1 KB multiple)
+constexpr uint32_t kTmemCols = 512;                // 2 accumulators x (hi, lo) x 128 columns
+constexpr uint64_t kWaitNs = 2000000000ull;        // 2 s per wait
+static_assert(kBBytes + kPBytes <= kStageBytes, "stage layout");
+
+// MMA instruction descriptor (kind::f16): D FP32 (bits 4-5 = 1), A and B FP16
+// (bits 7-9, 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 at bit 17,
+// M >> 4 at bit 24.
+constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(NCOL >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 struct Smem {
+  __half A[2][BM * 64];                   // Y_hi, Y_lo: canonical K-major, no swizzle
+  unsigned char stage[STAGES][kStageBytes];
   float Yst[BM][65];
   float two_q[BM];
   float inv_q[BM];
   int rowok[BM];
-  uint4 Bf[2][CH / 4][4][32];
-  float2 Gp[2][CH * PS];
-  unsigned long long mbar[2];
+  float red_g[4][BM];
+  uint32_t red_s[4][BM];
+  unsigned long long full[STAGES];        // bulk copies of a chunk landed
+  unsigned long long afull[2];            // MMAs of a chunk completed (tcgen05.commit)
+  unsigned long long aempty[2];           // epilogue warps done with an accumulator
+  uint32_t tmem_base;
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -63,6 +84,10 @@ __device__ __forceinline__ void mbar_expect_tx(unsigned long long* mb, uint32_t 
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(mb)),
                "r"(bytes)
                : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(unsigned long long* mb) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(mb)) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(unsigned long long* mb, uint32_t parity) {
@@ -96,28 +121,117 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-__device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+// Shared-memory matrix descriptor, canonical K-major layout without swizzle:
+// 8x16-byte core matrices, 128 B apart along K (leading byte offset) and
+// 1024 B apart along M/N (stride byte offset); bit 46 = descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)(128u >> 4) << 16) |
+         ((uint64_t)(1024u >> 4) << 32) | (1ull << 46);
 }
 
-// Two FP16 halves (exact small integers) packed low-first.
-__device__ __forceinline__ uint32_t pack_h2(int lo, int hi) {
-  return (uint32_t)__half_as_ushort(__int2half_rn(lo)) | ((uint32_t)__half_as_ushort(__int2half_rn(hi)) << 16);
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(unsigned long long* mb) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_addr(mb))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// 16 consecutive 32-bit TMEM columns of the warp's 32 lanes (one lane per thread).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
+// Byte offset of element (m, k) of a 128x64 FP16 operand in the canonical
+// K-major no-swizzle layout: core matrix (m/8, k/8) at ((m/8)*8 + k/8)*128.
+__device__ __forceinline__ int a_offset(int m, int k) {
+  return (((m >> 3) * 8 + (k >> 3)) << 7) + ((m & 7) << 4) + ((k & 7) << 1);
+}
+
+// Gains of one seed pair for this thread's row: hi/lo hold atom p of the two
+// seeds at [2p], [2p+1]; pe points at the pair's 18 float2 factors.
 template <bool FAST>
-__global__ void __launch_bounds__(NT, 2)
-    search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ bfrag,
+__device__ __forceinline__ float2 pair_gain(const Prm& pr, const float* hi, const float* lo, float2 tqc,
+                                            const float4* pe) {
+  float2 pv[PS];
+#pragma unroll
+  for (int i = 0; i < PS / 2; ++i) {
+    const float4 v = pe[i];
+    pv[2 * i] = make_float2(v.x, v.y);
+    pv[2 * i + 1] = make_float2(v.z, v.w);
+  }
+  const float2* nL = pv;       // -L
+  const float2* invD = pv + 6;
+  const float2* Go = pv + 10;  // G off-diagonal (doubled on the fast path)
+  const float2 gd = pv[16];
+  float2 bv[4], alpha[4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const float2 u = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
+                                make_float2(lo[2 * p], lo[2 * p + 1]));
+    bv[p] = __fmul2_rn(u, tqc);
+  }
+  ldl_solve2<4>(nL, invD, bv, alpha);
+  if constexpr (FAST) return quant_gain_fast2<4>(pr, alpha, bv, gd, Go);
+  float2 g;
+  float q[4];
+  int sf;
+  {
+    float G[6], a[4], b[4];
+#pragma unroll
+    for (int i = 0; i < 6; ++i) G[i] = Go[i].x;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].x; b[p] = bv[p].x; }
+    g.x = quant_gain<4>(pr, a, b, gd.x, G, q, &sf);
+  }
+  {
+    float G[6], a[4], b[4];
+#pragma unroll
+    for (int i = 0; i < 6; ++i) G[i] = Go[i].y;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].y; b[p] = bv[p].y; }
+    g.y = quant_gain<4>(pr, a, b, gd.y, G, q, &sf);
+  }
+  return g;
+}
+
+template <bool FAST>
+__global__ void __launch_bounds__(NT, 1)
+    search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ atoms,
                         const float2* __restrict__ pairs, float2* __restrict__ partials,
                         uint32_t* __restrict__ status) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  extern __shared__ unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int mi = find_mod(ld, blockIdx.x);
   const ModDesc& md = ld.m[mi];
@@ -133,21 +247,38 @@ __global__ void __launch_bounds__(NT, 2)
   const int c0 = min(nchunks, z * per);
   const int c1 = min(nchunks, c0 + per);
   const int nck = c1 - c0;
-  const uint4* bf_src = bfrag + (size_t)c0 * (kBBytes / 16);
-  const float2* gs_src = pairs + (size_t)(md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) * PS;
+  const unsigned char* at_src = reinterpret_cast<const unsigned char*>(atoms) + (size_t)c0 * kBBytes;
+  const unsigned char* pf_src =
+      reinterpret_cast<const unsigned char*>(pairs) +
+      (size_t)((md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) / 2) * PS * 8;
 
-  if (tid == 0) {
-    mbar_init(&sm.mbar[0], 1);
-    mbar_init(&sm.mbar[1], 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (warp == EW) {  // the producer warp owns the TMEM allocation
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_addr(&sm.tmem_base)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if (lane == 0) {
+      for (int i = 0; i < STAGES; ++i) mbar_init(&sm.full[i], 1);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&sm.afull[i], 1);
+        mbar_init(&sm.aempty[i], EW);
+      }
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    tc_fence_before();
   }
   if (tid < BM) sm.rowok[tid] = 1;
   __syncthreads();
-  if (tid == 0) {
-    for (int k = 0; k < 2 && k < nck; ++k) {
-      mbar_expect_tx(&sm.mbar[k], kBBytes + kGsBytes);
-      bulk_g2s(&sm.Bf[k][0][0][0], bf_src + (size_t)k * (kBBytes / 16), kBBytes, &sm.mbar[k]);
-      bulk_g2s(&sm.Gp[k][0], gs_src + (size_t)k * CH * PS, kGsBytes, &sm.mbar[k]);
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  int issued = 0;  // chunks whose copies the producer issued
+  if (warp == EW && lane == 0) {
+    for (; issued < STAGES && issued < nck; ++issued) {
+      mbar_expect_tx(&sm.full[issued], kBBytes + kPBytes);
+      bulk_g2s(&sm.stage[issued][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[issued]);
+      bulk_g2s(&sm.stage[issued][kBBytes], pf_src + (size_t)issued * kPBytes, kPBytes, &sm.full[issued]);
     }
   }
   // stage y = d * (W - W0): consecutive threads take consecutive columns of a row
@@ -174,185 +305,151 @@ __global__ void __launch_bounds__(NT, 2)
     sm.two_q[tid] = pow2f(q);
   }
   __syncthreads();
-
-  // A fragments of the warp's 16 rows: Y split into hi (a_h) and lo (a_l) halves
-  const int g = lane >> 2, t = lane & 3;
-  const int R0 = warp * 16 + g, R1 = R0 + 8;
-  uint32_t a_h[4][4], a_l[4][4];
-  {
-    const float i0 = sm.inv_q[R0], i1 = sm.inv_q[R1];
+  // A operands: one thread writes one 16-byte core-matrix row (8 values of k)
+  // of both halves
+  for (int e = tid; e < BM * 8; e += NT) {
+    const int m = e >> 3, k0 = (e & 7) * 8;
+    const float inv = sm.inv_q[m];
+    uint32_t wh[4], wl[4];
 #pragma unroll
-    for (int ks = 0; ks < 4; ++ks) {
-#pragma unroll
-      for (int reg = 0; reg < 4; ++reg) {
-        const int row = (reg & 1) ? R1 : R0;
-        const float inv = (reg & 1) ? i1 : i0;
-        const int k = 16 * ks + 2 * t + ((reg & 2) ? 8 : 0);
-        const int y0 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[row][k], inv);
-        const int y1 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[row][k + 1], inv);
-        a_h[ks][reg] = pack_h2(y0 >> 11, y1 >> 11);
-        a_l[ks][reg] = pack_h2(y0 & 2047, y1 & 2047);
-      }
+    for (int i = 0; i < 4; ++i) {
+      const int y0 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[m][k0 + 2 * i], inv);
+      const int y1 = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[m][k0 + 2 * i + 1], inv);
+      wh[i] = (uint32_t)__half_as_ushort(__int2half_rn(y0 >> 11)) |
+              ((uint32_t)__half_as_ushort(__int2half_rn(y1 >> 11)) << 16);
+      wl[i] = (uint32_t)__half_as_ushort(__int2half_rn(y0 & 2047)) |
+              ((uint32_t)__half_as_ushort(__int2half_rn(y1 & 2047)) << 16);
     }
+    const int off = a_offset(m, k0);
+    *reinterpret_cast<uint4*>(reinterpret_cast<unsigned char*>(sm.A[0]) + off) =
+        make_uint4(wh[0], wh[1], wh[2], wh[3]);
+    *reinterpret_cast<uint4*>(reinterpret_cast<unsigned char*>(sm.A[1]) + off) =
+        make_uint4(wl[0], wl[1], wl[2], wl[3]);
   }
-  // b = c * 2^q * RN(S) = RN(S) * (2^q c): c = 1/8 and 2^q >= 2^-120 keep every
-  // product exact (normal range), so one multiply per atom gives b.
-  const float2 tqc = make_float2(__fmul_rn(sm.two_q[R0], pr.c), __fmul_rn(sm.two_q[R1], pr.c));
-  float bg[2] = {neg_inf(), neg_inf()};
-  uint32_t bs[2] = {0xffffffffu, 0xffffffffu};
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // A is read by the tensor cores
+  __syncthreads();
 
-  // Seeds reach a lane in increasing order (chunk by chunk, group by group), so
-  // within a lane a strictly greater gain is the whole tie rule.
   bool timed_out = false;
-  for (int k = 0; k < nck; ++k) {
-    const int buf = k & 1;
-    const bool ok = mbar_wait(&sm.mbar[buf], (uint32_t)((k >> 1) & 1));
-    if (!ok) timed_out = true;
-    if (!timed_out) {
-      // 16 MMAs of one group of 4 seeds into acc[half][column tile][fragment]
-      auto mma_group = [&](int grp, float (&acc)[2][2][4]) {
-        uint32_t bb[4][4];
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-          const uint4 v = sm.Bf[buf][grp][ks][lane];
-          bb[ks][0] = v.x; bb[ks][1] = v.y; bb[ks][2] = v.z; bb[ks][3] = v.w;
+  if (warp == EW) {
+    // ------------------------------------------------------------ producer --
+    if (lane == 0) {
+      const uint32_t a0 = smem_addr(sm.A[0]), a1 = smem_addr(sm.A[1]);
+      int k = 0;
+      for (; k < nck; ++k) {
+        const int st = k % STAGES, tb = k & 1;
+        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
+        if (k >= 2) {
+          // the epilogue of chunk k-2 is done: its accumulator and its stage are free
+          if (!mbar_wait(&sm.aempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
+          if (issued < nck) {
+            const int ns = issued % STAGES;
+            mbar_expect_tx(&sm.full[ns], kBBytes + kPBytes);
+            bulk_g2s(&sm.stage[ns][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[ns]);
+            bulk_g2s(&sm.stage[ns][kBBytes], pf_src + (size_t)issued * kPBytes, kPBytes, &sm.full[ns]);
+            ++issued;
+          }
         }
+        tc_fence_after();
+        const uint32_t bsm = smem_addr(&sm.stage[st][0]);
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
+        for (int h = 0; h < 2; ++h) {
 #pragma unroll
-          for (int n = 0; n < 2; ++n)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) acc[h][n][i] = 0.0f;
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-          mma16816(acc[0][0], a_h[ks], bb[ks][0], bb[ks][1]);
-          mma16816(acc[0][1], a_h[ks], bb[ks][2], bb[ks][3]);
-          mma16816(acc[1][0], a_l[ks], bb[ks][0], bb[ks][1]);
-          mma16816(acc[1][1], a_l[ks], bb[ks][2], bb[ks][3]);
+          for (int ks = 0; ks < 4; ++ks) {
+            umma_f16(tmem + (uint32_t)(tb * 256 + h * 128), smem_desc((h ? a1 : a0) + ks * 256),
+                     smem_desc(bsm + ks * 256), ks > 0 ? 1u : 0u);
+          }
         }
-      };
-      auto epilogue = [&](int grp, const float (&acc)[2][2][4]) {
-        // epilogue: candidates (R0, seed t) and (R1, seed t) of this group, one
-        // per float2 component
-        const int sl = 4 * grp + t;
-        const uint32_t s = (uint32_t)((c0 + k) * CH + sl);
-        const float4* pe = reinterpret_cast<const float4*>(&sm.Gp[buf][sl * PS]);
-        float2 pv[PS];
-#pragma unroll
-        for (int i = 0; i < PS / 2; ++i) {
-          const float4 v = pe[i];
-          pv[2 * i] = make_float2(v.x, v.y);
-          pv[2 * i + 1] = make_float2(v.z, v.w);
-        }
-        const float2* nL = pv;          // -L
-        const float2* invD = pv + 6;
-        const float2* Go = pv + 10;     // G off-diagonal (doubled on the fast path)
-        const float2 gd = pv[16];
-        float2 bv[4], alpha[4];
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          // atoms p0, p1 sit in column tile 0, p2, p3 in tile 1; fragment
-          // elements 0,1 are row R0 and 2,3 row R1
-          const int n = p >> 1, e = p & 1;
-          const float2 u = make_float2(__fmaf_rn(2048.0f, acc[0][n][e], acc[1][n][e]),
-                                       __fmaf_rn(2048.0f, acc[0][n][2 + e], acc[1][n][2 + e]));
-          bv[p] = __fmul2_rn(u, tqc);
-        }
-        ldl_solve2<4>(nL, invD, bv, alpha);
-        float2 gn;
-        if (FAST) {
-          gn = quant_gain_fast2<4>(pr, alpha, bv, gd, Go);
-        } else {
-          float Gx[6], q[4];
-#pragma unroll
-          for (int i = 0; i < 6; ++i) Gx[i] = Go[i].x;
-          int sf;
-          float a0[4] = {alpha[0].x, alpha[1].x, alpha[2].x, alpha[3].x};
-          float b0[4] = {bv[0].x, bv[1].x, bv[2].x, bv[3].x};
-          float a1[4] = {alpha[0].y, alpha[1].y, alpha[2].y, alpha[3].y};
-          float b1[4] = {bv[0].y, bv[1].y, bv[2].y, bv[3].y};
-          gn.x = quant_gain<4>(pr, a0, b0, gd.x, Gx, q, &sf);
-          gn.y = quant_gain<4>(pr, a1, b1, gd.x, Gx, q, &sf);
-        }
-        if (gn.x > bg[0]) { bg[0] = gn.x; bs[0] = s; }
-        if (gn.y > bg[1]) { bg[1] = gn.y; bs[1] = s; }
-      };
-      // the MMAs of the next group are issued before the epilogue of the current
-      // one, so the tensor pipe and the FP32 pipe overlap within each warp
-      float accA[2][2][4], accB[2][2][4];
-      mma_group(0, accA);
+        umma_commit(&sm.afull[tb]);
+      }
+      if (timed_out) {
+        // wait (bounded) for this block's copies and MMAs still in flight
+        for (int j = max(0, issued - STAGES); j < issued; ++j)
+          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
+        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue --
+    const int m = 32 * (warp & 3) + lane;  // this thread's row = TMEM lane
+    const int sub = warp >> 2;             // seeds 8*sub .. 8*sub+7 of each chunk
+    const float tq = __fmul_rn(sm.two_q[m], pr.c);
+    const float2 tqc = make_float2(tq, tq);
+    const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
+    float bg = neg_inf();
+    uint32_t bsd = 0xffffffffu;
+    // Seeds reach a thread in increasing order, so a strictly greater gain is
+    // the whole tie rule within a thread.
+    for (int k = 0; k < nck; ++k) {
+      const int st = k % STAGES, tb = k & 1;
+      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1))) { timed_out = true; break; }
+      tc_fence_after();
+      const float4* pbase = reinterpret_cast<const float4*>(&sm.stage[st][kBBytes]);
 #pragma unroll 1
-      for (int grp = 0; grp < CH / 4; grp += 2) {
-        mma_group(grp + 1, accB);
-        epilogue(grp, accA);
-        if (grp + 2 < CH / 4) mma_group(grp + 2, accA);
-        epilogue(grp + 1, accB);
+      for (int rnd = 0; rnd < 2; ++rnd) {
+        const uint32_t col = (uint32_t)(tb * 256 + 32 * sub + 16 * rnd);
+        float hi[16], lo[16];
+        tmem_ld16(tmem + lane_base + col, hi);
+        tmem_ld16(tmem + lane_base + col + 128, lo);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const int ni = 4 * sub + 2 * rnd + j;  // seed pair within the chunk
+          const float2 g = pair_gain<FAST>(pr, hi + 8 * j, lo + 8 * j, tqc, pbase + ni * (PS / 2));
+          const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * ni);
+          if (g.x > bg) { bg = g.x; bsd = s; }
+          if (g.y > bg) { bg = g.y; bsd = s + 1; }
+        }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.aempty[tb]);
     }
-    // every thread is done with buffer `buf`; a timeout anywhere ends the block
-    if (__syncthreads_or(timed_out)) { timed_out = true; break; }
-    if (tid == 0 && k + 2 < nck) {
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_expect_tx(&sm.mbar[buf], kBBytes + kGsBytes);
-      bulk_g2s(&sm.Bf[buf][0][0][0], bf_src + (size_t)(k + 2) * (kBBytes / 16), kBBytes, &sm.mbar[buf]);
-      bulk_g2s(&sm.Gp[buf][0], gs_src + (size_t)(k + 2) * CH * PS, kGsBytes, &sm.mbar[buf]);
+    sm.red_g[sub][m] = bg;
+    sm.red_s[sub][m] = bsd;
+  }
+  tc_fence_before();
+  if (__syncthreads_or(timed_out)) {
+    if (tid == 0) atomicOr(status, kFaultTimeout);
+  } else if (tid < BM) {
+    // merge the four warps of each row (smaller seed on equal gains)
+    float g = sm.red_g[0][tid];
+    uint32_t s = sm.red_s[0][tid];
+#pragma unroll
+    for (int i = 1; i < 4; ++i) {
+      if (better(sm.red_g[i][tid], sm.red_s[i][tid], g, s)) { g = sm.red_g[i][tid]; s = sm.red_s[i][tid]; }
+    }
+    const int64_t row = rb * BM + tid;
+    if (row < md.rows) {
+      const int64_t tt = md.tile_off + row * md.n_cb + cb;
+      partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[tid] ? g : neg_inf(), __uint_as_float(s));
     }
   }
-  if (timed_out) {
-    // drain copies this block issued (bounded), record the fault and leave
-    if (tid == 0) {
-      atomicOr(status, kFaultTimeout);
-      for (int bb = 0; bb < 2; ++bb) (void)mbar_wait(&sm.mbar[bb], 0), (void)mbar_wait(&sm.mbar[bb], 1);
-    }
-    __syncthreads();
-    return;
-  }
-  // reduce the running argmax over the 4 lanes (t) that share rows R0, R1
-#pragma unroll
-  for (int rr = 0; rr < 2; ++rr) {
-#pragma unroll
-    for (int off = 1; off < 4; off <<= 1) {
-      const float og = __shfl_xor_sync(0xffffffffu, bg[rr], off);
-      const uint32_t os = __shfl_xor_sync(0xffffffffu, bs[rr], off);
-      if (better(og, os, bg[rr], bs[rr])) { bg[rr] = og; bs[rr] = os; }
-    }
-  }
-  if (t == 0) {
-#pragma unroll
-    for (int rr = 0; rr < 2; ++rr) {
-      const int r = rr ? R1 : R0;
-      const int64_t row = rb * BM + r;
-      if (row < md.rows) {
-        const int64_t tt = md.tile_off + row * md.n_cb + cb;
-        partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[r] ? bg[rr] : neg_inf(), __uint_as_float(bs[rr]));
-      }
-    }
+  if (warp == EW) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                 : "memory");
   }
 }
 
-// B fragments of the +-1 atoms in the order the kernel reads them:
-// out[((chunk*8 + grp)*4 + ks)*32 + lane] = {b0, b1 of column tile 0, b0, b1 of
-// tile 1} for k-step ks, where lane = 4g + t holds column g (seed 4*grp + g/2,
-// atom 2*tile + g%2) at rows k = 16ks + 2t (+1) and 16ks + 2t + 8 (+9).
-__global__ void bfrag_kernel(const uint64_t* __restrict__ masks, uint4* __restrict__ out, int S_pad) {
+// FP16 atoms in the order the MMAs read them: chunk c (32 seeds) is a 128x64
+// K-major operand in 16 KB; item i (16 bytes = one core-matrix row) is chunk
+// i >> 10, column group n8 = (i >> 6) & 15, k group (i >> 3) & 7, row i & 7,
+// and column 8*n8 + r carries atom r >> 1 of seed 32c + 2*n8 + (r & 1).
+__global__ void atoms_kernel(const uint64_t* __restrict__ masks, uint4* __restrict__ out, int S_pad) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t n = (int64_t)S_pad / 4 * 4 * 32;
+  const int64_t n = (int64_t)S_pad * 32;
   if (i >= n) return;
-  const int ln = (int)(i & 31), ks = (int)((i >> 5) & 3);
-  const int64_t grp = i >> 7;  // global group of 4 seeds
-  const int g = ln >> 2, t = ln & 3;
-  const int64_t seed = grp * 4 + (g >> 1);
+  const int r = (int)(i & 7), kg = (int)((i >> 3) & 7), n8 = (int)((i >> 6) & 15);
+  const int64_t chunk = i >> 10;
+  const int64_t seed = chunk * CH + 2 * n8 + (r & 1);
+  const uint64_t m = masks[(size_t)seed * 4 + (r >> 1)];
   uint32_t w[4];
 #pragma unroll
-  for (int tile = 0; tile < 2; ++tile) {
-    const uint64_t m = masks[(size_t)seed * 4 + 2 * tile + (g & 1)];
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int k = 16 * ks + 2 * t + 8 * half;
-      const uint32_t lo = ((m >> k) & 1ull) ? 0xBC00u : 0x3C00u;       // -1 : +1 in FP16
-      const uint32_t hi = ((m >> (k + 1)) & 1ull) ? 0xBC00u : 0x3C00u;
-      w[2 * tile + half] = lo | (hi << 16);
-    }
+  for (int h = 0; h < 4; ++h) {
+    const int k = 8 * kg + 2 * h;
+    const uint32_t lo = ((m >> k) & 1ull) ? 0xBC00u : 0x3C00u;  // -1 : +1 in FP16
+    const uint32_t hi = ((m >> (k + 1)) & 1ull) ? 0xBC00u : 0x3C00u;
+    w[h] = lo | (hi << 16);
   }
   out[i] = make_uint4(w[0], w[1], w[2], w[3]);
 }
@@ -361,11 +458,11 @@ __global__ void bfrag_kernel(const uint64_t* __restrict__ masks, uint4* __restri
 
 int search_c64p4_rows() { return BM; }
 int search_c64p4_chunk() { return CH; }
-size_t search_c64p4_table_bytes(int S_pad) { return (size_t)S_pad * 4 * 32 * 16 / 4; }
+size_t search_c64p4_table_bytes(int S_pad) { return (size_t)S_pad * 32 * 16; }
 
 cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st) {
-  const int64_t n = (int64_t)pr.S_pad / 4 * 4 * 32;
-  bfrag_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(masks, static_cast<uint4*>(out), pr.S_pad);
+  const int64_t n = (int64_t)pr.S_pad * 32;
+  atoms_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(masks, static_cast<uint4*>(out), pr.S_pad);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -373,7 +470,7 @@ cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, 
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
                                 const float2* pairs, int64_t n_blocks, float2* partials,
                                 uint32_t* status, cudaStream_t st) {
-  const size_t smem = sizeof(Smem);
+  const size_t smem = sizeof(Smem) + 1024;  // + alignment of the operand tiles
   auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
