@@ -108,10 +108,11 @@ __host__ __device__ constexpr int gram_stride(int P) {
 
 // float2 entries per (column block, seed pair) of the paired table the C = 64,
 // P = 4 search streams: -L, invD, G off-diagonal (2*G_pq on the fast
-// power-of-two path), gd, with seed 2i in component x and seed 2i+1 in y,
-// padded to an even count.
+// power-of-two path), gd, zero padding to an odd count, then the seed's
+// pruning-bound multiplier in the last entry; seed 2i in component x and
+// seed 2i+1 in y.
 __host__ __device__ constexpr int pair_stride(int P) {
-  return ((P * (P - 1) + P + 1) + 1) / 2 * 2;
+  return ((P * (P - 1) + P + 2) + 1) / 2 * 2;
 }
 
 // LDL^T of A = G + eps I with G_pp = gd, G_pq = Goff[tri(q, p)]. Writes L and
@@ -281,28 +282,32 @@ __device__ __forceinline__ void ldl_solve2(const float2* nL, const float2* invD,
   }
 }
 
-// Exponent of one candidate for quant_gain_fast2: scale bits, or 0 when amax is
-// outside [2^-100, 2^32] (NaN and inf included).
+// Scale bits 2^e of one candidate for quant_gain_fast2, or 0 when amax is
+// outside [2^-100, 2^32] (inf and NaN patterns included). Adding
+// 0x7FFFFF - mant_q carries into the exponent field exactly when the mantissa
+// field of amax exceeds that of qmax, which is the [f_a > f_qmax] step of
+// quant_gain_fast.
 __device__ __forceinline__ uint32_t fast_scale_bits(const Prm& pr, float amax) {
   const uint32_t ab = __float_as_uint(amax);
   const bool ok = (ab - 0x0D800000u) <= (0x4F800000u - 0x0D800000u);
-  const uint32_t sc_bits = (ab & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23) +
-                           (((ab & 0x007FFFFFu) > pr.mant_q) ? 0x00800000u : 0u);
+  const uint32_t sc_bits = ((ab + (0x007FFFFFu - pr.mant_q)) & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23);
   return ok ? sc_bits : 0u;
 }
 
 // quant_gain_fast on two candidates. Each code is RN(alpha*2^-e + 1.5*2^23) -
 // 1.5*2^23 with the product fused: alpha*2^-e is exact whenever it can reach
 // a rounding boundary, so this is the code of the scalar form. -t is formed as
-// (-sc)*Qq, the exact negation of sc*Qq.
+// (-sc)*Qq, the exact negation of sc*Qq. amax ignores NaN: a candidate with a
+// NaN coefficient but a valid amax gets a NaN gain (its code and Aq are NaN),
+// which no comparison of the seed argmax accepts, just as it accepts no -inf.
 template <int P>
 __device__ __forceinline__ float2 quant_gain_fast2(const Prm& pr, const float2* alpha, const float2* bv,
                                                    float2 gd, const float2* Goff2) {
   float m0 = fabsf(alpha[0].x), m1 = fabsf(alpha[0].y);
 #pragma unroll
   for (int p = 1; p < P; ++p) {
-    m0 = fmax_nan(m0, fabsf(alpha[p].x));
-    m1 = fmax_nan(m1, fabsf(alpha[p].y));
+    m0 = fmaxf(m0, fabsf(alpha[p].x));
+    m1 = fmaxf(m1, fabsf(alpha[p].y));
   }
   const uint32_t s0 = fast_scale_bits(pr, m0), s1 = fast_scale_bits(pr, m1);
   const float2 sc = make_float2(__uint_as_float(s0), __uint_as_float(s1));

@@ -24,6 +24,54 @@ constexpr int kGenThreads = kGenRows * kGenLanes;
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
+// ------------------------------------------------------------- seed bound --
+// Multiplier m of the search's pruning bound for one (column block, seed).
+//
+// For any coefficients x, the Eq. 4 gain 2x^T b - x^T G x is at most
+// U_G = b^T G^-1 b (its maximum over x), so the quantised gain of a candidate
+// can never exceed U_G. The search computes U = b^T alpha with alpha from the
+// ridge solve, i.e. U_eps = b^T (G + eps I)^-1 b up to rounding, and
+// U_G <= (1 + eps/lambda_min) U_eps <= (1 + eps tr(G^-1)) U_eps. With
+// kappa = tr(G) tr(G^-1) >= cond(G + eps I), the binary32 errors of the
+// solve, of b^T alpha and of the gain itself are each below a small multiple
+// of kappa*2^-24 relative to U (plus a few ulps), far inside the factor
+// 1 + 2^-10 + 2^-14 kappa. So a candidate with U * m < g_best cannot score
+// above g_best. m is +inf (no pruning) when G is not positive definite in
+// double precision or kappa > 2^16. Computed in double and rounded up.
+template <int P>
+__device__ float bound_multiplier(float gd, const float* Goff, float eps) {
+  double A[P][P];
+#pragma unroll
+  for (int i = 0; i < P; ++i) {
+    A[i][i] = gd;
+#pragma unroll
+    for (int j = 0; j < i; ++j) A[i][j] = A[j][i] = Goff[tri(i, j)];
+  }
+  // Gauss-Jordan on the symmetric positive definite candidate (no pivoting)
+  double Inv[P][P];
+#pragma unroll
+  for (int i = 0; i < P; ++i)
+#pragma unroll
+    for (int j = 0; j < P; ++j) Inv[i][j] = i == j ? 1.0 : 0.0;
+  for (int k = 0; k < P; ++k) {
+    const double piv = A[k][k];
+    if (!(piv > 0.0)) return __int_as_float(0x7f800000);
+    const double ip = 1.0 / piv;
+    for (int j = 0; j < P; ++j) { A[k][j] *= ip; Inv[k][j] *= ip; }
+    for (int i = 0; i < P; ++i) {
+      if (i == k) continue;
+      const double f = A[i][k];
+      for (int j = 0; j < P; ++j) { A[i][j] -= f * A[k][j]; Inv[i][j] -= f * Inv[k][j]; }
+    }
+  }
+  double tri_inv = 0.0;
+  for (int i = 0; i < P; ++i) tri_inv += Inv[i][i];
+  const double kappa = (double)P * gd * tri_inv;
+  if (!(tri_inv > 0.0) || !(kappa <= 65536.0)) return __int_as_float(0x7f800000);
+  const double m = (1.0 + (double)eps * tri_inv) * (1.0 + 0x1p-10 + 0x1p-14 * kappa);
+  return __double2float_ru(m);
+}
+
 // ----------------------------------------------------------------- gram_u --
 template <int P>
 __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
@@ -108,7 +156,8 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
 #pragma unroll
     for (int i = 0; i < nl; ++i) po[2 * (nl + P + i)] = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];
     po[2 * (2 * nl + P)] = gd;
-    for (int i = 2 * nl + P + 1; i < pair_stride(P); ++i) po[2 * i] = 0.0f;
+    for (int i = 2 * nl + P + 1; i < pair_stride(P) - 1; ++i) po[2 * i] = 0.0f;
+    po[2 * (pair_stride(P) - 1)] = ok ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
   }
 }
 

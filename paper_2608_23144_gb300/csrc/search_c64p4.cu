@@ -37,6 +37,11 @@ constexpr int CH = 32;              // seeds per chunk
 constexpr int NCOL = 4 * CH;        // MMA N: 128 columns per half
 constexpr int EW = 16;              // epilogue warps
 constexpr int NT = 32 * (EW + 1);   // + the producer warp
+constexpr int SUBS = EW / 4;        // epilogue warps per TMEM lane quarter
+constexpr int SUB_PAIRS = CH / 2 / SUBS;  // seed pairs of a chunk per epilogue warp
+constexpr int RPAIRS = 2;           // seed pairs per TMEM load (8 columns each)
+constexpr int ROUNDS = SUB_PAIRS / RPAIRS;
+static_assert(EW % 4 == 0 && SUB_PAIRS % RPAIRS == 0, "epilogue mapping");
 constexpr int STAGES = 4;
 constexpr int PS = pair_stride(4);  // 18 float2 per seed pair
 constexpr uint32_t kBBytes = NCOL * 64 * 2;        // 16 KB of FP16 atoms per chunk
@@ -58,8 +63,8 @@ struct Smem {
   float two_q[BM];
   float inv_q[BM];
   int rowok[BM];
-  float red_g[4][BM];
-  uint32_t red_s[4][BM];
+  float red_g[SUBS][BM];
+  uint32_t red_s[SUBS][BM];
   unsigned long long full[STAGES];        // bulk copies of a chunk landed
   unsigned long long afull[2];            // MMAs of a chunk completed (tcgen05.commit)
   unsigned long long aempty[2];           // epilogue warps done with an accumulator
@@ -166,6 +171,12 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 8 * RPAIRS consecutive columns (RPAIRS seed pairs) in 16-column loads.
+__device__ __forceinline__ void tmem_ld_pairs(uint32_t taddr, float* v) {
+#pragma unroll
+  for (int i = 0; i < RPAIRS / 2; ++i) tmem_ld16(taddr + 16 * i, v + 16 * i);
+}
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -178,51 +189,67 @@ __device__ __forceinline__ int a_offset(int m, int k) {
   return (((m >> 3) * 8 + (k >> 3)) << 7) + ((m & 7) << 4) + ((k & 7) << 1);
 }
 
-// Gains of one seed pair for this thread's row: hi/lo hold atom p of the two
-// seeds at [2p], [2p+1]; pe points at the pair's 18 float2 factors.
-template <bool FAST>
-__device__ __forceinline__ float2 pair_gain(const Prm& pr, const float* hi, const float* lo, float2 tqc,
-                                            const float4* pe) {
-  float2 pv[PS];
+// Fit of one seed pair for this thread's row: hi/lo hold atom p of the two
+// seeds at [2p], [2p+1]; pe points at the pair's 18 float2 factors (9 float4).
+__device__ __forceinline__ void pair_fit(const float* hi, const float* lo, float2 tqc, const float4* pe,
+                                         float2* bv, float2* alpha) {
+  float2 pv[10];
 #pragma unroll
-  for (int i = 0; i < PS / 2; ++i) {
+  for (int i = 0; i < 5; ++i) {
     const float4 v = pe[i];
     pv[2 * i] = make_float2(v.x, v.y);
     pv[2 * i + 1] = make_float2(v.z, v.w);
   }
-  const float2* nL = pv;       // -L
-  const float2* invD = pv + 6;
-  const float2* Go = pv + 10;  // G off-diagonal (doubled on the fast path)
-  const float2 gd = pv[16];
-  float2 bv[4], alpha[4];
 #pragma unroll
   for (int p = 0; p < 4; ++p) {
     const float2 u = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
                                 make_float2(lo[2 * p], lo[2 * p + 1]));
     bv[p] = __fmul2_rn(u, tqc);
   }
-  ldl_solve2<4>(nL, invD, bv, alpha);
-  if constexpr (FAST) return quant_gain_fast2<4>(pr, alpha, bv, gd, Go);
-  float2 g;
-  float q[4];
-  int sf;
-  {
-    float G[6], a[4], b[4];
+  ldl_solve2<4>(pv, pv + 6, bv, alpha);  // -L, invD
+}
+
+// Upper bound on the two candidates' gains: (b^T alpha) * m (see bound_multiplier).
+__device__ __forceinline__ float2 pair_bound(const float2* bv, const float2* alpha, const float4* pe) {
+  float2 U = __fmul2_rn(bv[0], alpha[0]);
+#pragma unroll
+  for (int p = 1; p < 4; ++p) U = __ffma2_rn(bv[p], alpha[p], U);
+  const float4 v = pe[8];
+  return __fmul2_rn(U, make_float2(v.z, v.w));
+}
+
+// Quantised gains of a fitted seed pair.
+template <bool FAST>
+__device__ __forceinline__ float2 pair_gain(const Prm& pr, const float2* bv, const float2* alpha,
+                                            const float4* pe) {
+  float2 Go[6];
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    const float4 v = pe[5 + i];
+    Go[2 * i] = make_float2(v.x, v.y);
+    Go[2 * i + 1] = make_float2(v.z, v.w);
+  }
+  const float4 v8 = pe[8];
+  const float2 gd = make_float2(v8.x, v8.y);
+  if constexpr (FAST) {
+    return quant_gain_fast2<4>(pr, alpha, bv, gd, Go);  // G off-diagonal doubled
+  } else {
+    float2 g;
+    float q[4];
+    int sf;
+    float G[6], a[4], bb[4];
 #pragma unroll
     for (int i = 0; i < 6; ++i) G[i] = Go[i].x;
 #pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].x; b[p] = bv[p].x; }
-    g.x = quant_gain<4>(pr, a, b, gd.x, G, q, &sf);
-  }
-  {
-    float G[6], a[4], b[4];
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].x; bb[p] = bv[p].x; }
+    g.x = quant_gain<4>(pr, a, bb, gd.x, G, q, &sf);
 #pragma unroll
     for (int i = 0; i < 6; ++i) G[i] = Go[i].y;
 #pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].y; b[p] = bv[p].y; }
-    g.y = quant_gain<4>(pr, a, b, gd.y, G, q, &sf);
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].y; bb[p] = bv[p].y; }
+    g.y = quant_gain<4>(pr, a, bb, gd.y, G, q, &sf);
+    return g;
   }
-  return g;
 }
 
 template <bool FAST>
@@ -371,7 +398,7 @@ __global__ void __launch_bounds__(NT, 1)
   } else {
     // ------------------------------------------------------------ epilogue --
     const int m = 32 * (warp & 3) + lane;  // this thread's row = TMEM lane
-    const int sub = warp >> 2;             // seeds 8*sub .. 8*sub+7 of each chunk
+    const int sub = warp >> 2;             // seed pairs SUB_PAIRS*sub .. of each chunk
     const float tq = __fmul_rn(sm.two_q[m], pr.c);
     const float2 tqc = make_float2(tq, tq);
     const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
@@ -385,19 +412,51 @@ __global__ void __launch_bounds__(NT, 1)
       tc_fence_after();
       const float4* pbase = reinterpret_cast<const float4*>(&sm.stage[st][kBBytes]);
 #pragma unroll 1
-      for (int rnd = 0; rnd < 2; ++rnd) {
-        const uint32_t col = (uint32_t)(tb * 256 + 32 * sub + 16 * rnd);
-        float hi[16], lo[16];
-        tmem_ld16(tmem + lane_base + col, hi);
-        tmem_ld16(tmem + lane_base + col + 128, lo);
+      for (int rnd = 0; rnd < ROUNDS; ++rnd) {
+        const int p0 = SUB_PAIRS * sub + RPAIRS * rnd;  // first seed pair of the round
+        const uint32_t col = (uint32_t)(tb * 256 + 8 * p0);
+        float hi[8 * RPAIRS], lo[8 * RPAIRS];
+        tmem_ld_pairs(tmem + lane_base + col, hi);
+        tmem_ld_pairs(tmem + lane_base + col + 128, lo);
         tmem_wait_ld();
+        float2 bv[RPAIRS][4], al[RPAIRS][4];
+        bool live[RPAIRS][2];
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          const int ni = 4 * sub + 2 * rnd + j;  // seed pair within the chunk
-          const float2 g = pair_gain<FAST>(pr, hi + 8 * j, lo + 8 * j, tqc, pbase + ni * (PS / 2));
-          const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * ni);
-          if (g.x > bg) { bg = g.x; bsd = s; }
-          if (g.y > bg) { bg = g.y; bsd = s + 1; }
+        for (int j = 0; j < RPAIRS; ++j) {
+          const float4* pe = pbase + (p0 + j) * (PS / 2);
+          pair_fit(hi + 8 * j, lo + 8 * j, tqc, pe, bv[j], al[j]);
+          if constexpr (FAST) {
+            // prune: a candidate whose gain bound is below the running best
+            // cannot win (NaN bounds stay live)
+            const float2 ub = pair_bound(bv[j], al[j], pe);
+            live[j][0] = !(ub.x < bg);
+            live[j][1] = !(ub.y < bg);
+          } else {
+            live[j][0] = live[j][1] = true;
+          }
+        }
+        float g[2 * RPAIRS];  // seeds 2*p0 + i of the chunk
+#pragma unroll
+        for (int j = 0; j < RPAIRS; ++j) {
+          float2 gp = make_float2(neg_inf(), neg_inf());
+          if (!FAST || __any_sync(0xffffffffu, live[j][0] || live[j][1])) {
+            gp = pair_gain<FAST>(pr, bv[j], al[j], pbase + (p0 + j) * (PS / 2));
+            if (!live[j][0]) gp.x = neg_inf();
+            if (!live[j][1]) gp.y = neg_inf();
+          }
+          g[2 * j] = gp.x;
+          g[2 * j + 1] = gp.y;
+        }
+        // running argmax: the first of the round's maxima, if it beats the best
+        float cm = g[0];
+#pragma unroll
+        for (int i = 1; i < 2 * RPAIRS; ++i) cm = fmaxf(cm, g[i]);
+        if (cm > bg) {
+          int i = 2 * RPAIRS - 1;
+#pragma unroll
+          for (int t = 2 * RPAIRS - 2; t >= 0; --t) if (g[t] == cm) i = t;
+          bg = cm;
+          bsd = (uint32_t)((c0 + k) * CH + 2 * p0 + i);
         }
       }
       tc_fence_before();
@@ -411,11 +470,11 @@ __global__ void __launch_bounds__(NT, 1)
   if (__syncthreads_or(timed_out)) {
     if (tid == 0) atomicOr(status, kFaultTimeout);
   } else if (tid < BM) {
-    // merge the four warps of each row (smaller seed on equal gains)
+    // merge the SUBS warps of each row (smaller seed on equal gains)
     float g = sm.red_g[0][tid];
     uint32_t s = sm.red_s[0][tid];
 #pragma unroll
-    for (int i = 1; i < 4; ++i) {
+    for (int i = 1; i < SUBS; ++i) {
       if (better(sm.red_g[i][tid], sm.red_s[i][tid], g, s)) { g = sm.red_g[i][tid]; s = sm.red_s[i][tid]; }
     }
     const int64_t row = rb * BM + tid;
