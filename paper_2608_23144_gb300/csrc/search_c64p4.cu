@@ -41,7 +41,7 @@ constexpr int SUBS = EW / 4;        // epilogue warps per TMEM lane quarter
 constexpr int SUB_PAIRS = CH / 2 / SUBS;  // seed pairs of a chunk per epilogue warp
 constexpr int RPAIRS = 2;           // seed pairs per TMEM load (8 columns each)
 constexpr int ROUNDS = SUB_PAIRS / RPAIRS;
-static_assert(EW % 4 == 0 && SUB_PAIRS % RPAIRS == 0, "epilogue mapping");
+static_assert(EW % 4 == 0 && SUB_PAIRS % RPAIRS == 0 && RPAIRS % 2 == 0, "epilogue mapping");
 constexpr int STAGES = 4;
 constexpr int PS = pair_stride(4);  // 18 float2 per seed pair
 constexpr uint32_t kBBytes = NCOL * 64 * 2;        // 16 KB of FP16 atoms per chunk
@@ -156,7 +156,8 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// 16 consecutive 32-bit TMEM columns of the warp's 32 lanes (one lane per thread).
+// 16 consecutive 32-bit TMEM columns of the warp's 32 lanes (one lane per
+// thread). The registers are valid only after tmem_wait_ld().
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   uint32_t r[16];
   asm volatile(
@@ -165,8 +166,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
         "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr)
-      : "memory");
+      : "r"(taddr));
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
@@ -177,8 +177,21 @@ __device__ __forceinline__ void tmem_ld_pairs(uint32_t taddr, float* v) {
   for (int i = 0; i < RPAIRS / 2; ++i) tmem_ld16(taddr + 16 * i, v + 16 * i);
 }
 
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+// Waits for this thread's TMEM loads; the operands tie 16 loaded registers to
+// the wait so that no use of them can be scheduled above it.
+__device__ __forceinline__ void tmem_wait_ld(float* v) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]), "+f"(v[6]),
+                 "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]), "+f"(v[12]),
+                 "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
+}
+
+// Ties further loaded registers to a wait already issued.
+__device__ __forceinline__ void tmem_tie(float* v) {
+  asm volatile(""
+               : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]), "+f"(v[6]),
+                 "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]), "+f"(v[12]),
+                 "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
 }
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
@@ -189,10 +202,14 @@ __device__ __forceinline__ int a_offset(int m, int k) {
   return (((m >> 3) * 8 + (k >> 3)) << 7) + ((m & 7) << 4) + ((k & 7) << 1);
 }
 
-// Fit of one seed pair for this thread's row: hi/lo hold atom p of the two
-// seeds at [2p], [2p+1]; pe points at the pair's 18 float2 factors (9 float4).
-__device__ __forceinline__ void pair_fit(const float* hi, const float* lo, float2 tqc, const float4* pe,
-                                         float2* bv, float2* alpha) {
+// Forward half of the ridge solve for one seed pair of this thread's row:
+// b from the exact correlations (hi/lo hold atom p of the two seeds at [2p],
+// [2p+1]), z = L^-1 b and w = D^-1 z, so that alpha = L^-T w. pe points at
+// the pair's 18 float2 factors (9 float4: -L, invD, G off-diagonal, gd and the
+// bound multiplier). Returns U = b^T (G + eps I)^-1 b = z^T w (a sum of
+// non-negative terms) times the seed's bound multiplier.
+__device__ __forceinline__ float2 pair_forward(const float* hi, const float* lo, float2 tqc, const float4* pe,
+                                               float2* bv, float2* w) {
   float2 pv[10];
 #pragma unroll
   for (int i = 0; i < 5; ++i) {
@@ -200,22 +217,46 @@ __device__ __forceinline__ void pair_fit(const float* hi, const float* lo, float
     pv[2 * i] = make_float2(v.x, v.y);
     pv[2 * i + 1] = make_float2(v.z, v.w);
   }
+  const float2* nL = pv;
+  const float2* invD = pv + 6;
 #pragma unroll
   for (int p = 0; p < 4; ++p) {
     const float2 u = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
                                 make_float2(lo[2 * p], lo[2 * p + 1]));
     bv[p] = __fmul2_rn(u, tqc);
   }
-  ldl_solve2<4>(pv, pv + 6, bv, alpha);  // -L, invD
+  float2 z[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    float2 v = bv[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) v = __ffma2_rn(nL[tri(k, i)], z[i], v);
+    z[k] = v;
+    w[k] = __fmul2_rn(v, invD[k]);
+  }
+  float2 U = __fmul2_rn(z[0], w[0]);
+#pragma unroll
+  for (int k = 1; k < 4; ++k) U = __ffma2_rn(z[k], w[k], U);
+  const float4 v8 = pe[8];
+  return __fmul2_rn(U, make_float2(v8.z, v8.w));
 }
 
-// Upper bound on the two candidates' gains: (b^T alpha) * m (see bound_multiplier).
-__device__ __forceinline__ float2 pair_bound(const float2* bv, const float2* alpha, const float4* pe) {
-  float2 U = __fmul2_rn(bv[0], alpha[0]);
+// Back half of the solve: alpha = L^-T w, in the order of ldl_solve2.
+__device__ __forceinline__ void pair_back(const float4* pe, const float2* w, float2* alpha) {
+  float2 nL[6];
 #pragma unroll
-  for (int p = 1; p < 4; ++p) U = __ffma2_rn(bv[p], alpha[p], U);
-  const float4 v = pe[8];
-  return __fmul2_rn(U, make_float2(v.z, v.w));
+  for (int i = 0; i < 3; ++i) {
+    const float4 v = pe[i];
+    nL[2 * i] = make_float2(v.x, v.y);
+    nL[2 * i + 1] = make_float2(v.z, v.w);
+  }
+#pragma unroll
+  for (int k = 3; k >= 0; --k) {
+    float2 v = w[k];
+#pragma unroll
+    for (int i = k + 1; i < 4; ++i) v = __ffma2_rn(nL[tri(i, k)], alpha[i], v);
+    alpha[k] = v;
+  }
 }
 
 // Quantised gains of a fitted seed pair.
@@ -409,40 +450,39 @@ __global__ void __launch_bounds__(NT, 1)
     for (int k = 0; k < nck; ++k) {
       const int st = k % STAGES, tb = k & 1;
       if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1))) { timed_out = true; break; }
+      // the stage's factors landed before the chunk's MMAs were issued; this
+      // wait (already complete) makes the copy visible to this warp's reads
+      if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
       tc_fence_after();
       const float4* pbase = reinterpret_cast<const float4*>(&sm.stage[st][kBBytes]);
-#pragma unroll 1
+#pragma unroll
       for (int rnd = 0; rnd < ROUNDS; ++rnd) {
         const int p0 = SUB_PAIRS * sub + RPAIRS * rnd;  // first seed pair of the round
         const uint32_t col = (uint32_t)(tb * 256 + 8 * p0);
         float hi[8 * RPAIRS], lo[8 * RPAIRS];
         tmem_ld_pairs(tmem + lane_base + col, hi);
         tmem_ld_pairs(tmem + lane_base + col + 128, lo);
-        tmem_wait_ld();
-        float2 bv[RPAIRS][4], al[RPAIRS][4];
-        bool live[RPAIRS][2];
+        tmem_wait_ld(hi);
 #pragma unroll
-        for (int j = 0; j < RPAIRS; ++j) {
-          const float4* pe = pbase + (p0 + j) * (PS / 2);
-          pair_fit(hi + 8 * j, lo + 8 * j, tqc, pe, bv[j], al[j]);
-          if constexpr (FAST) {
-            // prune: a candidate whose gain bound is below the running best
-            // cannot win (NaN bounds stay live)
-            const float2 ub = pair_bound(bv[j], al[j], pe);
-            live[j][0] = !(ub.x < bg);
-            live[j][1] = !(ub.y < bg);
-          } else {
-            live[j][0] = live[j][1] = true;
-          }
-        }
+        for (int i = 16; i < 8 * RPAIRS; i += 16) tmem_tie(hi + i);
+#pragma unroll
+        for (int i = 0; i < 8 * RPAIRS; i += 16) tmem_tie(lo + i);
         float g[2 * RPAIRS];  // seeds 2*p0 + i of the chunk
 #pragma unroll
         for (int j = 0; j < RPAIRS; ++j) {
+          const float4* pe = pbase + (p0 + j) * (PS / 2);
+          float2 bv[4], wv[4];
+          const float2 ub = pair_forward(hi + 8 * j, lo + 8 * j, tqc, pe, bv, wv);
+          // prune: a candidate whose gain bound is below the running best
+          // cannot win (NaN bounds stay live)
+          const bool lx = !FAST || !(ub.x < bg), ly = !FAST || !(ub.y < bg);
           float2 gp = make_float2(neg_inf(), neg_inf());
-          if (!FAST || __any_sync(0xffffffffu, live[j][0] || live[j][1])) {
-            gp = pair_gain<FAST>(pr, bv[j], al[j], pbase + (p0 + j) * (PS / 2));
-            if (!live[j][0]) gp.x = neg_inf();
-            if (!live[j][1]) gp.y = neg_inf();
+          if (__any_sync(0xffffffffu, lx || ly)) {
+            float2 al[4];
+            pair_back(pe, wv, al);
+            gp = pair_gain<FAST>(pr, bv, al, pe);
+            if (!lx) gp.x = neg_inf();
+            if (!ly) gp.y = neg_inf();
           }
           g[2 * j] = gp.x;
           g[2 * j + 1] = gp.y;
