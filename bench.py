@@ -9,7 +9,8 @@ decode-apply of every module. Inputs are resident in HBM (308 MB of W and W0,
 larger than the 129 MB L2) when the timed region starts.
 
 Reported: (tile, seed) candidates/s for the whole step (`value`), layers/s,
-decode-apply GB/s, the search kernel against the FP32 pipe (`roofline`), the
+decode-apply GB/s, the search kernel against the FP32 pipe (`roofline`: the
+FP32 work every candidate needs before pruning), the
 end-to-end figure through the public API with host buffers (`e2e`), and the
 CPU oracle on a bounded sample (`cpu_baseline`). `--impl reference` times the
 oracle alone (the baseline arm). Under torchrun each rank encodes its own layer
@@ -34,14 +35,18 @@ WORKLOAD = "qwen2.5-3b_layer"
 RATE = 0.162
 METRIC = "AWSRC encode (tile,seed) candidates/s + layers/s; decode-apply HBM GB/s"
 UNIT = "candidates/s"
-# FP32-pipe operations per (tile, seed) candidate of the C=64, P=4, U search:
-# C*P = 256 correlation FFMAs plus the 80-operation epilogue of the numeric
-# convention (solve 20, quantise 25, gain 34, compare 1).
-OPS_PER_CANDIDATE = 256 + 80
+# FP32-pipe operations every (tile, seed) candidate of the C=64, P=4, U search
+# needs before it can be pruned: the correlation's rounding and scaling (2 per
+# atom), the forward substitution (6), D^-1 (4), U = z^T D^-1 z (4) and the
+# bound multiplier (1). The ~1-2% of candidates that survive the bound add
+# about 35 more each (back substitution, quantiser, gain), not counted here.
+# The correlation itself is tensor-core work: 2 halves x C x P x 2 FLOP.
+OPS_PER_CANDIDATE = 8 + 6 + 4 + 4 + 1
+TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "b7550f8142e968b87e5cc09cd18cbf0704837c7c70751c8111b4f570691bdd1e",
-                  "bytes_per_launch": 447428352}
+SEARCH_TRAFFIC = {"source_sha256": "447e4f1a3e58f2d5ba2d9459b3199876759aa34ece504147a161a626f0b2d723",
+                  "bytes_per_launch": 418617088 + 8241152}
 
 
 def parse():
@@ -330,7 +335,8 @@ def run_ours(args):
                 "peak": fp32_peak / 1e9, "unit": "Gop/s", "frac": achieved / fp32_peak,
                 "traffic": traffic, "peak_kind": f"{peak_kind}: {nsm} SMs x 128 FP32 lanes x "
                 f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
-                "ops_per_candidate": OPS_PER_CANDIDATE, "search_ms": search_ms}
+                "ops_per_candidate": OPS_PER_CANDIDATE, "search_ms": search_ms,
+                "tensor_tflops": cands_per_step * TENSOR_FLOP_PER_CANDIDATE / (search_ms * 1e-3) / 1e12}
     decode = {"gbs": dec_gbs, "ms": dec_ms, "frac_of_hbm": dec_gbs / float(peaks.get("hbm_gbs", 6800.0)),
               "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0))}
 
