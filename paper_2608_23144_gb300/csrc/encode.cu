@@ -40,35 +40,42 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 // double precision or kappa > 2^16. Computed in double and rounded up.
 template <int P>
 __device__ float bound_multiplier(float gd, const float* Goff, float eps) {
-  double A[P][P];
+  // LDL^T of G in double; tr(G^-1) = sum_k |row k of L^-1|^2 / D_k
+  double L[P][P], d[P], inv_d[P];
 #pragma unroll
-  for (int i = 0; i < P; ++i) {
-    A[i][i] = gd;
-#pragma unroll
-    for (int j = 0; j < i; ++j) A[i][j] = A[j][i] = Goff[tri(i, j)];
-  }
-  // Gauss-Jordan on the symmetric positive definite candidate (no pivoting)
-  double Inv[P][P];
-#pragma unroll
-  for (int i = 0; i < P; ++i)
-#pragma unroll
-    for (int j = 0; j < P; ++j) Inv[i][j] = i == j ? 1.0 : 0.0;
   for (int k = 0; k < P; ++k) {
-    const double piv = A[k][k];
-    if (!(piv > 0.0)) return __int_as_float(0x7f800000);
-    const double ip = 1.0 / piv;
-    for (int j = 0; j < P; ++j) { A[k][j] *= ip; Inv[k][j] *= ip; }
-    for (int i = 0; i < P; ++i) {
-      if (i == k) continue;
-      const double f = A[i][k];
-      for (int j = 0; j < P; ++j) { A[i][j] -= f * A[k][j]; Inv[i][j] -= f * Inv[k][j]; }
+    double dk = gd;
+#pragma unroll
+    for (int i = 0; i < k; ++i) dk -= L[k][i] * L[k][i] * d[i];
+    if (!(dk > 0.0)) return __int_as_float(0x7f800000);
+    d[k] = dk;
+    inv_d[k] = 1.0 / dk;
+#pragma unroll
+    for (int j = k + 1; j < P; ++j) {
+      double v = Goff[tri(j, k)];
+#pragma unroll
+      for (int i = 0; i < k; ++i) v -= L[j][i] * L[k][i] * d[i];
+      L[j][k] = v * inv_d[k];
     }
   }
-  double tri_inv = 0.0;
-  for (int i = 0; i < P; ++i) tri_inv += Inv[i][i];
-  const double kappa = (double)P * gd * tri_inv;
-  if (!(tri_inv > 0.0) || !(kappa <= 65536.0)) return __int_as_float(0x7f800000);
-  const double m = (1.0 + (double)eps * tri_inv) * (1.0 + 0x1p-10 + 0x1p-14 * kappa);
+  double tr_inv = 0.0;
+#pragma unroll
+  for (int i = 0; i < P; ++i) {  // column i of X = L^-1, rows k >= i
+    double x[P];
+    x[i] = 1.0;
+    tr_inv += inv_d[i];
+#pragma unroll
+    for (int k = i + 1; k < P; ++k) {
+      double v = 0.0;
+#pragma unroll
+      for (int j = i; j < k; ++j) v -= L[k][j] * x[j];
+      x[k] = v;
+      tr_inv += v * v * inv_d[k];
+    }
+  }
+  const double kappa = (double)P * gd * tr_inv;
+  if (!(kappa <= 65536.0)) return __int_as_float(0x7f800000);
+  const double m = (1.0 + (double)eps * tr_inv) * (1.0 + 0x1p-10 + 0x1p-14 * kappa);
   return __double2float_ru(m);
 }
 

@@ -53,6 +53,36 @@ def test_encode_matches_oracle(aw, orc, label, kw, shapes, w_dtype, fisher):
     assert np.isfinite(got["gain"]).sum() > 0.5 * len(got)
 
 
+@pytest.mark.parametrize("kind", ["wide_range", "sparse_weights", "large_ridge", "one_hot_residual"])
+def test_pruned_search_matches_oracle_on_adversarial_tiles(aw, orc, kind):
+    """The specialised search skips candidates whose gain bound cannot beat the
+    running best. On tiles built to stress that bound (activation moments over
+    twelve decades, mostly-zero weights that make G singular, a large ridge,
+    one-hot residuals with many equal correlations) the winners must still be
+    the oracle's, bit for bit."""
+    mods = _mods([(300, 256)], "bf16", seed=3)
+    m = mods[0]
+    g = torch.Generator().manual_seed(7)
+    kw = dict(C=64, P=4, b=4, S=512)
+    if kind == "wide_range":
+        m["act"] = (10.0 ** (torch.rand(256, generator=g) * 12 - 6)).float()
+    elif kind == "sparse_weights":
+        m["act"] = m["act"] * (torch.rand(256, generator=g) < 0.1).float()
+    elif kind == "large_ridge":
+        kw["ridge_rel"] = 0.5
+    else:
+        W = m["W0"].clone()
+        W[:, ::64] += 0.25
+        m["W"] = W
+    prm, oprm = aw.params(**kw), orc.params(**kw)
+    cands = aw.awsrc_encode_tiles(prm, to_dev(mods))
+    flags = aw.awsrc_workspace_status(cands._awsrc_workspace)
+    got = aw.candidates_to_numpy(cands)
+    want = oracle_encode(orc, oprm, mods)[0]
+    assert flags == 0, f"device fault flags {flags:#x}"
+    assert_candidates_equal(got, want, kind)
+
+
 def test_degenerate_tiles(aw, orc):
     mods = _mods([(40, 192)], "f32")
     m = mods[0]
