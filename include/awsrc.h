@@ -280,7 +280,12 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  * Each corrected element is fl(W0 + fl(fl(k_j * C^-1/2) * scale)) with the exact
  * integer k_j = sum_p sign_{j,p} * code_p, rounded once more to BF16 when
  * out_dtype is BF16. Records naming a tile >= T or a seed >= S are skipped and
- * reported through awsrc_workspace_status(). Requires the same params as the encoder.
+ * reported through awsrc_workspace_status(). A stream names each tile at most
+ * once (the encoder never repeats one); DENSE decoding of a stream that does
+ * applies only the tile's later record and reports it the same way, INPLACE
+ * leaves such a tile unspecified. Requires the same params as the encoder.
+ * Workspace (awsrc_decode_workspace_bytes): the basis masks, plus for DENSE a
+ * tile -> record map and the unpacked records, 12 bytes per tile.
  */
 awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 const awsrc_module* mods, const uint8_t* stream,
@@ -323,7 +328,8 @@ awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t
  * device fault word kept in the first bytes of an encode/select/decode
  * workspace. Each of those entry points clears the word when it starts, so the
  * flags describe the last call made with this workspace; 0 means no fault.
- * Bit 0 (1): a record named a tile or seed out of range (decoder; skipped).
+ * Bit 0 (1): a record named a tile or seed out of range (decoder; skipped), or
+ *            a tile a second time (dense decoder).
  * Bit 1 (2): encoder self-check — the finalisation recomputed a different gain
  *            than the search found (never expected).
  * Bit 2 (4): a bounded wait inside a kernel gave up (never expected).

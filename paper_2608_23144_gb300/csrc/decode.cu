@@ -2,16 +2,23 @@
 // named by records, W0 elsewhere (Eq. 1); any prefix of a progressive stream
 // decodes the same way (Sec. 3.3).
 //
-//  copy      (dense mode) W_hat = W0 converted to the output dtype, a pure
-//            stream of 16-byte vectors, four in flight per thread.
-//  patch     one warp per record: unpack tile, seed, scale, codes; bounds-check
-//            tile < T and seed < S (a bad record is skipped and flagged); write
-//            W_hat_j = fl(W0_j + fl(fl(k_j * C^-1/2) * scale)) on the tile, with
-//            k_j = sum_p sign * code_p exact in integers. It reads W0, so W_hat
-//            may alias W0 (in-place mode).
-// Keeping the record lookup out of the streaming pass keeps dependent loads
-// (record -> masks) off the bandwidth-critical path; the patch re-touches only
-// the recorded tiles (about 16% of a layer at 0.162 bits/weight).
+//  dense mode (C >= one vector):
+//   prep     one grid slice generates the basis masks (one warp per selector);
+//            the other unpacks every record once: its codes go to a per-record
+//            array and the tile's map entry (k + 1, seed, scale field) is
+//            raised to it with atomicMax, so a tile named twice is flagged and
+//            takes its later record.
+//   fused    one streaming pass: 16-byte vectors, four in flight per thread
+//            with their tiles' map entries; vectors of unrecorded tiles are
+//            converted and stored at once, those of recorded tiles are queued
+//            in shared memory and patched densely by the whole block:
+//            W_hat_j = fl(W0_j + fl(fl(k_j * C^-1/2) * scale)) with
+//            k_j = sum_p sign * code_p exact in integers.
+//  in-place mode, and dense mode with tiles shorter than one vector (after a
+//  plain copy of W0):
+//   patch    one thread per vector of a recorded tile: unpack tile, seed, scale,
+//            codes; bounds-check tile < T and seed < S (a bad record is skipped
+//            and flagged); rewrite the tile from W0, which may be W_hat itself.
 #include <algorithm>
 
 #include "basis.cuh"
@@ -173,6 +180,75 @@ __device__ __forceinline__ void st_stream(V* p, const V& v) {
   }
 }
 
+// Pairs of converted elements: packed f32x2 arithmetic (each component
+// rounded like the scalar form) and paired BF16 rounding.
+template <typename T> struct Io2;
+template <> struct Io2<float> {
+  static __device__ __forceinline__ float2 ld(const float* p) { return make_float2(p[0], p[1]); }
+  static __device__ __forceinline__ void st(float* p, float2 v) { p[0] = v.x; p[1] = v.y; }
+};
+template <> struct Io2<__nv_bfloat16> {
+  static __device__ __forceinline__ float2 ld(const __nv_bfloat16* p) {
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+  }
+  static __device__ __forceinline__ void st(__nv_bfloat16* p, float2 v) {
+    *reinterpret_cast<__nv_bfloat162*>(p) = __float22bfloat162_rn(v);
+  }
+};
+
+// One G-element vector of a recorded tile: o_j = fl(w_j + fl(fl(k_j * c) * sc))
+// with k_j = sum_p sign_{j,p} * code_p = tot - 2 * sum_p bit_{j,p} * code_p
+// (exact integers); mk points at atom 0's mask word of the vector, j0 its first
+// element. PT = P when the atom count is fixed at compile time, else 0.
+template <typename TI, typename TO, int G, int PT>
+__device__ __forceinline__ void patch_vec(const Prm& pr, const Vec<TI, G>& w, uint2 cw,
+                                          const uint64_t* __restrict__ mk, int j0, float sc, Vec<TO, G>& o) {
+  const int P = PT ? PT : pr.P;
+  int tot = 0, acc[G];
+#pragma unroll
+  for (int e = 0; e < G; ++e) acc[e] = 0;
+#pragma unroll
+  for (int p = 0; p < (PT ? PT : kMaxP); ++p) {
+    if (p < P) {
+      const uint32_t bits = (uint32_t)(__ldg(mk + (size_t)p * pr.W) >> (j0 & 63));
+      const int cp = (int)(int8_t)((p < 4 ? cw.x : cw.y) >> (8 * (p & 3)));
+      tot += cp;
+#pragma unroll
+      for (int e = 0; e < G; ++e) acc[e] += (int)((bits >> e) & 1u) * cp;
+    }
+  }
+  const float2 c2 = make_float2(pr.c, pr.c), s2 = make_float2(sc, sc);
+#pragma unroll
+  for (int e = 0; e < G; e += 2) {
+    const float2 k = make_float2((float)(tot - 2 * acc[e]), (float)(tot - 2 * acc[e + 1]));
+    const float2 r = __fmul2_rn(__fmul2_rn(k, c2), s2);
+    Io2<TO>::st(o.v + e, __fadd2_rn(Io2<TI>::ld(w.v + e), r));
+  }
+}
+
+// Dense-mode record pass: record k's codes go to codes[k] and map[tile] is
+// raised to (k + 1) << 32 | seed << 16 | scale field (map cleared to 0
+// beforehand). Records naming a tile or seed out of range, and tiles named
+// twice, raise kFaultRecord. Threads [i0, i0 + n) of a grid-stride range.
+__device__ __forceinline__ void map_records(const Prm& pr, const DecArgs& a, const uint8_t* __restrict__ stream,
+                                            unsigned long long* __restrict__ map, uint2* __restrict__ codes,
+                                            uint32_t* __restrict__ status, int64_t i0, int64_t n) {
+  const int64_t Kd = stream_K(stream, a.K, a.kmax);
+  const int64_t end = a.h + a.kmax * a.L;
+  for (int64_t k = i0; k < Kd; k += n) {
+    DecRec d;
+    const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d, end);
+    if (tile < 0) {
+      atomicOr(status, kFaultRecord);
+      continue;
+    }
+    codes[k] = make_uint2(d.cw[0], d.cw[1]);
+    const unsigned long long e = ((unsigned long long)(k + 1) << 32) | ((unsigned long long)d.seed << 16) |
+                                 (unsigned long long)(uint16_t)d.scale;
+    if (atomicMax(map + tile, e) != 0ull) atomicOr(status, kFaultRecord);
+  }
+}
+
 // Dense pass: W_hat = convert(W0) for every element, a pure stream with U
 // independent 16-byte vectors in flight per thread and no dependent loads.
 // With `basis`, the blocks of grid slice y = 0 (dispatched first) generate the
@@ -182,15 +258,19 @@ template <typename TI, typename TO, int G>
 __global__ void __launch_bounds__(256) copy_kernel(Prm pr, const __grid_constant__ DecArgs a,
                                                    uint64_t* __restrict__ masks, int basis) {
   constexpr int U = 4;
-  if (basis && blockIdx.y == 0) {
-    __shared__ uint8_t perm_s[8][kMaxC], kidx_s[8][kMaxC], pool_s[8][kMaxC];
-    __shared__ int cols_s[8][kMaxP];
-    const int warp = threadIdx.x >> 5;
-    const int s = blockIdx.x * 8 + warp;
-    if (s < pr.S) basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
-    return;
+  int y = blockIdx.y;
+  if (basis) {
+    if (y == 0) {
+      __shared__ uint8_t perm_s[8][kMaxC], kidx_s[8][kMaxC], pool_s[8][kMaxC];
+      __shared__ int cols_s[8][kMaxP];
+      const int warp = threadIdx.x >> 5;
+      const int s = blockIdx.x * 8 + warp;
+      if (s < pr.S) basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
+      return;
+    }
+    --y;
   }
-  const DecodeMod& md = a.m[blockIdx.y - (basis ? 1 : 0)];
+  const DecodeMod& md = a.m[y];
   const int64_t ngroups = md.rows * md.cols / G;
   const Vec<TI, G>* __restrict__ src = static_cast<const Vec<TI, G>*>(md.W0);
   Vec<TO, G>* __restrict__ dst = static_cast<Vec<TO, G>*>(md.out);
@@ -245,24 +325,9 @@ __global__ void __launch_bounds__(256) patch_kernel(Prm pr, const __grid_constan
     const int j0 = gj * G;
     const int64_t e0 = (tile - md.tile_off) * pr.C + j0;
     const Vec<TI, G> v = *reinterpret_cast<const Vec<TI, G>*>(static_cast<const TI*>(md.W0) + e0);
-    const uint64_t* mk = masks + (size_t)d.seed * pr.P * pr.W + (j0 >> 6);
-    // k_j = sum_p (1 - 2 bit_pj) c_p = (sum_p c_p) - 2 sum_p bit_pj c_p, exact in integers
-    int tot = 0, acc[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) acc[g] = 0;
-    for (int p = 0; p < pr.P; ++p) {
-      const uint32_t bits = (uint32_t)(__ldg(mk + (size_t)p * pr.W) >> (j0 & 63));
-      const int cp = code_of(d, p);
-      tot += cp;
-#pragma unroll
-      for (int g = 0; g < G; ++g) acc[g] += (int)((bits >> g) & 1u) * cp;
-    }
-    const float sc = scale_of(pr, d.scale);
     Vec<TO, G> o;
-#pragma unroll
-    for (int g = 0; g < G; ++g)
-      o.v[g] = Io<TO>::cvt(__fadd_rn(Io<TI>::ld(v.v, g),
-                                     __fmul_rn(__fmul_rn((float)(tot - 2 * acc[g]), pr.c), sc)));
+    patch_vec<TI, TO, G, 0>(pr, v, make_uint2(d.cw[0], d.cw[1]),
+                            masks + (size_t)d.seed * pr.P * pr.W + (j0 >> 6), j0, scale_of(pr, d.scale), o);
     *reinterpret_cast<Vec<TO, G>*>(static_cast<TO*>(md.out) + e0) = o;
   }
 }
@@ -298,6 +363,139 @@ __global__ void __launch_bounds__(256) patch_small_kernel(Prm pr, const __grid_c
     const float w = Io<TI>::ld(static_cast<const TI*>(md.W0) + e, 0);
     static_cast<TO*>(md.out)[e] = Io<TO>::cvt(__fadd_rn(w, __fmul_rn(__fmul_rn((float)kj, pr.c), scale_of(pr, d.scale))));
   }
+}
+
+// Dense pass with the patches fused in. A block walks chunks of 1024 vectors (16 bytes each,
+// four per thread, coalesced): vectors of tiles without a record are converted
+// and stored at once; those of recorded tiles (about 16% at 0.162 bits/weight)
+// go, with their W0 data and map entry, to a queue in shared memory that all
+// threads then patch densely. C >= G.
+constexpr int kFusedThreads = 256;
+constexpr int kFusedU = 4;
+constexpr int kFusedChunk = kFusedThreads * kFusedU;
+
+struct FusedQ {
+  uint4 w0;                 // the vector's W0 bits
+  unsigned long long e;     // map entry
+  long long g;              // vector index within the module
+};
+
+template <typename TI, typename TO, int G, int PT>
+__global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                                 const unsigned long long* __restrict__ map,
+                                                                 const uint2* __restrict__ codes,
+                                                                 const uint64_t* __restrict__ masks) {
+  static_assert(sizeof(Vec<TI, G>) == 16, "16-byte vectors");
+  __shared__ FusedQ q[kFusedChunk];
+  __shared__ int qn;
+  const DecodeMod& md = a.m[blockIdx.y];
+  const int64_t ngroups = md.rows * md.cols / G;
+  const int vshift = pr.logC - (G == 8 ? 3 : 2);  // log2 of the vectors per tile
+  const Vec<TI, G>* __restrict__ src = static_cast<const Vec<TI, G>*>(md.W0);
+  Vec<TO, G>* __restrict__ dst = static_cast<Vec<TO, G>*>(md.out);
+  const unsigned long long* __restrict__ mmap = map + md.tile_off;
+  const int lane = threadIdx.x & 31;
+  for (int64_t c0 = (int64_t)blockIdx.x * kFusedChunk; c0 < ngroups; c0 += (int64_t)gridDim.x * kFusedChunk) {
+    if (threadIdx.x == 0) qn = 0;
+    __syncthreads();
+    Vec<TI, G> v[kFusedU];
+    unsigned long long r[kFusedU];
+#pragma unroll
+    for (int u = 0; u < kFusedU; ++u) {
+      const int64_t g = c0 + u * kFusedThreads + threadIdx.x;
+      r[u] = 0ull;
+      if (g < ngroups) {
+        v[u] = ld_stream(src + g);
+        r[u] = __ldg(mmap + (g >> vshift));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kFusedU; ++u) {
+      const int64_t g = c0 + u * kFusedThreads + threadIdx.x;
+      const bool in = g < ngroups;
+      const bool patch = in && r[u] != 0ull;
+      if (in && !patch) {
+        Vec<TO, G> o;
+#pragma unroll
+        for (int e = 0; e < G; e += 2) Io2<TO>::st(o.v + e, Io2<TI>::ld(v[u].v + e));
+        st_stream(dst + g, o);
+      }
+      const unsigned m = __ballot_sync(0xffffffffu, patch);  // warp-aggregated append
+      if (m) {
+        int base = 0;
+        if (lane == 0) base = atomicAdd(&qn, __popc(m));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (patch) {
+          FusedQ& x = q[base + __popc(m & ((1u << lane) - 1u))];
+          memcpy(&x.w0, &v[u], 16);
+          x.e = r[u];
+          x.g = g;
+        }
+      }
+    }
+    __syncthreads();
+    const int n = qn;
+    for (int i = threadIdx.x; i < n; i += kFusedThreads) {
+      const FusedQ x = q[i];
+      Vec<TI, G> w;
+      memcpy(&w, &x.w0, 16);
+      const int64_t k = (int64_t)(x.e >> 32) - 1;
+      const uint32_t seed = (uint32_t)(x.e >> 16) & 0xFFFFu;
+      const int j0 = (int)(x.g & ((1 << vshift) - 1)) * G;
+      Vec<TO, G> o;
+      patch_vec<TI, TO, G, PT>(pr, w, __ldg(codes + k), masks + (size_t)seed * pr.P * pr.W + (j0 >> 6), j0,
+                               scale_of(pr, (int16_t)(uint16_t)(x.e & 0xFFFFull)), o);
+      st_stream(dst + x.g, o);
+    }
+    __syncthreads();
+  }
+}
+
+// Dense-mode preparation for the fused pass: slice y = 0 generates the masks
+// (one warp per selector), slice y = 1 fills the tile map (map_records).
+__global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                   const uint8_t* __restrict__ stream,
+                                                   uint64_t* __restrict__ masks,
+                                                   unsigned long long* __restrict__ map,
+                                                   uint2* __restrict__ codes, uint32_t* __restrict__ status) {
+  if (blockIdx.y == 0) {
+    __shared__ uint8_t perm_s[8][kMaxC], kidx_s[8][kMaxC], pool_s[8][kMaxC];
+    __shared__ int cols_s[8][kMaxP];
+    const int warp = threadIdx.x >> 5;
+    const int s = blockIdx.x * 8 + warp;
+    if (s < pr.S) basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
+    return;
+  }
+  map_records(pr, a, stream, map, codes, status, (int64_t)blockIdx.x * blockDim.x + threadIdx.x,
+              (int64_t)gridDim.x * blockDim.x);
+}
+
+template <typename TI, typename TO, int G>
+cudaError_t launch_fused_t(const Prm& pr, const DecArgs& a, const unsigned long long* map,
+                           const uint2* codes, const uint64_t* masks, cudaStream_t st) {
+  int64_t maxg = 0;
+  for (int i = 0; i < a.n_mod; ++i) maxg = std::max<int64_t>(maxg, a.m[i].rows * a.m[i].cols / G);
+  int dev = 0, nsm = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (maxg + kFusedChunk - 1) / kFusedChunk;
+  const int64_t gx = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)nsm * 8));
+  if (pr.P == 4)
+    fused_kernel<TI, TO, G, 4><<<dim3((unsigned)gx, a.n_mod), kFusedThreads, 0, st>>>(pr, a, map, codes, masks);
+  else
+    fused_kernel<TI, TO, G, 0><<<dim3((unsigned)gx, a.n_mod), kFusedThreads, 0, st>>>(pr, a, map, codes, masks);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fused(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype,
+                         const unsigned long long* map, const uint2* codes, const uint64_t* masks,
+                         cudaStream_t st) {
+  const bool f32in = (w0_dtype == AWSRC_DTYPE_F32), f32out = (out_dtype == AWSRC_DTYPE_F32);
+  if (f32in && f32out) return launch_fused_t<float, float, 4>(pr, a, map, codes, masks, st);
+  if (f32in) return launch_fused_t<float, __nv_bfloat16, 4>(pr, a, map, codes, masks, st);
+  if (f32out) return launch_fused_t<__nv_bfloat16, float, 8>(pr, a, map, codes, masks, st);
+  return launch_fused_t<__nv_bfloat16, __nv_bfloat16, 8>(pr, a, map, codes, masks, st);
 }
 
 // copy: stream the modules of `a`; basis: also generate the masks (an extra
@@ -340,6 +538,7 @@ cudaError_t launch_patch_t(const Prm& pr, const DecArgs& a, const uint8_t* strea
   return cudaGetLastError();
 }
 
+// copy (dense) and/or the mask slice (basis), then the record-by-record patch.
 cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype, bool copy,
                          bool basis, const uint8_t* stream, uint64_t* masks, uint32_t* status,
                          cudaStream_t st) {
@@ -360,13 +559,31 @@ cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_
 
 }  // namespace
 
+// Launches over runs of at most 16 modules sharing the input dtype. DENSE with
+// C >= G: the first run's copy also generates the masks and fills the tile map,
+// then each run is patched in tile order; otherwise (INPLACE, or tiles shorter
+// than one vector) the copy (DENSE only) is followed by a record-by-record patch.
 cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
-  (void)scratch;
-  // launches over runs of at most 16 modules sharing the input dtype: DENSE
-  // copies every element (the first launch also generates the basis masks),
-  // then both modes patch the tiles named by records
+  const bool fused = mode == AWSRC_DECODE_DENSE && pr.C >= 8 && scratch != nullptr;
+  unsigned long long* map = nullptr;
+  uint2* codes = nullptr;
+  if (fused) {
+    map = static_cast<unsigned long long*>(scratch);
+    codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
+    cudaError_t e = cudaMemsetAsync(map, 0, (size_t)T * 8, st);
+    if (e != cudaSuccess) return e;
+    DecArgs a;
+    a.n_mod = 0;
+    a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
+    const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
+    const int64_t gx = std::max<int64_t>({(int64_t)1, (int64_t)(pr.S + 7) / 8,
+                                           std::min<int64_t>((work + 255) / 256, 1 << 20)});
+    prep_kernel<<<dim3((unsigned)gx, 2), 256, 0, st>>>(pr, a, stream, masks, map, codes, status);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   int i0 = 0;
   while (i0 < n_mod) {
     int i1 = i0 + 1;
@@ -375,8 +592,10 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     a.n_mod = i1 - i0;
     a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
     for (int i = 0; i < a.n_mod; ++i) a.m[i] = mods[i0 + i];
-    const cudaError_t e = launch_group(pr, a, mods[i0].w0_dtype, out_dtype, mode == AWSRC_DECODE_DENSE,
-                                       i0 == 0, stream, masks, status, st);
+    const cudaError_t e =
+        fused ? launch_fused(pr, a, mods[i0].w0_dtype, out_dtype, map, codes, masks, st)
+              : launch_group(pr, a, mods[i0].w0_dtype, out_dtype, mode == AWSRC_DECODE_DENSE, i0 == 0, stream,
+                             masks, status, st);
     if (e != cudaSuccess) return e;
     i0 = i1;
   }
@@ -384,9 +603,10 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
 }
 
 size_t decode_scratch_bytes(int64_t T, int mode) {
-  (void)T;
-  (void)mode;
-  return 0;
+  // dense: tile -> record map (8 B per tile) and each record's codes (8 B, at
+  // most one record per tile)
+  if (mode != AWSRC_DECODE_DENSE) return 0;
+  return align_up((size_t)T * 8, 256) + align_up((size_t)T * 8, 256);
 }
 
 }  // namespace awsrc

@@ -7,7 +7,7 @@
 // allocator of its own, or a recovery path that must not allocate while it
 // restores weights. awsrc_decode_apply_inplace_noalloc serves them: it runs the
 // same two kernels as the in-place mode of awsrc_decode_apply (basis masks,
-// then one warp per record), but its scratch — the fault word and the basis
+// then the patch of the recorded tiles), but its scratch — the fault word and the basis
 // mask table — lives in the file-scope device array below instead of a
 // caller-supplied workspace. It calls no cudaMalloc, cudaFree or allocating
 // library routine.

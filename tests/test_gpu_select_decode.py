@@ -130,3 +130,47 @@ def test_decode_rejects_K_beyond_stream(aw, orc):
     stream, counts, nbytes = aw.awsrc_select_records(prm, dmods, cands, [1.0])
     with pytest.raises(aw.AwsrcError):
         aw.awsrc_decode_apply(prm, dmods, stream[: int(nbytes[0])], int(counts.sum()) + 1)
+
+
+def test_decode_repeated_tile_takes_later_record(aw, orc):
+    """A stream that names a tile twice (never written by the encoder) is reported;
+    dense decoding applies the later record, i.e. it equals decoding the stream
+    without the earlier one."""
+    shapes = [(100, 256)]
+    mods, dmods, prm, oprm, cands, ocands = _setup(aw, orc, shapes, dict(C=64, P=4, b=4, S=64))
+    stream, counts, nbytes = aw.awsrc_select_records(prm, dmods, cands, [1.0])
+    K = int(counts.sum())
+    raw = stream.cpu().numpy()[: int(nbytes[0])].copy()
+    h, T = orc.header_bytes(1), 100 * 256 // 64
+    L = orc.record_bytes(oprm, T)
+    tb = int(np.ceil(np.log2(T)))
+    rec = lambda k: int.from_bytes(raw[h + k * L: h + (k + 1) * L].tobytes(), "little")
+    mask = (1 << tb) - 1
+    r1 = (rec(1) & ~mask) | (rec(0) & mask)        # record 1's payload on record 0's tile
+    dup = raw.copy()
+    dup[h + L: h + 2 * L] = np.frombuffer(r1.to_bytes(L, "little"), np.uint8)
+    fixed = np.concatenate([raw[:h], dup[h + L:]])  # record 0 removed
+    outs = aw.awsrc_decode_apply(prm, dmods, torch.from_numpy(dup).cuda(), K)
+    flags = aw.awsrc_workspace_status(outs[0]._awsrc_workspace)
+    assert flags & 1, "a repeated tile must be reported"
+    oouts, obad = orc.decode_apply(oprm, [mods[0]["W0"].float().numpy()], fixed.tobytes(), K - 1, out_bf16=True)
+    assert obad == 0
+    assert np.array_equal(outs[0].float().cpu().numpy(), oouts[0])
+
+
+@pytest.mark.parametrize("C,P", [(16, 4), (8, 2), (4, 1)])
+def test_decode_dense_many_modules_small_tiles(aw, orc, C, P):
+    """20 modules (two launch runs of at most 16) and tiles of one or two 16-byte
+    vectors (and a 4-element tile, below one BF16 vector)."""
+    shapes = [(6 + (i % 4), 32 if i % 3 else 64) for i in range(20)]
+    kw = dict(C=C, P=P, b=4, S=16)
+    mods, dmods, prm, oprm, cands, ocands = _setup(aw, orc, shapes, kw)
+    stream, counts, nbytes = aw.awsrc_select_records(prm, dmods, cands, [2.0])
+    ostream, ocounts, _ = orc.select_records(oprm, shapes, ocands, [2.0])
+    K = int(ocounts.sum())
+    assert K > 0
+    outs = aw.awsrc_decode_apply(prm, dmods, stream, -1)
+    oouts, _ = orc.decode_apply(oprm, [m["W0"].float().numpy() for m in mods], ostream, K, out_bf16=True)
+    for g, o in zip(outs, oouts):
+        assert np.array_equal(g.float().cpu().numpy(), o)
+    assert aw.awsrc_workspace_status(outs[0]._awsrc_workspace) == 0
