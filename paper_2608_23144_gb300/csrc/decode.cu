@@ -3,7 +3,7 @@
 // decodes the same way (Sec. 3.3).
 //
 //  dense mode (C >= one vector):
-//   prep     one grid slice generates the basis masks (one warp per selector);
+//   prep     one block range generates the basis masks (one warp per selector),
 //            the other unpacks every record once: its codes go to a per-record
 //            array and the tile's map entry (k + 1, seed, scale field) is
 //            raised to it with atomicMax, so a tile named twice is flagged and
@@ -451,14 +451,15 @@ __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const _
   }
 }
 
-// Dense-mode preparation for the fused pass: slice y = 0 generates the masks
-// (one warp per selector), slice y = 1 fills the tile map (map_records).
+// Dense-mode preparation for the fused pass: blocks [0, nb) generate the masks
+// (one warp per selector), the remaining blocks fill the tile map (map_records).
 __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant__ DecArgs a,
                                                    const uint8_t* __restrict__ stream,
                                                    uint64_t* __restrict__ masks,
                                                    unsigned long long* __restrict__ map,
-                                                   uint2* __restrict__ codes, uint32_t* __restrict__ status) {
-  if (blockIdx.y == 0) {
+                                                   uint2* __restrict__ codes, uint32_t* __restrict__ status,
+                                                   int nb) {
+  if ((int)blockIdx.x < nb) {
     __shared__ uint8_t perm_s[8][kMaxC], kidx_s[8][kMaxC], pool_s[8][kMaxC];
     __shared__ int cols_s[8][kMaxP];
     const int warp = threadIdx.x >> 5;
@@ -466,8 +467,8 @@ __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant
     if (s < pr.S) basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
     return;
   }
-  map_records(pr, a, stream, map, codes, status, (int64_t)blockIdx.x * blockDim.x + threadIdx.x,
-              (int64_t)gridDim.x * blockDim.x);
+  map_records(pr, a, stream, map, codes, status, (int64_t)(blockIdx.x - nb) * blockDim.x + threadIdx.x,
+              (int64_t)(gridDim.x - nb) * blockDim.x);
 }
 
 template <typename TI, typename TO, int G>
@@ -578,9 +579,12 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     a.n_mod = 0;
     a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
     const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
-    const int64_t gx = std::max<int64_t>({(int64_t)1, (int64_t)(pr.S + 7) / 8,
-                                           std::min<int64_t>((work + 255) / 256, 1 << 20)});
-    prep_kernel<<<dim3((unsigned)gx, 2), 256, 0, st>>>(pr, a, stream, masks, map, codes, status);
+    int dev = 0, nsm = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    const int nb = (pr.S + 7) / 8;  // mask blocks, then record blocks (grid-stride)
+    const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, nsm));
+    prep_kernel<<<(unsigned)(nb + nr), 256, 0, st>>>(pr, a, stream, masks, map, codes, status, nb);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
