@@ -30,6 +30,10 @@ bool use_c64p4(const Prm& pr) {
   return pr.C == 64 && pr.P == 4 && pr.variant == AWSRC_VARIANT_U;
 }
 
+bool use_c64p4_pf(const Prm& pr) {
+  return pr.C == 64 && pr.P == 4 && pr.variant == AWSRC_VARIANT_PF;
+}
+
 awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mods, bool encoder,
                            int64_t* T_out) {
   if (n_mod < 1 || mods == nullptr) return AWSRC_ERR_INVALID_ARG;
@@ -52,15 +56,17 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
 }
 
 struct EncodeLayout {
-  size_t masks, gram, pairs, mexp, partials, total;
+  size_t masks, gram, pairs, mexp, ptab, partials, total;
   int nsplit;
-  bool spec;
+  bool spec;     // U, C = 64, P = 4: tcgen05 search
+  bool spec_pf;  // P_F, C = 64, P = 4: tcgen05 search
 };
 
 EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mods, int64_t T) {
   EncodeLayout L{};
   L.spec = use_c64p4(pr);
-  const int rb = L.spec ? search_c64p4_rows() : generic_rows();
+  L.spec_pf = use_c64p4_pf(pr);
+  const int rb = (L.spec || L.spec_pf) ? search_c64p4_rows() : generic_rows();
   int64_t base_blocks = 0, ncb = 0;
   for (int m = 0; m < n_mod; ++m) {
     const int64_t n_cb = mods[m].cols / pr.C;
@@ -68,7 +74,8 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
     base_blocks += n_cb * ((mods[m].rows + rb - 1) / rb);
   }
   const int64_t units = L.spec ? pr.S_pad / search_c64p4_chunk()
-                               : (pr.S + generic_chunk() - 1) / generic_chunk();
+                       : L.spec_pf ? pr.S_pad / search_pf_c64p4_chunk()
+                                   : (pr.S + generic_chunk() - 1) / generic_chunk();
   int64_t ns = (kTargetBlocks + base_blocks - 1) / base_blocks;
   ns = std::max<int64_t>(1, std::min<int64_t>(ns, units));
   L.nsplit = (int)ns;
@@ -80,7 +87,9 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   L.pairs = off;
   if (L.spec) off += align_up((size_t)ncb * (pr.S_pad / 2) * pair_stride(pr.P) * 8, 256);
   L.mexp = off;
-  if (L.spec) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
+  if (L.spec || L.spec_pf) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
+  L.ptab = off;
+  if (L.spec_pf) off += align_up(search_pf_c64p4_table_bytes(pr.S_pad), 256);
   L.partials = off;
   off += align_up((size_t)L.nsplit * T * 8, 256);
   L.total = off;
@@ -238,9 +247,12 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   if (e != cudaSuccess) return cuda_fail(e, "encode: clear status");
   e = launch_gen_basis(pr, masks, pr.S_pad, st);
   if (e != cudaSuccess) return cuda_fail(e, "encode: gen_basis");
-  if (lay.spec && (e = launch_bfrag_c64p4(pr, masks, mexp, st)) != cudaSuccess)
-    return cuda_fail(e, "encode: atom fragments");
-  const int rb = lay.spec ? search_c64p4_rows() : generic_rows();
+  void* ptab = ws + lay.ptab;
+  if ((lay.spec || lay.spec_pf) && (e = launch_bfrag_c64p4(pr, masks, mexp, st)) != cudaSuccess)
+    return cuda_fail(e, "encode: atom table");
+  if (lay.spec_pf && (e = launch_products_pf_c64p4(pr, masks, ptab, st)) != cudaSuccess)
+    return cuda_fail(e, "encode: atom product table");
+  const int rb = (lay.spec || lay.spec_pf) ? search_c64p4_rows() : generic_rows();
   int64_t tile_off = 0, gram_off = 0;
   for (int g0 = 0; g0 < n_mod; g0 += kMaxModsPerLaunch) {
     LaunchDesc ld;
@@ -269,6 +281,7 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
     if (g0 == 0 && g_ev_before && (e = cudaEventRecord(g_ev_before, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
     if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, pairs, blocks, partials, status, st);
+    else if (lay.spec_pf) e = launch_search_pf_c64p4(pr, ld, mexp, ptab, blocks, partials, status, st);
     else e = launch_search_generic(pr, ld, masks, gram, blocks, partials, st);
     if (e != cudaSuccess) return cuda_fail(e, "encode: search");
     if (g0 + kMaxModsPerLaunch >= n_mod && g_ev_after && (e = cudaEventRecord(g_ev_after, st)) != cudaSuccess)

@@ -47,6 +47,13 @@ cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void*
                                 uint32_t* status, cudaStream_t st);
 int search_c64p4_rows();   // rows per block of the specialised kernel
 int search_c64p4_chunk();  // seeds per chunk of the specialised kernel
+// search_pf_c64p4.cu: P_F with C = 64, P = 4 on tcgen05 (atoms from the table
+// above, plus a table of atom products), same partials layout.
+int search_pf_c64p4_chunk();
+size_t search_pf_c64p4_table_bytes(int S_pad);
+cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
+cudaError_t launch_search_pf_c64p4(const Prm& pr, const LaunchDesc& ld, const void* atoms, const void* prods,
+                                   int64_t n_blocks, float2* partials, uint32_t* status, cudaStream_t st);
 
 // select.cu
 struct SelectPlan {

@@ -1,0 +1,421 @@
+// search_pf_c64p4.cu — seed search (Sec. 3.2) for AWSRC-P_F with C = 64, P = 4
+// on the tcgen05 tensor cores.
+//
+// P_F weights every element (d_ij = w_act a_j + w_fisher F_ij), so the Gram
+// matrix G = B_s^T D B_s / C differs per (tile, seed): its off-diagonal entries
+// are the +-1 correlations of the tile's D with the pairwise products
+// m_p * m_q of the seed's atoms, and its diagonal is the tile's gd. Both the
+// correlations b_p (with y = d r) and the six off-diagonals are exact integer
+// sums on the tile's fixed-point grids (|Y|, |D| <= 2^21, FP16 halves
+// hi = X >> 11, lo = X & 2047), computed by tcgen05.mma and rounded once in the
+// epilogue, which then factors G + eps I (LDL^T), solves, quantises and scores
+// every candidate exactly as the binary32 recipe does.
+//
+// Block: 128 tiles of one column block (row m = TMEM lane m), 17 warps. The
+// producer warp streams 8-seed chunks (FP16 atoms 4 KB, a slice of the U
+// search's atom table, and FP16 atom products 6 KB) through a 4-stage
+// bulk-copy ring and issues per chunk 16 MMAs into one of two TMEM
+// accumulators: Y_hi, Y_lo x atoms (N = 32) and D_hi, D_lo x products (N = 48).
+// Epilogue warp w takes TMEM lanes 32(w%4).. and seed pair w/4 of each chunk,
+// as a float2 stream over the pair's two seeds. Every mbarrier wait is bounded.
+#include "internal.h"
+#include "tc05.cuh"
+
+namespace awsrc {
+
+namespace {
+
+using namespace tc05;
+
+constexpr int BM = 128;             // rows (tiles) per block = TMEM lanes
+constexpr int CH = 8;               // seeds per chunk
+constexpr int NA = 4 * CH;          // atom columns per chunk
+constexpr int NQ = 6 * CH;          // product columns per chunk
+constexpr int EW = 16;              // epilogue warps: 4 lane quarters x 4 seed pairs
+constexpr int NT = 32 * (EW + 1);
+constexpr int STAGES = 4;
+constexpr uint32_t kABytes = NA * 64 * 2;      // 4 KB
+constexpr uint32_t kQBytes = NQ * 64 * 2;      // 6 KB
+constexpr uint32_t kStageBytes = kABytes + kQBytes;
+constexpr uint32_t kTmemCols = 512;            // 2 accumulators of 256 columns
+constexpr int kYH = 0, kYL = 32, kDH = 64, kDL = 112;  // columns within an accumulator
+constexpr uint32_t kIdA = idesc_f16(BM, NA);
+constexpr uint32_t kIdQ = idesc_f16(BM, NQ);
+static_assert(EW / 4 == CH / 2, "one seed pair per epilogue warp and chunk");
+
+struct Smem {
+  __half A[4][BM * 64];  // Y_hi, Y_lo, D_hi, D_lo: canonical K-major, no swizzle
+  unsigned char stage[STAGES][kStageBytes];
+  float Yst[BM][65];
+  float Dst[BM][65];
+  float tqc[BM];      // 2^qy * c
+  float tqdc[BM];     // 2^qd * c2
+  float gd[BM];       // G_pp
+  float diag[BM];     // fl(gd + eps)
+  float invd0[BM];    // 1 / D_0 = 1 / diag
+  float inv_qy[BM], inv_qd[BM];
+  int rowok[BM];
+  float red_g[4][BM];
+  uint32_t red_s[4][BM];
+  unsigned long long full[STAGES], afull[2], tempty[2];
+  uint32_t tmem_base;
+};
+
+__device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
+
+__device__ __forceinline__ int a_offset(int m, int k) {
+  return (((m >> 3) * 8 + (k >> 3)) << 7) + ((m & 7) << 4) + ((k & 7) << 1);
+}
+
+// Exact sums RN(2048*hi + lo) of two seeds, scaled by a power of two.
+__device__ __forceinline__ float2 pair_sum(const float* hi, const float* lo, int i, float2 scale) {
+  const float2 u = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[i], hi[i + 1]),
+                              make_float2(lo[i], lo[i + 1]));
+  return __fmul2_rn(u, scale);
+}
+
+__device__ __forceinline__ float2 neg2(float2 v) { return make_float2(-v.x, -v.y); }
+
+__device__ __forceinline__ bool pivot_ok(float d) { return d > 0.0f && d <= 3.402823466e38f; }
+
+// Gains of one seed pair of this thread's row; ah/al: atom p of the two seeds
+// at [2p], [2p+1]; qh/ql: product q (tri order) at [2q], [2q+1].
+template <bool FAST>
+__device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, const float* al, const float* qh,
+                                               const float* ql, float tqc, float tqdc, float gd, float diag,
+                                               float invd0) {
+  const float2 tq2 = make_float2(tqc, tqc), td2 = make_float2(tqdc, tqdc);
+  float2 bv[4], G[6];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) bv[p] = pair_sum(ah, al, 2 * p, tq2);
+#pragma unroll
+  for (int q = 0; q < 6; ++q) G[q] = pair_sum(qh, ql, 2 * q, td2);
+  // LDL^T of G + eps I in the recipe's order; D_0 = diag for every seed
+  const float2 dg = make_float2(diag, diag);
+  float2 nL[6], E[6], invD[4];
+  invD[0] = make_float2(invd0, invd0);
+  bool okx = true, oky = true;
+#pragma unroll
+  for (int k = 1; k < 4; ++k) {
+#pragma unroll
+    for (int j = 0; j < k; ++j) {
+      float2 v = G[tri(k, j)];
+#pragma unroll
+      for (int i = 0; i < j; ++i) v = __ffma2_rn(nL[tri(k, i)], E[tri(j, i)], v);
+      E[tri(k, j)] = v;
+      nL[tri(k, j)] = __fmul2_rn(v, neg2(invD[j]));  // -(v * invD_j), exact negation
+    }
+    float2 dk = dg;
+#pragma unroll
+    for (int i = 0; i < k; ++i) dk = __ffma2_rn(nL[tri(k, i)], E[tri(k, i)], dk);
+    okx = okx && pivot_ok(dk.x);
+    oky = oky && pivot_ok(dk.y);
+    invD[k] = make_float2(__frcp_rn(dk.x), __frcp_rn(dk.y));
+  }
+  float2 alpha[4];
+  ldl_solve2<4>(nL, invD, bv, alpha);
+  float2 g;
+  if constexpr (FAST) {
+    float2 G2[6];
+#pragma unroll
+    for (int q = 0; q < 6; ++q) G2[q] = __fmul2_rn(G[q], make_float2(2.0f, 2.0f));  // exact
+    g = quant_gain_fast2<4>(pr, alpha, bv, make_float2(gd, gd), G2);
+  } else {
+    float q4[4];
+    int sf;
+    float Gx[6], a[4], b[4];
+#pragma unroll
+    for (int i = 0; i < 6; ++i) Gx[i] = G[i].x;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].x; b[p] = bv[p].x; }
+    g.x = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
+#pragma unroll
+    for (int i = 0; i < 6; ++i) Gx[i] = G[i].y;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].y; b[p] = bv[p].y; }
+    g.y = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
+  }
+  if (!okx) g.x = neg_inf();
+  if (!oky) g.y = neg_inf();
+  return g;
+}
+
+template <bool FAST>
+__global__ void __launch_bounds__(NT, 1)
+    search_pf_kernel(Prm pr, LaunchDesc ld, const unsigned char* __restrict__ atoms,
+                     const unsigned char* __restrict__ prods, float2* __restrict__ partials,
+                     uint32_t* __restrict__ status) {
+  extern __shared__ unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int mi = find_mod(ld, blockIdx.x);
+  const ModDesc& md = ld.m[mi];
+  const int64_t b = blockIdx.x - md.block_off;
+  const int z = (int)(b % md.nsplit);
+  const int64_t rest = b / md.nsplit;
+  const int64_t rb = rest % md.n_rb;
+  const int64_t cb = rest / md.n_rb;
+
+  const int nchunks = pr.S_pad / CH;
+  const int per = (nchunks + md.nsplit - 1) / md.nsplit;
+  const int c0 = min(nchunks, z * per);
+  const int c1 = min(nchunks, c0 + per);
+  const int nck = c1 - c0;
+  const unsigned char* a_src = atoms + (size_t)c0 * kABytes;
+  const unsigned char* q_src = prods + (size_t)c0 * kQBytes;
+
+  if (warp == EW) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_addr(&sm.tmem_base)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if (lane == 0) {
+      for (int i = 0; i < STAGES; ++i) mbar_init(&sm.full[i], 1);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&sm.afull[i], 1);
+        mbar_init(&sm.tempty[i], EW);
+      }
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    tc_fence_before();
+  }
+  if (tid < BM) sm.rowok[tid] = 1;
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  int issued = 0;
+  if (warp == EW && lane == 0) {
+    for (; issued < STAGES && issued < nck; ++issued) {
+      mbar_expect_tx(&sm.full[issued], kStageBytes);
+      bulk_g2s(&sm.stage[issued][0], a_src + (size_t)issued * kABytes, kABytes, &sm.full[issued]);
+      bulk_g2s(&sm.stage[issued][kABytes], q_src + (size_t)issued * kQBytes, kQBytes, &sm.full[issued]);
+    }
+  }
+  // stage y = d * r and d, d = w_act * a + w_fisher * F (per element)
+  for (int e = tid; e < BM * 64; e += NT) {
+    const int r = e >> 6, j = e & 63;
+    const int64_t row = rb * BM + r;
+    float y = 0.0f, d = 0.0f;
+    if (row < md.rows) {
+      const int64_t idx = row * md.cols + cb * 64 + j;
+      const float rr = __fsub_rn(load_elem(md.W, idx, md.w_dtype), load_elem(md.W0, idx, md.w0_dtype));
+      d = __fadd_rn(__fmul_rn(md.w_act, md.act[cb * 64 + j]), __fmul_rn(md.w_fisher, md.fisher[idx]));
+      if (!in_domain(rr, d)) sm.rowok[r] = 0;
+      y = __fmul_rn(d, rr);
+    }
+    sm.Yst[r][j] = y;
+    sm.Dst[r][j] = d;
+  }
+  __syncthreads();
+  if (tid < BM) {  // per row: fixed-point exponents, gd, eps and the first pivot
+    float my = 0.0f, mdd = 0.0f;
+    for (int j = 0; j < 64; ++j) {
+      my = fmaxf(my, fabsf(sm.Yst[tid][j]));
+      mdd = fmaxf(mdd, fabsf(sm.Dst[tid][j]));
+    }
+    int qy, qd;
+    const float iy = fixed_point_inv(my, &qy);
+    const float idd = fixed_point_inv(mdd, &qd);
+    const float two_qd = pow2f(qd);
+    int sd = 0;
+    for (int j = 0; j < 64; ++j) sd += idd == 0.0f ? 0 : fixed_point_int(sm.Dst[tid][j], idd);
+    const float gd = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(sd), two_qd));
+    const float eps = __fmul_rn(pr.ridge_rel, gd);
+    const float diag = __fadd_rn(gd, eps);
+    const bool ok = sm.rowok[tid] && pivot_ok(diag);
+    sm.rowok[tid] = ok ? 1 : 0;
+    sm.inv_qy[tid] = ok ? iy : 0.0f;
+    sm.inv_qd[tid] = ok ? idd : 0.0f;
+    sm.tqc[tid] = __fmul_rn(pow2f(qy), pr.c);
+    sm.tqdc[tid] = __fmul_rn(two_qd, pr.c2);
+    sm.gd[tid] = gd;
+    sm.diag[tid] = diag;
+    sm.invd0[tid] = __frcp_rn(diag);
+  }
+  __syncthreads();
+  // A operands: one thread writes one 16-byte core-matrix row of both halves
+  for (int e = tid; e < 2 * BM * 8; e += NT) {
+    const int which = e >= BM * 8;  // 0: Y, 1: D
+    const int ee = e - which * BM * 8;
+    const int m = ee >> 3, k0 = (ee & 7) * 8;
+    const float inv = which ? sm.inv_qd[m] : sm.inv_qy[m];
+    const float* src = which ? &sm.Dst[m][k0] : &sm.Yst[m][k0];
+    uint32_t wh[4], wl[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int x0 = inv == 0.0f ? 0 : fixed_point_int(src[2 * i], inv);
+      const int x1 = inv == 0.0f ? 0 : fixed_point_int(src[2 * i + 1], inv);
+      wh[i] = (uint32_t)__half_as_ushort(__int2half_rn(x0 >> 11)) |
+              ((uint32_t)__half_as_ushort(__int2half_rn(x1 >> 11)) << 16);
+      wl[i] = (uint32_t)__half_as_ushort(__int2half_rn(x0 & 2047)) |
+              ((uint32_t)__half_as_ushort(__int2half_rn(x1 & 2047)) << 16);
+    }
+    const int off = a_offset(m, k0);
+    *reinterpret_cast<uint4*>(reinterpret_cast<unsigned char*>(sm.A[2 * which]) + off) =
+        make_uint4(wh[0], wh[1], wh[2], wh[3]);
+    *reinterpret_cast<uint4*>(reinterpret_cast<unsigned char*>(sm.A[2 * which + 1]) + off) =
+        make_uint4(wl[0], wl[1], wl[2], wl[3]);
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  __syncthreads();
+
+  bool timed_out = false;
+  if (warp == EW) {
+    // ------------------------------------------------------------ producer --
+    if (lane == 0) {
+      uint32_t ab[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ab[i] = smem_addr(sm.A[i]);
+      int k = 0;
+      for (; k < nck; ++k) {
+        const int st = k % STAGES, tb = k & 1;
+        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
+        if (k >= 2 && !mbar_wait(&sm.tempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
+        tc_fence_after();
+        const uint32_t sa = smem_addr(&sm.stage[st][0]), sq = sa + kABytes;
+        const uint32_t acc = tmem + (uint32_t)(tb * 256);
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+          const uint32_t kb = (uint32_t)ks * 256u, en = ks > 0 ? 1u : 0u;
+          umma_f16(acc + kYH, smem_desc(ab[0] + kb), smem_desc(sa + kb), kIdA, en);
+          umma_f16(acc + kYL, smem_desc(ab[1] + kb), smem_desc(sa + kb), kIdA, en);
+          umma_f16(acc + kDH, smem_desc(ab[2] + kb), smem_desc(sq + kb), kIdQ, en);
+          umma_f16(acc + kDL, smem_desc(ab[3] + kb), smem_desc(sq + kb), kIdQ, en);
+        }
+        umma_commit(&sm.afull[tb]);
+        if (k >= 2 && issued < nck) {
+          // chunk k+2 takes the stage of chunk k-2, whose MMAs completed before
+          // its accumulator was loaded (tempty above)
+          const int ps = (k - 2) % STAGES;
+          mbar_expect_tx(&sm.full[ps], kStageBytes);
+          bulk_g2s(&sm.stage[ps][0], a_src + (size_t)issued * kABytes, kABytes, &sm.full[ps]);
+          bulk_g2s(&sm.stage[ps][kABytes], q_src + (size_t)issued * kQBytes, kQBytes, &sm.full[ps]);
+          ++issued;
+        }
+      }
+      if (timed_out) {
+        for (int j = max(0, issued - STAGES); j < issued; ++j)
+          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
+        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue --
+    const int m = 32 * (warp & 3) + lane;
+    const int pi = warp >> 2;  // seed pair of each chunk
+    const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
+    const float tqc = sm.tqc[m], tqdc = sm.tqdc[m], gd = sm.gd[m], diag = sm.diag[m], invd0 = sm.invd0[m];
+    float bg = neg_inf();
+    uint32_t bsd = 0xffffffffu;
+    for (int k = 0; k < nck; ++k) {
+      const int tb = k & 1;
+      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1))) { timed_out = true; break; }
+      tc_fence_after();
+      const uint32_t base = tmem + lane_base + (uint32_t)(tb * 256);
+      float ah[8], al[8], qh[12], ql[12];
+      tmem_ld4(base + kYH + 8 * pi, ah);
+      tmem_ld4(base + kYH + 8 * pi + 4, ah + 4);
+      tmem_ld4(base + kYL + 8 * pi, al);
+      tmem_ld4(base + kYL + 8 * pi + 4, al + 4);
+#pragma unroll
+      for (int i = 0; i < 3; ++i) {
+        tmem_ld4(base + kDH + 12 * pi + 4 * i, qh + 4 * i);
+        tmem_ld4(base + kDL + 12 * pi + 4 * i, ql + 4 * i);
+      }
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      tmem_tie4(ah); tmem_tie4(ah + 4); tmem_tie4(al); tmem_tie4(al + 4);
+#pragma unroll
+      for (int i = 0; i < 3; ++i) { tmem_tie4(qh + 4 * i); tmem_tie4(ql + 4 * i); }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.tempty[tb]);
+      const float2 g = pf_pair_gain<FAST>(pr, ah, al, qh, ql, tqc, tqdc, gd, diag, invd0);
+      // seeds reach a thread in increasing order: a strictly greater gain wins
+      const float cm = fmaxf(g.x, g.y);
+      if (cm > bg) {
+        bg = cm;
+        bsd = (uint32_t)((c0 + k) * CH + 2 * pi + (g.x == cm ? 0 : 1));
+      }
+    }
+    sm.red_g[pi][m] = bg;
+    sm.red_s[pi][m] = bsd;
+  }
+  tc_fence_before();
+  if (__syncthreads_or(timed_out)) {
+    if (tid == 0) atomicOr(status, kFaultTimeout);
+  } else if (tid < BM) {
+    float g = sm.red_g[0][tid];
+    uint32_t s = sm.red_s[0][tid];
+#pragma unroll
+    for (int i = 1; i < 4; ++i) {
+      if (better(sm.red_g[i][tid], sm.red_s[i][tid], g, s)) { g = sm.red_g[i][tid]; s = sm.red_s[i][tid]; }
+    }
+    const int64_t row = rb * BM + tid;
+    if (row < md.rows) {
+      const int64_t tt = md.tile_off + row * md.n_cb + cb;
+      partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[tid] ? g : neg_inf(), __uint_as_float(s));
+    }
+  }
+  if (warp == EW) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+// FP16 products of atom pairs in the order the MMAs read them: chunk c
+// (8 seeds) is a 48 x 64 K-major operand in 6 KB; item i (16 bytes, one
+// core-matrix row) is chunk i / 384, column group n8 = (i >> 6) % 6, k group
+// (i >> 3) & 7, row i & 7; column n = 8*n8 + r carries product q = (n % 12) / 2
+// (pairs (1,0), (2,0), (2,1), (3,0), (3,1), (3,2)) of seed 8c + 2*(n / 12) + n % 2.
+__global__ void products_kernel(const uint64_t* __restrict__ masks, uint4* __restrict__ out, int S_pad) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t n_items = (int64_t)(S_pad / CH) * 384;
+  if (i >= n_items) return;
+  const int64_t chunk = i / 384;
+  const int w = (int)(i % 384);
+  const int r = w & 7, kg = (w >> 3) & 7, n8 = w >> 6;
+  const int n = 8 * n8 + r;
+  const int q = (n % 12) >> 1;
+  const int64_t seed = chunk * CH + 2 * (n / 12) + (n & 1);
+  const int pa = q < 1 ? 1 : (q < 3 ? 2 : 3);
+  const int pb = q - (pa * (pa - 1)) / 2;
+  const uint64_t m = masks[(size_t)seed * 4 + pa] ^ masks[(size_t)seed * 4 + pb];
+  uint32_t wv[4];
+#pragma unroll
+  for (int h = 0; h < 4; ++h) {
+    const int k = 8 * kg + 2 * h;
+    const uint32_t lo = ((m >> k) & 1ull) ? 0xBC00u : 0x3C00u;  // -1 : +1 in FP16
+    const uint32_t hi = ((m >> (k + 1)) & 1ull) ? 0xBC00u : 0x3C00u;
+    wv[h] = lo | (hi << 16);
+  }
+  out[i] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+}
+
+}  // namespace
+
+int search_pf_c64p4_chunk() { return CH; }
+size_t search_pf_c64p4_table_bytes(int S_pad) { return (size_t)(S_pad / CH) * kQBytes; }
+
+cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st) {
+  const int64_t n = (int64_t)(pr.S_pad / CH) * 384;
+  products_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(masks, static_cast<uint4*>(out), pr.S_pad);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_search_pf_c64p4(const Prm& pr, const LaunchDesc& ld, const void* atoms, const void* prods,
+                                   int64_t n_blocks, float2* partials, uint32_t* status, cudaStream_t st) {
+  const size_t smem = sizeof(Smem) + 1024;
+  auto kern = pr.fast_pow2 ? search_pf_kernel<true> : search_pf_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const unsigned char*>(atoms),
+                                             static_cast<const unsigned char*>(prods), partials, status);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace awsrc
