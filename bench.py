@@ -45,8 +45,8 @@ OPS_PER_CANDIDATE = 8 + 6 + 4 + 4 + 1
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "447e4f1a3e58f2d5ba2d9459b3199876759aa34ece504147a161a626f0b2d723",
-                  "bytes_per_launch": 418617088 + 8241152}
+SEARCH_TRAFFIC = {"source_sha256": "eb3c0657891a1ae9405bc97349a5771be0d62e110b29fc534ad6a15f4cb2340b",
+                  "bytes_per_launch": 419272704 + 8250880}
 
 
 def parse():
@@ -59,6 +59,7 @@ def parse():
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-pf", action="store_true", help="skip the P_F encode measurement")
     ap.add_argument("--modules", default="",
                     help="comma-separated subset of the layer's modules (profiling runs only)")
     return ap.parse_args()
@@ -375,6 +376,31 @@ def run_ours(args):
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": 1e3 * dt / args.steps}
 
+    # the P_F variant of the search on one Qwen2.5-7B-shaped layer (blended
+    # activation/Fisher weights), timed on the device outside the step
+    pf = None
+    if rank == 0 and not args.no_pf and not args.modules:
+        wl7 = WORKLOADS["qwen2.5-7b_stack_pf"]
+        m7 = make_layer(wl7, layer=0, device=dev)
+        p7 = aw.params(C=wl7.C, P=wl7.P, b=wl7.b, S=wl7.S, variant=1)
+        c7 = aw.awsrc_encode_tiles(p7, m7)
+        ws7 = c7._awsrc_workspace
+        torch.cuda.synchronize()
+        e7 = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        reps = 3
+        e7[0].record()
+        for _ in range(reps):
+            aw.awsrc_encode_tiles(p7, m7, out=c7, workspace=ws7)
+        e7[1].record()
+        torch.cuda.synchronize()
+        assert aw.awsrc_workspace_status(ws7) == 0, "P_F encoder self-check fault"
+        ms7 = e7[0].elapsed_time(e7[1]) / reps
+        T7 = wl7.tiles_per_layer
+        pf = {"workload": "one Qwen2.5-7B-shaped layer (7 modules, 233,046,016 weights) BF16, "
+                          "AWSRC-P_F 0.5/0.5 activation/Fisher blend, C=64 P=4 b=4 S=4096",
+              "encode_ms": ms7, "candidates_per_s": T7 * wl7.S / (ms7 * 1e-3)}
+        del m7, c7, ws7
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, cores, desc = oracle_sample(wl, host_modules(mods), args.cpu_seconds)
@@ -395,7 +421,7 @@ def run_ours(args):
             "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf,
             "gpu_launches": launches, "clocks": clk.summary(),
         }
         print(json.dumps(line), flush=True)
