@@ -11,22 +11,20 @@
 
 namespace awsrc {
 
-constexpr int kBasisWarps = 4;  // seeds per block of the stand-alone kernel
+constexpr int kBasisWarps = 4;  // warps per block of the stand-alone kernel
 
 __global__ void __launch_bounds__(32 * kBasisWarps) gen_basis_kernel(Prm pr, uint64_t* __restrict__ masks,
                                                                      int S_out) {
-  __shared__ uint8_t perm_s[kBasisWarps][kMaxC];
-  __shared__ uint8_t kidx_s[kBasisWarps][kMaxC];
-  __shared__ uint8_t pool_s[kBasisWarps][kMaxC];
-  __shared__ int cols_s[kBasisWarps][kMaxP];
+  __shared__ __align__(16) uint8_t smem[kBasisWarps][kBasisWarp4Smem];
   const int warp = threadIdx.x >> 5;
-  const int s = blockIdx.x * kBasisWarps + warp;
-  if (s >= S_out) return;  // whole warp leaves together
-  basis_warp(pr, masks, s, perm_s[warp], kidx_s[warp], pool_s[warp], cols_s[warp]);
+  const int s0 = (blockIdx.x * kBasisWarps + warp) * kWarpSeeds;
+  if (s0 >= S_out) return;  // whole warp leaves together
+  basis_warp4(pr, masks, s0, S_out, smem[warp]);
 }
 
 cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st) {
-  gen_basis_kernel<<<(S_out + kBasisWarps - 1) / kBasisWarps, 32 * kBasisWarps, 0, st>>>(pr, masks, S_out);
+  const int per = kBasisWarps * kWarpSeeds;
+  gen_basis_kernel<<<(S_out + per - 1) / per, 32 * kBasisWarps, 0, st>>>(pr, masks, S_out);
   note_launches(1);
   return cudaGetLastError();
 }
