@@ -330,8 +330,9 @@ awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t
  * flags describe the last call made with this workspace; 0 means no fault.
  * Bit 0 (1): a record named a tile or seed out of range (decoder; skipped), or
  *            a tile a second time (dense decoder).
- * Bit 1 (2): encoder self-check — the finalisation recomputed a different gain
- *            than the search found (never expected).
+ * Bit 1 (2): encoder self-check — recomputing the winning candidate of a tile
+ *            (for its codes) gave a different gain than the search found
+ *            (never expected).
  * Bit 2 (4): a bounded wait inside a kernel gave up (never expected).
  */
 awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags);

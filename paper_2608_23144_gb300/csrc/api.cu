@@ -56,7 +56,7 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
 }
 
 struct EncodeLayout {
-  size_t masks, gram, pairs, mexp, ptab, partials, total;
+  size_t masks, gram, pairs, mexp, ptab, partials, pcands, total;
   int nsplit;
   bool spec;     // U, C = 64, P = 4: tcgen05 search
   bool spec_pf;  // P_F, C = 64, P = 4: tcgen05 search
@@ -82,16 +82,20 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   size_t off = kStatusBytes;
   L.masks = off;
   off += align_up((size_t)pr.S_pad * pr.P * pr.W * 8, 256);
-  L.gram = off;
-  if (pr.variant == AWSRC_VARIANT_U) off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
+  L.gram = off;  // read by the finalisation pass of the other search paths
+  if (pr.variant == AWSRC_VARIANT_U && !L.spec)
+    off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
   L.pairs = off;
   if (L.spec) off += align_up((size_t)ncb * (pr.S_pad / 2) * pair_stride(pr.P) * 8, 256);
   L.mexp = off;
   if (L.spec || L.spec_pf) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
   L.ptab = off;
   if (L.spec_pf) off += align_up(search_pf_c64p4_table_bytes(pr.S_pad), 256);
-  L.partials = off;
-  off += align_up((size_t)L.nsplit * T * 8, 256);
+  const bool whole = L.spec || L.spec_pf;  // the search writes whole candidates
+  L.partials = off;  // (gain, seed) per tile and split, for the finalisation pass
+  if (!whole) off += align_up((size_t)L.nsplit * T * 8, 256);
+  L.pcands = off;    // whole candidates per tile and split, merged when nsplit > 1
+  if (whole && L.nsplit > 1) off += align_up((size_t)L.nsplit * T * sizeof(awsrc_candidate), 256);
   L.total = off;
   return L;
 }
@@ -239,7 +243,8 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   uint32_t* status = reinterpret_cast<uint32_t*>(ws);
   uint64_t* masks = reinterpret_cast<uint64_t*>(ws + lay.masks);
-  float* gram = reinterpret_cast<float*>(ws + lay.gram);
+  float* gram = lay.spec ? nullptr : reinterpret_cast<float*>(ws + lay.gram);
+  awsrc_candidate* pcands = lay.nsplit > 1 ? reinterpret_cast<awsrc_candidate*>(ws + lay.pcands) : out;
   float2* pairs = lay.spec ? reinterpret_cast<float2*>(ws + lay.pairs) : nullptr;
   void* mexp = ws + lay.mexp;
   float2* partials = reinterpret_cast<float2*>(ws + lay.partials);
@@ -280,14 +285,22 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
       return cuda_fail(e, "encode: gram");
     if (g0 == 0 && g_ev_before && (e = cudaEventRecord(g_ev_before, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
-    if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, pairs, blocks, partials, status, st);
-    else if (lay.spec_pf) e = launch_search_pf_c64p4(pr, ld, mexp, ptab, blocks, partials, status, st);
+    if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, pairs, masks, blocks, pcands, status, st);
+    else if (lay.spec_pf) e = launch_search_pf_c64p4(pr, ld, mexp, ptab, masks, blocks, pcands, status, st);
     else e = launch_search_generic(pr, ld, masks, gram, blocks, partials, st);
     if (e != cudaSuccess) return cuda_fail(e, "encode: search");
     if (g0 + kMaxModsPerLaunch >= n_mod && g_ev_after && (e = cudaEventRecord(g_ev_after, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
-    if ((e = launch_finalize(pr, ld, masks, gram, partials, lay.nsplit, out, status, st)) != cudaSuccess)
+    if (lay.spec || lay.spec_pf) {  // the search wrote whole candidates
+      if (lay.nsplit > 1) {
+        const int64_t t0 = ld.m[0].tile_off;
+        const int64_t t1 = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
+        if ((e = launch_merge_candidates(pcands, lay.nsplit, T, t0, t1, out, st)) != cudaSuccess)
+          return cuda_fail(e, "encode: merge");
+      }
+    } else if ((e = launch_finalize(pr, ld, masks, gram, partials, lay.nsplit, out, status, st)) != cudaSuccess) {
       return cuda_fail(e, "encode: finalize");
+    }
   }
   return AWSRC_OK;
 }

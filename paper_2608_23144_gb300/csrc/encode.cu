@@ -142,15 +142,17 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   const float eps = __fmul_rn(pr.ridge_rel, gd);
   bool ok = ldl_factor<P>(gd, eps, Goff, L, invD);
   ok = ok && dok && (s < pr.S);
-  float* out = gram + (size_t)(md.gram_off + cb * pr.S_pad + s) * gram_stride(P);
   const float qnan = __int_as_float(0x7fc00000);
+  if (gram) {
+    float* out = gram + (size_t)(md.gram_off + cb * pr.S_pad + s) * gram_stride(P);
 #pragma unroll
-  for (int i = 0; i < P * (P - 1) / 2; ++i) out[i] = L[i];
+    for (int i = 0; i < P * (P - 1) / 2; ++i) out[i] = L[i];
 #pragma unroll
-  for (int k = 0; k < P; ++k) out[P * (P - 1) / 2 + k] = ok ? invD[k] : qnan;
+    for (int k = 0; k < P; ++k) out[P * (P - 1) / 2 + k] = ok ? invD[k] : qnan;
 #pragma unroll
-  for (int i = 0; i < P * (P - 1) / 2; ++i) out[P * (P - 1) / 2 + P + i] = Goff[i];
-  out[P * (P - 1) + P] = gd;
+    for (int i = 0; i < P * (P - 1) / 2; ++i) out[P * (P - 1) / 2 + P + i] = Goff[i];
+    out[P * (P - 1) + P] = gd;
+  }
   if (pairs) {
     // seed s is component s & 1 of seed pair s >> 1 (entries start on even seeds)
     float* po = reinterpret_cast<float*>(pairs) +

@@ -42,9 +42,14 @@ cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t*
 // FP16 table of the +-1 atoms in MMA operand order, then the tcgen05 search.
 size_t search_c64p4_table_bytes(int S_pad);
 cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
+// Writes each tile's best candidate (codes included) to cands[z * T + t] for
+// seed split z; launch_merge_candidates reduces the splits of tiles [t0, t1).
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
-                                const float2* pairs, int64_t n_blocks, float2* partials,
+                                const float2* pairs, const uint64_t* masks, int64_t n_blocks,
+                                awsrc_candidate* cands,
                                 uint32_t* status, cudaStream_t st);
+cudaError_t launch_merge_candidates(const awsrc_candidate* pc, int nsplit, int64_t T, int64_t t0, int64_t t1,
+                                   awsrc_candidate* out, cudaStream_t st);
 int search_c64p4_rows();   // rows per block of the specialised kernel
 int search_c64p4_chunk();  // seeds per chunk of the specialised kernel
 // search_pf_c64p4.cu: P_F with C = 64, P = 4 on tcgen05 (atoms from the table
@@ -53,7 +58,8 @@ int search_pf_c64p4_chunk();
 size_t search_pf_c64p4_table_bytes(int S_pad);
 cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
 cudaError_t launch_search_pf_c64p4(const Prm& pr, const LaunchDesc& ld, const void* atoms, const void* prods,
-                                   int64_t n_blocks, float2* partials, uint32_t* status, cudaStream_t st);
+                                   const uint64_t* masks, int64_t n_blocks, awsrc_candidate* cands,
+                                   uint32_t* status, cudaStream_t st);
 
 // select.cu
 struct SelectPlan {

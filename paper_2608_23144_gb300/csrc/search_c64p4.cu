@@ -19,7 +19,8 @@
 //  * Warps 0..15 (epilogue): warp w reads TMEM lanes 32(w%4).. (its threads'
 //    rows) and the columns of seeds 8(w/4)..8(w/4)+7 of each chunk, and runs the
 //    fit / quantise / score epilogue on seed pairs as float2 streams, keeping a
-//    running argmax per row. The four warps of a row merge at the end.
+//    running argmax per row with the winner's codes and scale. The four warps
+//    of a row merge at the end and write the tile's candidate.
 // Columns of a chunk are seed-pair major: column 8i + 2p + e holds atom p of
 // seed 2i + e, so one 32x32b.x16 TMEM load gives a thread two seed pairs with
 // each atom's two seeds in adjacent registers.
@@ -141,7 +142,6 @@ __device__ __forceinline__ void pair_back(const float4* pe, const float2* w, flo
   }
 }
 
-// Quantised gains of a fitted seed pair.
 template <bool FAST>
 __device__ __forceinline__ float2 pair_gain(const Prm& pr, const float2* bv, const float2* alpha,
                                             const float4* pe) {
@@ -175,10 +175,56 @@ __device__ __forceinline__ float2 pair_gain(const Prm& pr, const float2* bv, con
   }
 }
 
+// Codes and scale field of the winning seed of row m. The search keeps only
+// (gain, seed), so the seed's correlations are formed again here as the exact
+// integer sums sum_j +-Y_j that the tensor cores accumulate (hi/lo split so
+// that 2048*hi + lo is that sum and the fma of pair_forward rounds it once),
+// then go through the same solve and quantiser instructions as in the search.
+// The pair's other half gets the same correlations and is ignored. Returns the
+// gain once more, which must equal the one the search found.
+template <bool FAST>
+__device__ __forceinline__ float winner_codes(const Prm& pr, const Smem& sm, int m, const uint64_t* mk,
+                                              const float4* pe, bool odd, uint32_t* cw, int* sf) {
+  const float inv = sm.inv_q[m];
+  uint64_t w[4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) w[p] = mk[p];
+  int tot = 0, neg[4] = {0, 0, 0, 0};
+  for (int j = 0; j < 64; ++j) {
+    const int y = inv == 0.0f ? 0 : fixed_point_int(sm.Yst[m][j], inv);
+    tot += y;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) neg[p] += ((w[p] >> j) & 1ull) ? y : 0;
+  }
+  float hi[8], lo[8];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const int u = tot - 2 * neg[p];  // |u| <= 64 * 2^21
+    hi[2 * p] = hi[2 * p + 1] = (float)(u >> 11);
+    lo[2 * p] = lo[2 * p + 1] = (float)(u & 2047);
+  }
+  const float tq = __fmul_rn(sm.two_q[m], pr.c);
+  float2 bv[4], wv[4], al[4];
+  (void)pair_forward(hi, lo, make_float2(tq, tq), pe, bv, wv);
+  pair_back(pe, wv, al);
+  float a[4], q[4], zero[6] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+  for (int p = 0; p < 4; ++p) a[p] = odd ? al[p].y : al[p].x;
+  if constexpr (FAST) (void)quant_gain_fast<4>(pr, a, zero, 0.0f, zero, q, sf);
+  else (void)quant_gain<4>(pr, a, zero, 0.0f, zero, q, sf);
+  uint32_t c = 0u;
+#pragma unroll
+  for (int p = 0; p < 4; ++p) c |= ((uint32_t)(int)q[p] & 0xFFu) << (8 * p);
+  *cw = c;
+  const float2 g = pair_gain<FAST>(pr, bv, al, pe);
+  return odd ? g.y : g.x;
+}
+
 template <bool FAST>
 __global__ void __launch_bounds__(NT, 1)
     search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ atoms,
-                        const float2* __restrict__ pairs, float2* __restrict__ partials,
+                        const float2* __restrict__ pairs, const uint64_t* __restrict__ masks,
+                        awsrc_candidate* __restrict__ cands,
                         uint32_t* __restrict__ status) {
   extern __shared__ unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -349,7 +395,6 @@ __global__ void __launch_bounds__(NT, 1)
         for (int i = 16; i < 8 * RPAIRS; i += 16) tmem_tie(hi + i);
 #pragma unroll
         for (int i = 0; i < 8 * RPAIRS; i += 16) tmem_tie(lo + i);
-        float g[2 * RPAIRS];  // seeds 2*p0 + i of the chunk
 #pragma unroll
         for (int j = 0; j < RPAIRS; ++j) {
           const float4* pe = pbase + (p0 + j) * (PS / 2);
@@ -358,27 +403,15 @@ __global__ void __launch_bounds__(NT, 1)
           // prune: a candidate whose gain bound is below the running best
           // cannot win (NaN bounds stay live)
           const bool lx = !FAST || !(ub.x < bg), ly = !FAST || !(ub.y < bg);
-          float2 gp = make_float2(neg_inf(), neg_inf());
           if (__any_sync(0xffffffffu, lx || ly)) {
             float2 al[4];
             pair_back(pe, wv, al);
-            gp = pair_gain<FAST>(pr, bv, al, pe);
-            if (!lx) gp.x = neg_inf();
-            if (!ly) gp.y = neg_inf();
+            const float2 gp = pair_gain<FAST>(pr, bv, al, pe);
+            // running argmax in seed order: a strictly greater gain wins
+            const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * (p0 + j));
+            if (lx && gp.x > bg) { bg = gp.x; bsd = s; }
+            if (ly && gp.y > bg) { bg = gp.y; bsd = s + 1; }
           }
-          g[2 * j] = gp.x;
-          g[2 * j + 1] = gp.y;
-        }
-        // running argmax: the first of the round's maxima, if it beats the best
-        float cm = g[0];
-#pragma unroll
-        for (int i = 1; i < 2 * RPAIRS; ++i) cm = fmaxf(cm, g[i]);
-        if (cm > bg) {
-          int i = 2 * RPAIRS - 1;
-#pragma unroll
-          for (int t = 2 * RPAIRS - 2; t >= 0; --t) if (g[t] == cm) i = t;
-          bg = cm;
-          bsd = (uint32_t)((c0 + k) * CH + 2 * p0 + i);
         }
       }
       tc_fence_before();
@@ -392,17 +425,35 @@ __global__ void __launch_bounds__(NT, 1)
   if (__syncthreads_or(timed_out)) {
     if (tid == 0) atomicOr(status, kFaultTimeout);
   } else if (tid < BM) {
-    // merge the SUBS warps of each row (smaller seed on equal gains)
-    float g = sm.red_g[0][tid];
-    uint32_t s = sm.red_s[0][tid];
+    // merge the SUBS warps of each row (smaller seed on equal gains) and write
+    // the row's candidate (split z of it when the seeds are split over blocks)
+    int best = 0;
 #pragma unroll
-    for (int i = 1; i < SUBS; ++i) {
-      if (better(sm.red_g[i][tid], sm.red_s[i][tid], g, s)) { g = sm.red_g[i][tid]; s = sm.red_s[i][tid]; }
-    }
+    for (int i = 1; i < SUBS; ++i)
+      if (better(sm.red_g[i][tid], sm.red_s[i][tid], sm.red_g[best][tid], sm.red_s[best][tid])) best = i;
     const int64_t row = rb * BM + tid;
     if (row < md.rows) {
       const int64_t tt = md.tile_off + row * md.n_cb + cb;
-      partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[tid] ? g : neg_inf(), __uint_as_float(s));
+      const float g = sm.red_g[best][tid];
+      const uint32_t s = sm.red_s[best][tid];
+      awsrc_candidate cd;
+      const bool valid = sm.rowok[tid] && g > neg_inf();
+      uint32_t cw = 0u;
+      int sf = 0;
+      if (valid) {
+        const float4* pe = reinterpret_cast<const float4*>(
+            pairs + (size_t)((md.gram_off + cb * pr.S_pad + s) / 2) * PS);
+        const float gw = winner_codes<FAST>(pr, sm, tid, masks + (size_t)s * 4, pe, (s & 1u) != 0u, &cw, &sf);
+        if (__float_as_uint(gw) != __float_as_uint(g)) atomicOr(status, kFaultSelfCheck);
+      }
+      cd.gain = valid ? g : neg_inf();
+      cd.seed = valid ? (uint16_t)s : (uint16_t)0;
+      cd.scale = (int16_t)sf;
+#pragma unroll
+      for (int p = 0; p < 4; ++p) cd.code[p] = (int8_t)(cw >> (8 * p));
+#pragma unroll
+      for (int p = 4; p < 8; ++p) cd.code[p] = 0;
+      cands[(size_t)z * ld.T + tt] = cd;
     }
   }
   if (warp == EW) {
@@ -435,6 +486,20 @@ __global__ void atoms_kernel(const uint64_t* __restrict__ masks, uint4* __restri
   out[i] = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+// Best of the per-split candidates of tiles [t0, t1): larger gain, then the
+// smaller seed (an invalid tile's candidates are all zero with gain -inf).
+__global__ void merge_kernel(const awsrc_candidate* __restrict__ pc, int nsplit, int64_t T, int64_t t0,
+                             int64_t t1, awsrc_candidate* __restrict__ out) {
+  const int64_t t = t0 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= t1) return;
+  awsrc_candidate b = pc[t];
+  for (int z = 1; z < nsplit; ++z) {
+    const awsrc_candidate c = pc[(size_t)z * T + t];
+    if (better(c.gain, c.seed, b.gain, b.seed)) b = c;
+  }
+  out[t] = b;
+}
+
 }  // namespace
 
 int search_c64p4_rows() { return BM; }
@@ -448,14 +513,24 @@ cudaError_t launch_bfrag_c64p4(const Prm& pr, const uint64_t* masks, void* out, 
   return cudaGetLastError();
 }
 
+cudaError_t launch_merge_candidates(const awsrc_candidate* pc, int nsplit, int64_t T, int64_t t0, int64_t t1,
+                                   awsrc_candidate* out, cudaStream_t st) {
+  if (t1 <= t0) return cudaSuccess;
+  merge_kernel<<<(unsigned)((t1 - t0 + 255) / 256), 256, 0, st>>>(pc, nsplit, T, t0, t1, out);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void* table,
-                                const float2* pairs, int64_t n_blocks, float2* partials,
+                                const float2* pairs, const uint64_t* masks, int64_t n_blocks,
+                                awsrc_candidate* cands,
                                 uint32_t* status, cudaStream_t st) {
   const size_t smem = sizeof(Smem) + 1024;  // + alignment of the operand tiles
   auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), pairs, partials, status);
+  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), pairs, masks, cands,
+                                            status);
   note_launches(1);
   return cudaGetLastError();
 }

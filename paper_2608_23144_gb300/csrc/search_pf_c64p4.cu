@@ -78,14 +78,13 @@ __device__ __forceinline__ float2 neg2(float2 v) { return make_float2(-v.x, -v.y
 
 __device__ __forceinline__ bool pivot_ok(float d) { return d > 0.0f && d <= 3.402823466e38f; }
 
-// Gains of one seed pair of this thread's row; ah/al: atom p of the two seeds
-// at [2p], [2p+1]; qh/ql: product q (tri order) at [2q], [2q+1].
-template <bool FAST>
-__device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, const float* al, const float* qh,
-                                               const float* ql, float tqc, float tqdc, float gd, float diag,
-                                               float invd0) {
+// Fit of one seed pair of this thread's row; ah/al: atom p of the two seeds
+// at [2p], [2p+1]; qh/ql: product q (tri order) at [2q], [2q+1]. Returns b, the
+// off-diagonal G, alpha and whether each candidate's pivots are valid.
+__device__ __forceinline__ void pf_pair_fit(const float* ah, const float* al, const float* qh, const float* ql,
+                                            float tqc, float tqdc, float diag, float invd0, float2* bv,
+                                            float2* G, float2* alpha, bool* okx, bool* oky) {
   const float2 tq2 = make_float2(tqc, tqc), td2 = make_float2(tqdc, tqdc);
-  float2 bv[4], G[6];
 #pragma unroll
   for (int p = 0; p < 4; ++p) bv[p] = pair_sum(ah, al, 2 * p, tq2);
 #pragma unroll
@@ -94,7 +93,8 @@ __device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, c
   const float2 dg = make_float2(diag, diag);
   float2 nL[6], E[6], invD[4];
   invD[0] = make_float2(invd0, invd0);
-  bool okx = true, oky = true;
+  *okx = true;
+  *oky = true;
 #pragma unroll
   for (int k = 1; k < 4; ++k) {
 #pragma unroll
@@ -108,12 +108,25 @@ __device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, c
     float2 dk = dg;
 #pragma unroll
     for (int i = 0; i < k; ++i) dk = __ffma2_rn(nL[tri(k, i)], E[tri(k, i)], dk);
-    okx = okx && pivot_ok(dk.x);
-    oky = oky && pivot_ok(dk.y);
+    *okx = *okx && pivot_ok(dk.x);
+    *oky = *oky && pivot_ok(dk.y);
     invD[k] = make_float2(__frcp_rn(dk.x), __frcp_rn(dk.y));
   }
-  float2 alpha[4];
   ldl_solve2<4>(nL, invD, bv, alpha);
+}
+
+// Gains of one seed pair (operands as for pf_pair_fit).
+template <bool FAST>
+__device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, const float* al, const float* qh,
+                                               const float* ql, float tqc, float tqdc, float gd, float diag,
+                                               float invd0, float2* alpha_out = nullptr) {
+  float2 bv[4], G[6], alpha[4];
+  bool okx, oky;
+  pf_pair_fit(ah, al, qh, ql, tqc, tqdc, diag, invd0, bv, G, alpha, &okx, &oky);
+  if (alpha_out) {
+#pragma unroll
+    for (int p = 0; p < 4; ++p) alpha_out[p] = alpha[p];
+  }
   float2 g;
   if constexpr (FAST) {
     float2 G2[6];
@@ -140,11 +153,69 @@ __device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, c
   return g;
 }
 
+// Codes and scale field of the winning seed of row m. The search keeps only
+// (gain, seed), so the seed's correlations with Y (atoms) and D (atom
+// products) are formed again as the exact integer sums the tensor cores
+// accumulate, split into hi/lo so that 2048*hi + lo is the sum and the fma of
+// pair_sum rounds it once, and go through the same fit and quantiser. Both
+// halves of the pair get the winner's sums; one is read. Returns the gain
+// once more, which must equal the one the search found.
+template <bool FAST>
+__device__ __forceinline__ float pf_winner(const Prm& pr, const Smem& sm, int m, const uint64_t* mk, bool odd,
+                                           uint32_t* cw, int* sf) {
+  const float iy = sm.inv_qy[m], idd = sm.inv_qd[m];
+  uint64_t w[4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) w[p] = mk[p];
+  uint64_t wq[6];
+#pragma unroll
+  for (int a = 1, q = 0; a < 4; ++a)
+#pragma unroll
+    for (int c = 0; c < a; ++c, ++q) wq[q] = w[a] ^ w[c];  // products in tri order
+  int ty = 0, td = 0, ny[4] = {0, 0, 0, 0}, nd[6] = {0, 0, 0, 0, 0, 0};
+  for (int j = 0; j < 64; ++j) {
+    const int y = iy == 0.0f ? 0 : fixed_point_int(sm.Yst[m][j], iy);
+    const int d = idd == 0.0f ? 0 : fixed_point_int(sm.Dst[m][j], idd);
+    ty += y;
+    td += d;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) ny[p] += ((w[p] >> j) & 1ull) ? y : 0;
+#pragma unroll
+    for (int q = 0; q < 6; ++q) nd[q] += ((wq[q] >> j) & 1ull) ? d : 0;
+  }
+  float ah[8], al[8], qh[12], ql[12];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const int u = ty - 2 * ny[p];  // |u| <= 64 * 2^21
+    ah[2 * p] = ah[2 * p + 1] = (float)(u >> 11);
+    al[2 * p] = al[2 * p + 1] = (float)(u & 2047);
+  }
+#pragma unroll
+  for (int q = 0; q < 6; ++q) {
+    const int u = td - 2 * nd[q];
+    qh[2 * q] = qh[2 * q + 1] = (float)(u >> 11);
+    ql[2 * q] = ql[2 * q + 1] = (float)(u & 2047);
+  }
+  float2 alpha[4];
+  const float2 g = pf_pair_gain<FAST>(pr, ah, al, qh, ql, sm.tqc[m], sm.tqdc[m], sm.gd[m], sm.diag[m],
+                                      sm.invd0[m], alpha);
+  float a[4], q4[4], zero[6] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+  for (int p = 0; p < 4; ++p) a[p] = odd ? alpha[p].y : alpha[p].x;
+  if constexpr (FAST) (void)quant_gain_fast<4>(pr, a, zero, 0.0f, zero, q4, sf);
+  else (void)quant_gain<4>(pr, a, zero, 0.0f, zero, q4, sf);
+  uint32_t c = 0u;
+#pragma unroll
+  for (int p = 0; p < 4; ++p) c |= ((uint32_t)(int)q4[p] & 0xFFu) << (8 * p);
+  *cw = c;
+  return odd ? g.y : g.x;
+}
+
 template <bool FAST>
 __global__ void __launch_bounds__(NT, 1)
     search_pf_kernel(Prm pr, LaunchDesc ld, const unsigned char* __restrict__ atoms,
-                     const unsigned char* __restrict__ prods, float2* __restrict__ partials,
-                     uint32_t* __restrict__ status) {
+                     const unsigned char* __restrict__ prods, const uint64_t* __restrict__ masks,
+                     awsrc_candidate* __restrict__ cands, uint32_t* __restrict__ status) {
   extern __shared__ unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -355,7 +426,22 @@ __global__ void __launch_bounds__(NT, 1)
     const int64_t row = rb * BM + tid;
     if (row < md.rows) {
       const int64_t tt = md.tile_off + row * md.n_cb + cb;
-      partials[(size_t)z * ld.T + tt] = make_float2(sm.rowok[tid] ? g : neg_inf(), __uint_as_float(s));
+      const bool valid = sm.rowok[tid] && g > neg_inf();
+      uint32_t cw = 0u;
+      int sf = 0;
+      if (valid) {
+        const float gw = pf_winner<FAST>(pr, sm, tid, masks + (size_t)s * 4, (s & 1u) != 0u, &cw, &sf);
+        if (__float_as_uint(gw) != __float_as_uint(g)) atomicOr(status, kFaultSelfCheck);
+      }
+      awsrc_candidate cd;
+      cd.gain = valid ? g : neg_inf();
+      cd.seed = valid ? (uint16_t)s : (uint16_t)0;
+      cd.scale = (int16_t)sf;
+#pragma unroll
+      for (int p = 0; p < 4; ++p) cd.code[p] = (int8_t)(cw >> (8 * p));
+#pragma unroll
+      for (int p = 4; p < 8; ++p) cd.code[p] = 0;
+      cands[(size_t)z * ld.T + tt] = cd;
     }
   }
   if (warp == EW) {
@@ -407,13 +493,14 @@ cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void*
 }
 
 cudaError_t launch_search_pf_c64p4(const Prm& pr, const LaunchDesc& ld, const void* atoms, const void* prods,
-                                   int64_t n_blocks, float2* partials, uint32_t* status, cudaStream_t st) {
+                                   const uint64_t* masks, int64_t n_blocks, awsrc_candidate* cands,
+                                   uint32_t* status, cudaStream_t st) {
   const size_t smem = sizeof(Smem) + 1024;
   auto kern = pr.fast_pow2 ? search_pf_kernel<true> : search_pf_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const unsigned char*>(atoms),
-                                             static_cast<const unsigned char*>(prods), partials, status);
+                                             static_cast<const unsigned char*>(prods), masks, cands, status);
   note_launches(1);
   return cudaGetLastError();
 }
