@@ -11,19 +11,17 @@
 
 namespace awsrc {
 
-constexpr int kBasisWarps = 4;  // warps per block of the stand-alone kernel
+constexpr int kBasisWarps = 8;  // warps per block of the stand-alone kernel
 
 __global__ void __launch_bounds__(32 * kBasisWarps) gen_basis_kernel(Prm pr, uint64_t* __restrict__ masks,
                                                                      int S_out) {
-  __shared__ __align__(16) uint8_t smem[kBasisWarps][kBasisWarp4Smem];
+  __shared__ __align__(16) uint8_t smem[kBasisWarps][kBasisSmem];
   const int warp = threadIdx.x >> 5;
-  const int s0 = (blockIdx.x * kBasisWarps + warp) * kWarpSeeds;
-  if (s0 >= S_out) return;  // whole warp leaves together
-  basis_warp4(pr, masks, s0, S_out, smem[warp]);
+  basis_warp(pr, masks, (int64_t)blockIdx.x * kBasisWarps + warp, S_out, smem[warp]);
 }
 
 cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStream_t st) {
-  const int per = kBasisWarps * kWarpSeeds;
+  const int per = kBasisWarps * basis_warp_seeds(pr.C);
   gen_basis_kernel<<<(S_out + per - 1) / per, 32 * kBasisWarps, 0, st>>>(pr, masks, S_out);
   note_launches(1);
   return cudaGetLastError();

@@ -3,7 +3,7 @@
 // decodes the same way (Sec. 3.3).
 //
 //  dense mode (C >= one vector):
-//   prep     one block range generates the basis masks (one warp per 4 selectors),
+//   prep     one block range generates the basis masks (basis_warp),
 //            the other unpacks every record once: its codes go to a per-record
 //            array and the tile's map entry (k + 1, seed, scale field) is
 //            raised to it with atomicMax, so a tile named twice is flagged and
@@ -252,7 +252,7 @@ __device__ __forceinline__ void map_records(const Prm& pr, const DecArgs& a, con
 // Dense pass: W_hat = convert(W0) for every element, a pure stream with U
 // independent 16-byte vectors in flight per thread and no dependent loads.
 // With `basis`, the blocks of grid slice y = 0 (dispatched first) generate the
-// basis masks, one warp per 4 selectors, overlapping GenBasis with the
+// basis masks (8 warps per block, basis_warp), overlapping GenBasis with the
 // memory-bound stream of the other slices.
 template <typename TI, typename TO, int G>
 __global__ void __launch_bounds__(256) copy_kernel(Prm pr, const __grid_constant__ DecArgs a,
@@ -261,10 +261,9 @@ __global__ void __launch_bounds__(256) copy_kernel(Prm pr, const __grid_constant
   int y = blockIdx.y;
   if (basis) {
     if (y == 0) {
-      __shared__ __align__(16) uint8_t bsm[8][kBasisWarp4Smem];
+      __shared__ __align__(16) uint8_t bsm[8][kBasisSmem];
       const int warp = threadIdx.x >> 5;
-      const int s0 = (blockIdx.x * 8 + warp) * kWarpSeeds;
-      if (s0 < pr.S) basis_warp4(pr, masks, s0, pr.S, bsm[warp]);
+      basis_warp(pr, masks, (int64_t)blockIdx.x * 8 + warp, pr.S, bsm[warp]);
       return;
     }
     --y;
@@ -451,7 +450,8 @@ __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const _
 }
 
 // Dense-mode preparation for the fused pass: blocks [0, nb) generate the masks
-// (one warp per 4 selectors), the remaining blocks fill the tile map (map_records).
+// (8 warps per block, basis_warp), the remaining blocks fill the tile map
+// (map_records).
 __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant__ DecArgs a,
                                                    const uint8_t* __restrict__ stream,
                                                    uint64_t* __restrict__ masks,
@@ -459,10 +459,9 @@ __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant
                                                    uint2* __restrict__ codes, uint32_t* __restrict__ status,
                                                    int nb) {
   if ((int)blockIdx.x < nb) {
-    __shared__ __align__(16) uint8_t bsm[8][kBasisWarp4Smem];
+    __shared__ __align__(16) uint8_t bsm[8][kBasisSmem];
     const int warp = threadIdx.x >> 5;
-    const int s0 = (blockIdx.x * 8 + warp) * kWarpSeeds;
-    if (s0 < pr.S) basis_warp4(pr, masks, s0, pr.S, bsm[warp]);
+    basis_warp(pr, masks, (int64_t)blockIdx.x * 8 + warp, pr.S, bsm[warp]);
     return;
   }
   map_records(pr, a, stream, map, codes, status, (int64_t)(blockIdx.x - nb) * blockDim.x + threadIdx.x,
@@ -510,7 +509,10 @@ cudaError_t launch_copy_t(const Prm& pr, DecArgs a, bool copy, bool basis, uint6
   cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (maxg + 4 * 256 - 1) / (4 * 256);
   int64_t gx = std::min<int64_t>(want, (int64_t)nsm * 8);
-  if (basis) gx = std::max<int64_t>(gx, (pr.S + 8 * kWarpSeeds - 1) / (8 * kWarpSeeds));
+  if (basis) {
+    const int per = 8 * basis_warp_seeds(pr.C);
+    gx = std::max<int64_t>(gx, (pr.S + per - 1) / per);
+  }
   gx = std::max<int64_t>(gx, 1);
   copy_kernel<TI, TO, G><<<dim3((unsigned)gx, a.n_mod + (basis ? 1 : 0)), 256, 0, st>>>(pr, a, masks,
                                                                                       basis ? 1 : 0);
@@ -580,8 +582,9 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     int dev = 0, nsm = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    const int nb = (pr.S + 8 * kWarpSeeds - 1) / (8 * kWarpSeeds);  // mask blocks, then record blocks
-    const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, nsm));
+    const int per = 8 * basis_warp_seeds(pr.C);
+    const int nb = (pr.S + per - 1) / per;  // mask blocks, then record blocks (one record per thread)
+    const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, (int64_t)nsm * 64));
     prep_kernel<<<(unsigned)(nb + nr), 256, 0, st>>>(pr, a, stream, masks, map, codes, status, nb);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

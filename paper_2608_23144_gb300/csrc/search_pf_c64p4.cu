@@ -217,7 +217,9 @@ __global__ void __launch_bounds__(NT, 1)
                      const unsigned char* __restrict__ prods, const uint64_t* __restrict__ masks,
                      awsrc_candidate* __restrict__ cands, uint32_t* __restrict__ status) {
   extern __shared__ unsigned char smem_raw[];
-  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1 KB aligned by pointer arithmetic on the shared array, so that the
+  // compiler keeps the shared address space (LDS/STS, not generic accesses)
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int mi = find_mod(ld, blockIdx.x);
   const ModDesc& md = ld.m[mi];

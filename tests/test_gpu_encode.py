@@ -115,11 +115,19 @@ def test_seed_splits_do_not_change_the_result(aw, orc):
 
 
 def test_gen_basis_matches_oracle(aw, orc):
-    for C, P, permute, S in [(64, 4, 1, 4096), (16, 4, 1, 64), (128, 2, 1, 64), (256, 8, 0, 32), (8, 3, 1, 100)]:
+    """Every selector's masks, bit for bit (C <= 64 takes the warp-parallel
+    Fisher-Yates evaluation, C > 64 the sequential one)."""
+    cases = [(64, 4, 1, 4096), (64, 8, 1, 300), (64, 4, 0, 100), (32, 4, 1, 500), (16, 4, 1, 64), (8, 3, 1, 100),
+             (4, 2, 1, 200), (4, 4, 1, 64), (4, 1, 0, 8), (128, 2, 1, 64), (256, 8, 0, 32), (256, 4, 1, 40)]
+    for C, P, permute, S in cases:
         prm = aw.params(C=C, P=P, S=S, permute=permute, gen_seed=12345)
-        masks = aw.awsrc_gen_basis(prm).cpu().numpy().view(np.uint64).reshape(S, P, (C + 63) // 64)
-        for s in list(range(min(S, 64))) + [S - 1]:
+        W = (C + 63) // 64
+        masks = aw.awsrc_gen_basis(prm).cpu().numpy().view(np.uint64).reshape(S, P, W)
+        bits = ((masks[..., None] >> np.arange(64, dtype=np.uint64)) & np.uint64(1)).astype(np.uint8)
+        bits = bits.reshape(S, P, W * 64)
+        assert not bits[:, :, C:].any(), (C, P)
+        for s in range(S):
             neg = orc.gen_basis(12345, s, C, P, permute)[3]
-            bits = np.array([(int(masks[s, p, j // 64]) >> (j % 64)) & 1 for p in range(P) for j in range(C)],
-                            np.uint8).reshape(P, C)
-            assert np.array_equal(bits, neg), (C, P, s)
+            assert np.array_equal(bits[s, :, :C], neg), (C, P, permute, s)
+
+
