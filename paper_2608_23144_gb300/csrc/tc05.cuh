@@ -41,11 +41,13 @@ __device__ __forceinline__ void mbar_arrive(unsigned long long* mb) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(mb)) : "memory");
 }
 
+// One potentially blocking test of the phase; the 20 us suspend hint lets a
+// waiting thread sleep until the phase completes instead of spinning.
 __device__ __forceinline__ bool mbar_try_wait(unsigned long long* mb, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, 20000;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
       : "r"(smem_addr(mb)), "r"(parity)

@@ -83,6 +83,26 @@ def test_pruned_search_matches_oracle_on_adversarial_tiles(aw, orc, kind):
     assert_candidates_equal(got, want, kind)
 
 
+@pytest.mark.parametrize("variant", [0, 1])
+def test_padding_selectors_never_win(aw, orc, variant):
+    """Seeds are searched in chunks padded up to a multiple of 32 with all-zero
+    masks; such a basis is four copies of the constant vector, which would fit a
+    constant residual exactly. The padding must never be chosen."""
+    mods = _mods([(64, 128)], "f32", fisher=bool(variant), seed=5)
+    m = mods[0]
+    m["W"] = m["W0"] + 0.01                          # constant residual on every tile
+    m["W"][::3, :64] += 0.002 * torch.randn(22, 64)  # and some ordinary tiles
+    kw = dict(C=64, P=4, b=4, S=37, variant=variant)
+    prm, oprm = aw.params(**kw), orc.params(**kw)
+    cands = aw.awsrc_encode_tiles(prm, to_dev(mods))
+    flags = aw.awsrc_workspace_status(cands._awsrc_workspace)
+    got = aw.candidates_to_numpy(cands)
+    want = oracle_encode(orc, oprm, mods)[0]
+    assert flags == 0, f"device fault flags {flags:#x}"
+    assert (got["seed"] < 37).all()
+    assert_candidates_equal(got, want, f"padding v{variant}")
+
+
 def test_degenerate_tiles(aw, orc):
     mods = _mods([(40, 192)], "f32")
     m = mods[0]
