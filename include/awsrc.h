@@ -129,6 +129,10 @@ typedef struct awsrc_params {
 } awsrc_params;
 
 /*
+ * Pointer alignment (checked; a violation returns AWSRC_ERR_INVALID_ARG before
+ * any launch): device arrays at least at their element size; workspaces at 256
+ * bytes (as cudaMalloc returns them); W0 and W_hat of the decoder at 16 bytes.
+ *
  * One linear module (a weight matrix W with backbone reconstruction W0 = Q(W),
  * Eq. 1) and its per-input-channel statistics (Sec. 3.2).
  *   rows, cols  output and input dimensions; cols % C == 0.
@@ -285,7 +289,7 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  * applies only the tile's later record and reports it the same way, INPLACE
  * leaves such a tile unspecified. Requires the same params as the encoder.
  * Workspace (awsrc_decode_workspace_bytes): the basis masks, plus for DENSE a
- * tile -> record map and the unpacked records, 12 bytes per tile.
+ * tile -> record map and the unpacked records, 16 bytes per tile.
  */
 awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 const awsrc_module* mods, const uint8_t* stream,

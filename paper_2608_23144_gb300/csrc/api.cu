@@ -34,6 +34,11 @@ bool use_c64p4_pf(const Prm& pr) {
   return pr.C == 64 && pr.P == 4 && pr.variant == AWSRC_VARIANT_PF;
 }
 
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+uintptr_t elt_bytes(int32_t dtype) { return dtype == AWSRC_DTYPE_BF16 ? 2 : 4; }
+
+// Shapes, dtypes and, for the encoder, pointers: it reads W, W0 and the
+// statistics element by element (natural alignment).
 awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mods, bool encoder,
                            int64_t* T_out) {
   if (n_mod < 1 || mods == nullptr) return AWSRC_ERR_INVALID_ARG;
@@ -47,6 +52,9 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
       if (md.w_dtype != AWSRC_DTYPE_F32 && md.w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
       if (!md.W || !md.W0 || !md.act) return AWSRC_ERR_INVALID_ARG;
       if (pr.variant == AWSRC_VARIANT_PF && !md.fisher) return AWSRC_ERR_INVALID_ARG;
+      if (!aligned(md.W, elt_bytes(md.w_dtype)) || !aligned(md.W0, elt_bytes(md.w0_dtype)) ||
+          !aligned(md.act, 4) || !aligned(md.fisher, 4))
+        return AWSRC_ERR_INVALID_ARG;
     }
     T += md.rows * (md.cols / pr.C);
   }
@@ -236,9 +244,10 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   if (s != AWSRC_OK) return s;
   int64_t T;
   if ((s = check_modules(pr, n_mod, mods, true, &T)) != AWSRC_OK) return s;
-  if (!out) return AWSRC_ERR_INVALID_ARG;
+  if (!out || !aligned(out, 4)) return AWSRC_ERR_INVALID_ARG;
   const EncodeLayout lay = encode_layout(pr, n_mod, mods, T);
   if (!workspace || workspace_bytes < lay.total) return AWSRC_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return AWSRC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   uint32_t* status = reinterpret_cast<uint32_t*>(ws);
@@ -409,8 +418,10 @@ awsrc_status awsrc_select_records(const awsrc_params* prm, int32_t n_mod, const 
   std::vector<int64_t> to, kc;
   if ((s = select_plan(pr, n_mod, mods, rates_bpw, n_rates, &sp, &to, &kc)) != AWSRC_OK) return s;
   if (!cands || !stream_out || !d_counts || !d_bytes) return AWSRC_ERR_INVALID_ARG;
+  if (!aligned(cands, 4) || !aligned(d_counts, 8) || !aligned(d_bytes, 8)) return AWSRC_ERR_INVALID_ARG;
   if (stream_capacity < (size_t)(sp.h + sp.cap_records * sp.L)) return AWSRC_ERR_CAPACITY;
   if (!workspace || workspace_bytes < select_ws_bytes(sp)) return AWSRC_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return AWSRC_ERR_INVALID_ARG;
   std::vector<int64_t> mt(n_mod);
   for (int m = 0; m < n_mod; ++m) mt[m] = to[m + 1] - to[m];
   const cudaError_t e = cudaMemsetAsync(workspace, 0, sizeof(uint32_t), (cudaStream_t)stream);
@@ -449,8 +460,9 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const aw
   std::vector<DecodeMod> dm(n_mod);
   int64_t off = 0;
   for (int m = 0; m < n_mod; ++m) {
-    if (!W_hat[m]) return AWSRC_ERR_INVALID_ARG;
-    if (mode == AWSRC_DECODE_DENSE && !mods[m].W0) return AWSRC_ERR_INVALID_ARG;
+    if (!W_hat[m] || !aligned(W_hat[m], 16)) return AWSRC_ERR_INVALID_ARG;
+    // the decoder moves W0 and W_hat in 16-byte vectors
+    if (mode == AWSRC_DECODE_DENSE && (!mods[m].W0 || !aligned(mods[m].W0, 16))) return AWSRC_ERR_INVALID_ARG;
     if (mode == AWSRC_DECODE_INPLACE && mods[m].w0_dtype != out_dtype) return AWSRC_ERR_INVALID_ARG;
     dm[m].W0 = mods[m].W0;
     dm[m].out = W_hat[m];
@@ -464,6 +476,7 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const aw
   size_t need;
   if ((s = awsrc_decode_workspace_bytes(prm, n_mod, mods, mode, &need)) != AWSRC_OK) return s;
   if (!workspace || workspace_bytes < need) return AWSRC_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return AWSRC_ERR_INVALID_ARG;
   const int64_t L = awsrc_record_bytes(prm, T), h = awsrc_header_bytes(n_mod);
   if (stream_len < (size_t)h) return AWSRC_ERR_INVALID_ARG;
   const int64_t kmax = std::min<int64_t>(((int64_t)stream_len - h) / L, T);
@@ -473,8 +486,9 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const aw
   uint64_t* masks = reinterpret_cast<uint64_t*>(ws + kStatusBytes);
   void* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
   cudaStream_t st = (cudaStream_t)stream_handle;
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
-  if (e != cudaSuccess) return cuda_fail(e, "decode: clear status");
+  cudaError_t e = cudaSuccess;
+  if (!decode_clears_status(pr, mode) && (e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st)) != cudaSuccess)
+    return cuda_fail(e, "decode: clear status");
   e = launch_decode(pr, n_mod, dm.data(), T, L, h, stream, K, kmax, out_dtype, mode, masks, scratch, status, st);
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "decode");
 }

@@ -20,6 +20,7 @@
 //            codes; bounds-check tile < T and seed < S (a bad record is skipped
 //            and flagged); rewrite the tile from W0, which may be W_hat itself.
 #include <algorithm>
+#include <utility>
 
 #include "basis.cuh"
 #include "internal.h"
@@ -27,6 +28,13 @@
 namespace awsrc {
 
 namespace {
+
+// Programmatic dependent launch: a kernel launched with
+// cudaLaunchAttributeProgrammaticStreamSerialization may start while the
+// previous kernel of the stream runs; it must call pdl_wait() before touching
+// anything that kernel writes. pdl_trigger() lets the next kernel launch early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 struct DecRec {   // an unpacked record; codes packed as signed bytes, code p in byte p
   uint16_t seed;
@@ -238,6 +246,7 @@ __device__ __forceinline__ void map_records(const Prm& pr, const DecArgs& a, con
   for (int64_t k = i0; k < Kd; k += n) {
     DecRec d;
     const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d, end);
+    pdl_wait();  // the map is cleared by the previous kernel
     if (tile < 0) {
       atomicOr(status, kFaultRecord);
       continue;
@@ -393,6 +402,7 @@ __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const _
   Vec<TO, G>* __restrict__ dst = static_cast<Vec<TO, G>*>(md.out);
   const unsigned long long* __restrict__ mmap = map + md.tile_off;
   const int lane = threadIdx.x & 31;
+  pdl_wait();  // masks, map and codes come from the preparation kernel
   for (int64_t c0 = (int64_t)blockIdx.x * kFusedChunk; c0 < ngroups; c0 += (int64_t)gridDim.x * kFusedChunk) {
     if (threadIdx.x == 0) qn = 0;
     __syncthreads();
@@ -449,6 +459,32 @@ __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const _
   }
 }
 
+// Clears the dense tile map (16-byte stores) and lets the preparation kernel
+// launch at once: its mask generation and record unpacking overlap this pass.
+__global__ void __launch_bounds__(256) zero_map_kernel(uint4* __restrict__ p, int64_t n16,
+                                                       uint32_t* __restrict__ status) {
+  pdl_trigger();
+  if (blockIdx.x == 0 && threadIdx.x == 0) *status = 0u;  // the call's fault word
+  for (int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x; i < n16; i += (int64_t)gridDim.x * 256)
+    p[i] = make_uint4(0u, 0u, 0u, 0u);
+}
+
+// Launch with programmatic serialisation after the previous kernel of `st`.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
 // Dense-mode preparation for the fused pass: blocks [0, nb) generate the masks
 // (8 warps per block, basis_warp), the remaining blocks fill the tile map
 // (map_records).
@@ -458,6 +494,7 @@ __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant
                                                    unsigned long long* __restrict__ map,
                                                    uint2* __restrict__ codes, uint32_t* __restrict__ status,
                                                    int nb) {
+  pdl_trigger();  // the fused pass may launch now; it waits for this grid
   if ((int)blockIdx.x < nb) {
     __shared__ __align__(16) uint8_t bsm[8][kBasisSmem];
     const int warp = threadIdx.x >> 5;
@@ -478,12 +515,13 @@ cudaError_t launch_fused_t(const Prm& pr, const DecArgs& a, const unsigned long 
   cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (maxg + kFusedChunk - 1) / kFusedChunk;
   const int64_t gx = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)nsm * 8));
-  if (pr.P == 4)
-    fused_kernel<TI, TO, G, 4><<<dim3((unsigned)gx, a.n_mod), kFusedThreads, 0, st>>>(pr, a, map, codes, masks);
-  else
-    fused_kernel<TI, TO, G, 0><<<dim3((unsigned)gx, a.n_mod), kFusedThreads, 0, st>>>(pr, a, map, codes, masks);
+  const dim3 grid((unsigned)gx, (unsigned)a.n_mod);
+  cudaError_t e = pr.P == 4 ? launch_pdl(fused_kernel<TI, TO, G, 4>, grid, dim3(kFusedThreads), st, pr, a, map,
+                                         codes, masks)
+                            : launch_pdl(fused_kernel<TI, TO, G, 0>, grid, dim3(kFusedThreads), st, pr, a, map,
+                                         codes, masks);
   note_launches(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_fused(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype,
@@ -567,14 +605,12 @@ cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_
 cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
-  const bool fused = mode == AWSRC_DECODE_DENSE && pr.C >= 8 && scratch != nullptr;
+  const bool fused = decode_clears_status(pr, mode) && scratch != nullptr;
   unsigned long long* map = nullptr;
   uint2* codes = nullptr;
   if (fused) {
     map = static_cast<unsigned long long*>(scratch);
     codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
-    cudaError_t e = cudaMemsetAsync(map, 0, (size_t)T * 8, st);
-    if (e != cudaSuccess) return e;
     DecArgs a;
     a.n_mod = 0;
     a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
@@ -585,9 +621,17 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     const int per = 8 * basis_warp_seeds(pr.C);
     const int nb = (pr.S + per - 1) / per;  // mask blocks, then record blocks (one record per thread)
     const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, (int64_t)nsm * 64));
-    prep_kernel<<<(unsigned)(nb + nr), 256, 0, st>>>(pr, a, stream, masks, map, codes, status, nb);
+    // the map region is align_up(T * 8, 256) bytes, so whole 16-byte words stay inside it
+    const int64_t n16 = (T * 8 + 15) / 16;
+    const unsigned gz = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n16 + 255) / 256, (int64_t)nsm * 8));
+    zero_map_kernel<<<gz, 256, 0, st>>>(reinterpret_cast<uint4*>(map), n16, status);
     note_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(prep_kernel, dim3((unsigned)(nb + nr)), dim3(256), st, pr, a, stream, masks, map, codes, status,
+                   nb);
+    note_launches(1);
+    if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
   }
   int i0 = 0;
   while (i0 < n_mod) {
@@ -606,6 +650,8 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
   }
   return cudaSuccess;
 }
+
+bool decode_clears_status(const Prm& pr, int mode) { return mode == AWSRC_DECODE_DENSE && pr.C >= 8; }
 
 size_t decode_scratch_bytes(int64_t T, int mode) {
   // dense: tile -> record map (8 B per tile) and each record's codes (8 B, at

@@ -91,7 +91,7 @@ extern "C" awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* p
     const awsrc_module& md = mods[m];
     if (md.rows < 1 || md.cols < 1 || md.cols % pr.C != 0) return AWSRC_ERR_SHAPE;
     if (md.w0_dtype != AWSRC_DTYPE_F32 && md.w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
-    if (!W_hat[m]) return AWSRC_ERR_INVALID_ARG;
+    if (!W_hat[m] || (reinterpret_cast<uintptr_t>(W_hat[m]) & 15) != 0) return AWSRC_ERR_INVALID_ARG;
     dm[m].W0 = W_hat[m];
     dm[m].out = W_hat[m];
     dm[m].rows = md.rows;

@@ -86,6 +86,8 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
 size_t decode_scratch_bytes(int64_t T, int mode);
+// The dense fused decoder clears the fault word itself (no separate memset).
+bool decode_clears_status(const Prm& pr, int mode);
 int generic_rows();
 int generic_chunk();
 

@@ -103,3 +103,33 @@ def test_stream_capacity_matches_oracle_budget(libpath, orc):
     quotas = [((B - h) * r * c) // N for r, c in shapes]
     assert n.value == h + sum(qm // L for qm in quotas) * L
     assert n.value <= B
+
+
+def test_misaligned_pointers_are_refused_before_any_launch(libpath):
+    """Pointer values are only compared here (no device memory exists): each
+    call must return INVALID_ARG on the host, before touching the GPU."""
+    import paper_2608_23144_gb300 as aw
+    lib = aw.lib
+    p = aw.params(C=64, S=64)
+    mods = (aw.Module * 1)()
+    mods[0].rows, mods[0].cols = 8, 128
+    mods[0].w_dtype = mods[0].w0_dtype = aw.DTYPE_BF16
+    mods[0].W, mods[0].W0, mods[0].act = 0x10000, 0x20000, 0x30000
+    big = 1 << 40
+    assert lib.awsrc_encode_tiles(ct.byref(p), 1, mods, 0x40000, 0x50001, big, None) == 1    # workspace
+    assert lib.awsrc_encode_tiles(ct.byref(p), 1, mods, 0x40002, 0x50000, big, None) == 1    # candidates
+    mods[0].W = 0x10001                                                                      # BF16 needs 2
+    assert lib.awsrc_encode_tiles(ct.byref(p), 1, mods, 0x40000, 0x50000, big, None) == 1
+    mods[0].W, mods[0].act = 0x10000, 0x30002                                                # f32 needs 4
+    assert lib.awsrc_encode_tiles(ct.byref(p), 1, mods, 0x40000, 0x50000, big, None) == 1
+    mods[0].act = 0x30000
+    what = (ct.c_void_p * 1)(0x60008)                                                        # W_hat needs 16
+    assert lib.awsrc_decode_apply(ct.byref(p), 1, mods, 0x70000, 1 << 20, 0, what, aw.DTYPE_BF16,
+                                  aw.DECODE_DENSE, 0x80000, big, None) == 1
+    what[0] = 0x60000
+    mods[0].W0 = 0x20008                                                                     # dense W0 needs 16
+    assert lib.awsrc_decode_apply(ct.byref(p), 1, mods, 0x70000, 1 << 20, 0, what, aw.DTYPE_BF16,
+                                  aw.DECODE_DENSE, 0x80000, big, None) == 1
+    mods[0].W0 = 0x20000
+    assert lib.awsrc_decode_apply(ct.byref(p), 1, mods, 0x70000, 1 << 20, 0, what, aw.DTYPE_BF16,
+                                  aw.DECODE_DENSE, 0x80040, big, None) == 1                  # workspace
