@@ -197,6 +197,58 @@ def host_modules(mods):
 
 
 # ------------------------------------------------------------- reference --
+def paper_points(dev, hbm_gbs):
+    """The paper's own operating points (Sec. 4) on the three MLP projections of
+    one Qwen2.5-3B-shaped layer (gate/up 11008x2048, down 2048x11008, BF16):
+    AWSRC-U at (C, P, b, S) = (128, 2, 4, 2) and AWSRC-P_F at (16, 4, 4, 16) with
+    the 0.25/0.75 activation/Fisher blend. Encode, select (0.162 bpw) and dense
+    decode, each timed on the device (mean of 3 runs after one warm-up)."""
+    import torch
+    import paper_2608_23144_gb300 as aw
+    from synth.workloads import make_module, module_seed
+    shapes = [(11008, 2048), (11008, 2048), (2048, 11008)]
+    out = {}
+    for name, kw, fisher, blend in [
+            ("U_c128_p2_s2", dict(C=128, P=2, b=4, S=2), False, (1.0, 0.0)),
+            ("PF_c16_p4_s16", dict(C=16, P=4, b=4, S=16, variant=1), True, (0.25, 0.75))]:
+        mods = [make_module(r, c, seed=module_seed(0, 0, 4 + i), device=dev, fisher=fisher, blend=blend)
+                for i, (r, c) in enumerate(shapes)]
+        prm = aw.params(**kw)
+        N = sum(r * c for r, c in shapes)
+        T = N // kw["C"]
+        cands = aw.awsrc_encode_tiles(prm, mods)
+        ws = cands._awsrc_workspace
+        stream, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, [0.162])
+        outs = aw.awsrc_decode_apply(prm, mods, stream, -1)
+        torch.cuda.synchronize()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        reps = 3
+        ev[0].record()
+        for _ in range(reps):
+            aw.awsrc_encode_tiles(prm, mods, out=cands, workspace=ws)
+        ev[1].record()
+        for _ in range(reps):
+            aw.awsrc_select_records(prm, mods, cands, [0.162])
+        ev[2].record()
+        for _ in range(reps):
+            aw.awsrc_decode_apply(prm, mods, stream, -1, outs=outs)
+        ev[3].record()
+        torch.cuda.synchronize()
+        assert aw.awsrc_workspace_status(ws) == 0, "encoder self-check fault"
+        enc, sel, dec = (ev[i].elapsed_time(ev[i + 1]) / reps for i in range(3))
+        read = N * (2 + 2 + (4 if fisher else 0))  # W, W0 (BF16) and the Fisher diagonal
+        out[name] = {"params": kw, "blend": list(blend), "tiles": T, "records": int(counts.sum().item()),
+                     "encode_ms": enc, "candidates_per_s": T * kw["S"] / (enc * 1e-3),
+                     "encode_read_gbs": read / (enc * 1e-3) / 1e9,
+                     "encode_frac_of_hbm": read / (enc * 1e-3) / 1e9 / hbm_gbs,
+                     "select_ms": sel, "decode_ms": dec,
+                     "decode_gbs": N * 4 / (dec * 1e-3) / 1e9}
+        del mods, cands, ws, stream, outs
+    out["workload"] = ("gate/up/down projections of one Qwen2.5-3B-shaped layer (67,633,152 BF16 weights); "
+                       "the paper's (C,P,b,S) points, 0.162 bpw")
+    return out
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -432,6 +484,10 @@ def run_ours(args):
               "encode_ms": ms7, "candidates_per_s": T7 * wl7.S / (ms7 * 1e-3)}
         del m7, c7, ws7
 
+    paper = None
+    if rank == 0 and not args.no_pf and not args.modules:
+        paper = paper_points(dev, float(peaks.get("hbm_gbs", 6800.0)))
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, cores, desc = oracle_sample(wl, host_modules(mods), args.cpu_seconds)
@@ -452,7 +508,7 @@ def run_ours(args):
             "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper,
             "gpu_launches": launches, "clocks": clk.summary(),
         }
         print(json.dumps(line), flush=True)

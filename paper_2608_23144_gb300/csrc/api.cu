@@ -64,7 +64,7 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
 }
 
 struct EncodeLayout {
-  size_t masks, gram, pairs, mexp, ptab, partials, pcands, total;
+  size_t masks, gram, pairs, mexp, ptab, pcands, total;
   int nsplit;
   bool spec;     // U, C = 64, P = 4: tcgen05 search
   bool spec_pf;  // P_F, C = 64, P = 4: tcgen05 search
@@ -74,23 +74,24 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   EncodeLayout L{};
   L.spec = use_c64p4(pr);
   L.spec_pf = use_c64p4_pf(pr);
-  const int rb = (L.spec || L.spec_pf) ? search_c64p4_rows() : generic_rows();
+  const GenShape gs = gen_shape(pr);
   int64_t base_blocks = 0, ncb = 0;
   for (int m = 0; m < n_mod; ++m) {
     const int64_t n_cb = mods[m].cols / pr.C;
     ncb += n_cb;
-    base_blocks += n_cb * ((mods[m].rows + rb - 1) / rb);
+    if (L.spec || L.spec_pf) base_blocks += n_cb * ((mods[m].rows + search_c64p4_rows() - 1) / search_c64p4_rows());
   }
+  if (!(L.spec || L.spec_pf)) base_blocks = (T + gs.tiles - 1) / gs.tiles;
   const int64_t units = L.spec ? pr.S_pad / search_c64p4_chunk()
                        : L.spec_pf ? pr.S_pad / search_pf_c64p4_chunk()
-                                   : (pr.S + generic_chunk() - 1) / generic_chunk();
+                                   : (pr.S + gs.lanes - 1) / gs.lanes;
   int64_t ns = (kTargetBlocks + base_blocks - 1) / base_blocks;
   ns = std::max<int64_t>(1, std::min<int64_t>(ns, units));
   L.nsplit = (int)ns;
   size_t off = kStatusBytes;
   L.masks = off;
   off += align_up((size_t)pr.S_pad * pr.P * pr.W * 8, 256);
-  L.gram = off;  // read by the finalisation pass of the other search paths
+  L.gram = off;  // read by the generic U search
   if (pr.variant == AWSRC_VARIANT_U && !L.spec)
     off += align_up((size_t)ncb * pr.S_pad * gram_stride(pr.P) * 4, 256);
   L.pairs = off;
@@ -99,11 +100,8 @@ EncodeLayout encode_layout(const Prm& pr, int32_t n_mod, const awsrc_module* mod
   if (L.spec || L.spec_pf) off += align_up(search_c64p4_table_bytes(pr.S_pad), 256);
   L.ptab = off;
   if (L.spec_pf) off += align_up(search_pf_c64p4_table_bytes(pr.S_pad), 256);
-  const bool whole = L.spec || L.spec_pf;  // the search writes whole candidates
-  L.partials = off;  // (gain, seed) per tile and split, for the finalisation pass
-  if (!whole) off += align_up((size_t)L.nsplit * T * 8, 256);
-  L.pcands = off;    // whole candidates per tile and split, merged when nsplit > 1
-  if (whole && L.nsplit > 1) off += align_up((size_t)L.nsplit * T * sizeof(awsrc_candidate), 256);
+  L.pcands = off;  // candidates per tile and seed split, merged when nsplit > 1
+  if (L.nsplit > 1) off += align_up((size_t)L.nsplit * T * sizeof(awsrc_candidate), 256);
   L.total = off;
   return L;
 }
@@ -256,7 +254,6 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   awsrc_candidate* pcands = lay.nsplit > 1 ? reinterpret_cast<awsrc_candidate*>(ws + lay.pcands) : out;
   float2* pairs = lay.spec ? reinterpret_cast<float2*>(ws + lay.pairs) : nullptr;
   void* mexp = ws + lay.mexp;
-  float2* partials = reinterpret_cast<float2*>(ws + lay.partials);
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(uint32_t), st);
   if (e != cudaSuccess) return cuda_fail(e, "encode: clear status");
   e = launch_gen_basis(pr, masks, pr.S_pad, st);
@@ -266,7 +263,9 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
     return cuda_fail(e, "encode: atom table");
   if (lay.spec_pf && (e = launch_products_pf_c64p4(pr, masks, ptab, st)) != cudaSuccess)
     return cuda_fail(e, "encode: atom product table");
-  const int rb = (lay.spec || lay.spec_pf) ? search_c64p4_rows() : generic_rows();
+  const bool spec = lay.spec || lay.spec_pf;
+  const int rb = search_c64p4_rows();
+  const GenShape gs = gen_shape(pr);
   int64_t tile_off = 0, gram_off = 0;
   for (int g0 = 0; g0 < n_mod; g0 += kMaxModsPerLaunch) {
     LaunchDesc ld;
@@ -290,25 +289,25 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
       tile_off += d.rows * d.n_cb;
       gram_off += d.n_cb * pr.S_pad;
     }
+    if (!spec) {  // the generic search takes runs of consecutive tiles
+      const int64_t tiles = tile_off - ld.m[0].tile_off;
+      blocks = (tiles + gs.tiles - 1) / gs.tiles * lay.nsplit;
+    }
     if (pr.variant == AWSRC_VARIANT_U && (e = launch_gram_u(pr, ld, masks, gram, pairs, st)) != cudaSuccess)
       return cuda_fail(e, "encode: gram");
     if (g0 == 0 && g_ev_before && (e = cudaEventRecord(g_ev_before, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
     if (lay.spec) e = launch_search_c64p4(pr, ld, mexp, pairs, masks, blocks, pcands, status, st);
     else if (lay.spec_pf) e = launch_search_pf_c64p4(pr, ld, mexp, ptab, masks, blocks, pcands, status, st);
-    else e = launch_search_generic(pr, ld, masks, gram, blocks, partials, st);
+    else e = launch_search_generic(pr, ld, masks, gram, blocks, pcands, st);
     if (e != cudaSuccess) return cuda_fail(e, "encode: search");
     if (g0 + kMaxModsPerLaunch >= n_mod && g_ev_after && (e = cudaEventRecord(g_ev_after, st)) != cudaSuccess)
       return cuda_fail(e, "encode: timing event");
-    if (lay.spec || lay.spec_pf) {  // the search wrote whole candidates
-      if (lay.nsplit > 1) {
-        const int64_t t0 = ld.m[0].tile_off;
-        const int64_t t1 = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
-        if ((e = launch_merge_candidates(pcands, lay.nsplit, T, t0, t1, out, st)) != cudaSuccess)
-          return cuda_fail(e, "encode: merge");
-      }
-    } else if ((e = launch_finalize(pr, ld, masks, gram, partials, lay.nsplit, out, status, st)) != cudaSuccess) {
-      return cuda_fail(e, "encode: finalize");
+    if (lay.nsplit > 1) {  // best of the seed splits of each tile
+      const int64_t t0 = ld.m[0].tile_off;
+      const int64_t t1 = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
+      if ((e = launch_merge_candidates(pcands, lay.nsplit, T, t0, t1, out, st)) != cudaSuccess)
+        return cuda_fail(e, "encode: merge");
     }
   }
   return AWSRC_OK;

@@ -23,7 +23,7 @@ constexpr int kMaxModsPerLaunch = 16;
 
 // Fault bits of the device status word kept at the start of every workspace.
 constexpr uint32_t kFaultRecord = 1u;     // decoder: record names a tile/seed out of range
-constexpr uint32_t kFaultSelfCheck = 2u;  // encoder: finalisation disagrees with the search
+constexpr uint32_t kFaultSelfCheck = 2u;  // encoder: the winner's recomputation disagrees with the search
 constexpr uint32_t kFaultTimeout = 4u;    // a bounded wait gave up
 constexpr size_t kStatusBytes = 256;
 

@@ -1,15 +1,13 @@
 // encode.cu — the seed search of Sec. 3.2 for any supported (C, P) and both
-// variants, plus the two kernels around every search:
+// variants, and the U Gram tables every U search reads:
 //
 //  gram_u      U only. The activation diagonal is shared by all rows of a module
 //              (Sec. 3.2), so the Gram matrix B_s^T D B_s of Eq. 3 and its LDL^T
 //              depend on (column block, seed) only. They are computed once per
 //              (cb, s) and reused by every row.
 //  search      per (tile, seed): correlation b = B_s^T D r, solve, quantise,
-//              gain; running argmax over the seeds of one split.
-//  finalize    per tile: argmax over splits, then recomputation of the winning
-//              seed's codes and scale with the same operations; the recomputed
-//              gain must equal the searched one bit for bit (self-check bit).
+//              gain; the best seed of each tile (over one seed split) is
+//              written as a whole candidate.
 #include <cfloat>
 
 #include "internal.h"
@@ -18,9 +16,6 @@ namespace awsrc {
 
 namespace {
 
-constexpr int kGenRows = 32;      // rows per block of the generic search
-constexpr int kGenLanes = 8;      // seed lanes per row
-constexpr int kGenThreads = kGenRows * kGenLanes;
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
@@ -170,23 +165,9 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   }
 }
 
-// Tile staging shared by search and finalisation: r = W - W0, d, y = d*r.
-__device__ __forceinline__ void tile_elem(const Prm& pr, const ModDesc& md, int64_t row,
-                                          int64_t cb, int j, float* y, float* d, bool* ok) {
-  const int64_t idx = row * md.cols + cb * pr.C + j;
-  const float r = __fsub_rn(load_elem(md.W, idx, md.w_dtype), load_elem(md.W0, idx, md.w0_dtype));
-  const float a = md.act[cb * pr.C + j];
-  float dv;
-  if (pr.variant == AWSRC_VARIANT_U) dv = a;
-  else dv = __fadd_rn(__fmul_rn(md.w_act, a), __fmul_rn(md.w_fisher, md.fisher[idx]));
-  *ok = in_domain(r, dv);
-  *d = dv;
-  *y = __fmul_rn(dv, r);
-}
-
 // Score of seed s for one tile from its fixed-point Y (and D for PF): the +-1
 // correlations are exact integer sums, rounded once and scaled by 2^q.
-template <int P, int VAR, bool ALLOW_FAST = true>
+template <int P, int VAR>
 __device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const int* Di, float two_qy,
                                             float two_qd, float gd_row, const uint64_t* __restrict__ masks,
                                             const float* __restrict__ gram_cb, uint32_t s, float* q,
@@ -231,7 +212,7 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const 
     for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = gt[P * (P - 1) / 2 + P + i];
     const float gd = gt[P * (P - 1) + P];
     ldl_solve<P>(L, invD, bv, alpha);
-    if (ALLOW_FAST && pr.fast_pow2) {
+    if (pr.fast_pow2) {
 #pragma unroll
       for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(2.0f, Goff[i]);
       return quant_gain_fast<P>(pr, alpha, bv, gd, Goff, q, sf);
@@ -245,7 +226,7 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const 
     const bool ok = ldl_factor<P>(gd_row, eps, Goff, L, invD);
     ldl_solve<P>(L, invD, bv, alpha);
     float g;
-    if (ALLOW_FAST && pr.fast_pow2) {
+    if (pr.fast_pow2) {
 #pragma unroll
       for (int i = 0; i < P * (P - 1) / 2; ++i) Goff[i] = __fmul_rn(2.0f, Goff[i]);
       g = quant_gain_fast<P>(pr, alpha, bv, gd_row, Goff, q, sf);
@@ -283,82 +264,6 @@ __device__ __forceinline__ void split_range(int S, int chunk, int nsplit, int z,
   *s1 = min(S, (z + 1) * per * chunk);
 }
 
-// ---------------------------------------------------------- generic search --
-template <int P, int VAR>
-__global__ void __launch_bounds__(kGenThreads) search_generic_kernel(
-    Prm pr, LaunchDesc ld, const uint64_t* __restrict__ masks, const float* __restrict__ gram,
-    float2* __restrict__ partials) {
-  extern __shared__ float smem[];
-  const int mi = find_mod(ld, blockIdx.x);
-  const ModDesc& md = ld.m[mi];
-  const int64_t b = blockIdx.x - md.block_off;
-  const int z = (int)(b % md.nsplit);
-  const int64_t rest = b / md.nsplit;
-  const int64_t rb = rest % md.n_rb;
-  const int64_t cb = rest / md.n_rb;
-  const int C = pr.C, ldc = C + 1;
-  float* ys = smem;
-  float* ds = smem + kGenRows * ldc;
-  __shared__ int rowok[kGenRows];
-  __shared__ float gds[kGenRows];
-  const int tid = threadIdx.x;
-  if (tid < kGenRows) rowok[tid] = 1;
-  __syncthreads();
-  for (int e = tid; e < kGenRows * C; e += kGenThreads) {
-    const int r = e / C, j = e % C;
-    const int64_t row = rb * kGenRows + r;
-    float y = 0.0f, d = 0.0f;
-    if (row < md.rows) {
-      bool ok;
-      tile_elem(pr, md, row, cb, j, &y, &d, &ok);
-      if (!ok) rowok[r] = 0;
-    }
-    ys[r * ldc + j] = y;
-    if (VAR == AWSRC_VARIANT_PF) ds[r * ldc + j] = d;
-  }
-  __syncthreads();
-  __shared__ float tqy[kGenRows], tqd[kGenRows];
-  if (tid < kGenRows) {
-    tqy[tid] = row_to_fixed(ys + tid * ldc, C);
-    if (VAR == AWSRC_VARIANT_PF) {
-      tqd[tid] = row_to_fixed(ds + tid * ldc, C);
-      gds[tid] = row_gd(pr, reinterpret_cast<const int*>(ds + tid * ldc), tqd[tid]);
-    }
-  }
-  __syncthreads();
-  const int r = tid / kGenLanes, sl = tid % kGenLanes;
-  const int64_t row = rb * kGenRows + r;
-  int s0, s1;
-  split_range(pr.S, kGenLanes, md.nsplit, z, &s0, &s1);
-  float bg = neg_inf();
-  uint32_t bs = 0xffffffffu;
-  const float* gram_cb = (VAR == AWSRC_VARIANT_U)
-                             ? gram + (size_t)(md.gram_off + cb * pr.S_pad) * gram_stride(P)
-                             : nullptr;
-  if (row < md.rows && rowok[r]) {
-    for (int s = s0 + sl; s < s1; s += kGenLanes) {
-      float q[P];
-      int sf;
-      const float g = score_seed<P, VAR>(pr, reinterpret_cast<const int*>(ys + r * ldc),
-                                         reinterpret_cast<const int*>(ds + r * ldc), tqy[r],
-                                         VAR == AWSRC_VARIANT_PF ? tqd[r] : 0.0f,
-                                         VAR == AWSRC_VARIANT_PF ? gds[r] : 0.0f, masks, gram_cb,
-                                         (uint32_t)s, q, &sf);
-      if (better(g, (uint32_t)s, bg, bs)) { bg = g; bs = (uint32_t)s; }
-    }
-  }
-#pragma unroll
-  for (int off = 1; off < kGenLanes; off <<= 1) {
-    const float og = __shfl_xor_sync(0xffffffffu, bg, off);
-    const uint32_t os = __shfl_xor_sync(0xffffffffu, bs, off);
-    if (better(og, os, bg, bs)) { bg = og; bs = os; }
-  }
-  if (sl == 0 && row < md.rows) {
-    const int64_t t = md.tile_off + row * md.n_cb + cb;
-    partials[(size_t)z * ld.T + t] = make_float2(rowok[r] ? bg : neg_inf(), __uint_as_float(bs));
-  }
-}
-
 // V consecutive elements (V = 4 or 8) of a weight array as floats; idx is a
 // multiple of V. Vector loads when the array is 16-byte aligned.
 template <int V>
@@ -383,12 +288,14 @@ __device__ __forceinline__ void load_run(const void* p, int64_t idx, int dtype, 
   }
 }
 
-// --------------------------------------------------------------- finalize --
-// One thread per tile; a block stages its tiles' y (and d) in shared memory with
-// coalesced loads: tiles are numbered row-major, so consecutive tiles of a
-// module are consecutive C-element runs of its weight arrays.
-__host__ __device__ inline int fin_tiles(int C) { return C <= 64 ? 128 : 16384 / C; }
-
+// ---------------------------------------------------------- generic search --
+// Any (C, P, variant): a block takes TB consecutive tiles of the launch (a
+// module's tiles are consecutive C-element runs of its weight arrays, so the
+// staging loads are coalesced vectors), converts each tile to its fixed-point
+// grid, and `lanes` threads per tile score interleaved seeds with score_seed;
+// the best seed of each tile (larger gain, then smaller seed) is merged across
+// lanes with its codes and scale field and written as a whole candidate (seed
+// split z of it when the seeds are split over blocks).
 // Stage y = d*(W - W0) (and d) of tiles [t0, t0 + TB) in shared memory, V
 // elements per load, loads of four runs issued before any is used.
 template <int V, int VAR>
@@ -439,21 +346,21 @@ __device__ __forceinline__ void stage_tiles(const Prm& pr, const LaunchDesc& ld,
 }
 
 template <int P, int VAR>
-__global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
-                                                       const uint64_t* __restrict__ masks,
-                                                       const float* __restrict__ gram,
-                                                       const float2* __restrict__ partials,
-                                                       awsrc_candidate* __restrict__ out,
-                                                       uint32_t* __restrict__ status) {
+__global__ void __launch_bounds__(256) search_tiles_kernel(Prm pr, LaunchDesc ld, const uint64_t* __restrict__ masks,
+                                                           const float* __restrict__ gram,
+                                                           awsrc_candidate* __restrict__ cands, int lanes, int TB) {
   extern __shared__ float fsm[];
-  const int C = pr.C, ldc = C + 1, TB = fin_tiles(C);
+  const int C = pr.C, ldc = C + 1;
   float* ys = fsm;
   float* ds = fsm + TB * ldc;
-  __shared__ int tmod[128];
-  __shared__ int tok[128];
+  __shared__ int tmod[256];
+  __shared__ int tok[256];
+  __shared__ float tqy[256], tqd[256], gds[256];
+  const int nsplit = ld.m[0].nsplit;
+  const int z = (int)(blockIdx.x % nsplit);
   const int64_t first = ld.m[0].tile_off;
   const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
-  const int64_t t0 = first + (int64_t)blockIdx.x * TB;
+  const int64_t t0 = first + (int64_t)(blockIdx.x / nsplit) * TB;
   const int tid = threadIdx.x;
   if (tid < TB) {
     const int64_t t = t0 + tid;
@@ -467,53 +374,74 @@ __global__ void __launch_bounds__(128) finalize_kernel(Prm pr, LaunchDesc ld,
   if (C >= 8) stage_tiles<8, VAR>(pr, ld, t0, last, TB, tmod, tok, ys, ds);
   else stage_tiles<4, VAR>(pr, ld, t0, last, TB, tmod, tok, ys, ds);
   __syncthreads();
-  if (tid >= TB) return;
-  const int64_t t = t0 + tid;
-  if (t >= last) return;
-  const ModDesc& md = ld.m[tmod[tid]];
-  const int64_t cb = (t - md.tile_off) % md.n_cb;
+  if (tid < TB) {
+    tqy[tid] = row_to_fixed(ys + tid * ldc, C);
+    if (VAR == AWSRC_VARIANT_PF) {
+      tqd[tid] = row_to_fixed(ds + tid * ldc, C);
+      gds[tid] = row_gd(pr, reinterpret_cast<const int*>(ds + tid * ldc), tqd[tid]);
+    }
+  }
+  __syncthreads();
+  const int lt = tid / lanes, sl = tid % lanes;
+  const int64_t t = t0 + lt;
   float bg = neg_inf();
   uint32_t bs = 0xffffffffu;
-  for (int z = 0; z < md.nsplit; ++z) {
-    const float2 pz = partials[(size_t)z * ld.T + t];
-    const float g = pz.x;
-    const uint32_t s = __float_as_uint(pz.y);
-    if (better(g, s, bg, bs)) { bg = g; bs = s; }
-  }
-  awsrc_candidate cd;
-  cd.gain = neg_inf();
-  cd.seed = 0;
-  cd.scale = 0;
+  float bq[P];
 #pragma unroll
-  for (int p = 0; p < 8; ++p) cd.code[p] = 0;
-  if (bg > neg_inf() && bs < (uint32_t)pr.S) {
-    const bool ok = tok[tid] != 0;
-    const float two_qy = row_to_fixed(ys + tid * ldc, C);
-    float two_qd = 0.0f, gd_row = 0.0f;
-    if (VAR == AWSRC_VARIANT_PF) {
-      two_qd = row_to_fixed(ds + tid * ldc, C);
-      gd_row = row_gd(pr, reinterpret_cast<const int*>(ds + tid * ldc), two_qd);
-    }
+  for (int p = 0; p < P; ++p) bq[p] = 0.0f;
+  int bsf = 0;
+  const bool live = t < last && tok[lt] != 0;
+  if (live) {
+    const ModDesc& md = ld.m[tmod[lt]];
+    const int64_t cb = (t - md.tile_off) % md.n_cb;
     const float* gram_cb = (VAR == AWSRC_VARIANT_U)
                                ? gram + (size_t)(md.gram_off + cb * pr.S_pad) * gram_stride(P)
                                : nullptr;
-    float q[P];
-    int sf = 0;
-    // the general quantiser here, so the self-check also compares it with the
-    // fast path the search used
-    const float g = score_seed<P, VAR, false>(pr, reinterpret_cast<const int*>(ys + tid * ldc),
-                                              reinterpret_cast<const int*>(ds + tid * ldc), two_qy, two_qd,
-                                              gd_row, masks, gram_cb, bs, q, &sf);
-    if (!ok || __float_as_uint(g) != __float_as_uint(bg)) atomicOr(status, kFaultSelfCheck);
-    if (ok && g > neg_inf()) {
-      cd.gain = g;
-      cd.seed = (uint16_t)bs;
-      cd.scale = (int16_t)sf;
+    int s0, s1;
+    split_range(pr.S, lanes, nsplit, z, &s0, &s1);
+    for (int s = s0 + sl; s < s1; s += lanes) {
+      float q[P];
+      int sf;
+      const float g = score_seed<P, VAR>(pr, reinterpret_cast<const int*>(ys + lt * ldc),
+                                         reinterpret_cast<const int*>(ds + lt * ldc), tqy[lt],
+                                         VAR == AWSRC_VARIANT_PF ? tqd[lt] : 0.0f,
+                                         VAR == AWSRC_VARIANT_PF ? gds[lt] : 0.0f, masks, gram_cb,
+                                         (uint32_t)s, q, &sf);
+      if (better(g, (uint32_t)s, bg, bs)) {
+        bg = g;
+        bs = (uint32_t)s;
+        bsf = sf;
 #pragma unroll
-      for (int p = 0; p < P; ++p) cd.code[p] = (int8_t)(int)q[p];
+        for (int p = 0; p < P; ++p) bq[p] = q[p];
+      }
     }
   }
-  out[t] = cd;
+  // lanes of a tile are consecutive threads of one warp (lanes <= 8, blockDim a multiple of 32)
+  for (int off = 1; off < lanes; off <<= 1) {
+    const float og = __shfl_xor_sync(0xffffffffu, bg, off);
+    const uint32_t os = __shfl_xor_sync(0xffffffffu, bs, off);
+    const int osf = __shfl_xor_sync(0xffffffffu, bsf, off);
+    float oq[P];
+#pragma unroll
+    for (int p = 0; p < P; ++p) oq[p] = __shfl_xor_sync(0xffffffffu, bq[p], off);
+    if (better(og, os, bg, bs)) {
+      bg = og;
+      bs = os;
+      bsf = osf;
+#pragma unroll
+      for (int p = 0; p < P; ++p) bq[p] = oq[p];
+    }
+  }
+  if (sl == 0 && t < last) {
+    awsrc_candidate cd;
+    const bool valid = live && bg > neg_inf() && bs < (uint32_t)pr.S;
+    cd.gain = valid ? bg : neg_inf();
+    cd.seed = valid ? (uint16_t)bs : (uint16_t)0;
+    cd.scale = valid ? (int16_t)bsf : (int16_t)0;
+#pragma unroll
+    for (int p = 0; p < 8; ++p) cd.code[p] = (p < P && valid) ? (int8_t)(int)bq[p < P ? p : 0] : (int8_t)0;
+    cands[(size_t)z * ld.T + t] = cd;
+  }
 }
 
 template <int P>
@@ -528,30 +456,14 @@ cudaError_t launch_gram_p(const Prm& pr, const LaunchDesc& ld, const uint64_t* m
 }
 
 template <int P, int VAR>
-cudaError_t launch_search_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                             const float* gram, int64_t n_blocks, float2* partials,
-                             cudaStream_t st) {
-  const size_t smem = (size_t)kGenRows * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
-  auto k = search_generic_kernel<P, VAR>;
+cudaError_t launch_search_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, const float* gram,
+                             int64_t n_blocks, awsrc_candidate* cands, cudaStream_t st) {
+  const GenShape gs = gen_shape(pr);
+  const size_t smem = (size_t)gs.tiles * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
+  auto k = search_tiles_kernel<P, VAR>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<(unsigned)n_blocks, kGenThreads, smem, st>>>(pr, ld, masks, gram, partials);
-  note_launches(1);
-  return cudaGetLastError();
-}
-
-template <int P, int VAR>
-cudaError_t launch_finalize_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                               const float* gram, const float2* partials, awsrc_candidate* out,
-                               uint32_t* status, cudaStream_t st) {
-  const int64_t first = ld.m[0].tile_off;
-  const int64_t last = ld.m[ld.n - 1].tile_off + ld.m[ld.n - 1].rows * ld.m[ld.n - 1].n_cb;
-  const int TB = fin_tiles(pr.C);
-  const size_t smem = (size_t)TB * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
-  auto k = finalize_kernel<P, VAR>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  k<<<(unsigned)((last - first + TB - 1) / TB), 128, smem, st>>>(pr, ld, masks, gram, partials, out, status);
+  k<<<(unsigned)n_blocks, gs.tiles * gs.lanes, smem, st>>>(pr, ld, masks, gram, cands, gs.lanes, gs.tiles);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -577,25 +489,23 @@ cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* m
 }
 
 cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                                  const float* gram, int64_t n_blocks, float2* partials,
+                                  const float* gram, int64_t n_blocks, awsrc_candidate* cands,
                                   cudaStream_t st) {
   if (pr.variant == AWSRC_VARIANT_U) {
-    AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_U>(pr, ld, masks, gram, n_blocks, partials, st)));
+    AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_U>(pr, ld, masks, gram, n_blocks, cands, st)));
   }
-  AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_PF>(pr, ld, masks, gram, n_blocks, partials, st)));
+  AWSRC_DISPATCH_P(pr.P, (launch_search_pv<PP, AWSRC_VARIANT_PF>(pr, ld, masks, gram, n_blocks, cands, st)));
 }
 
-cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                            const float* gram, const float2* partials, int nsplit_max,
-                            awsrc_candidate* out, uint32_t* status, cudaStream_t st) {
-  (void)nsplit_max;
-  if (pr.variant == AWSRC_VARIANT_U) {
-    AWSRC_DISPATCH_P(pr.P, (launch_finalize_pv<PP, AWSRC_VARIANT_U>(pr, ld, masks, gram, partials, out, status, st)));
-  }
-  AWSRC_DISPATCH_P(pr.P, (launch_finalize_pv<PP, AWSRC_VARIANT_PF>(pr, ld, masks, gram, partials, out, status, st)));
+GenShape gen_shape(const Prm& pr) {
+  // one lane per four seeds (at most 8), 256 threads, shared memory for the
+  // staged tiles at most 96 KB (but at least 32 threads)
+  int lanes = 1;
+  while (lanes < 8 && lanes * 4 < pr.S) lanes <<= 1;
+  int tiles = 256 / lanes;
+  const size_t per_tile = (size_t)(pr.C + 1) * sizeof(float) * (pr.variant == AWSRC_VARIANT_PF ? 2 : 1);
+  while (tiles * lanes > 32 && tiles * per_tile > 96 * 1024) tiles >>= 1;
+  return {lanes, tiles};
 }
-
-int generic_rows() { return kGenRows; }
-int generic_chunk() { return kGenLanes; }
 
 }  // namespace awsrc

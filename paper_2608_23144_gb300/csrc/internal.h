@@ -32,12 +32,16 @@ cudaError_t launch_gen_basis(const Prm& pr, uint64_t* masks, int S_out, cudaStre
 // (pair_stride(P) float2 per seed pair) the C = 64, P = 4 search reads.
 cudaError_t launch_gram_u(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
                           float* gram, float2* pairs, cudaStream_t st);
+// The generic search (any C, P, variant): blocks of gen_shape(pr).tiles
+// consecutive tiles, `lanes` threads per tile; writes whole candidates to
+// cands[z * T + t] like the specialised kernels.
+struct GenShape {
+  int lanes, tiles;
+};
+GenShape gen_shape(const Prm& pr);
 cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                                  const float* gram, int64_t n_blocks, float2* partials,
+                                  const float* gram, int64_t n_blocks, awsrc_candidate* cands,
                                   cudaStream_t st);
-cudaError_t launch_finalize(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks,
-                            const float* gram, const float2* partials, int nsplit_max,
-                            awsrc_candidate* out, uint32_t* status, cudaStream_t st);
 // search_c64p4.cu
 // FP16 table of the +-1 atoms in MMA operand order, then the tcgen05 search.
 size_t search_c64p4_table_bytes(int S_pad);
@@ -53,7 +57,7 @@ cudaError_t launch_merge_candidates(const awsrc_candidate* pc, int nsplit, int64
 int search_c64p4_rows();   // rows per block of the specialised kernel
 int search_c64p4_chunk();  // seeds per chunk of the specialised kernel
 // search_pf_c64p4.cu: P_F with C = 64, P = 4 on tcgen05 (atoms from the table
-// above, plus a table of atom products), same partials layout.
+// above, plus a table of atom products), same candidate output.
 int search_pf_c64p4_chunk();
 size_t search_pf_c64p4_table_bytes(int S_pad);
 cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st);
@@ -88,7 +92,5 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
 size_t decode_scratch_bytes(int64_t T, int mode);
 // The dense fused decoder clears the fault word itself (no separate memset).
 bool decode_clears_status(const Prm& pr, int mode);
-int generic_rows();
-int generic_chunk();
 
 }  // namespace awsrc
