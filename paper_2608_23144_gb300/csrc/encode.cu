@@ -165,19 +165,20 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   }
 }
 
-// Score of seed s for one tile from its fixed-point Y (and D for PF): the +-1
-// correlations are exact integer sums, rounded once and scaled by 2^q.
+// The score of seed s for one tile works on its fixed-point Y (and D for PF):
+// the +-1 correlations are exact integer sums, rounded once and scaled by 2^q.
+template <int P>
+__host__ __device__ constexpr int n_off() { return P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1; }
+
+// The +-1 correlations of seed s with the tile's fixed-point Y (u) and, for
+// PF, of the pairwise atom products with D (v), element by element.
 template <int P, int VAR>
-__device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const int* Di, float two_qy,
-                                            float two_qd, float gd_row, const uint64_t* __restrict__ masks,
-                                            const float* __restrict__ gram_cb, uint32_t s, float* q,
-                                            int* sf) {
-  constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
+__device__ __forceinline__ void seed_sums(const Prm& pr, const int* Yi, const int* Di,
+                                          const uint64_t* __restrict__ masks, uint32_t s, int* u, int* v) {
+  constexpr int NL = n_off<P>();
   const uint64_t* mk = masks + (size_t)s * P * pr.W;
-  int u[P];
 #pragma unroll
   for (int p = 0; p < P; ++p) u[p] = 0;
-  int v[NL];
 #pragma unroll
   for (int i = 0; i < NL; ++i) v[i] = 0;
   for (int wd = 0; wd < pr.W; ++wd) {
@@ -198,6 +199,47 @@ __device__ __forceinline__ float score_seed(const Prm& pr, const int* Yi, const 
       }
     }
   }
+}
+
+// The same sums from per-tile nibble tables (C <= 64, one mask word):
+// Ty[16 g + m] = sum_{i<4} (bit i of m ? -Y : Y)[4 g + i], likewise Td for D,
+// so each correlation is C/4 table reads. Integer sums: exact in any order.
+template <int P, int VAR>
+__device__ __forceinline__ void seed_sums_tab(const Prm& pr, const int* Ty, const int* Td,
+                                              const uint64_t* __restrict__ masks, uint32_t s, int* u, int* v) {
+  const uint64_t* mk = masks + (size_t)s * P;
+  uint64_t m[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    m[p] = mk[p];
+    u[p] = 0;
+  }
+  if (VAR == AWSRC_VARIANT_PF) {
+#pragma unroll
+    for (int i = 0; i < n_off<P>(); ++i) v[i] = 0;
+  }
+  const int ng = pr.C >> 2;
+  for (int g = 0; g < ng; ++g) {
+    const int* ty = Ty + 16 * g;
+#pragma unroll
+    for (int p = 0; p < P; ++p) u[p] += ty[(uint32_t)(m[p] >> (4 * g)) & 15u];
+    if (VAR == AWSRC_VARIANT_PF) {
+      const int* td = Td + 16 * g;
+#pragma unroll
+      for (int qq = 1; qq < P; ++qq)
+#pragma unroll
+        for (int p = 0; p < qq; ++p) v[tri(qq, p)] += td[(uint32_t)((m[p] ^ m[qq]) >> (4 * g)) & 15u];
+    }
+  }
+}
+
+// Score of a seed from its correlation sums: b and (PF) the Gram off-diagonals
+// rounded once and scaled, the ridge solve, quantiser and gain.
+template <int P, int VAR>
+__device__ __forceinline__ float score_sums(const Prm& pr, const int* u, const int* v, float two_qy,
+                                            float two_qd, float gd_row, const float* __restrict__ gram_cb,
+                                            uint32_t s, float* q, int* sf) {
+  constexpr int NL = n_off<P>();
   float bv[P], alpha[P];
 #pragma unroll
   for (int p = 0; p < P; ++p) bv[p] = __fmul_rn(pr.c, __fmul_rn(__int2float_rn(u[p]), two_qy));
@@ -289,6 +331,16 @@ __device__ __forceinline__ void load_run(const void* p, int64_t idx, int dtype, 
 }
 
 // ---------------------------------------------------------- generic search --
+// Nibble tables pay off when a tile is one mask word (C <= 64) and each table
+// serves several seeds.
+__host__ __device__ inline bool gen_tables(const Prm& pr) { return pr.C <= 64 && pr.S >= 4; }
+
+// Shared memory per tile: staged y (and d), plus the nibble tables.
+__host__ __device__ inline size_t gen_tile_smem(const Prm& pr) {
+  const size_t nb = pr.variant == AWSRC_VARIANT_PF ? 2 : 1;
+  return (nb * (size_t)(pr.C + 1) + (gen_tables(pr) ? nb * 4 * (size_t)pr.C + 1 : 0)) * sizeof(float);
+}
+
 // Any (C, P, variant): a block takes TB consecutive tiles of the launch (a
 // module's tiles are consecutive C-element runs of its weight arrays, so the
 // staging loads are coalesced vectors), converts each tile to its fixed-point
@@ -351,8 +403,14 @@ __global__ void __launch_bounds__(256) search_tiles_kernel(Prm pr, LaunchDesc ld
                                                            awsrc_candidate* __restrict__ cands, int lanes, int TB) {
   extern __shared__ float fsm[];
   const int C = pr.C, ldc = C + 1;
+  const int nb = VAR == AWSRC_VARIANT_PF ? 2 : 1;
   float* ys = fsm;
   float* ds = fsm + TB * ldc;
+  const bool tab = gen_tables(pr);
+  // nibble tables when tab: per tile [Y, D][C/4 groups][16], tiles one word
+  // apart beyond their size so that tiles read from different banks
+  const int tstride = nb * 4 * C + 1;
+  int* tabs = reinterpret_cast<int*>(fsm + (size_t)nb * TB * ldc);
   __shared__ int tmod[256];
   __shared__ int tok[256];
   __shared__ float tqy[256], tqd[256], gds[256];
@@ -383,6 +441,20 @@ __global__ void __launch_bounds__(256) search_tiles_kernel(Prm pr, LaunchDesc ld
   }
   __syncthreads();
   const int lt = tid / lanes, sl = tid % lanes;
+  if (tab) {  // the tile's lanes build its nibble tables
+    const int per = 4 * C;  // C/4 groups x 16 patterns
+    int* T = tabs + lt * tstride;
+    for (int k = sl; k < nb * per; k += lanes) {
+      const int which = k >= per ? 1 : 0, kk = k - which * per;
+      const int g = kk >> 4, m = kk & 15;
+      const int* X = reinterpret_cast<const int*>((which ? ds : ys) + lt * ldc) + 4 * g;
+      int acc = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc += ((m >> i) & 1) ? -X[i] : X[i];
+      T[k] = acc;
+    }
+    __syncthreads();
+  }
   const int64_t t = t0 + lt;
   float bg = neg_inf();
   uint32_t bs = 0xffffffffu;
@@ -399,14 +471,17 @@ __global__ void __launch_bounds__(256) search_tiles_kernel(Prm pr, LaunchDesc ld
                                : nullptr;
     int s0, s1;
     split_range(pr.S, lanes, nsplit, z, &s0, &s1);
+    const int* Ty = tabs + (size_t)lt * tstride;
     for (int s = s0 + sl; s < s1; s += lanes) {
       float q[P];
       int sf;
-      const float g = score_seed<P, VAR>(pr, reinterpret_cast<const int*>(ys + lt * ldc),
-                                         reinterpret_cast<const int*>(ds + lt * ldc), tqy[lt],
-                                         VAR == AWSRC_VARIANT_PF ? tqd[lt] : 0.0f,
-                                         VAR == AWSRC_VARIANT_PF ? gds[lt] : 0.0f, masks, gram_cb,
-                                         (uint32_t)s, q, &sf);
+      int u[P], v[n_off<P>()];
+      if (tab) seed_sums_tab<P, VAR>(pr, Ty, Ty + 4 * C, masks, (uint32_t)s, u, v);
+      else
+        seed_sums<P, VAR>(pr, reinterpret_cast<const int*>(ys + lt * ldc),
+                          reinterpret_cast<const int*>(ds + lt * ldc), masks, (uint32_t)s, u, v);
+      const float g = score_sums<P, VAR>(pr, u, v, tqy[lt], VAR == AWSRC_VARIANT_PF ? tqd[lt] : 0.0f,
+                                         VAR == AWSRC_VARIANT_PF ? gds[lt] : 0.0f, gram_cb, (uint32_t)s, q, &sf);
       if (better(g, (uint32_t)s, bg, bs)) {
         bg = g;
         bs = (uint32_t)s;
@@ -459,7 +534,7 @@ template <int P, int VAR>
 cudaError_t launch_search_pv(const Prm& pr, const LaunchDesc& ld, const uint64_t* masks, const float* gram,
                              int64_t n_blocks, awsrc_candidate* cands, cudaStream_t st) {
   const GenShape gs = gen_shape(pr);
-  const size_t smem = (size_t)gs.tiles * (pr.C + 1) * sizeof(float) * (VAR == AWSRC_VARIANT_PF ? 2 : 1);
+  const size_t smem = (size_t)gs.tiles * gen_tile_smem(pr);
   auto k = search_tiles_kernel<P, VAR>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -499,12 +574,11 @@ cudaError_t launch_search_generic(const Prm& pr, const LaunchDesc& ld, const uin
 
 GenShape gen_shape(const Prm& pr) {
   // one lane per four seeds (at most 8), 256 threads, shared memory for the
-  // staged tiles at most 96 KB (but at least 32 threads)
+  // staged tiles (and nibble tables) at most 96 KB (but at least 32 threads)
   int lanes = 1;
   while (lanes < 8 && lanes * 4 < pr.S) lanes <<= 1;
   int tiles = 256 / lanes;
-  const size_t per_tile = (size_t)(pr.C + 1) * sizeof(float) * (pr.variant == AWSRC_VARIANT_PF ? 2 : 1);
-  while (tiles * lanes > 32 && tiles * per_tile > 96 * 1024) tiles >>= 1;
+  while (tiles * lanes > 32 && tiles * gen_tile_smem(pr) > 96 * 1024) tiles >>= 1;
   return {lanes, tiles};
 }
 

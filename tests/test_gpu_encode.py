@@ -37,6 +37,9 @@ CASES = [
     ("c256p8_b8_u", dict(C=256, P=8, b=8, S=12), [(20, 512)], "bf16", False),
     ("c4p1_u", dict(C=4, P=1, b=4, S=9), [(11, 20)], "f32", False),
     ("c64p4_u_fp16_pf", dict(C=64, P=4, b=4, S=24, variant=1, scale_mode=1, b_e=16), [(40, 128)], "f32", True),
+    ("c64p3_u_generic", dict(C=64, P=3, b=4, S=70), [(90, 192), (5, 64)], "bf16", False),
+    ("c64p2_pf_generic", dict(C=64, P=2, b=3, S=21, variant=1), [(77, 128)], "bf16", True),
+    ("c32p4_pf_s3", dict(C=32, P=4, b=4, S=3, variant=1), [(50, 96)], "f32", True),
 ]
 
 
