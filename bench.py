@@ -45,8 +45,17 @@ OPS_PER_CANDIDATE = 8 + 6 + 4 + 4 + 1
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "eb3c0657891a1ae9405bc97349a5771be0d62e110b29fc534ad6a15f4cb2340b",
-                  "bytes_per_launch": 419272704 + 8250880}
+SEARCH_TRAFFIC = {"source_sha256": "29a1d54133a735296ac6bf130b08523e709c4b0ca9bb0357ebbafb796f3b2478",
+                  "bytes_per_launch": 419800000 + 16400000}
+
+
+def search_source_sha() -> str:
+    """SHA-256 of the search kernel's source and the headers it includes: the
+    committed DRAM traffic figure holds only for that exact kernel."""
+    h = hashlib.sha256()
+    for f in ("search_c64p4.cu", "tc05.cuh", "common.cuh", "internal.h"):
+        h.update(open(os.path.join(ROOT, "paper_2608_23144_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
 
 
 def parse():
@@ -382,9 +391,8 @@ def run_ours(args):
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
     fp32_peak = nsm * 128 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
     achieved = cands_per_step * OPS_PER_CANDIDATE / (search_ms * 1e-3)
-    src = open(os.path.join(ROOT, "paper_2608_23144_gb300", "csrc", "search_c64p4.cu"), "rb").read()
     traffic = (SEARCH_TRAFFIC["bytes_per_launch"]
-               if SEARCH_TRAFFIC["source_sha256"] == hashlib.sha256(src).hexdigest() else None)
+               if SEARCH_TRAFFIC["source_sha256"] == search_source_sha() else None)
     roofline = {"bound": "alu", "kernel": "search_c64p4", "achieved": achieved / 1e9,
                 "peak": fp32_peak / 1e9, "unit": "Gop/s", "frac": achieved / fp32_peak,
                 "traffic": traffic, "peak_kind": f"{peak_kind}: {nsm} SMs x 128 FP32 lanes x "
