@@ -675,3 +675,123 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
   }
   return bad;
 }
+
+/* ------------------------------------------------------------------------ */
+/* RTN-INT4 backbone (Eq. 1's W0 = Q(W); Sec. 4: round to nearest, groups of */
+/* `group` consecutive input coordinates of a row) and scale double          */
+/* quantisation (SDQ, Sec. 3.3: the group scales are themselves quantised,   */
+/* after QLoRA's double quantisation; the paper gives no format):            */
+/*  first level, group g (groups are consecutive runs since cols % group ==  */
+/*  0): s_g = binary16(max|w| / 7); q = clamp(rint(w / s_g), -8, 7), q = 0    */
+/*  when s_g == 0;                                                            */
+/*  second level (sdq != 0), per block of `block` consecutive groups:        */
+/*  mu = binary32((sum of the block's s_g, exact in double) / n), d = s_g -   */
+/*  mu, a = max|d|, step = a / 127, c_g = clamp(rint(d / step), -127, 127)   */
+/*  (0 when step == 0), s~_g = mu + c_g * step (two roundings);              */
+/*  W0 = q * s_eff in binary32, s_eff = s_g, or s~_g with SDQ.               */
+/* Outputs: q (rows*cols), s16 (G), c8 and consts (mu, step per block; SDQ   */
+/* only), s_eff (G), W0 (rows*cols).                                         */
+/* ------------------------------------------------------------------------ */
+void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block, const float* W, int8_t* q,
+                      uint16_t* s16, int8_t* c8, float* consts, float* s_eff, float* W0) {
+  const int64_t G = rows * cols / group;
+  for (int64_t g = 0; g < G; ++g) {
+    const float* w = W + g * group;
+    float amax = 0.0f;
+    for (int j = 0; j < group; ++j) {
+      const float a = fabsf(w[j]);
+      if (a > amax) amax = a;
+    }
+    const uint16_t h = orc_f32_to_f16(amax / 7.0f);
+    s16[g] = h;
+    const float s = orc_f16_to_f32(h);
+    for (int j = 0; j < group; ++j) {
+      float v = 0.0f;
+      if (s > 0.0f) {
+        v = rintf(w[j] / s);
+        if (v < -8.0f) v = -8.0f;
+        if (v > 7.0f) v = 7.0f;
+      }
+      q[g * group + j] = (int8_t)v;
+    }
+    s_eff[g] = s;
+  }
+  if (sdq) {
+    for (int64_t b0 = 0; b0 < G; b0 += block) {
+      const int64_t n = G - b0 < block ? G - b0 : block;
+      double sum = 0.0;
+      for (int64_t g = b0; g < b0 + n; ++g) sum += (double)s_eff[g];
+      const float mu = (float)(sum / (double)n);
+      float a = 0.0f;
+      for (int64_t g = b0; g < b0 + n; ++g) {
+        const float d = fabsf(s_eff[g] - mu);
+        if (d > a) a = d;
+      }
+      const float step = a / 127.0f;
+      consts[2 * (b0 / block)] = mu;
+      consts[2 * (b0 / block) + 1] = step;
+      for (int64_t g = b0; g < b0 + n; ++g) {
+        float cv = 0.0f;
+        if (step > 0.0f) {
+          cv = rintf((s_eff[g] - mu) / step);
+          if (cv < -127.0f) cv = -127.0f;
+          if (cv > 127.0f) cv = 127.0f;
+        }
+        c8[g] = (int8_t)cv;
+        s_eff[g] = mu + cv * step;
+      }
+    }
+  }
+  for (int64_t i = 0; i < rows * cols; ++i) W0[i] = (float)q[i] * s_eff[i / group];
+}
+
+/* ------------------------------------------------------------------------ */
+/* Definition of the packed product (the decoded weights applied to x        */
+/* without forming them): y[m][i] = sum_j (W0_ij + r_ij) x[m][j] in double,  */
+/* W0_ij = q_ij * s_eff (the backbone's binary32 value), r the decoder's      */
+/* residual (Sec. 3.2) on the                                                 */
+/* tiles named by the first K records of a one-module stream, in double:      */
+/* k_j * C^-1/2 * scale. yabs = sum_j |(W0_ij + r_ij) x[m][j]| bounds the    */
+/* rounding of any binary32 evaluation. x: M x cols, y and yabs: M x rows.   */
+/* ------------------------------------------------------------------------ */
+int orc_packed_gemv(const orc_params* prm, int64_t rows, int64_t cols, int group, const int8_t* q,
+                    const float* s_eff, const uint8_t* stream, int64_t K, int M, const float* x, double* y,
+                    double* yabs) {
+  const int C = prm->C, P = prm->P;
+  const int64_t T = rows * cols / C, n_cb = cols / C;
+  const int64_t h = orc_header_bytes(1), L = orc_record_bytes(prm, T);
+  double* Wt = (double*)malloc(sizeof(double) * (size_t)(rows * cols));
+  if (!Wt) return -1;
+  for (int64_t i = 0; i < rows * cols; ++i) Wt[i] = (double)((float)q[i] * s_eff[i / group]);
+  const double c = 1.0 / sqrt((double)C);
+  uint8_t sign[256], neg[8 * 256];
+  int32_t perm[256], colsel[8];
+  int bad = 0;
+  for (int64_t k = 0; k < K; ++k) {
+    int64_t tile;
+    orc_candidate cd;
+    orc_unpack_record(prm, T, stream + h + k * L, &tile, &cd);
+    if (tile >= T || cd.seed >= prm->S) { bad = 1; continue; }
+    const int64_t base = (tile / n_cb) * cols + (tile % n_cb) * C;
+    orc_gen_basis(prm->gen_seed, cd.seed, C, P, prm->permute, sign, perm, colsel, neg);
+    const double sc = prm->scale_mode == 0 ? ldexp(1.0, cd.scale) : (double)orc_f16_to_f32((uint16_t)cd.scale);
+    for (int j = 0; j < C; ++j) {
+      int kj = 0;
+      for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
+      Wt[base + j] += (double)kj * c * sc;
+    }
+  }
+  for (int m = 0; m < M; ++m)
+    for (int64_t i = 0; i < rows; ++i) {
+      double acc = 0.0, aabs = 0.0;
+      for (int64_t j = 0; j < cols; ++j) {
+        const double t = Wt[i * cols + j] * (double)x[(int64_t)m * cols + j];
+        acc += t;
+        aabs += fabs(t);
+      }
+      y[(int64_t)m * rows + i] = acc;
+      yabs[(int64_t)m * rows + i] = aabs;
+    }
+  free(Wt);
+  return bad;
+}

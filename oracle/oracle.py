@@ -10,6 +10,8 @@ the C file, which follows the paper step by step:
 * ``def_fit/def_gain``  Eq. 3 and Eq. 4 in double (definition mode)
 * ``select_records``    Sec. 3.3 allocation and Sec. 3.4 serialisation (Eq. 5)
 * ``decode_apply``      Sec. 3.2 decoder
+* ``rtn_quantize``      the RTN-INT4 g128 backbone (Eq. 1, Sec. 4) and SDQ (Sec. 3.3)
+* ``packed_gemv``       (W0 + r_hat) x in double from the packed backbone and a stream
 """
 from __future__ import annotations
 
@@ -101,6 +103,11 @@ def lib():
                                              vp, ct.c_int64, vp, vp]
             L.orc_decode_apply.restype = ct.c_int
             L.orc_decode_apply.argtypes = [P(Params), ct.c_int32, vp, vp, vp, ct.c_int64, vp, ct.c_int]
+            L.orc_rtn_quantize.argtypes = [ct.c_int64, ct.c_int64, ct.c_int, ct.c_int, ct.c_int, vp, vp, vp, vp,
+                                           vp, vp, vp]
+            L.orc_packed_gemv.restype = ct.c_int
+            L.orc_packed_gemv.argtypes = [P(Params), ct.c_int64, ct.c_int64, ct.c_int, vp, vp, vp, ct.c_int64,
+                                          ct.c_int, vp, vp, vp]
             _lib = L
     return _lib
 
@@ -312,3 +319,38 @@ def decode_apply(prm: Params, W0_list, stream: bytes, K: int, out_bf16: bool = F
     bad = lib().orc_decode_apply(ct.byref(prm), len(outs), _ptr(rows), _ptr(cols), _ptr(buf), K,
                                  ptrs, int(out_bf16))
     return outs, int(bad)
+
+
+def rtn_quantize(W, group: int = 128, sdq: bool = False, block: int = 256):
+    """RTN-INT4 backbone and optional scale double quantisation of one module.
+    Returns dict(q, s16, c8, consts, s_eff, W0) (W0 in float32)."""
+    W = np.ascontiguousarray(W, np.float32)
+    rows, cols = W.shape
+    assert cols % group == 0
+    G = rows * cols // group
+    nb = (G + block - 1) // block
+    q = np.zeros((rows, cols), np.int8)
+    s16 = np.zeros(G, np.uint16)
+    c8 = np.zeros(G, np.int8)
+    consts = np.zeros(2 * nb, np.float32)
+    s_eff = np.zeros(G, np.float32)
+    W0 = np.zeros((rows, cols), np.float32)
+    lib().orc_rtn_quantize(ct.c_int64(rows), ct.c_int64(cols), group, int(sdq), block, _ptr(W), _ptr(q),
+                           _ptr(s16), _ptr(c8), _ptr(consts), _ptr(s_eff), _ptr(W0))
+    return {"q": q, "s16": s16, "c8": c8, "consts": consts, "s_eff": s_eff, "W0": W0}
+
+
+def packed_gemv(prm: Params, q, s_eff, group: int, stream: bytes, K: int, x):
+    """y = (W0 + r_hat) x in double (one module). Returns (y, yabs, bad): y and
+    yabs of shape (M, rows), yabs = sum_j |(W0 + r_hat)_ij x_j|."""
+    q = np.ascontiguousarray(q, np.int8)
+    rows, cols = q.shape
+    x = np.ascontiguousarray(np.atleast_2d(x), np.float32)
+    M = x.shape[0]
+    y = np.zeros((M, rows), np.float64)
+    yabs = np.zeros((M, rows), np.float64)
+    buf = np.frombuffer(stream, np.uint8).copy()
+    bad = lib().orc_packed_gemv(ct.byref(prm), ct.c_int64(rows), ct.c_int64(cols), group, _ptr(q),
+                                _ptr(np.ascontiguousarray(s_eff, np.float32)), _ptr(buf), ct.c_int64(K), M,
+                                _ptr(x), _ptr(y), _ptr(yabs))
+    return y, yabs, int(bad)
