@@ -197,6 +197,46 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod,
                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * awsrc_rtn_quantize — the RTN-INT4 backbone W0 = Q(W) of Eq. 1 that the
+ * residual R = W - W0 is coded against: symmetric round to nearest with groups
+ * of 128 consecutive input coordinates of a row (Sec. 4), optionally with scale
+ * double quantisation (SDQ, Sec. 3.3, after QLoRA's double quantisation; the
+ * paper gives no format, this is the library's). All binary32, one rounding per
+ * operation:
+ *   group g (row-major, cols % 128 == 0): s_g = binary16(max|w| / 7);
+ *     q = clamp(rint(w / s_g), -8, 7), q = 0 when s_g == 0 (|q| <= 7 in fact);
+ *   SDQ block b of 256 consecutive groups (the last may be shorter, n groups):
+ *     mu = binary32((sum of the block's s_g, exact in double) / n);
+ *     step = max_g |s_g - mu| / 127;
+ *     c_g = clamp(rint((s_g - mu) / step), -127, 127), 0 when step == 0;
+ *     s~_g = mu + c_g * step;
+ *   W0 = q * s_eff with s_eff = s_g, or s~_g under SDQ (codes stay those of s_g).
+ * Metadata: binary16 scales cost 2 bytes per group (0.125 bits/weight); SDQ
+ * 1 byte per group plus 8 per block (0.0645 bits/weight on whole blocks), see
+ * awsrc_backbone_metadata_bytes. W must be finite.
+ *   W           device, rows*cols elements of w_dtype, 16-byte aligned.
+ *   codes       device, rows*cols/2 bytes: element 2i in the low nibble of byte
+ *               i, 4-bit two's complement.
+ *   scales      device, G = rows*cols/128 binary16 s_g, or NULL.
+ *   sdq_codes   device, G int8 c_g (SDQ), or NULL.
+ *   sdq_consts  device, 2*ceil(G/256) floats (mu, step) per block (SDQ), or NULL.
+ *   W0          device, rows*cols elements of w0_dtype (16-byte aligned), or NULL.
+ * Errors: INVALID_ARG, SHAPE (cols % 128), CUDA.
+ */
+awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32_t w_dtype, int32_t sdq,
+                                uint8_t* codes, uint16_t* scales, int8_t* sdq_codes, float* sdq_consts,
+                                void* W0, int32_t w0_dtype, void* stream);
+
+/*
+ * awsrc_backbone_metadata_bytes — scale metadata of a rows x cols RTN-INT4
+ * backbone: 2 bytes per group of 128, or with SDQ 1 per group plus 8 per block
+ * of 256 groups. Under a fixed total budget the bytes SDQ saves can go to the
+ * residual records (Sec. 3.3): raise the rate given to awsrc_select_records by
+ * 8 * saved / N_scope bits/weight. Returns -1 for a bad shape.
+ */
+int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq);
+
+/*
  * awsrc_gen_basis — writes the sign masks of GenBasis (Eq. 2) for seeds [0, S):
  * masks[(s*P + p)*W + w], W = ceil(C/64) words, bit j%64 of word j/64 set when
  * entry (j, p) of B_s is negative. Device array of S*P*W uint64. Used by the

@@ -8,6 +8,8 @@ binding with the same entry-point names:
 * ``awsrc_encode_tiles``   per-(tile, seed) search of Sec. 3.2 (Eqs. 2-4)
 * ``awsrc_select_records`` byte-aware allocation and stream (Sec. 3.3-3.4, Eq. 5)
 * ``awsrc_decode_apply``   decoder, W_hat = W0 + B_s alpha_hat (Eq. 1)
+* ``awsrc_rtn_quantize``   the RTN-INT4 backbone W0 = Q(W) with optional scale
+  double quantisation (Sec. 3.3)
 """
 from ._binding import (  # noqa: F401
     CANDIDATE_DTYPE,
@@ -28,6 +30,8 @@ from ._binding import (  # noqa: F401
     awsrc_encode_tiles,
     awsrc_encode_workspace_bytes,
     awsrc_gen_basis,
+    awsrc_rtn_quantize,
+    awsrc_backbone_metadata_bytes,
     awsrc_header_bytes,
     awsrc_kernel_launches,
     awsrc_record_bytes,

@@ -225,6 +225,27 @@ awsrc_status awsrc_encode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
   return AWSRC_OK;
 }
 
+awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32_t w_dtype, int32_t sdq,
+                                uint8_t* codes, uint16_t* scales, int8_t* sdq_codes, float* sdq_consts,
+                                void* W0, int32_t w0_dtype, void* stream) {
+  if (rows < 1 || cols < 1 || cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
+  if (w_dtype != AWSRC_DTYPE_F32 && w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+  if (w0_dtype != AWSRC_DTYPE_F32 && w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+  if (sdq != 0 && sdq != 1) return AWSRC_ERR_INVALID_ARG;
+  if (!W || !codes || !aligned(W, 16) || !aligned(codes, 2) || !aligned(scales, 2) || !aligned(sdq_consts, 4) ||
+      !aligned(W0, 16))
+    return AWSRC_ERR_INVALID_ARG;
+  const cudaError_t e = launch_rtn(W, w_dtype, rows, cols, sdq, codes, scales, sdq_codes, sdq_consts, W0,
+                                   w0_dtype, (cudaStream_t)stream);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "rtn_quantize");
+}
+
+int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq) {
+  if (rows < 1 || cols < 1 || cols % rtn_group() != 0) return -1;
+  const int64_t G = rows * cols / rtn_group();
+  return sdq ? G + 8 * ((G + sdq_block() - 1) / sdq_block()) : 2 * G;
+}
+
 awsrc_status awsrc_gen_basis(const awsrc_params* prm, uint64_t* masks, void* stream) {
   Prm pr;
   awsrc_status s = make_prm(prm, &pr);

@@ -93,4 +93,11 @@ size_t decode_scratch_bytes(int64_t T, int mode);
 // The dense fused decoder clears the fault word itself (no separate memset).
 bool decode_clears_status(const Prm& pr, int mode);
 
+// backbone.cu: RTN-INT4 groups of rtn_group() inputs, SDQ blocks of sdq_block() groups.
+int rtn_group();
+int sdq_block();
+cudaError_t launch_rtn(const void* W, int w_dtype, int64_t rows, int64_t cols, int sdq, uint8_t* codes,
+                       uint16_t* scales, int8_t* sdq_codes, float* sdq_consts, void* W0, int w0_dtype,
+                       cudaStream_t st);
+
 }  // namespace awsrc

@@ -133,3 +133,14 @@ def test_misaligned_pointers_are_refused_before_any_launch(libpath):
     mods[0].W0 = 0x20000
     assert lib.awsrc_decode_apply(ct.byref(p), 1, mods, 0x70000, 1 << 20, 0, what, aw.DTYPE_BF16,
                                   aw.DECODE_DENSE, 0x80040, big, None) == 1                  # workspace
+
+
+def test_backbone_metadata_bytes(libpath):
+    """Host-only byte count of the backbone's scale metadata (Sec. 3.3):
+    binary16 per group of 128, or SDQ's byte per group plus 8 per 256 groups."""
+    import paper_2608_23144_gb300 as aw
+    G = 11008 * 2048 // 128
+    assert aw.awsrc_backbone_metadata_bytes(11008, 2048, False) == 2 * G
+    assert aw.awsrc_backbone_metadata_bytes(11008, 2048, True) == G + 8 * 688
+    assert aw.awsrc_backbone_metadata_bytes(4, 100, True) == -1
+    assert aw.awsrc_backbone_metadata_bytes(1, 128, True) == 1 + 8

@@ -1,0 +1,52 @@
+"""GPU parity of the RTN-INT4 backbone and its scale double quantisation
+(Eq. 1, Sec. 3.3, Sec. 4) against the oracle: packed codes, binary16 scales,
+SDQ codes and constants and W0, bit for bit, over input and output dtypes,
+partial SDQ blocks, zero groups and a full Qwen2.5-3B-sized gate projection."""
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def aw():
+    import paper_2608_23144_gb300 as aw
+    assert torch.cuda.is_available()
+    return aw
+
+
+def _weights(seed, rows, cols):
+    rng = np.random.default_rng(seed)
+    W = rng.normal(0, 0.02, (rows, cols)).astype(np.float32)
+    W[:, rng.choice(cols, max(1, cols // 100), replace=False)] *= 8.0
+    W[0, :128] = 0.0
+    W[-1, -128:] *= 1e-3
+    return W
+
+
+def _pack(q):
+    q = q.reshape(-1).astype(np.int16) & 15
+    return (q[0::2] | (q[1::2] << 4)).astype(np.uint8)
+
+
+@pytest.mark.parametrize("rows,cols", [(40, 512), (300, 1024), (11008, 2048)])
+@pytest.mark.parametrize("w_dtype,w0_dtype", [(torch.bfloat16, torch.bfloat16), (torch.float32, torch.float32),
+                                              (torch.bfloat16, torch.float32)])
+@pytest.mark.parametrize("sdq", [False, True])
+def test_backbone_matches_oracle(aw, orc, rows, cols, w_dtype, w0_dtype, sdq):
+    if rows == 11008 and w_dtype != w0_dtype:
+        pytest.skip("full size once per dtype")
+    W = torch.from_numpy(_weights(rows + cols, rows, cols)).to(w_dtype)
+    got = aw.awsrc_rtn_quantize(W.cuda(), sdq=sdq, w0_dtype=w0_dtype)
+    torch.cuda.synchronize()
+    want = orc.rtn_quantize(W.float().numpy(), sdq=sdq)
+    assert np.array_equal(got["codes"].cpu().numpy(), _pack(want["q"]))
+    assert np.array_equal(got["scales"].cpu().numpy().view(np.uint16), want["s16"])
+    if sdq:
+        assert np.array_equal(got["sdq_codes"].cpu().numpy(), want["c8"])
+        assert np.array_equal(got["sdq_consts"].cpu().numpy().view(np.uint32), want["consts"].view(np.uint32))
+    W0 = torch.from_numpy(want["W0"]).to(w0_dtype)
+    assert torch.equal(got["W0"].cpu().view(torch.int16 if w0_dtype == torch.bfloat16 else torch.int32),
+                       W0.view(torch.int16 if w0_dtype == torch.bfloat16 else torch.int32))
+
