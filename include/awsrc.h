@@ -368,6 +368,47 @@ awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t
 /* ------------------------------------------------------------------ misc -- */
 
 /*
+ * Serving with the sidecar applied on the fly (the fused packed inference the
+ * paper leaves to future work, Sec. 5): a stream is unpacked once for a model,
+ * then each module's product with a few vectors reads the packed RTN-INT4
+ * backbone and the sidecar, never a dense W_hat.
+ *
+ * awsrc_sidecar_workspace_bytes — device bytes of a prepared sidecar for the
+ *   stream's module list (the dense decoder's workspace: basis masks, tile ->
+ *   record map, per-record codes).
+ * awsrc_sidecar_prepare — unpacks the first K records of `stream` (K < 0: the
+ *   header's count) into `workspace`, as awsrc_decode_apply's first step does;
+ *   faults are reported through awsrc_workspace_status(workspace).
+ * awsrc_packed_gemv — y[m][i] = sum_j (W0_ij + r_ij) x[m][j] for module `m` of
+ *   the list and the M <= 8 vectors x[m] (rows of x, M x cols, 16-byte
+ *   aligned; y is M x rows): W0_ij = fl(q_ij * s_eff) from the packed backbone
+ *   (awsrc_rtn_quantize's outputs; binary16 scales or SDQ), r_ij =
+ *   fl(fl(k_j * C^-1/2) * scale) on the tiles the sidecar names (none when
+ *   `sidecar` is NULL), both accumulated in binary32 with fma. The result
+ *   equals the double-precision product of those values within binary32
+ *   summation error (bounded by (2*cols/32 + 8) * 2^-24 * sum_j |(W0 + r) x|).
+ *   The module needs cols % 128 == 0.
+ * Errors: INVALID_ARG, SHAPE, UNSUPPORTED, WORKSPACE, CUDA.
+ */
+typedef struct awsrc_packed_weights {
+  const uint8_t* codes;      /* rows*cols/2 bytes, 4-byte aligned */
+  const uint16_t* scales;    /* binary16 per group (sdq == 0) */
+  const int8_t* sdq_codes;   /* per group (sdq == 1) */
+  const float* sdq_consts;   /* (mean, step) per 256 groups (sdq == 1), 8-byte aligned */
+  int32_t sdq;
+  int32_t pad_;
+} awsrc_packed_weights;
+
+awsrc_status awsrc_sidecar_workspace_bytes(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                           size_t* bytes);
+awsrc_status awsrc_sidecar_prepare(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                   const uint8_t* stream, size_t stream_len, int64_t K, void* workspace,
+                                   size_t workspace_bytes, void* stream_handle);
+awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods, int32_t m,
+                               const awsrc_packed_weights* pw, const void* sidecar, size_t sidecar_bytes,
+                               int32_t M, const float* x, float* y, void* stream);
+
+/*
  * awsrc_workspace_status — synchronises `stream`, then reads and clears the
  * device fault word kept in the first bytes of an encode/select/decode
  * workspace. Each of those entry points clears the word when it starts, so the

@@ -747,19 +747,24 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
 
 /* ------------------------------------------------------------------------ */
 /* Definition of the packed product (the decoded weights applied to x        */
-/* without forming them): y[m][i] = sum_j (W0_ij + r_ij) x[m][j] in double,  */
-/* W0_ij = q_ij * s_eff (the backbone's binary32 value), r the decoder's      */
-/* residual (Sec. 3.2) on the                                                 */
-/* tiles named by the first K records of a one-module stream, in double:      */
-/* k_j * C^-1/2 * scale. yabs = sum_j |(W0_ij + r_ij) x[m][j]| bounds the    */
+/* without forming them) for module m of a stream over n_mod modules:        */
+/* y[v][i] = sum_j (W0_ij + r_ij) x[v][j] in double, W0_ij = q_ij * s_eff    */
+/* (the backbone's binary32 value), r the decoder's residual (Sec. 3.2) on    */
+/* the module's tiles named by the first K records, in double:                */
+/* k_j * C^-1/2 * scale. yabs = sum_j |(W0_ij + r_ij) x[v][j]| bounds the    */
 /* rounding of any binary32 evaluation. x: M x cols, y and yabs: M x rows.   */
 /* ------------------------------------------------------------------------ */
-int orc_packed_gemv(const orc_params* prm, int64_t rows, int64_t cols, int group, const int8_t* q,
-                    const float* s_eff, const uint8_t* stream, int64_t K, int M, const float* x, double* y,
-                    double* yabs) {
+int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_rows, const int64_t* mod_cols,
+                    int32_t m, int group, const int8_t* q, const float* s_eff, const uint8_t* stream, int64_t K,
+                    int M, const float* x, double* y, double* yabs) {
   const int C = prm->C, P = prm->P;
-  const int64_t T = rows * cols / C, n_cb = cols / C;
-  const int64_t h = orc_header_bytes(1), L = orc_record_bytes(prm, T);
+  int64_t T = 0, off = 0;
+  for (int i = 0; i < n_mod; ++i) {
+    if (i == m) off = T;
+    T += mod_rows[i] * mod_cols[i] / C;
+  }
+  const int64_t rows = mod_rows[m], cols = mod_cols[m], Tm = rows * cols / C, n_cb = cols / C;
+  const int64_t h = orc_header_bytes(n_mod), L = orc_record_bytes(prm, T);
   double* Wt = (double*)malloc(sizeof(double) * (size_t)(rows * cols));
   if (!Wt) return -1;
   for (int64_t i = 0; i < rows * cols; ++i) Wt[i] = (double)((float)q[i] * s_eff[i / group]);
@@ -772,7 +777,9 @@ int orc_packed_gemv(const orc_params* prm, int64_t rows, int64_t cols, int group
     orc_candidate cd;
     orc_unpack_record(prm, T, stream + h + k * L, &tile, &cd);
     if (tile >= T || cd.seed >= prm->S) { bad = 1; continue; }
-    const int64_t base = (tile / n_cb) * cols + (tile % n_cb) * C;
+    if (tile < off || tile >= off + Tm) continue;  /* another module's record */
+    const int64_t lt = tile - off;
+    const int64_t base = (lt / n_cb) * cols + (lt % n_cb) * C;
     orc_gen_basis(prm->gen_seed, cd.seed, C, P, prm->permute, sign, perm, colsel, neg);
     const double sc = prm->scale_mode == 0 ? ldexp(1.0, cd.scale) : (double)orc_f16_to_f32((uint16_t)cd.scale);
     for (int j = 0; j < C; ++j) {
@@ -781,16 +788,16 @@ int orc_packed_gemv(const orc_params* prm, int64_t rows, int64_t cols, int group
       Wt[base + j] += (double)kj * c * sc;
     }
   }
-  for (int m = 0; m < M; ++m)
+  for (int v = 0; v < M; ++v)
     for (int64_t i = 0; i < rows; ++i) {
       double acc = 0.0, aabs = 0.0;
       for (int64_t j = 0; j < cols; ++j) {
-        const double t = Wt[i * cols + j] * (double)x[(int64_t)m * cols + j];
+        const double t = Wt[i * cols + j] * (double)x[(int64_t)v * cols + j];
         acc += t;
         aabs += fabs(t);
       }
-      y[(int64_t)m * rows + i] = acc;
-      yabs[(int64_t)m * rows + i] = aabs;
+      y[(int64_t)v * rows + i] = acc;
+      yabs[(int64_t)v * rows + i] = aabs;
     }
   free(Wt);
   return bad;

@@ -106,8 +106,8 @@ def lib():
             L.orc_rtn_quantize.argtypes = [ct.c_int64, ct.c_int64, ct.c_int, ct.c_int, ct.c_int, vp, vp, vp, vp,
                                            vp, vp, vp]
             L.orc_packed_gemv.restype = ct.c_int
-            L.orc_packed_gemv.argtypes = [P(Params), ct.c_int64, ct.c_int64, ct.c_int, vp, vp, vp, ct.c_int64,
-                                          ct.c_int, vp, vp, vp]
+            L.orc_packed_gemv.argtypes = [P(Params), ct.c_int32, vp, vp, ct.c_int32, ct.c_int, vp, vp, vp,
+                                          ct.c_int64, ct.c_int, vp, vp, vp]
             _lib = L
     return _lib
 
@@ -340,17 +340,23 @@ def rtn_quantize(W, group: int = 128, sdq: bool = False, block: int = 256):
     return {"q": q, "s16": s16, "c8": c8, "consts": consts, "s_eff": s_eff, "W0": W0}
 
 
-def packed_gemv(prm: Params, q, s_eff, group: int, stream: bytes, K: int, x):
-    """y = (W0 + r_hat) x in double (one module). Returns (y, yabs, bad): y and
-    yabs of shape (M, rows), yabs = sum_j |(W0 + r_hat)_ij x_j|."""
+def packed_gemv(prm: Params, q, s_eff, group: int, stream: bytes, K: int, x, shapes=None, m: int = 0):
+    """y = (W0 + r_hat) x in double for module m of a stream over `shapes`
+    (default: the one module of q). Returns (y, yabs, bad): y and yabs of
+    shape (M, rows), yabs = sum_j |(W0 + r_hat)_ij x_j|."""
     q = np.ascontiguousarray(q, np.int8)
     rows, cols = q.shape
+    if shapes is None:
+        shapes = [(rows, cols)]
+    assert tuple(shapes[m]) == (rows, cols)
+    mr = np.array([r for r, _ in shapes], np.int64)
+    mc = np.array([c for _, c in shapes], np.int64)
     x = np.ascontiguousarray(np.atleast_2d(x), np.float32)
     M = x.shape[0]
     y = np.zeros((M, rows), np.float64)
     yabs = np.zeros((M, rows), np.float64)
     buf = np.frombuffer(stream, np.uint8).copy()
-    bad = lib().orc_packed_gemv(ct.byref(prm), ct.c_int64(rows), ct.c_int64(cols), group, _ptr(q),
+    bad = lib().orc_packed_gemv(ct.byref(prm), len(shapes), _ptr(mr), _ptr(mc), m, group, _ptr(q),
                                 _ptr(np.ascontiguousarray(s_eff, np.float32)), _ptr(buf), ct.c_int64(K), M,
                                 _ptr(x), _ptr(y), _ptr(yabs))
     return y, yabs, int(bad)

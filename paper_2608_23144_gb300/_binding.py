@@ -55,6 +55,11 @@ class Module(ct.Structure):
     ]
 
 
+class PackedWeights(ct.Structure):
+    _fields_ = [("codes", ct.c_void_p), ("scales", ct.c_void_p), ("sdq_codes", ct.c_void_p),
+                ("sdq_consts", ct.c_void_p), ("sdq", ct.c_int32), ("pad_", ct.c_int32)]
+
+
 def params(C=64, P=4, b=4, S=4096, b_e=8, e_bias=0, scale_mode=SCALE_POW2, permute=1,
            variant=VARIANT_U, ridge_rel=1e-6, gen_seed=0) -> Params:
     return Params(C, P, b, S, b_e, e_bias, scale_mode, permute, variant,
@@ -110,6 +115,13 @@ def _load():
                                      ct.c_int32, vp]
     L.awsrc_backbone_metadata_bytes.restype = ct.c_int64
     L.awsrc_backbone_metadata_bytes.argtypes = [ct.c_int64, ct.c_int64, ct.c_int32]
+    L.awsrc_sidecar_workspace_bytes.restype = st
+    L.awsrc_sidecar_workspace_bytes.argtypes = [P(Params), ct.c_int32, P(Module), P(sz)]
+    L.awsrc_sidecar_prepare.restype = st
+    L.awsrc_sidecar_prepare.argtypes = [P(Params), ct.c_int32, P(Module), vp, sz, ct.c_int64, vp, sz, vp]
+    L.awsrc_packed_gemv.restype = st
+    L.awsrc_packed_gemv.argtypes = [P(Params), ct.c_int32, P(Module), ct.c_int32, P(PackedWeights), vp, sz,
+                                    ct.c_int32, vp, vp, vp]
     return L
 
 
@@ -225,6 +237,47 @@ def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream
 
 def awsrc_backbone_metadata_bytes(rows: int, cols: int, sdq: bool) -> int:
     return int(lib.awsrc_backbone_metadata_bytes(rows, cols, int(sdq)))
+
+
+def shape_modules(shapes):
+    """awsrc_module[] carrying only shapes (serving calls read no weights)."""
+    arr = (Module * len(shapes))()
+    for i, (r, c) in enumerate(shapes):
+        arr[i].rows, arr[i].cols = r, c
+        arr[i].w0_dtype = DTYPE_BF16
+    return arr
+
+
+def awsrc_sidecar_prepare(prm: Params, shapes, stream_bytes: torch.Tensor, K: int = -1,
+                          workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Unpack a stream once for serving; returns the prepared sidecar workspace."""
+    mods = shape_modules(shapes)
+    n = ct.c_size_t()
+    _check(lib.awsrc_sidecar_workspace_bytes(ct.byref(prm), len(shapes), mods, ct.byref(n)), "sidecar_workspace_bytes")
+    if workspace is None or workspace.numel() < n.value:
+        workspace = torch.empty(n.value, dtype=torch.uint8, device=stream_bytes.device)
+    _check(lib.awsrc_sidecar_prepare(ct.byref(prm), len(shapes), mods, _dev_ptr(stream_bytes), stream_bytes.numel(),
+                                     K, _dev_ptr(workspace), workspace.numel(), _stream(stream)), "sidecar_prepare")
+    return workspace
+
+
+def awsrc_packed_gemv(prm: Params, shapes, m: int, backbone: Dict[str, torch.Tensor], x: torch.Tensor,
+                      sidecar: Optional[torch.Tensor] = None, y: Optional[torch.Tensor] = None,
+                      stream=None) -> torch.Tensor:
+    """y = (W0 + r_hat) x for module m (x: M x cols float32); backbone holds
+    awsrc_rtn_quantize's codes and scales (or SDQ codes and constants)."""
+    mods = shape_modules(shapes)
+    rows, cols = shapes[m]
+    x = x.reshape(-1, cols)
+    if y is None:
+        y = torch.empty(x.shape[0], rows, dtype=torch.float32, device=x.device)
+    sdq = "sdq_codes" in backbone
+    pw = PackedWeights(_dev_ptr(backbone["codes"]), None if sdq else _dev_ptr(backbone["scales"]),
+                       _dev_ptr(backbone.get("sdq_codes")), _dev_ptr(backbone.get("sdq_consts")), int(sdq), 0)
+    _check(lib.awsrc_packed_gemv(ct.byref(prm), len(shapes), mods, m, ct.byref(pw), _dev_ptr(sidecar),
+                                 0 if sidecar is None else sidecar.numel(), x.shape[0], _dev_ptr(x), _dev_ptr(y),
+                                 _stream(stream)), "packed_gemv")
+    return y
 
 
 def awsrc_gen_basis(prm: Params, stream=None, device="cuda") -> torch.Tensor:

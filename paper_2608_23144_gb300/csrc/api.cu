@@ -513,6 +513,79 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod, const aw
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "decode");
 }
 
+// ----------------------------------------------------------------- serving --
+
+awsrc_status awsrc_sidecar_workspace_bytes(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                           size_t* bytes) {
+  return awsrc_decode_workspace_bytes(prm, n_mod, mods, AWSRC_DECODE_DENSE, bytes);
+}
+
+awsrc_status awsrc_sidecar_prepare(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                   const uint8_t* stream, size_t stream_len, int64_t K, void* workspace,
+                                   size_t workspace_bytes, void* stream_handle) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  if (!stream) return AWSRC_ERR_INVALID_ARG;
+  size_t need;
+  if ((s = awsrc_sidecar_workspace_bytes(prm, n_mod, mods, &need)) != AWSRC_OK) return s;
+  if (!workspace || workspace_bytes < need) return AWSRC_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return AWSRC_ERR_INVALID_ARG;
+  const int64_t L = awsrc_record_bytes(prm, T), h = awsrc_header_bytes(n_mod);
+  if (stream_len < (size_t)h) return AWSRC_ERR_INVALID_ARG;
+  const int64_t kmax = std::min<int64_t>(((int64_t)stream_len - h) / L, T);
+  if (K > kmax) return AWSRC_ERR_INVALID_ARG;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint64_t* masks = reinterpret_cast<uint64_t*>(ws + kStatusBytes);
+  void* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
+  const cudaError_t e = launch_dense_prep(pr, T, L, h, stream, K, kmax, masks, scratch,
+                                          reinterpret_cast<uint32_t*>(ws), (cudaStream_t)stream_handle);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "sidecar_prepare");
+}
+
+awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods, int32_t m,
+                               const awsrc_packed_weights* pw, const void* sidecar, size_t sidecar_bytes,
+                               int32_t M, const float* x, float* y, void* stream) {
+  Prm pr;
+  awsrc_status s = make_prm(prm, &pr);
+  if (s != AWSRC_OK) return s;
+  int64_t T;
+  if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
+  if (m < 0 || m >= n_mod || !pw || !x || !y || M < 1 || M > 8) return AWSRC_ERR_INVALID_ARG;
+  if (mods[m].cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
+  if (pw->sdq != 0 && pw->sdq != 1) return AWSRC_ERR_INVALID_ARG;
+  if (!pw->codes || (pw->sdq ? (!pw->sdq_codes || !pw->sdq_consts) : !pw->scales)) return AWSRC_ERR_INVALID_ARG;
+  if (!aligned(pw->codes, 4) || !aligned(pw->scales, 2) || !aligned(pw->sdq_consts, 8) || !aligned(x, 16) ||
+      !aligned(y, 4))
+    return AWSRC_ERR_INVALID_ARG;
+  GemvArgs a{};
+  a.rows = mods[m].rows;
+  a.cols = mods[m].cols;
+  for (int i = 0; i < m; ++i) a.tile_off += mods[i].rows * (mods[i].cols / pr.C);
+  a.sdq = pw->sdq;
+  a.codes = reinterpret_cast<const uint16_t*>(pw->codes);
+  a.scales = pw->scales;
+  a.sdq_codes = pw->sdq_codes;
+  a.sdq_consts = pw->sdq_consts;
+  a.x = x;
+  a.y = y;
+  if (sidecar) {
+    size_t need;
+    if ((s = awsrc_sidecar_workspace_bytes(prm, n_mod, mods, &need)) != AWSRC_OK) return s;
+    if (sidecar_bytes < need) return AWSRC_ERR_WORKSPACE;
+    if (!aligned(sidecar, 256)) return AWSRC_ERR_INVALID_ARG;
+    const uint8_t* ws = static_cast<const uint8_t*>(sidecar);
+    a.masks = reinterpret_cast<const uint64_t*>(ws + kStatusBytes);
+    const uint8_t* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
+    a.map = reinterpret_cast<const unsigned long long*>(scratch);
+    a.rcodes = reinterpret_cast<const uint2*>(scratch + align_up((size_t)T * 8, 256));
+  }
+  const cudaError_t e = launch_gemv(pr, a, M, (cudaStream_t)stream);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "packed_gemv");
+}
+
 awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags) {
   if (!workspace || !flags) return AWSRC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;

@@ -598,6 +598,37 @@ cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_
 
 }  // namespace
 
+// Dense preparation: clear the tile map (and the fault word), then generate
+// the masks and unpack the records into the map and the code array of
+// `scratch` (map: align_up(T * 8, 256) bytes, then 8 bytes per record).
+cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, const uint8_t* stream, int64_t K,
+                              int64_t kmax, uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
+  unsigned long long* map = static_cast<unsigned long long*>(scratch);
+  uint2* codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
+  DecArgs a;
+  a.n_mod = 0;
+  a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
+  const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
+  int dev = 0, nsm = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  const int per = 8 * basis_warp_seeds(pr.C);
+  const int nb = (pr.S + per - 1) / per;  // mask blocks, then record blocks (one record per thread)
+  const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, (int64_t)nsm * 64));
+  // the map region is align_up(T * 8, 256) bytes, so whole 16-byte words stay inside it
+  const int64_t n16 = (T * 8 + 15) / 16;
+  const unsigned gz = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n16 + 255) / 256, (int64_t)nsm * 8));
+  zero_map_kernel<<<gz, 256, 0, st>>>(reinterpret_cast<uint4*>(map), n16, status);
+  note_launches(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(prep_kernel, dim3((unsigned)(nb + nr)), dim3(256), st, pr, a, stream, masks, map, codes, status,
+                 nb);
+  note_launches(1);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  return e;
+}
+
 // Launches over runs of at most 16 modules sharing the input dtype. DENSE with
 // C >= G: the first run's copy also generates the masks and fills the tile map,
 // then each run is patched in tile order; otherwise (INPLACE, or tiles shorter
@@ -611,27 +642,8 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
   if (fused) {
     map = static_cast<unsigned long long*>(scratch);
     codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
-    DecArgs a;
-    a.n_mod = 0;
-    a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
-    const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
-    int dev = 0, nsm = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    const int per = 8 * basis_warp_seeds(pr.C);
-    const int nb = (pr.S + per - 1) / per;  // mask blocks, then record blocks (one record per thread)
-    const int64_t nr = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, (int64_t)nsm * 64));
-    // the map region is align_up(T * 8, 256) bytes, so whole 16-byte words stay inside it
-    const int64_t n16 = (T * 8 + 15) / 16;
-    const unsigned gz = (unsigned)std::max<int64_t>(1, std::min<int64_t>((n16 + 255) / 256, (int64_t)nsm * 8));
-    zero_map_kernel<<<gz, 256, 0, st>>>(reinterpret_cast<uint4*>(map), n16, status);
-    note_launches(1);
-    cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_dense_prep(pr, T, L, h, stream, K, kmax, masks, scratch, status, st);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(prep_kernel, dim3((unsigned)(nb + nr)), dim3(256), st, pr, a, stream, masks, map, codes, status,
-                   nb);
-    note_launches(1);
-    if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
   }
   int i0 = 0;
   while (i0 < n_mod) {

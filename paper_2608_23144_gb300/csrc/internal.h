@@ -90,8 +90,26 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
 size_t decode_scratch_bytes(int64_t T, int mode);
+cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, const uint8_t* stream, int64_t K,
+                              int64_t kmax, uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
 // The dense fused decoder clears the fault word itself (no separate memset).
 bool decode_clears_status(const Prm& pr, int mode);
+
+// gemv.cu: y[m] = (W0 + r_hat) x[m] for one module of a prepared sidecar.
+struct GemvArgs {
+  int64_t rows, cols, tile_off;  // tile_off: the module's first global tile
+  int32_t sdq, pad_;
+  const uint16_t* codes;         // 4 codes per uint16, element 2i in the low nibble of byte i
+  const uint16_t* scales;        // binary16 per group (sdq == 0)
+  const int8_t* sdq_codes;       // per group (sdq)
+  const float* sdq_consts;       // (mean, step) per 256 groups (sdq)
+  const unsigned long long* map; // tile map of the prepared sidecar, or null (no residual)
+  const uint2* rcodes;           // per-record codes of the prepared sidecar
+  const uint64_t* masks;         // basis masks of the prepared sidecar
+  const float* x;                // M x cols
+  float* y;                      // M x rows
+};
+cudaError_t launch_gemv(const Prm& pr, const GemvArgs& a, int M, cudaStream_t st);
 
 // backbone.cu: RTN-INT4 groups of rtn_group() inputs, SDQ blocks of sdq_block() groups.
 int rtn_group();

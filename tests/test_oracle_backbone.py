@@ -120,3 +120,23 @@ def test_packed_product_definition(orc):
     ref = x.astype(np.float64) @ dec[0].astype(np.float64).T
     assert (np.abs(y - ref) <= 2.0 ** -22 * yabs + 1e-30).all()
     assert (yabs >= np.abs(y)).all() and not np.allclose(y, y0)
+
+
+def test_packed_product_second_module_of_a_stream(orc):
+    """Module 1 of a two-module stream: only its own records apply (tile
+    offsets), matching the oracle decoder's weights of that module."""
+    rng = np.random.default_rng(6)
+    shapes = [(32, 256), (40, 384)]
+    Ws = [_weights(rng, r, c, zero_groups=False) for r, c in shapes]
+    bbs = [orc.rtn_quantize(W) for W in Ws]
+    prm = orc.params(C=64, P=4, b=4, S=32)
+    cands = np.concatenate([orc.encode_tiles(prm, W, bb["W0"], (rng.lognormal(0, 1, W.shape[1]) ** 2)
+                                             .astype(np.float32)) for W, bb in zip(Ws, bbs)])
+    stream, counts, _ = orc.select_records(prm, shapes, cands, [2.0])
+    K = int(counts.sum())
+    x = rng.normal(0, 1, (2, shapes[1][1])).astype(np.float32)
+    y, yabs, bad = orc.packed_gemv(prm, bbs[1]["q"], bbs[1]["s_eff"], 128, stream, K, x, shapes=shapes, m=1)
+    dec, _ = orc.decode_apply(prm, [bb["W0"] for bb in bbs], stream, K)
+    ref = x.astype(np.float64) @ dec[1].astype(np.float64).T
+    assert bad == 0 and counts[1] > 0
+    assert (np.abs(y - ref) <= 2.0 ** -22 * yabs + 1e-30).all()
