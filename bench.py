@@ -36,12 +36,14 @@ RATE = 0.162
 METRIC = "AWSRC encode (tile,seed) candidates/s + layers/s; decode-apply HBM GB/s"
 UNIT = "candidates/s"
 # FP32-pipe operations every (tile, seed) candidate of the C=64, P=4, U search
-# needs before it can be pruned: the correlation's rounding and scaling (2 per
-# atom), the forward substitution (6), D^-1 (4), U = z^T D^-1 z (4) and the
-# bound multiplier (1). The ~1-2% of candidates that survive the bound add
-# about 35 more each (back substitution, quantiser, gain), not counted here.
+# needs before it can be pruned: forming the rounded correlation from its two
+# halves (1 per atom), the forward substitution (6), z * (D^-1 m) (4) and the
+# bound z^T (z D^-1 m) (4); the bound is taken on the unscaled correlations, so
+# no scaling is needed before the decision. The ~0.5% of candidates that
+# survive the bound add about 50 more each (scaling, the forward substitution
+# in the recipe's units, back substitution, quantiser, gain), not counted here.
 # The correlation itself is tensor-core work: 2 halves x C x P x 2 FLOP.
-OPS_PER_CANDIDATE = 8 + 6 + 4 + 4 + 1
+OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.

@@ -107,12 +107,12 @@ __host__ __device__ constexpr int gram_stride(int P) {
 }
 
 // float2 entries per (column block, seed pair) of the paired table the C = 64,
-// P = 4 search streams: -L, invD, G off-diagonal (2*G_pq on the fast
-// power-of-two path), gd, zero padding to an odd count, then the seed's
-// pruning-bound multiplier in the last entry; seed 2i in component x and
-// seed 2i+1 in y.
+// P = 4 search streams: -L, invD rounded up after multiplying by the seed's
+// pruning-bound multiplier (used only by the bound), invD, G off-diagonal
+// (2*G_pq on the fast power-of-two path), gd, zero padding to an even count;
+// seed 2i in component x and seed 2i+1 in y.
 __host__ __device__ constexpr int pair_stride(int P) {
-  return ((P * (P - 1) + P + 2) + 1) / 2 * 2;
+  return ((P * (P - 1) + 2 * P + 1) + 1) / 2 * 2;
 }
 
 // LDL^T of A = G + eps I with G_pp = gd, G_pq = Goff[tri(q, p)]. Writes L and

@@ -153,15 +153,19 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     float* po = reinterpret_cast<float*>(pairs) +
                 (size_t)((md.gram_off + cb * pr.S_pad + s) >> 1) * pair_stride(P) * 2 + (s & 1);
     constexpr int nl = P * (P - 1) / 2;
+    const float m = ok ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
 #pragma unroll
     for (int i = 0; i < nl; ++i) po[2 * i] = -L[i];
+    // invD * m rounded up: the bound's terms z_k (z_k invD_k m) are then never
+    // below the exact z_k^2 invD_k m (m = +inf disables pruning)
 #pragma unroll
-    for (int k = 0; k < P; ++k) po[2 * (nl + k)] = ok ? invD[k] : qnan;
+    for (int k = 0; k < P; ++k) po[2 * (nl + k)] = ok ? __double2float_ru((double)invD[k] * (double)m) : qnan;
 #pragma unroll
-    for (int i = 0; i < nl; ++i) po[2 * (nl + P + i)] = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];
-    po[2 * (2 * nl + P)] = gd;
-    for (int i = 2 * nl + P + 1; i < pair_stride(P) - 1; ++i) po[2 * i] = 0.0f;
-    po[2 * (pair_stride(P) - 1)] = ok ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
+    for (int k = 0; k < P; ++k) po[2 * (nl + P + k)] = ok ? invD[k] : qnan;
+#pragma unroll
+    for (int i = 0; i < nl; ++i) po[2 * (nl + 2 * P + i)] = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];
+    po[2 * (2 * nl + 2 * P)] = gd;
+    for (int i = 2 * nl + 2 * P + 1; i < pair_stride(P); ++i) po[2 * i] = 0.0f;
   }
 }
 

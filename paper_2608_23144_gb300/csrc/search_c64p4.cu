@@ -13,14 +13,16 @@
 // Block: 128 rows (tiles of one column block; row m = TMEM lane m) and 17 warps.
 //  * Warp 16 (producer): one thread streams each chunk of 32 seeds — FP16 atoms
 //    in the canonical K-major layout (16 KB) and the chunk's paired Gram factors
-//    (2.3 KB) — by bulk copies into a 4-stage shared-memory ring, and issues the
+//    (2.8 KB) — by bulk copies into a 4-stage shared-memory ring, and issues the
 //    chunk's 8 MMAs (M = 128, N = 128, K = 16; halves hi and lo, 4 k-steps) into
 //    one of two 256-column TMEM accumulators, committed to an mbarrier.
 //  * Warps 0..15 (epilogue): warp w reads TMEM lanes 32(w%4).. (its threads'
 //    rows) and the columns of seeds 8(w/4)..8(w/4)+7 of each chunk, and runs the
 //    fit / quantise / score epilogue on seed pairs as float2 streams, keeping a
-//    running argmax per row with the winner's codes and scale. The four warps
-//    of a row merge at the end and write the tile's candidate.
+//    running (gain, seed) argmax per row. The four warps of a row publish
+//    their running best gains in shared memory and prune against the largest;
+//    they merge at the end, form the winner's codes again and write the
+//    tile's candidate.
 // Columns of a chunk are seed-pair major: column 8i + 2p + e holds atom p of
 // seed 2i + e, so one 32x32b.x16 TMEM load gives a thread two seed pairs with
 // each atom's two seeds in adjacent registers.
@@ -47,9 +49,9 @@ constexpr int RPAIRS = 2;           // seed pairs per TMEM load (8 columns each)
 constexpr int ROUNDS = SUB_PAIRS / RPAIRS;
 static_assert(EW % 4 == 0 && SUB_PAIRS % RPAIRS == 0 && RPAIRS % 2 == 0, "epilogue mapping");
 constexpr int STAGES = 4;
-constexpr int PS = pair_stride(4);  // 18 float2 per seed pair
+constexpr int PS = pair_stride(4);  // 22 float2 per seed pair
 constexpr uint32_t kBBytes = NCOL * 64 * 2;        // 16 KB of FP16 atoms per chunk
-constexpr uint32_t kPBytes = (CH / 2) * PS * 8u;   // 2304 B of paired factors per chunk
+constexpr uint32_t kPBytes = (CH / 2) * PS * 8u;   // 2816 B of paired factors per chunk
 constexpr uint32_t kStageBytes = 19456;            // B at 0, factors at kBBytes (1 KB multiple)
 constexpr uint32_t kTmemCols = 512;                // 2 accumulators x (hi, lo) x 128 columns
 static_assert(kBBytes + kPBytes <= kStageBytes, "stage layout");
@@ -65,6 +67,7 @@ struct Smem {
   int rowok[BM];
   float red_g[SUBS][BM];
   uint32_t red_s[SUBS][BM];
+  float cur_g[SUBS][BM];                  // running best gain of each (sub, row) in u units, for pruning
   unsigned long long full[STAGES];        // bulk copies of a chunk landed
   unsigned long long afull[2];            // MMAs of a chunk completed (tcgen05.commit)
   unsigned long long aempty[2];           // epilogue warps done with an accumulator
@@ -85,14 +88,15 @@ __device__ __forceinline__ int a_offset(int m, int k) {
   return (((m >> 3) * 8 + (k >> 3)) << 7) + ((m & 7) << 4) + ((k & 7) << 1);
 }
 
-// Forward half of the ridge solve for one seed pair of this thread's row:
-// b from the exact correlations (hi/lo hold atom p of the two seeds at [2p],
-// [2p+1]), z = L^-1 b and w = D^-1 z, so that alpha = L^-T w. pe points at
-// the pair's 18 float2 factors (9 float4: -L, invD, G off-diagonal, gd and the
-// bound multiplier). Returns U = b^T (G + eps I)^-1 b = z^T w (a sum of
-// non-negative terms) times the seed's bound multiplier.
-__device__ __forceinline__ float2 pair_forward(const float* hi, const float* lo, float2 tqc, const float4* pe,
-                                               float2* bv, float2* w) {
+// Pruning bound of one seed pair for this thread's row, in the units of the
+// unscaled correlations u = b / (2^q c) (c 2^q is a power of two for C = 64,
+// so the comparison against a threshold scaled by (2^q c)^-2 is exact). hi/lo
+// hold atom p of the two seeds at [2p], [2p+1]; u = RN(2048 hi + lo) is the
+// exact integer correlation rounded once. pe points at the pair's factors
+// (-L, then invD m rounded up). Returns U = u^T (G + eps I)^-1 u times the
+// seed's bound multiplier, as z^T (z * invD m) with z = L^-1 u: a sum of
+// non-negative terms.
+__device__ __forceinline__ float2 pair_bound(const float* hi, const float* lo, const float4* pe, float2* u) {
   float2 pv[10];
 #pragma unroll
   for (int i = 0; i < 5; ++i) {
@@ -101,13 +105,44 @@ __device__ __forceinline__ float2 pair_forward(const float* hi, const float* lo,
     pv[2 * i + 1] = make_float2(v.z, v.w);
   }
   const float2* nL = pv;
-  const float2* invD = pv + 6;
+  const float2* invDm = pv + 6;
 #pragma unroll
-  for (int p = 0; p < 4; ++p) {
-    const float2 u = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
-                                make_float2(lo[2 * p], lo[2 * p + 1]));
-    bv[p] = __fmul2_rn(u, tqc);
+  for (int p = 0; p < 4; ++p)
+    u[p] = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
+                      make_float2(lo[2 * p], lo[2 * p + 1]));
+  float2 z[4];
+  float2 U = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    float2 v = u[k];
+#pragma unroll
+    for (int i = 0; i < k; ++i) v = __ffma2_rn(nL[tri(k, i)], z[i], v);
+    z[k] = v;
+    const float2 wm = __fmul2_rn(v, invDm[k]);
+    U = k == 0 ? __fmul2_rn(v, wm) : __ffma2_rn(v, wm, U);
   }
+  return U;
+}
+
+// Forward half of the ridge solve in the recipe's units: b = u (2^q c),
+// z = L^-1 b and w = D^-1 z, so that alpha = L^-T w.
+__device__ __forceinline__ void pair_forward(const float2* u, float2 tqc, const float4* pe, float2* bv,
+                                             float2* w) {
+  float2 nL[6], invD[4];
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    const float4 v = pe[i];
+    nL[2 * i] = make_float2(v.x, v.y);
+    nL[2 * i + 1] = make_float2(v.z, v.w);
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float4 v = pe[5 + i];
+    invD[2 * i] = make_float2(v.x, v.y);
+    invD[2 * i + 1] = make_float2(v.z, v.w);
+  }
+#pragma unroll
+  for (int p = 0; p < 4; ++p) bv[p] = __fmul2_rn(u[p], tqc);
   float2 z[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
@@ -117,11 +152,6 @@ __device__ __forceinline__ float2 pair_forward(const float* hi, const float* lo,
     z[k] = v;
     w[k] = __fmul2_rn(v, invD[k]);
   }
-  float2 U = __fmul2_rn(z[0], w[0]);
-#pragma unroll
-  for (int k = 1; k < 4; ++k) U = __ffma2_rn(z[k], w[k], U);
-  const float4 v8 = pe[8];
-  return __fmul2_rn(U, make_float2(v8.z, v8.w));
 }
 
 // Back half of the solve: alpha = L^-T w, in the order of ldl_solve2.
@@ -148,12 +178,12 @@ __device__ __forceinline__ float2 pair_gain(const Prm& pr, const float2* bv, con
   float2 Go[6];
 #pragma unroll
   for (int i = 0; i < 3; ++i) {
-    const float4 v = pe[5 + i];
+    const float4 v = pe[7 + i];
     Go[2 * i] = make_float2(v.x, v.y);
     Go[2 * i + 1] = make_float2(v.z, v.w);
   }
-  const float4 v8 = pe[8];
-  const float2 gd = make_float2(v8.x, v8.y);
+  const float4 v10 = pe[10];
+  const float2 gd = make_float2(v10.x, v10.y);
   if constexpr (FAST) {
     return quant_gain_fast2<4>(pr, alpha, bv, gd, Go);  // G off-diagonal doubled
   } else {
@@ -204,8 +234,12 @@ __device__ __forceinline__ float winner_codes(const Prm& pr, const Smem& sm, int
     lo[2 * p] = lo[2 * p + 1] = (float)(u & 2047);
   }
   const float tq = __fmul_rn(sm.two_q[m], pr.c);
-  float2 bv[4], wv[4], al[4];
-  (void)pair_forward(hi, lo, make_float2(tq, tq), pe, bv, wv);
+  float2 u[4], bv[4], wv[4], al[4];
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+    u[p] = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
+                      make_float2(lo[2 * p], lo[2 * p + 1]));
+  pair_forward(u, make_float2(tq, tq), pe, bv, wv);
   pair_back(pe, wv, al);
   float a[4], q[4], zero[6] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
@@ -266,7 +300,11 @@ __global__ void __launch_bounds__(NT, 1)
     }
     tc_fence_before();
   }
-  if (tid < BM) sm.rowok[tid] = 1;
+  if (tid < BM) {
+    sm.rowok[tid] = 1;
+#pragma unroll
+    for (int i = 0; i < SUBS; ++i) sm.cur_g[i][tid] = neg_inf();
+  }
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
@@ -372,9 +410,19 @@ __global__ void __launch_bounds__(NT, 1)
     const int sub = warp >> 2;             // seed pairs SUB_PAIRS*sub .. of each chunk
     const float tq = __fmul_rn(sm.two_q[m], pr.c);
     const float2 tqc = make_float2(tq, tq);
+    // A gain g in the units of the bound: g (2^q c)^-2 = g 2^(6 - 2q), formed
+    // by two power-of-two factors (each a normal float), so exactly unless it
+    // overflows (to +inf: every finite bound is then below the scaled gain,
+    // as it is below the unscaled one) or falls far below every non-zero
+    // bound (which is at least ~2^-36: u is integral, D_k <= 2^33).
+    const int qrow = (int)((__float_as_uint(sm.two_q[m]) >> 23) & 0xffu) - 127;
+    const int eu = min(250, max(-250, 6 - 2 * qrow)), eu1 = eu / 2, eu2 = eu - eu1;
+    const float fu1 = __uint_as_float((uint32_t)(eu1 + 127) << 23);
+    const float fu2 = __uint_as_float((uint32_t)(eu2 + 127) << 23);
     const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
     float bg = neg_inf();
     uint32_t bsd = 0xffffffffu;
+    volatile float* cur_g = &sm.cur_g[0][m];  // written by the row's other warps
     // Seeds reach a thread in increasing order, so a strictly greater gain is
     // the whole tie rule within a thread.
     for (int k = 0; k < nck; ++k) {
@@ -384,6 +432,15 @@ __global__ void __launch_bounds__(NT, 1)
       // wait (already complete) makes the copy visible to this warp's reads
       if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
       tc_fence_after();
+      // Pruning threshold: the best gain any of the row's SUBS warps has found
+      // so far. Each of them is a gain some candidate of this row reaches, so
+      // a candidate whose bound is strictly below it cannot win. The entries
+      // of the other warps may be stale, which only weakens the threshold.
+      float thr = neg_inf();
+      if constexpr (FAST) {
+#pragma unroll
+        for (int i = 0; i < SUBS; ++i) thr = fmaxf(thr, cur_g[i * BM]);
+      }
       const float4* pbase = reinterpret_cast<const float4*>(&sm.stage[st][kBBytes]);
 #pragma unroll
       for (int rnd = 0; rnd < ROUNDS; ++rnd) {
@@ -400,19 +457,25 @@ __global__ void __launch_bounds__(NT, 1)
 #pragma unroll
         for (int j = 0; j < RPAIRS; ++j) {
           const float4* pe = pbase + (p0 + j) * (PS / 2);
-          float2 bv[4], wv[4];
-          const float2 ub = pair_forward(hi + 8 * j, lo + 8 * j, tqc, pe, bv, wv);
+          float2 u[4];
+          const float2 ub = pair_bound(hi + 8 * j, lo + 8 * j, pe, u);
           // prune: a candidate whose gain bound is below the running best
           // cannot win (NaN bounds stay live)
-          const bool lx = !FAST || !(ub.x < bg), ly = !FAST || !(ub.y < bg);
+          const bool lx = !FAST || !(ub.x < thr), ly = !FAST || !(ub.y < thr);
           if (__any_sync(0xffffffffu, lx || ly)) {
-            float2 al[4];
+            float2 bv[4], wv[4], al[4];
+            pair_forward(u, tqc, pe, bv, wv);
             pair_back(pe, wv, al);
             const float2 gp = pair_gain<FAST>(pr, bv, al, pe);
             // running argmax in seed order: a strictly greater gain wins
             const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * (p0 + j));
             if (lx && gp.x > bg) { bg = gp.x; bsd = s; }
             if (ly && gp.y > bg) { bg = gp.y; bsd = s + 1; }
+            if constexpr (FAST) {
+              const float bgu = __fmul_rn(__fmul_rn(bg, fu1), fu2);
+              cur_g[sub * BM] = bgu;
+              thr = fmaxf(thr, bgu);
+            }
           }
         }
       }
