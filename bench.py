@@ -47,8 +47,8 @@ OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "29a1d54133a735296ac6bf130b08523e709c4b0ca9bb0357ebbafb796f3b2478",
-                  "bytes_per_launch": 419800000 + 16400000}
+SEARCH_TRAFFIC = {"source_sha256": "f20aba940c0b1abed772390d1dd1810af0150b95162d17bb1f186427e25956e6",
+                  "bytes_per_launch": 442798336 + 16855296}
 
 
 def search_source_sha() -> str:
@@ -258,6 +258,68 @@ def paper_points(dev, hbm_gbs):
     out["workload"] = ("gate/up/down projections of one Qwen2.5-3B-shaped layer (67,633,152 BF16 weights); "
                        "the paper's (C,P,b,S) points, 0.162 bpw")
     return out
+
+
+def backbone_and_serving(dev, prm, mods, outs, stream, records, hbm_gbs):
+    """The RTN-INT4 backbone with scale double quantisation (Sec. 3.3) and the
+    sidecar applied inside an INT4 GEMV (the packed inference of Sec. 5) on the
+    benchmark layer, each timed on the device (mean of 5 runs after one
+    warm-up) against the HBM copy ceiling. Algorithmic bytes: the backbone
+    reads W (2 B/weight) and writes the 4-bit codes, the SDQ scale codes and
+    W0 (BF16); the GEMV (one vector) reads the codes, the SDQ scale codes and
+    constants, the prepared sidecar's tile map (8 B per tile) and record codes
+    (8 B per record), x and writes y. cuBLAS's BF16 GEMV of the decoded weights
+    (2 B/weight) is timed beside it for context."""
+    import torch
+    import paper_2608_23144_gb300 as aw
+    reps = 5
+    N = sum(m["rows"] * m["cols"] for m in mods)
+    G = N // 128
+    bb = [aw.awsrc_rtn_quantize(m["W"], sdq=True) for m in mods]
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    for _ in range(reps):
+        for m, b in zip(mods, bb):
+            aw.awsrc_rtn_quantize(m["W"], sdq=True)
+    ev[1].record()
+    torch.cuda.synchronize()
+    q_ms = ev[0].elapsed_time(ev[1]) / reps
+    q_bytes = N * 2 + N // 2 + G + 8 * ((G + 255) // 256) + N * 2
+    shapes = [(m["rows"], m["cols"]) for m in mods]
+    side = aw.awsrc_sidecar_prepare(prm, shapes, stream)
+    T = N // prm.C
+    xs = [torch.randn(1, m["cols"], device=dev, dtype=torch.float32) for m in mods]
+    ys = [torch.empty(1, m["rows"], device=dev, dtype=torch.float32) for m in mods]
+    for i in range(len(mods)):
+        aw.awsrc_packed_gemv(prm, shapes, i, bb[i], xs[i], sidecar=side, y=ys[i])
+    torch.cuda.synchronize()
+    ev[0].record()
+    for _ in range(reps):
+        for i in range(len(mods)):
+            aw.awsrc_packed_gemv(prm, shapes, i, bb[i], xs[i], sidecar=side, y=ys[i])
+    ev[1].record()
+    torch.cuda.synchronize()
+    g_ms = ev[0].elapsed_time(ev[1]) / reps
+    xb = [x.to(torch.bfloat16) for x in xs]
+    for o, x in zip(outs, xb):
+        torch.nn.functional.linear(x, o)
+    torch.cuda.synchronize()
+    ev[0].record()
+    for _ in range(reps):
+        for o, x in zip(outs, xb):
+            torch.nn.functional.linear(x, o)
+    ev[1].record()
+    torch.cuda.synchronize()
+    d_ms = ev[0].elapsed_time(ev[1]) / reps
+    g_bytes = (N // 2 + G + 8 * ((G + 255) // 256) + 8 * T + 8 * records + 8 * prm.S * prm.P
+               + 4 * sum(m["cols"] + m["rows"] for m in mods))
+    return {"workload": "the 7 modules of the benchmark layer (77,070,336 weights), 0.162-bpw stream",
+            "rtn_sdq": {"ms": q_ms, "gbs": q_bytes / (q_ms * 1e-3) / 1e9,
+                        "frac_of_hbm": q_bytes / (q_ms * 1e-3) / 1e9 / hbm_gbs, "bytes": q_bytes},
+            "packed_gemv_m1": {"ms": g_ms, "gbs": g_bytes / (g_ms * 1e-3) / 1e9,
+                               "frac_of_hbm": g_bytes / (g_ms * 1e-3) / 1e9 / hbm_gbs, "bytes": g_bytes},
+            "cublas_bf16_gemv_of_decoded_m1_ms": d_ms}
 
 
 def run_reference(args):
@@ -494,9 +556,11 @@ def run_ours(args):
               "encode_ms": ms7, "candidates_per_s": T7 * wl7.S / (ms7 * 1e-3)}
         del m7, c7, ws7
 
-    paper = None
+    paper = serving = None
     if rank == 0 and not args.no_pf and not args.modules:
         paper = paper_points(dev, float(peaks.get("hbm_gbs", 6800.0)))
+        serving = backbone_and_serving(dev, prm, mods, outs, s, int(counts.sum().item()),
+                                       float(peaks.get("hbm_gbs", 6800.0)))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -518,7 +582,7 @@ def run_ours(args):
             "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper, "backbone_and_serving": serving,
             "gpu_launches": launches, "clocks": clk.summary(),
         }
         print(json.dumps(line), flush=True)
