@@ -215,8 +215,8 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod,
  * 1 byte per group plus 8 per block (0.0645 bits/weight on whole blocks), see
  * awsrc_backbone_metadata_bytes. W must be finite.
  *   W           device, rows*cols elements of w_dtype, 16-byte aligned.
- *   codes       device, rows*cols/2 bytes: element 2i in the low nibble of byte
- *               i, 4-bit two's complement.
+ *   codes       device, rows*cols/2 bytes (4-byte aligned): element 2i in the
+ *               low nibble of byte i, 4-bit two's complement.
  *   scales      device, G = rows*cols/128 binary16 s_g, or NULL.
  *   sdq_codes   device, G int8 c_g (SDQ), or NULL.
  *   sdq_consts  device, 2*ceil(G/256) floats (mu, step) per block (SDQ), or NULL.

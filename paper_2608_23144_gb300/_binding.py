@@ -213,21 +213,24 @@ def awsrc_encode_tiles(prm: Params, modules, out: Optional[torch.Tensor] = None,
     return out
 
 
-def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream=None) -> Dict[str, torch.Tensor]:
+def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream=None,
+                       out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
     """RTN-INT4 backbone of one module (groups of 128 inputs), optional SDQ.
     Returns codes (uint8, two per byte), scales (binary16 bits as int16),
     sdq_codes (int8) and sdq_consts (float32 mean, step per 256 groups) when
-    sdq, and W0 (in w0_dtype, default W's dtype)."""
+    sdq, and W0 (in w0_dtype, default W's dtype). `out` reuses the buffers of
+    an earlier call on the same shape."""
     rows, cols = W.shape
     dev = W.device
     G = rows * cols // 128
-    out = {"codes": torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev),
-           "scales": torch.empty(G, dtype=torch.int16, device=dev)}
-    if sdq:
-        out["sdq_codes"] = torch.empty(G, dtype=torch.int8, device=dev)
-        out["sdq_consts"] = torch.empty(2 * ((G + 255) // 256), dtype=torch.float32, device=dev)
-    w0t = W.dtype if w0_dtype is None else w0_dtype
-    out["W0"] = torch.empty(rows, cols, dtype=w0t, device=dev)
+    if out is None:
+        out = {"codes": torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev),
+               "scales": torch.empty(G, dtype=torch.int16, device=dev)}
+        if sdq:
+            out["sdq_codes"] = torch.empty(G, dtype=torch.int8, device=dev)
+            out["sdq_consts"] = torch.empty(2 * ((G + 255) // 256), dtype=torch.float32, device=dev)
+        w0t = W.dtype if w0_dtype is None else w0_dtype
+        out["W0"] = torch.empty(rows, cols, dtype=w0t, device=dev)
     _check(lib.awsrc_rtn_quantize(rows, cols, _dev_ptr(W), _dtype_code(W), int(sdq), _dev_ptr(out["codes"]),
                                   _dev_ptr(out["scales"]), _dev_ptr(out.get("sdq_codes")),
                                   _dev_ptr(out.get("sdq_consts")), _dev_ptr(out["W0"]), _dtype_code(out["W0"]),

@@ -232,7 +232,7 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
   if (w_dtype != AWSRC_DTYPE_F32 && w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
   if (w0_dtype != AWSRC_DTYPE_F32 && w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
   if (sdq != 0 && sdq != 1) return AWSRC_ERR_INVALID_ARG;
-  if (!W || !codes || !aligned(W, 16) || !aligned(codes, 2) || !aligned(scales, 2) || !aligned(sdq_consts, 4) ||
+  if (!W || !codes || !aligned(W, 16) || !aligned(codes, 4) || !aligned(scales, 2) || !aligned(sdq_consts, 4) ||
       !aligned(W0, 16))
     return AWSRC_ERR_INVALID_ARG;
   const cudaError_t e = launch_rtn(W, w_dtype, rows, cols, sdq, codes, scales, sdq_codes, sdq_consts, W0,
