@@ -47,8 +47,8 @@ OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "f20aba940c0b1abed772390d1dd1810af0150b95162d17bb1f186427e25956e6",
-                  "bytes_per_launch": 442798336 + 16855296}
+SEARCH_TRAFFIC = {"source_sha256": "656d472e5f2cdb59b3b26ea2ab1e1eb97c044a07bc33e965458909d707f60de2",
+                  "bytes_per_launch": 442162432 + 16630528}
 
 
 def search_source_sha() -> str:

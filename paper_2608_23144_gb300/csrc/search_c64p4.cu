@@ -24,8 +24,9 @@
 //    they merge at the end, form the winner's codes again and write the
 //    tile's candidate.
 // Columns of a chunk are seed-pair major: column 8i + 2p + e holds atom p of
-// seed 2i + e, so one 32x32b.x16 TMEM load gives a thread two seed pairs with
-// each atom's two seeds in adjacent registers.
+// seed 2i + e, so one 32x32b.x8 TMEM load gives a thread one seed pair with
+// each atom's two seeds in adjacent registers; the next pair's loads are in
+// flight while a pair is scored.
 // Every mbarrier wait is bounded in time; on expiry the block records a timeout
 // fault, waits (bounded) for its own copies and MMAs in flight, frees its TMEM
 // and returns.
@@ -45,9 +46,7 @@ constexpr int EW = 16;              // epilogue warps
 constexpr int NT = 32 * (EW + 1);   // + the producer warp
 constexpr int SUBS = EW / 4;        // epilogue warps per TMEM lane quarter
 constexpr int SUB_PAIRS = CH / 2 / SUBS;  // seed pairs of a chunk per epilogue warp
-constexpr int RPAIRS = 2;           // seed pairs per TMEM load (8 columns each)
-constexpr int ROUNDS = SUB_PAIRS / RPAIRS;
-static_assert(EW % 4 == 0 && SUB_PAIRS % RPAIRS == 0 && RPAIRS % 2 == 0, "epilogue mapping");
+static_assert(EW % 4 == 0 && SUB_PAIRS >= 1, "epilogue mapping");
 constexpr int STAGES = 4;
 constexpr int PS = pair_stride(4);  // 22 float2 per seed pair
 constexpr uint32_t kBBytes = NCOL * 64 * 2;        // 16 KB of FP16 atoms per chunk
@@ -73,12 +72,6 @@ struct Smem {
   unsigned long long aempty[2];           // epilogue warps done with an accumulator
   uint32_t tmem_base;
 };
-
-// 8 * RPAIRS consecutive columns (RPAIRS seed pairs) in 16-column loads.
-__device__ __forceinline__ void tmem_ld_pairs(uint32_t taddr, float* v) {
-#pragma unroll
-  for (int i = 0; i < RPAIRS / 2; ++i) tmem_ld16(taddr + 16 * i, v + 16 * i);
-}
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
@@ -442,23 +435,28 @@ __global__ void __launch_bounds__(NT, 1)
         for (int i = 0; i < SUBS; ++i) thr = fmaxf(thr, cur_g[i * BM]);
       }
       const float4* pbase = reinterpret_cast<const float4*>(&sm.stage[st][kBBytes]);
+      // The warp's SUB_PAIRS seed pairs, one at a time, with the next pair's
+      // TMEM loads in flight while a pair is scored: wait (only pair i's
+      // loads are outstanding), issue pair i + 1's, then score pair i.
+      const uint32_t cbase = tmem + lane_base + (uint32_t)(tb * 256 + 8 * SUB_PAIRS * sub);
+      float hb[2][8], lb[2][8];
+      tmem_ld8(cbase, hb[0]);
+      tmem_ld8(cbase + 128, lb[0]);
 #pragma unroll
-      for (int rnd = 0; rnd < ROUNDS; ++rnd) {
-        const int p0 = SUB_PAIRS * sub + RPAIRS * rnd;  // first seed pair of the round
-        const uint32_t col = (uint32_t)(tb * 256 + 8 * p0);
-        float hi[8 * RPAIRS], lo[8 * RPAIRS];
-        tmem_ld_pairs(tmem + lane_base + col, hi);
-        tmem_ld_pairs(tmem + lane_base + col + 128, lo);
-        tmem_wait_ld(hi);
-#pragma unroll
-        for (int i = 16; i < 8 * RPAIRS; i += 16) tmem_tie(hi + i);
-#pragma unroll
-        for (int i = 0; i < 8 * RPAIRS; i += 16) tmem_tie(lo + i);
-#pragma unroll
-        for (int j = 0; j < RPAIRS; ++j) {
-          const float4* pe = pbase + (p0 + j) * (PS / 2);
+      for (int i = 0; i < SUB_PAIRS; ++i) {
+        float* hi = hb[i & 1];
+        float* lo = lb[i & 1];
+        tmem_wait_ld8(hi);
+        tmem_tie8(lo);
+        if (i + 1 < SUB_PAIRS) {
+          tmem_ld8(cbase + 8 * (i + 1), hb[(i + 1) & 1]);
+          tmem_ld8(cbase + 128 + 8 * (i + 1), lb[(i + 1) & 1]);
+        }
+        const int pj = SUB_PAIRS * sub + i;  // seed pair within the chunk
+        {
+          const float4* pe = pbase + pj * (PS / 2);
           float2 u[4];
-          const float2 ub = pair_bound(hi + 8 * j, lo + 8 * j, pe, u);
+          const float2 ub = pair_bound(hi, lo, pe, u);
           // prune: a candidate whose gain bound is below the running best
           // cannot win (NaN bounds stay live)
           const bool lx = !FAST || !(ub.x < thr), ly = !FAST || !(ub.y < thr);
@@ -468,7 +466,7 @@ __global__ void __launch_bounds__(NT, 1)
             pair_back(pe, wv, al);
             const float2 gp = pair_gain<FAST>(pr, bv, al, pe);
             // running argmax in seed order: a strictly greater gain wins
-            const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * (p0 + j));
+            const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * pj);
             if (lx && gp.x > bg) { bg = gp.x; bsd = s; }
             if (ly && gp.y > bg) { bg = gp.y; bsd = s + 1; }
             if constexpr (FAST) {

@@ -137,6 +137,31 @@ __device__ __forceinline__ void tmem_tie(float* v) {
                  "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
 }
 
+// 8 consecutive 32-bit TMEM columns of the warp's 32 lanes (valid after a
+// tcgen05.wait::ld, see tmem_wait_ld8).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
+  uint32_t r[8];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+                 "=r"(r[7])
+               : "r"(taddr));
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Waits for this thread's TMEM loads, tying 8 loaded registers to the wait.
+__device__ __forceinline__ void tmem_wait_ld8(float* v) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]), "+f"(v[6]),
+                 "+f"(v[7]));
+}
+
+// Ties 8 further loaded registers to a wait already issued.
+__device__ __forceinline__ void tmem_tie8(float* v) {
+  asm volatile("" : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]), "+f"(v[6]),
+               "+f"(v[7]));
+}
+
 // 4 consecutive 32-bit TMEM columns of the warp's 32 lanes.
 __device__ __forceinline__ void tmem_ld4(uint32_t taddr, float* v) {
   uint32_t r[4];
