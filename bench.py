@@ -71,6 +71,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pf", action="store_true", help="skip the P_F encode measurement")
+    ap.add_argument("--no-model", action="store_true",
+                    help="skip the whole 36-layer Qwen2.5-3B stack (encode, select, decode)")
     ap.add_argument("--modules", default="",
                     help="comma-separated subset of the layer's modules (profiling runs only)")
     return ap.parse_args()
@@ -333,6 +335,80 @@ def backbone_and_serving(dev, prm, mods, outs, stream, records, hbm_gbs):
             "cublas_bf16_gemv_of_decoded_m1_ms": d_ms}
 
 
+def model_stack(dev, hbm_gbs):
+    """The full Qwen2.5-3B-shaped stack (36 layers x 7 modules, 2,774,532,096
+    BF16 weights): every layer encoded (S = 4096) into one candidate array,
+    one AWSRC-U selection over all 252 modules at 0.162 bits/weight, then one
+    dense decode-apply call over every module. Timed on the device with CUDA
+    events, each phase once after a warm-up pass over the whole model. The
+    decode's algorithmic bytes are W0 read + W_hat written (4 B/weight) +
+    the stream."""
+    import torch
+    import paper_2608_23144_gb300 as aw
+    from synth import WORKLOADS, make_layer
+    wl = WORKLOADS["qwen2.5-3b_stack"]
+    mods = []
+    for layer in range(wl.layers):
+        for m in make_layer(wl, layer=layer, device=dev):
+            del m["W"]  # the encoder reads W; it is regenerated per layer below
+            mods.append(m)
+    prm = aw.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
+    per_layer = len(wl.shapes)
+    T_layer = wl.tiles_per_layer
+    cands = torch.empty((T_layer * wl.layers, 16), dtype=torch.uint8, device=dev)
+    ws = None
+    outs = [torch.empty_like(m["W0"]) for m in mods]
+
+    def encode_all():
+        nonlocal ws
+        ms = 0.0
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        for layer in range(wl.layers):
+            lm = make_layer(wl, layer=layer, device=dev)  # W and W0 of this layer, regenerated
+            sl = cands[layer * T_layer:(layer + 1) * T_layer]
+            torch.cuda.synchronize()
+            e[0].record()
+            out = aw.awsrc_encode_tiles(prm, lm, out=sl, workspace=ws)
+            e[1].record()
+            torch.cuda.synchronize()
+            ws = out._awsrc_workspace
+            ms += e[0].elapsed_time(e[1])
+            del lm
+        return ms
+
+    encode_all()                       # warm-up
+    enc_ms = encode_all()
+    assert aw.awsrc_workspace_status(ws) == 0, "encoder self-check fault"
+    stream, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, [RATE])
+    sel_ws = stream._awsrc_workspace
+    aw.awsrc_decode_apply(prm, mods, stream, -1, outs=outs)
+    dec_ws = outs[0]._awsrc_workspace
+    torch.cuda.synchronize()
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    e[0].record()
+    aw.awsrc_select_records(prm, mods, cands, [RATE], workspace=sel_ws, out=stream, counts=counts, nbytes=nbytes)
+    e[1].record()
+    aw.awsrc_decode_apply(prm, mods, stream, -1, outs=outs, workspace=dec_ws)
+    e[2].record()
+    torch.cuda.synchronize()
+    assert aw.awsrc_workspace_status(dec_ws) == 0, "decoder fault"
+    sel_ms, dec_ms = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2])
+    N = sum(m["rows"] * m["cols"] for m in mods)
+    sb = int(nbytes[0].item())
+    dec_bytes = 4 * N + sb
+    out = {"workload": wl.description, "layers": wl.layers, "modules": len(mods), "weights": N,
+           "encode_ms": enc_ms, "layers_per_s": wl.layers / (enc_ms * 1e-3),
+           "encode_candidates_per_s": T_layer * wl.layers * wl.S / (enc_ms * 1e-3),
+           "select_ms": sel_ms, "records": int(counts.sum().item()), "stream_bytes": sb,
+           "decode_ms": dec_ms, "decode_gbs": dec_bytes / (dec_ms * 1e-3) / 1e9,
+           "decode_frac_of_hbm": dec_bytes / (dec_ms * 1e-3) / 1e9 / hbm_gbs,
+           "timing": "encode: 36 calls (one per layer, W regenerated between calls, outside the timed "
+                     "events); select and decode: one call over all 252 modules"}
+    del mods, outs, cands, stream
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -572,6 +648,9 @@ def run_ours(args):
         paper = paper_points(dev, float(peaks.get("hbm_gbs", 6800.0)))
         serving = backbone_and_serving(dev, prm, mods, outs, s, int(counts.sum().item()),
                                        float(peaks.get("hbm_gbs", 6800.0)))
+    model = None
+    if rank == 0 and world == 1 and not args.no_model and not args.modules:
+        model = model_stack(dev, float(peaks.get("hbm_gbs", 6800.0)))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -593,7 +672,7 @@ def run_ours(args):
             "encode_candidates_per_s_kernel": cands_per_step / (search_ms * 1e-3),
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper, "backbone_and_serving": serving,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper, "backbone_and_serving": serving, "model_stack": model,
             "gpu_launches": launches, "clocks": clk.summary(),
         }
         print(json.dumps(line), flush=True)
