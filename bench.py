@@ -71,6 +71,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pf", action="store_true", help="skip the P_F encode measurement")
+    ap.add_argument("--full-models", action="store_true",
+                    help="also encode, select and decode the whole 28-layer Qwen2.5-7B (P_F) and 64-layer "
+                         "Qwen2.5-32B (U and P_F) synthetic models (about a minute of GPU time)")
     ap.add_argument("--no-model", action="store_true",
                     help="skip the whole 36-layer Qwen2.5-3B stack (encode, select, decode)")
     ap.add_argument("--modules", default="",
@@ -409,6 +412,97 @@ def model_stack(dev, hbm_gbs):
     return out
 
 
+def full_model(dev, hbm_gbs, name):
+    """A whole synthetic model of the Qwen2.5-7B (28 layers, AWSRC-P_F) or
+    Qwen2.5-32B (64 layers, AWSRC-U plus AWSRC-P_F) shape, streamed one layer
+    at a time: each layer's W, W0, activation moments and Fisher diagonal are
+    generated on the device, encoded for every variant into model-wide
+    candidate arrays, then W and F are dropped (W0 stays for the decoder).
+    After the last layer: one selection per variant over all modules (U at
+    0.162 bits/weight; P_F prefixes at 0.05/0.10/0.162/0.25 with the 0.5/0.5
+    activation/Fisher blend) and one dense decode-apply call over every
+    module (the U stream, else each P_F prefix). Encode time is the sum of the
+    per-layer CUDA-event times (generation outside them); select and decode
+    are single calls, timed likewise."""
+    import torch
+    import paper_2608_23144_gb300 as aw
+    from synth import WORKLOADS
+    from synth.workloads import make_module, module_seed
+    wl = WORKLOADS[name]
+    PF_RATES = [0.05, 0.10, 0.162, 0.25]
+    variants = [1] if wl.variant == 1 else [0, 1]
+    prm = {v: aw.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S, variant=v) for v in variants}
+    T_layer = wl.tiles_per_layer
+    cands = {v: torch.empty((T_layer * wl.layers, 16), dtype=torch.uint8, device=dev) for v in variants}
+    ws = {v: None for v in variants}
+    enc_ms = {v: 0.0 for v in variants}
+    keep = []  # W0 and shapes of every module, for selection and decode
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for layer in range(wl.layers):
+        lm = []
+        for mi, (_, rows, cols) in enumerate(wl.shapes):
+            m = make_module(rows, cols, seed=module_seed(wl.seed, layer, mi), device=dev, w_dtype=wl.w_dtype,
+                            outlier=wl.outlier, fisher=True, blend=(0.5, 0.5))
+            lm.append(m)
+        for v in variants:
+            mv = lm if v == 1 else [{**m, "fisher": None, "w_act": 1.0, "w_fisher": 0.0} for m in lm]
+            torch.cuda.synchronize()
+            ev[0].record()
+            out = aw.awsrc_encode_tiles(prm[v], mv, out=cands[v][layer * T_layer:(layer + 1) * T_layer],
+                                        workspace=ws[v])
+            ev[1].record()
+            torch.cuda.synchronize()
+            ws[v] = out._awsrc_workspace
+            enc_ms[v] += ev[0].elapsed_time(ev[1])
+        for m in lm:
+            keep.append({"W0": m["W0"], "rows": m["rows"], "cols": m["cols"], "act": m["act"], "fisher": None,
+                         "w_act": 1.0, "w_fisher": 0.0})
+        del lm
+    for v in variants:
+        assert aw.awsrc_workspace_status(ws[v]) == 0, "encoder self-check fault"
+    N = sum(m["rows"] * m["cols"] for m in keep)
+    outs = [torch.empty_like(m["W0"]) for m in keep]
+    res = {"workload": wl.description, "layers": wl.layers, "modules": len(keep), "weights": N}
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    for v in variants:
+        rates = PF_RATES if v == 1 else [RATE]
+        stream, counts, nbytes = aw.awsrc_select_records(prm[v], keep, cands[v], rates)   # warm-up
+        torch.cuda.synchronize()
+        e[0].record()
+        aw.awsrc_select_records(prm[v], keep, cands[v], rates, workspace=stream._awsrc_workspace, out=stream,
+                                counts=counts, nbytes=nbytes)
+        e[1].record()
+        torch.cuda.synchronize()
+        key = "U" if v == 0 else "P_F"
+        r = {"encode_ms": enc_ms[v], "layers_per_s": wl.layers / (enc_ms[v] * 1e-3),
+             "encode_candidates_per_s": T_layer * wl.layers * wl.S / (enc_ms[v] * 1e-3),
+             "select_ms": e[0].elapsed_time(e[1]), "rates_bpw": rates,
+             "records": [int(x) for x in counts.tolist()] if v == 1 else int(counts.sum().item()),
+             "stream_bytes": [int(x) for x in nbytes.tolist()]}
+        Ks = [int(x) for x in counts.tolist()] if v == 1 else [-1]
+        dec = []
+        dws = None
+        for ki, K in enumerate(Ks):
+            aw.awsrc_decode_apply(prm[v], keep, stream, K, outs=outs, workspace=dws)
+            dws = outs[0]._awsrc_workspace
+            torch.cuda.synchronize()
+            e[1].record()
+            aw.awsrc_decode_apply(prm[v], keep, stream, K, outs=outs, workspace=dws)
+            e[2].record()
+            torch.cuda.synchronize()
+            assert aw.awsrc_workspace_status(dws) == 0, "decoder fault"
+            ms = e[1].elapsed_time(e[2])
+            sb = int(nbytes[ki].item())  # the bytes of this prefix of the stream
+            gbs = (4 * N + sb) / (ms * 1e-3) / 1e9
+            dec.append({"K": K, "ms": ms, "gbs": gbs, "frac_of_hbm": gbs / hbm_gbs})
+        r["decode"] = dec
+        res[key] = r
+        del stream
+    del keep, outs, cands
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -651,6 +745,10 @@ def run_ours(args):
     model = None
     if rank == 0 and world == 1 and not args.no_model and not args.modules:
         model = model_stack(dev, float(peaks.get("hbm_gbs", 6800.0)))
+    models = None
+    if rank == 0 and world == 1 and args.full_models:
+        models = {n: full_model(dev, float(peaks.get("hbm_gbs", 6800.0)), n)
+                  for n in ("qwen2.5-7b_stack_pf", "qwen2.5-32b_stack")}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -673,6 +771,7 @@ def run_ours(args):
             "decode_apply": decode,
             "records_per_step": int(counts.sum().item()), "stream_bytes": stream_bytes,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "pf": pf, "paper_points": paper, "backbone_and_serving": serving, "model_stack": model,
+            "full_models": models,
             "gpu_launches": launches, "clocks": clk.summary(),
         }
         print(json.dumps(line), flush=True)
