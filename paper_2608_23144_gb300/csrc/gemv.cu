@@ -126,8 +126,8 @@ __global__ void __launch_bounds__(32 * kGemvWarps) gemv_kernel(Prm pr, GemvArgs 
 // (u the offset-binary code) and one packed subtraction, and are accumulated
 // with packed FMAs; each chunk's sum is scaled by its group's s. The row's
 // recorded tiles follow, 32 tiles at a time: one map entry per lane, the
-// recorded lanes fetch their record codes, and the warp walks the tiles
-// together (elements lane + 32e, mask words by uniform loads, x from global).
+// recorded lanes fetch their record codes and mask words, and the warp walks
+// the tiles together (elements lane + 32e, x from the staged copy).
 constexpr int kUnroll = 2;
 constexpr float kNibbleBias = 8388616.0f;  // 2^23 + 8
 constexpr int kPrefetchWords = 4;          // mask words (P * W) a recorded lane prefetches
@@ -241,7 +241,8 @@ __global__ void __launch_bounds__(32 * kGemvWarps) gemv_warp_kernel(Prm pr, Gemv
   __syncthreads();
   const int n_cb = (int)(a.cols / pr.C);
   const int nch = (int)((a.cols + 1023) >> 10);
-  const float* xb = reinterpret_cast<const float*>(xs4) + 4 * lane;
+  const float* xsm = reinterpret_cast<const float*>(xs4);  // x in shared memory (permuted)
+  const float* xb = xsm + 4 * lane;
   const int64_t stride = (int64_t)gridDim.x * kGemvWarps;
   const bool pre = a.map && pr.P * pr.W <= kPrefetchWords;  // recorded lanes prefetch their mask words
   int64_t row = (int64_t)blockIdx.x * kGemvWarps + warp;
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(32 * kGemvWarps) gemv_warp_kernel(Prm pr, Gemv
             }
             const float r = __fmul_rn(__fmul_rn((float)kj, pr.c), sc);
 #pragma unroll
-            for (int m = 0; m < M; ++m) acc[m] = __fmaf_rn(r, __ldg(a.x + m * a.cols + col0 + j), acc[m]);
+            for (int m = 0; m < M; ++m) acc[m] = __fmaf_rn(r, xsm[m * xs_stride + xs_index(col0 + j)], acc[m]);
           }
         }
       }
