@@ -48,7 +48,10 @@ TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
 SEARCH_TRAFFIC = {"source_sha256": "656d472e5f2cdb59b3b26ea2ab1e1eb97c044a07bc33e965458909d707f60de2",
-                  "bytes_per_launch": 442162432 + 16630528}
+                  "bytes_per_launch": 442162432 + 16630528,
+                  # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
+                  "ncu_fma_pipe_pct": 37.07, "ncu_issue_active_pct": 43.50,
+                  "ncu_tensor_pipe_pct": 23.16}
 
 
 def search_source_sha() -> str:
@@ -636,14 +639,16 @@ def run_ours(args):
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
     fp32_peak = nsm * 128 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
     achieved = cands_per_step * OPS_PER_CANDIDATE / (search_ms * 1e-3)
-    traffic = (SEARCH_TRAFFIC["bytes_per_launch"]
-               if SEARCH_TRAFFIC["source_sha256"] == search_source_sha() else None)
+    counters_valid = SEARCH_TRAFFIC["source_sha256"] == search_source_sha()
+    traffic = SEARCH_TRAFFIC["bytes_per_launch"] if counters_valid else None
     roofline = {"bound": "alu", "kernel": "search_c64p4", "achieved": achieved / 1e9,
                 "peak": fp32_peak / 1e9, "unit": "Gop/s", "frac": achieved / fp32_peak,
                 "traffic": traffic, "peak_kind": f"{peak_kind}: {nsm} SMs x 128 FP32 lanes x "
                 f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
                 "ops_per_candidate": OPS_PER_CANDIDATE, "search_ms": search_ms,
-                "tensor_tflops": cands_per_step * TENSOR_FLOP_PER_CANDIDATE / (search_ms * 1e-3) / 1e12}
+                "tensor_tflops": cands_per_step * TENSOR_FLOP_PER_CANDIDATE / (search_ms * 1e-3) / 1e12,
+                "ncu": ({k: SEARCH_TRAFFIC[k] for k in ("ncu_fma_pipe_pct", "ncu_issue_active_pct",
+                                                         "ncu_tensor_pipe_pct")} if counters_valid else None)}
     decode = {"gbs": dec_gbs, "ms": dec_ms, "frac_of_hbm": dec_gbs / float(peaks.get("hbm_gbs", 6800.0)),
               "hbm_peak_gbs": float(peaks.get("hbm_gbs", 6800.0))}
 
