@@ -31,47 +31,56 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 // solve, of b^T alpha and of the gain itself are each below a small multiple
 // of kappa*2^-24 relative to U (plus a few ulps), far inside the factor
 // 1 + 2^-10 + 2^-14 kappa. So a candidate with U * m < g_best cannot score
-// above g_best. m is +inf (no pruning) when G is not positive definite in
-// double precision or kappa > 2^16. Computed in double and rounded up.
+// above g_best. m is +inf (no pruning) when G is not positive definite or
+// kappa > 2^16.
+//
+// Evaluated in binary32 (the GPU's double rate is low): the LDL^T of G and
+// tr(G^-1) = sum_k |row k of L^-1|^2 / D_k. For kappa <= 2^16 the computed
+// factors are those of G + dG with |dG| <= ~5 P 2^-24 kappa |G| (<= ~8% in
+// eigenvalue terms), and the inverse trace from them is within ~10% of the
+// exact one; it enters m inflated by 1.5, with every operation of m rounded
+// up, so m is at least the value the exact trace gives.
 template <int P>
 __device__ float bound_multiplier(float gd, const float* Goff, float eps) {
-  // LDL^T of G in double; tr(G^-1) = sum_k |row k of L^-1|^2 / D_k
-  double L[P][P], d[P], inv_d[P];
+  float L[P][P], d[P], inv_d[P];
 #pragma unroll
   for (int k = 0; k < P; ++k) {
-    double dk = gd;
+    float dk = gd;
 #pragma unroll
-    for (int i = 0; i < k; ++i) dk -= L[k][i] * L[k][i] * d[i];
-    if (!(dk > 0.0)) return __int_as_float(0x7f800000);
+    for (int i = 0; i < k; ++i) dk = __fmaf_rn(-L[k][i] * L[k][i], d[i], dk);
+    if (!(dk > 0.0f)) return __int_as_float(0x7f800000);
     d[k] = dk;
-    inv_d[k] = 1.0 / dk;
+    inv_d[k] = __frcp_rn(dk);
 #pragma unroll
     for (int j = k + 1; j < P; ++j) {
-      double v = Goff[tri(j, k)];
+      float v = Goff[tri(j, k)];
 #pragma unroll
-      for (int i = 0; i < k; ++i) v -= L[j][i] * L[k][i] * d[i];
-      L[j][k] = v * inv_d[k];
+      for (int i = 0; i < k; ++i) v = __fmaf_rn(-L[j][i] * L[k][i], d[i], v);
+      L[j][k] = __fmul_rn(v, inv_d[k]);
     }
   }
-  double tr_inv = 0.0;
+  float tr_inv = 0.0f;
 #pragma unroll
   for (int i = 0; i < P; ++i) {  // column i of X = L^-1, rows k >= i
-    double x[P];
-    x[i] = 1.0;
-    tr_inv += inv_d[i];
+    float x[P];
+    x[i] = 1.0f;
+    tr_inv = __fadd_rn(tr_inv, inv_d[i]);
 #pragma unroll
     for (int k = i + 1; k < P; ++k) {
-      double v = 0.0;
+      float v = 0.0f;
 #pragma unroll
-      for (int j = i; j < k; ++j) v -= L[k][j] * x[j];
+      for (int j = i; j < k; ++j) v = __fmaf_rn(-L[k][j], x[j], v);
       x[k] = v;
-      tr_inv += v * v * inv_d[k];
+      tr_inv = __fmaf_rn(__fmul_rn(v, v), inv_d[k], tr_inv);
     }
   }
-  const double kappa = (double)P * gd * tr_inv;
-  if (!(kappa <= 65536.0)) return __int_as_float(0x7f800000);
-  const double m = (1.0 + (double)eps * tr_inv) * (1.0 + 0x1p-10 + 0x1p-14 * kappa);
-  return __double2float_ru(m);
+  if (!(tr_inv > 0.0f && tr_inv < 3.0e38f)) return __int_as_float(0x7f800000);
+  const float kappa = __fmul_rn(__fmul_rn((float)P, gd), tr_inv);
+  if (!(kappa <= 65536.0f)) return __int_as_float(0x7f800000);
+  const float ts = __fmul_ru(1.5f, tr_inv), ks = __fmul_ru(1.5f, __fmul_ru(__fmul_ru((float)P, gd), tr_inv));
+  const float f1 = __fmaf_ru(eps, ts, 1.0f);
+  const float f2 = __fmaf_ru(0x1p-14f, ks, 1.0f + 0x1p-10f);
+  return __fmul_ru(f1, f2);
 }
 
 // ----------------------------------------------------------------- gram_u --
@@ -88,6 +97,7 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   const int C = pr.C;
   __shared__ float d[kMaxC];
   __shared__ int Dq[kMaxC];
+  __shared__ int Dt[kMaxC / 4][16];  // subset sums of each 4-input group of Dq
   __shared__ int dok;
   __shared__ float dmax;
   __shared__ float two_qd;
@@ -110,6 +120,15 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   for (int j = threadIdx.x; j < C; j += blockDim.x) Dq[j] = inv == 0.0f ? 0 : fixed_point_int(d[j], inv);
   if (threadIdx.x == 0) two_qd = pow2f(qd);
   __syncthreads();
+  for (int i = threadIdx.x; i < (C / 4) * 16; i += blockDim.x) {
+    const int g = i >> 4, nb = i & 15;
+    int v = 0;
+#pragma unroll
+    for (int bb = 0; bb < 4; ++bb)
+      if ((nb >> bb) & 1) v += Dq[4 * g + bb];
+    Dt[g][nb] = v;
+  }
+  __syncthreads();
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s >= pr.S_pad) return;
   constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
@@ -122,15 +141,15 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   for (int q = 1; q < P; ++q) {
 #pragma unroll
     for (int p = 0; p < q; ++p) {
-      int v = 0;
+      // sum_j (+-1) Dq_j with the sign of atom product p*q: the total minus
+      // twice the inputs where the two masks differ, by nibble-table reads
+      int v = sd, neg = 0;
       for (int wd = 0; wd < pr.W; ++wd) {
         const uint64_t x = mk[p * pr.W + wd] ^ mk[q * pr.W + wd];
-        const int jn = min(64, C - 64 * wd);
-        for (int jj = 0; jj < jn; ++jj) {
-          const int dj = Dq[64 * wd + jj];
-          v += ((x >> jj) & 1ull) ? -dj : dj;
-        }
+        const int gn = min(16, (C - 64 * wd) >> 2);
+        for (int g = 0; g < gn; ++g) neg += Dt[16 * wd + g][(int)((x >> (4 * g)) & 15ull)];
       }
+      v -= 2 * neg;
       Goff[tri(q, p)] = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(v), two_qd));
     }
   }
