@@ -440,6 +440,17 @@ void awsrc_set_timing_events(void* before_search, void* after_search);
 /* Number of kernels this library has launched in the process so far. */
 uint64_t awsrc_kernel_launches(void);
 
+/*
+ * awsrc_verify_reciprocal — a check of the library's own arithmetic (no
+ * counterpart in the paper): the LDL^T factorisations take 1/D_k correctly
+ * rounded from a cheaper sequence on [2^-125, 2^125); this compares that
+ * sequence with CUDA's correctly rounded reciprocal on every binary32 bit
+ * pattern in [first, last) and adds the number that differ to *mismatches
+ * (device, 8-byte aligned; the caller zeroes it). Asynchronous on `stream`.
+ * Errors: INVALID_ARG (null, misaligned, first > last), CUDA.
+ */
+awsrc_status awsrc_verify_reciprocal(uint32_t first, uint32_t last, uint64_t* mismatches, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -39,6 +39,7 @@ from ._binding import (  # noqa: F401
     shape_modules,
     awsrc_header_bytes,
     awsrc_kernel_launches,
+    awsrc_verify_reciprocal,
     awsrc_record_bytes,
     awsrc_select_records,
     awsrc_set_timing_events,

@@ -108,6 +108,8 @@ def _load():
     L.awsrc_set_timing_events.argtypes = [vp, vp]
     L.awsrc_kernel_launches.restype = ct.c_uint64
     L.awsrc_kernel_launches.argtypes = []
+    L.awsrc_verify_reciprocal.restype = st
+    L.awsrc_verify_reciprocal.argtypes = [ct.c_uint32, ct.c_uint32, vp, vp]
     L.awsrc_workspace_status.restype = st
     L.awsrc_workspace_status.argtypes = [vp, vp, P(ct.c_uint32)]
     L.awsrc_rtn_quantize.restype = st
@@ -382,6 +384,14 @@ def awsrc_set_timing_events(before: Optional[torch.cuda.Event], after: Optional[
 
 def awsrc_kernel_launches() -> int:
     return int(lib.awsrc_kernel_launches())
+
+
+def awsrc_verify_reciprocal(first: int, last: int, stream=None, device="cuda") -> int:
+    """Bit patterns in [first, last) where the library's reciprocal differs from
+    CUDA's correctly rounded one (synchronises)."""
+    bad = torch.zeros(1, dtype=torch.int64, device=device)
+    _check(lib.awsrc_verify_reciprocal(first, last, _dev_ptr(bad), _stream(stream)), "verify_reciprocal")
+    return int(bad.item())
 
 
 def candidates_to_numpy(cands: torch.Tensor) -> np.ndarray:

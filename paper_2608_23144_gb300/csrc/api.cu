@@ -586,6 +586,13 @@ awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const aws
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "packed_gemv");
 }
 
+awsrc_status awsrc_verify_reciprocal(uint32_t first, uint32_t last, uint64_t* mismatches, void* stream) {
+  if (!mismatches || !aligned(mismatches, 8) || first > last) return AWSRC_ERR_INVALID_ARG;
+  const cudaError_t e = launch_verify_rcp(first, last, reinterpret_cast<unsigned long long*>(mismatches),
+                                          (cudaStream_t)stream);
+  return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "verify_reciprocal");
+}
+
 awsrc_status awsrc_workspace_status(void* workspace, void* stream, uint32_t* flags) {
   if (!workspace || !flags) return AWSRC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)stream;

@@ -115,6 +115,25 @@ __host__ __device__ constexpr int pair_stride(int P) {
   return ((P * (P - 1) + 2 * P + 1) + 1) / 2 * 2;
 }
 
+// Correctly rounded binary32 reciprocal, as __frcp_rn, cheaper on the range
+// the LDL^T pivots live in. For positive normal x in [2^-125, 2^125) the
+// hardware approximation y (rcp.approx, within one ulp) is corrected once,
+// y + y (1 - x y) with both steps fused (Markstein's final correction: P.
+// Markstein, "Computation of elementary functions on the IBM RISC System/6000
+// processor", IBM J. Res. Dev. 34(1), 1990): 1 - x y is exact and the fused
+// update rounds the corrected value once. Every other input takes __frcp_rn.
+// The fast path equals __frcp_rn on every float of its range, checked
+// exhaustively on the GPU (awsrc_verify_reciprocal).
+__device__ __forceinline__ float rcp_rn(float x) {
+  const uint32_t b = __float_as_uint(x);
+  if (b - 0x01000000u < 0x7D000000u - 0x01000000u) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return __fmaf_rn(y, __fmaf_rn(-x, y, 1.0f), y);
+  }
+  return __frcp_rn(x);
+}
+
 // LDL^T of A = G + eps I with G_pp = gd, G_pq = Goff[tri(q, p)]. Writes L and
 // invD; returns false if some pivot is not in (0, FLT_MAX].
 template <int P>
@@ -137,7 +156,7 @@ __device__ __forceinline__ bool ldl_factor(float gd, float eps, const float* Gof
 #pragma unroll
     for (int i = 0; i < k; ++i) dk = __fmaf_rn(-L[tri(k, i)], E[tri(k, i)], dk);
     ok = ok && (dk > 0.0f) && (dk <= 3.402823466e38f);
-    invD[k] = __frcp_rn(dk);
+    invD[k] = rcp_rn(dk);
   }
   return ok;
 }

@@ -118,4 +118,8 @@ cudaError_t launch_rtn(const void* W, int w_dtype, int64_t rows, int64_t cols, i
                        uint16_t* scales, int8_t* sdq_codes, float* sdq_consts, void* W0, int w0_dtype,
                        cudaStream_t st);
 
+// numerics.cu: bit patterns in [first, last) where rcp_rn differs from __frcp_rn
+// are added to *bad (device).
+cudaError_t launch_verify_rcp(uint32_t first, uint32_t last, unsigned long long* bad, cudaStream_t st);
+
 }  // namespace awsrc

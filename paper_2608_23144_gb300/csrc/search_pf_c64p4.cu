@@ -110,7 +110,7 @@ __device__ __forceinline__ void pf_pair_fit(const float* ah, const float* al, co
     for (int i = 0; i < k; ++i) dk = __ffma2_rn(nL[tri(k, i)], E[tri(k, i)], dk);
     *okx = *okx && pivot_ok(dk.x);
     *oky = *oky && pivot_ok(dk.y);
-    invD[k] = make_float2(__frcp_rn(dk.x), __frcp_rn(dk.y));
+    invD[k] = make_float2(rcp_rn(dk.x), rcp_rn(dk.y));
   }
   ldl_solve2<4>(nL, invD, bv, alpha);
 }
