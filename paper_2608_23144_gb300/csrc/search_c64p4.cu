@@ -69,7 +69,8 @@ struct Smem {
   float cur_g[SUBS][BM];                  // running best gain of each (sub, row) in u units, for pruning
   unsigned long long full[STAGES];        // bulk copies of a chunk landed
   unsigned long long afull[2];            // MMAs of a chunk completed (tcgen05.commit)
-  unsigned long long aempty[2];           // epilogue warps done with an accumulator
+  unsigned long long aempty[2];           // epilogue warps done loading an accumulator
+  unsigned long long sempty[STAGES];      // epilogue warps done with a stage's factors
   uint32_t tmem_base;
 };
 
@@ -289,6 +290,7 @@ __global__ void __launch_bounds__(NT, 1)
         mbar_init(&sm.afull[i], 1);
         mbar_init(&sm.aempty[i], EW);
       }
+      for (int i = 0; i < STAGES; ++i) mbar_init(&sm.sempty[i], EW);
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     tc_fence_before();
@@ -367,17 +369,8 @@ __global__ void __launch_bounds__(NT, 1)
       for (; k < nck; ++k) {
         const int st = k % STAGES, tb = k & 1;
         if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
-        if (k >= 2) {
-          // the epilogue of chunk k-2 is done: its accumulator and its stage are free
-          if (!mbar_wait(&sm.aempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
-          if (issued < nck) {
-            const int ns = issued % STAGES;
-            mbar_expect_tx(&sm.full[ns], kBBytes + kPBytes);
-            bulk_g2s(&sm.stage[ns][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[ns]);
-            bulk_g2s(&sm.stage[ns][kBBytes], pf_src + (size_t)issued * kPBytes, kPBytes, &sm.full[ns]);
-            ++issued;
-          }
-        }
+        // every epilogue warp has loaded chunk k-2 from its accumulator
+        if (k >= 2 && !mbar_wait(&sm.aempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
         tc_fence_after();
         const uint32_t bsm = smem_addr(&sm.stage[st][0]);
 #pragma unroll
@@ -389,6 +382,16 @@ __global__ void __launch_bounds__(NT, 1)
           }
         }
         umma_commit(&sm.afull[tb]);
+        if (k >= 2 && issued < nck) {
+          // chunk k-2's factors are no longer read: its stage takes chunk k+2
+          const int ps = (k - 2) % STAGES;
+          if (!mbar_wait(&sm.sempty[ps], (uint32_t)(((k - 2) / STAGES) & 1))) { timed_out = true; ++k; break; }
+          const int ns = issued % STAGES;
+          mbar_expect_tx(&sm.full[ns], kBBytes + kPBytes);
+          bulk_g2s(&sm.stage[ns][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[ns]);
+          bulk_g2s(&sm.stage[ns][kBBytes], pf_src + (size_t)issued * kPBytes, kPBytes, &sm.full[ns]);
+          ++issued;
+        }
       }
       if (timed_out) {
         // wait (bounded) for this block's copies and MMAs still in flight
@@ -451,6 +454,12 @@ __global__ void __launch_bounds__(NT, 1)
         if (i + 1 < SUB_PAIRS) {
           tmem_ld8(cbase + 8 * (i + 1), hb[(i + 1) & 1]);
           tmem_ld8(cbase + 128 + 8 * (i + 1), lb[(i + 1) & 1]);
+        } else {
+          // the warp's last loads of this accumulator are complete: release it
+          // now, so that chunk k+2's MMAs need not wait for the last scores
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.aempty[tb]);
         }
         const int pj = SUB_PAIRS * sub + i;  // seed pair within the chunk
         {
@@ -477,9 +486,8 @@ __global__ void __launch_bounds__(NT, 1)
           }
         }
       }
-      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.aempty[tb]);
+      if (lane == 0) mbar_arrive(&sm.sempty[st]);  // done with the stage's factors
     }
     sm.red_g[sub][m] = bg;
     sm.red_s[sub][m] = bsd;
