@@ -47,11 +47,11 @@ OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "8a10118677a5dd6f84f011dccab41be76e99d15d5d3fca47ba286318d460d595",
-                  "bytes_per_launch": 442225920 + 16615424,
+SEARCH_TRAFFIC = {"source_sha256": "7d5c53ca340a84740acee414cdd963193738a988b6fdd19aabbf0a6e10243f83",
+                  "bytes_per_launch": 443179008 + 16896512,
                   # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
-                  "ncu_fma_pipe_pct": 37.23, "ncu_issue_active_pct": 43.59,
-                  "ncu_tensor_pipe_pct": 23.06}
+                  "ncu_fma_pipe_pct": 38.26, "ncu_issue_active_pct": 45.31,
+                  "ncu_tensor_pipe_pct": 23.66}
 
 
 def search_source_sha() -> str:
