@@ -47,7 +47,7 @@ OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
 TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "7d5c53ca340a84740acee414cdd963193738a988b6fdd19aabbf0a6e10243f83",
+SEARCH_TRAFFIC = {"source_sha256": "6d1079712f4600ea47f9057a1375d6b7b73847b96f7a4fb1e394b59ed11273ca",
                   "bytes_per_launch": 443179008 + 16896512,
                   # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
                   "ncu_fma_pipe_pct": 38.26, "ncu_issue_active_pct": 45.31,
@@ -55,11 +55,16 @@ SEARCH_TRAFFIC = {"source_sha256": "7d5c53ca340a84740acee414cdd963193738a988b6fd
 
 
 def search_source_sha() -> str:
-    """SHA-256 of the search kernel's source and the headers it includes: the
-    committed DRAM traffic figure holds only for that exact kernel."""
+    """SHA-256 of the search kernel's source and the headers it includes, with
+    comments and blank lines removed: the committed DRAM traffic and ncu
+    figures hold only for that exact code."""
+    import re
     h = hashlib.sha256()
     for f in ("search_c64p4.cu", "tc05.cuh", "common.cuh", "internal.h"):
-        h.update(open(os.path.join(ROOT, "paper_2608_23144_gb300", "csrc", f), "rb").read())
+        src = open(os.path.join(ROOT, "paper_2608_23144_gb300", "csrc", f)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        src = "\n".join(l.split("//")[0].rstrip() for l in src.splitlines())
+        h.update("\n".join(l for l in src.splitlines() if l.strip()).encode())
     return h.hexdigest()
 
 

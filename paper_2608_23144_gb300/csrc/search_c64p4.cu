@@ -15,7 +15,10 @@
 //    in the canonical K-major layout (16 KB) and the chunk's paired Gram factors
 //    (2.8 KB) — by bulk copies into a 4-stage shared-memory ring, and issues the
 //    chunk's 8 MMAs (M = 128, N = 128, K = 16; halves hi and lo, 4 k-steps) into
-//    one of two 256-column TMEM accumulators, committed to an mbarrier.
+//    one of two 256-column TMEM accumulators, committed to an mbarrier. Chunk
+//    k's MMAs wait only until every epilogue warp has loaded chunk k-2 from
+//    that accumulator; chunk k-2's stage is refilled once every warp has also
+//    finished reading its factors (two release barriers).
 //  * Warps 0..15 (epilogue): warp w reads TMEM lanes 32(w%4).. (its threads'
 //    rows) and the columns of seeds 8(w/4)..8(w/4)+7 of each chunk, and runs the
 //    fit / quantise / score epilogue on seed pairs as float2 streams, keeping a
