@@ -104,3 +104,84 @@ def test_bound_is_tight_on_typical_tiles(orc):
             U = b @ np.linalg.solve(G + eps * np.eye(P), b)
             ratios.append(U * m / (b @ np.linalg.solve(G, b)))
     assert np.median(ratios) < 1.01 and min(ratios) >= 1.0
+
+
+def multiplier_binary32(gd, Goff, eps):
+    """The multiplier as the GPU table builder evaluates it: LDL^T of G and the
+    inverse trace in binary32 (fused multiply-adds emulated by one rounding of
+    the double-precision result), the trace inflated by 1.5, the last steps
+    rounded up (emulated by one step towards +inf after rounding)."""
+    f = np.float32
+    up = lambda x: np.nextafter(f(x), f(np.inf))
+    fma = lambda a, b, c: f(np.float64(a) * np.float64(b) + np.float64(c))
+    L = np.zeros((P, P), np.float32)
+    d = np.zeros(P, np.float32)
+    inv = np.zeros(P, np.float32)
+    for k in range(P):
+        dk = f(gd)
+        for i in range(k):
+            dk = fma(-f(L[k, i] * L[k, i]), d[i], dk)
+        if not dk > 0:
+            return np.inf
+        d[k], inv[k] = dk, f(1.0 / np.float64(dk))
+        for j in range(k + 1, P):
+            v = f(Goff[j][k])
+            for i in range(k):
+                v = fma(-f(L[j, i] * L[k, i]), d[i], v)
+            L[j, k] = f(v * inv[k])
+    tr = f(0)
+    for i in range(P):
+        x = np.zeros(P, np.float32)
+        x[i] = 1
+        tr = f(tr + inv[i])
+        for k in range(i + 1, P):
+            v = f(0)
+            for j in range(i, k):
+                v = fma(-L[k, j], x[j], v)
+            x[k] = v
+            tr = fma(f(v * v), inv[k], tr)
+    kappa = f(f(P * f(gd)) * tr)
+    if not (tr > 0 and kappa <= 65536):
+        return np.inf
+    ts = up(1.5 * np.float64(tr))
+    ks = up(1.5 * np.float64(up(np.float64(up(P * np.float64(gd))) * tr)))
+    f1 = up(np.float64(eps) * ts + 1)
+    f2 = up(2.0 ** -14 * np.float64(ks) + (1 + 2.0 ** -10))
+    return float(up(np.float64(f1) * f2))
+
+
+def test_binary32_multiplier_is_never_below_the_double_one():
+    """The GPU builds the pruning multiplier in binary32 with a 1.5 safety factor
+    on tr(G^-1); over Gram matrices of +-1 atoms under weights spanning twelve
+    decades (condition numbers up to the 2^16 cutoff) it must stay at or above
+    the double-precision multiplier, or be +inf (no pruning)."""
+    rng = np.random.default_rng(17)
+    checked, kappas = 0, []
+    for trial in range(4000):
+        scale = 10.0 ** rng.uniform(-6, 6)
+        kind = trial % 4
+        if kind == 0:
+            dv = rng.lognormal(0, 2.0, C)
+        elif kind == 1:
+            dv = 10.0 ** rng.uniform(-6, 6, C)
+        elif kind == 2:
+            dv = rng.lognormal(0, 1.0, C) * (rng.random(C) < 0.2)
+        else:  # weight on a few coordinates over a small floor: G nearly rank-deficient
+            dv = np.full(C, 10.0 ** rng.uniform(-6, -2))
+            dv[rng.choice(C, rng.integers(2, 5), replace=False)] = 1.0
+        dv = (dv * scale).astype(np.float32).astype(np.float64)
+        sgn = rng.choice([-1.0, 1.0], size=(P, C))
+        G = (sgn * dv) @ sgn.T / C
+        G = G.astype(np.float32).astype(np.float64)
+        gd = float(np.float32(dv.sum() / C))
+        np.fill_diagonal(G, gd)
+        eps = float(np.float32(np.float32(1e-6) * np.float32(gd)))
+        m64 = multiplier(G, eps)
+        m32 = multiplier_binary32(gd, G, eps)
+        if not np.isfinite(m32):
+            continue
+        checked += 1
+        kappas.append(np.trace(G) * np.trace(np.linalg.inv(G)))
+        assert np.isfinite(m64) and m32 >= m64, (trial, m32, m64)
+    kappas = np.array(kappas)
+    assert checked > 1000 and (kappas > 1e3).sum() >= 50 and (kappas > 1e4).sum() >= 10
