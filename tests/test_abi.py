@@ -144,3 +144,32 @@ def test_backbone_metadata_bytes(libpath):
     assert aw.awsrc_backbone_metadata_bytes(11008, 2048, True) == G + 8 * 688
     assert aw.awsrc_backbone_metadata_bytes(4, 100, True) == -1
     assert aw.awsrc_backbone_metadata_bytes(1, 128, True) == 1 + 8
+
+
+def test_serving_and_diagnostic_arguments_are_refused_on_the_host(libpath):
+    """Pointer values are only compared (no device memory exists): the backbone
+    quantiser, the packed GEMV and the reciprocal check return INVALID_ARG or
+    SHAPE on the host, before any launch."""
+    import paper_2608_23144_gb300 as aw
+    lib = aw.lib
+    bf16 = aw.DTYPE_BF16
+    # awsrc_rtn_quantize: cols % 128, 16-byte W and W0, 4-byte codes
+    assert lib.awsrc_rtn_quantize(8, 100, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40000, bf16, None) == 2
+    assert lib.awsrc_rtn_quantize(8, 128, 0x10008, bf16, 0, 0x20000, 0x30000, None, None, 0x40000, bf16, None) == 1
+    assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 0, 0x20002, 0x30000, None, None, 0x40000, bf16, None) == 1
+    assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40004, bf16, None) == 1
+    assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 2, 0x20000, 0x30000, None, None, 0x40000, bf16, None) == 1
+    # awsrc_packed_gemv: M in [1, 8], module index, 16-byte x, 4-byte codes
+    from paper_2608_23144_gb300._binding import PackedWeights, shape_modules
+    p = aw.params(C=64, S=64)
+    mods = shape_modules([(8, 128)])
+    pw = PackedWeights(0x10000, 0x20000, None, None, 0, 0)
+    assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 0, ct.byref(pw), None, 0, 9, 0x30000, 0x40000, None) == 1
+    assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 1, ct.byref(pw), None, 0, 1, 0x30000, 0x40000, None) == 1
+    assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 0, ct.byref(pw), None, 0, 1, 0x30008, 0x40000, None) == 1
+    pw.codes = 0x10002
+    assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 0, ct.byref(pw), None, 0, 1, 0x30000, 0x40000, None) == 1
+    # awsrc_verify_reciprocal: null, misaligned counter, empty-range order
+    assert lib.awsrc_verify_reciprocal(0, 1, None, None) == 1
+    assert lib.awsrc_verify_reciprocal(0, 1, 0x50004, None) == 1
+    assert lib.awsrc_verify_reciprocal(2, 1, 0x50000, None) == 1
