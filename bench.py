@@ -76,6 +76,8 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--ref-step-seconds", type=float, default=4.0,
+                    help="target CPU time of one step of the reference (oracle) arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pf", action="store_true", help="skip the P_F encode measurement")
@@ -525,22 +527,29 @@ def run_reference(args):
     oprm = orc.params(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
     masks = orc.basis_masks(oprm)
     rng = np.random.default_rng(1)
-    # one step = one whole row of every module (1 row x n_cb tiles each)
-    def step():
+    tiles_per_row = sum(m["W"].shape[1] // wl.C for m in mods)
+
+    # one step = `rows` random whole rows of every module, enough tiles per
+    # oracle call to keep every host core busy
+    def step(rows):
         n = 0
         for m in mods:
-            r = int(rng.integers(m["W"].shape[0]))
-            orc.encode_tiles(oprm, m["W"][r:r + 1], m["W0"][r:r + 1], m["act"], masks=masks)
-            n += m["W"].shape[1] // wl.C
+            r = rng.choice(m["W"].shape[0], rows, replace=False)
+            orc.encode_tiles(oprm, m["W"][r], m["W0"][r], m["act"], masks=masks)
+            n += rows * m["W"].shape[1] // wl.C
         return n * wl.S
-    for _ in range(args.warmup):
-        step()
     t0 = time.perf_counter()
-    cands = sum(step() for _ in range(args.steps))
+    step(4)                                          # calibration (and warm-up)
+    per_row = (time.perf_counter() - t0) / 4
+    rows = max(1, min(min(m["W"].shape[0] for m in mods), int(args.ref_step_seconds / per_row)))
+    for _ in range(args.warmup):
+        step(rows)
+    t0 = time.perf_counter()
+    cands = sum(step(rows) for _ in range(args.steps))
     dt = time.perf_counter() - t0
     v = cands / dt
-    sample = (f"per step one random whole row of each of the 7 modules "
-              f"({cands // args.steps:,} candidates, S = {wl.S})")
+    sample = (f"per step {rows} random whole rows of each of the 7 modules "
+              f"({rows * tiles_per_row:,} tiles x {wl.S} seeds = {cands // args.steps:,} candidates)")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
