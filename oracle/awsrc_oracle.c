@@ -37,6 +37,13 @@
 #define ORC_MAXP 8
 #define ORC_GAMMA 0x9E3779B97F4A7C15ULL
 
+/* Planted mistakes for the mutation test of the pins: a build with
+ * -DORC_MUTANT=k carries mistake k (listed in the test), and the pins must
+ * catch every one. The default, 0, is the oracle itself. */
+#ifndef ORC_MUTANT
+#define ORC_MUTANT 0
+#endif
+
 /* Candidate record layout mirrors the ABI's 16-byte struct (an interface, not code). */
 typedef struct {
   float gain;
@@ -103,7 +110,11 @@ void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
   if (permute) {
     for (int i = C - 1; i >= 1; --i) {
       uint64_t x = orc_splitmix64_output(key, n++) >> 32;
+#if ORC_MUTANT == 12
+      int k = (int)((x * (uint64_t)i) >> 32);
+#else
       int k = (int)((x * (uint64_t)(i + 1)) >> 32);
+#endif
       int32_t t = perm[i]; perm[i] = perm[k]; perm[k] = t;
     }
   }
@@ -119,7 +130,11 @@ void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
   /* B_s[j][p] = C^-1/2 * sigma_j * H[pi(j), c_p],  H[i][k] = (-1)^popcount(i & k) */
   for (int p = 0; p < P; ++p)
     for (int j = 0; j < C; ++j)
+#if ORC_MUTANT == 13
+      negmask[p * C + j] = (uint8_t)((sign[j] + orc_popcount((uint32_t)(perm[j] | cols[p]))) & 1);
+#else
       negmask[p * C + j] = (uint8_t)((sign[j] + orc_popcount((uint32_t)(perm[j] & cols[p]))) & 1);
+#endif
 }
 
 /* ------------------------------------------------------------------------ */
@@ -195,7 +210,11 @@ int orc_fixed_point(int C, const float* x, int32_t* X) {
     for (int j = 0; j < C; ++j) X[j] = 0;
     return 0;
   }
+#if ORC_MUTANT == 17
+  int q = ilogbf(m) - 19;
+#else
   int q = ilogbf(m) - 20;
+#endif
   for (int j = 0; j < C; ++j) X[j] = (int32_t)rintf(ldexpf(x[j], -q));
   return q;
 }
@@ -231,7 +250,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     int64_t su = 0;
     for (int j = 0; j < C; ++j) su += negmask[p * C + j] ? -(int64_t)Y[j] : (int64_t)Y[j];
     float u = ldexpf((float)su, qy);
+#if ORC_MUTANT == 3
+    bvec[p] = u;
+#else
     bvec[p] = c * u;
+#endif
   }
   /* Gram G = B_s^T D B_s */
   float G[ORC_MAXP][ORC_MAXP];
@@ -243,12 +266,22 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     for (int q = p + 1; q < P; ++q) {
       int64_t sv = 0;
       for (int j = 0; j < C; ++j)
+#if ORC_MUTANT == 1
+        sv += (negmask[p * C + j] ^ negmask[q * C + j]) ? (int64_t)Dq[j] : -(int64_t)Dq[j];
+#elif ORC_MUTANT == 2
+        sv += (negmask[p * C + j] ^ negmask[p * C + (j ^ 1)]) ? -(int64_t)Dq[j] : (int64_t)Dq[j];
+#else
         sv += (negmask[p * C + j] ^ negmask[q * C + j]) ? -(int64_t)Dq[j] : (int64_t)Dq[j];
+#endif
       G[p][q] = G[q][p] = c2 * ldexpf((float)sv, qd);
     }
   }
   /* ridge (Eq. 3): A = G + eps I */
+#if ORC_MUTANT == 5
+  float eps = prm->ridge_rel;
+#else
   float eps = prm->ridge_rel * gd;
+#endif
   float A[ORC_MAXP][ORC_MAXP];
   for (int p = 0; p < P; ++p)
     for (int q = 0; q < P; ++q) A[p][q] = G[p][q];
@@ -272,7 +305,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
   float z[ORC_MAXP], alpha[ORC_MAXP];
   for (int k = 0; k < P; ++k) {
     float v = bvec[k];
+#if ORC_MUTANT == 16
+    for (int i = 0; i < k - 1; ++i) v = fmaf(-L[k][i], z[i], v);
+#else
     for (int i = 0; i < k; ++i) v = fmaf(-L[k][i], z[i], v);
+#endif
     z[k] = v;
   }
   for (int k = P - 1; k >= 0; --k) {
@@ -298,7 +335,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     int lo, hi;
     orc_exp_range(prm, &lo, &hi);
     int e0 = ilogbf(amax) - (prm->b - 2);   /* ilogb(qmax) = b - 2 */
+#if ORC_MUTANT == 4
+    int e = e0 + (amax > ldexpf((float)qmax, e0) ? 1 : 0) + 1;
+#else
     int e = e0 + (amax > ldexpf((float)qmax, e0) ? 1 : 0);
+#endif
     if (e < lo) e = lo;
     if (e > hi) e = hi;
     float inv = ldexpf(1.0f, -e);
@@ -331,7 +372,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     for (int q = p + 1; q < P; ++q) Qq = fmaf((float)(2 * codes[p] * codes[q]), G[p][q], Qq);
   }
   float t = sc * Qq;
+#if ORC_MUTANT == 6
+  float g = sc * (Aq - t);
+#else
   float g = sc * (2.0f * Aq - t);
+#endif
   *gain_out = g;
   *scale_out = scale_field;
   for (int p = 0; p < ORC_MAXP; ++p) codes_out[p] = (int8_t)(p < P ? codes[p] : 0);
@@ -374,7 +419,11 @@ void orc_encode_tiles(const orc_params* prm, int64_t rows, int64_t cols, const f
       for (int s = 0; s < prm->S; ++s) {
         float g; int16_t sf; int8_t codes[8];
         if (!orc_score_candidate(prm, r, d, masks + (size_t)s * P * C, &g, &sf, codes, NULL)) continue;
+#if ORC_MUTANT == 7
+        if (g >= best.gain) {
+#else
         if (g > best.gain) {
+#endif
           best.gain = g;
           best.seed = (uint16_t)s;
           best.scale = sf;
@@ -473,7 +522,11 @@ int64_t orc_header_bytes(int32_t n_mod) { return 40 + 8 * (int64_t)n_mod; }
 int64_t orc_record_bytes(const orc_params* prm, int64_t T) {
   int64_t bits = orc_ceil_log2((uint64_t)T) + orc_ceil_log2((uint64_t)prm->S) + prm->b_e +
                  (int64_t)prm->P * prm->b;
+#if ORC_MUTANT == 10
+  return (bits + 8) / 8;
+#else
   return (bits + 7) / 8;
+#endif
 }
 
 int64_t orc_budget_bytes(double rate_bpw, int64_t n_scope) {
@@ -537,7 +590,11 @@ static int orc_key_cmp(const void* a, const void* b) {
   const orc_key* y = (const orc_key*)b;
   if (x->gain > y->gain) return -1;   /* rho = gain / L with one L: gain descending */
   if (x->gain < y->gain) return 1;
+#if ORC_MUTANT == 8
+  return (x->tile < y->tile) - (x->tile > y->tile);
+#else
   return (x->tile > y->tile) - (x->tile < y->tile);  /* ties: tile ascending */
+#endif
 }
 
 /*
@@ -588,7 +645,11 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
     for (int r = 0; r < n_rates; ++r) {
       int64_t B = orc_budget_bytes(rates[r], Nscope);
       if (B < h) { rc = 4; goto done; }
+#if ORC_MUTANT == 9
+      int64_t K = (B - h) / L + 1;
+#else
       int64_t K = (B - h) / L;
+#endif
       if (K > npos) K = npos;
       counts[r] = K;
       bytes_out[r] = h + K * L;
@@ -664,7 +725,11 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
     for (int j = 0; j < C; ++j) {
       int kj = 0;
       for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
+#if ORC_MUTANT == 11
+      float rh = ((float)kj * c) * (0.5f * sc);
+#else
       float rh = ((float)kj * c) * sc;
+#endif
       out[m][base + j] = out[m][base + j] + rh;
     }
   }
@@ -702,7 +767,11 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
       const float a = fabsf(w[j]);
       if (a > amax) amax = a;
     }
+#if ORC_MUTANT == 14
+    const uint16_t h = orc_f32_to_f16(amax / 8.0f);
+#else
     const uint16_t h = orc_f32_to_f16(amax / 7.0f);
+#endif
     s16[g] = h;
     const float s = orc_f16_to_f32(h);
     for (int j = 0; j < group; ++j) {
@@ -727,7 +796,11 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
         const float d = fabsf(s_eff[g] - mu);
         if (d > a) a = d;
       }
+#if ORC_MUTANT == 15
+      const float step = a / 128.0f;
+#else
       const float step = a / 127.0f;
+#endif
       consts[2 * (b0 / block)] = mu;
       consts[2 * (b0 / block) + 1] = step;
       for (int64_t g = b0; g < b0 + n; ++g) {

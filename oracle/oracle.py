@@ -44,25 +44,31 @@ class Params(ct.Structure):
     ]
 
 
-def build(force: bool = False) -> str:
+def _mutant() -> int:
+    """Planted-mistake build selected by AWSRC_ORACLE_MUTANT (the mutation test
+    of the pins only; 0 or unset is the oracle itself)."""
+    return int(os.environ.get("AWSRC_ORACLE_MUTANT", "0") or 0)
+
+
+def build(force: bool = False, mutant: int = 0) -> str:
     """Compile the oracle with gcc (-ffp-contract=off: no implicit fusion)."""
     os.makedirs(_BUILD, exist_ok=True)
-    if not force and os.path.exists(_LIB_PATH) and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC):
-        return _LIB_PATH
-    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    path = _LIB_PATH if mutant == 0 else os.path.join(_BUILD, f"liboracle_mutant{mutant}.so")
+    if not force and os.path.exists(path) and os.path.getmtime(path) >= os.path.getmtime(_SRC):
+        return path
+    tmp = path + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=gnu11", "-ffp-contract=off", "-fno-fast-math", "-fopenmp",
-           "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"]
+           "-fPIC", "-shared", f"-DORC_MUTANT={mutant}", "-o", tmp, _SRC, "-lm"]
     subprocess.run(cmd, check=True)
-    os.replace(tmp, _LIB_PATH)
-    return _LIB_PATH
+    os.replace(tmp, path)
+    return path
 
 
 def lib():
     global _lib
     with _lock:
         if _lib is None:
-            build()
-            L = ct.CDLL(_LIB_PATH)
+            L = ct.CDLL(build(mutant=_mutant()))
             P = ct.POINTER
             vp = ct.c_void_p
             L.orc_num_threads.restype = ct.c_int

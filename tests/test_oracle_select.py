@@ -125,3 +125,30 @@ def test_no_positive_gain_gives_empty_stream(orc):
     cands["gain"] = -np.inf
     stream, counts, nbytes = orc.select_records(prm, [(64, 16)], cands, [8.0])
     assert counts[0] == 0 and len(stream) == orc.header_bytes(1)
+
+
+@pytest.mark.parametrize("variant", [0, 1])
+def test_equal_gains_are_ranked_by_tile_ascending(orc, variant):
+    """Ties in rho = gain / L (one L for every record) are broken by the global
+    tile index, smallest first, in both allocations: with every gain drawn
+    from three values and a budget that keeps part of each tie class, the
+    stream lists each class's tiles in ascending order and keeps the smallest
+    ones of the class that is cut."""
+    prm = orc.params(C=16, P=2, b=4, S=4, variant=variant)
+    shapes = [(64, 64)]
+    T = 64 * 64 // 16
+    rng = np.random.default_rng(31)
+    cands = np.zeros(T, orc.CANDIDATE_DTYPE)
+    cands["gain"] = rng.choice(np.array([1.0, 2.0, 3.0], np.float32), T)
+    cands["seed"] = rng.integers(0, 4, T)
+    stream, counts, _ = orc.select_records(prm, shapes, cands, [0.75])
+    K, _, recs = _parse(orc, prm, stream, shapes)
+    assert 0 < K < T
+    tiles = [t for t, _ in recs]
+    gains = [float(cands[t]["gain"]) for t in tiles]
+    assert gains == sorted(gains, reverse=True)
+    for g in set(gains):
+        cls = [t for t, gg in zip(tiles, gains) if gg == g]
+        assert cls == sorted(cls)
+        everyone = np.flatnonzero(cands["gain"] == g)
+        assert cls == sorted(everyone.tolist())[: len(cls)]   # the smallest tiles of the class

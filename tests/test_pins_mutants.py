@@ -1,0 +1,42 @@
+"""Mutation test of the oracle's pins: the oracle built with
+-DORC_MUTANT=k carries one plausible mistake (below), and the pin files
+(tests/test_oracle_*.py) run against that build in a subprocess must fail.
+A mistake that no pin catches means the oracle is not pinned there."""
+import glob
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+PIN_FILES = sorted(glob.glob(os.path.join(ROOT, "tests", "test_oracle_*.py")))
+
+MUTANTS = {
+    1: "Gram off-diagonal sums with the sign of the atom product flipped",
+    2: "Gram off-diagonal sums taking a wrong atom index",
+    3: "b = B^T D r without the C^-1/2 normalisation",
+    4: "power-of-two scale exponent one too large",
+    5: "ridge eps absolute instead of relative to mean(d)",
+    6: "Eq. 4 gain without the factor 2 on alpha^T b",
+    7: "seed ties keep the larger selector",
+    8: "records with equal gains ordered by tile descending",
+    9: "progressive prefix one record longer than the budget allows",
+    10: "record width rounded up one byte too far",
+    11: "decoder adds half the correction",
+    12: "Fisher-Yates permutation draw range one short",
+    13: "Hadamard entry sign from OR instead of AND",
+    14: "RTN group scale max|w| / 8 instead of / 7",
+    15: "SDQ step max deviation / 128 instead of / 127",
+    16: "forward substitution dropping its last term",
+    17: "fixed-point grid one bit coarser",
+}
+
+
+@pytest.mark.parametrize("k", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(k):
+    env = dict(os.environ, AWSRC_ORACLE_MUTANT=str(k))
+    r = subprocess.run([sys.executable, "-m", "pytest", *PIN_FILES, "-x", "-q", "-m", "not gpu",
+                        "-p", "no:cacheprovider"], env=env, cwd=ROOT, capture_output=True, text=True,
+                       timeout=900)
+    assert r.returncode == 1, f"mistake {k} ({MUTANTS[k]}) not caught by any pin:\n{r.stdout[-3000:]}"
