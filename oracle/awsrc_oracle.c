@@ -103,7 +103,11 @@ void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
   /* sign pattern: one 64-bit draw per 64 coordinates */
   for (int w = 0; w * 64 < C; ++w) {
     uint64_t word = orc_splitmix64_output(key, n++);
+#if ORC_MUTANT == 20
+    for (int j = w * 64; j < C && j < w * 64 + 64; ++j) sign[j] = (uint8_t)((word >> (63 - (j - w * 64))) & 1u);
+#else
     for (int j = w * 64; j < C && j < w * 64 + 64; ++j) sign[j] = (uint8_t)((word >> (j - w * 64)) & 1u);
+#endif
   }
   /* coordinate permutation: Fisher-Yates (Durstenfeld), index by multiply-shift */
   for (int j = 0; j < C; ++j) perm[j] = j;
@@ -555,8 +559,13 @@ void orc_pack_record(const orc_params* prm, int64_t T, int64_t tile, const orc_c
   int64_t L = orc_record_bytes(prm, T);
   memset(rec, 0, (size_t)L);
   int pos = 0;
+#if ORC_MUTANT == 18
+  orc_put_bits(rec, &pos, cd->seed, orc_ceil_log2((uint64_t)prm->S));
+  orc_put_bits(rec, &pos, (uint64_t)tile, orc_ceil_log2((uint64_t)T));
+#else
   orc_put_bits(rec, &pos, (uint64_t)tile, orc_ceil_log2((uint64_t)T));
   orc_put_bits(rec, &pos, cd->seed, orc_ceil_log2((uint64_t)prm->S));
+#endif
   uint64_t sf;
   if (prm->scale_mode == 0) sf = (uint64_t)(int64_t)(cd->scale - prm->e_bias);
   else sf = (uint16_t)cd->scale;
@@ -858,7 +867,11 @@ int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_row
     for (int j = 0; j < C; ++j) {
       int kj = 0;
       for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
+#if ORC_MUTANT == 19
+      Wt[base + j] -= (double)kj * c * sc;
+#else
       Wt[base + j] += (double)kj * c * sc;
+#endif
     }
   }
   for (int v = 0; v < M; ++v)

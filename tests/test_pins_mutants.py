@@ -30,6 +30,9 @@ MUTANTS = {
     15: "SDQ step max deviation / 128 instead of / 127",
     16: "forward substitution dropping its last term",
     17: "fixed-point grid one bit coarser",
+    18: "record fields packed seed before tile",
+    19: "packed GEMV subtracting the sidecar correction",
+    20: "sign word bits read most-significant first",
 }
 
 
