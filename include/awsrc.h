@@ -135,7 +135,9 @@ typedef struct awsrc_params {
  *
  * One linear module (a weight matrix W with backbone reconstruction W0 = Q(W),
  * Eq. 1) and its per-input-channel statistics (Sec. 3.2).
- *   rows, cols  output and input dimensions; cols % C == 0.
+ *   rows, cols  output and input dimensions; cols % C == 0. The tiles of all
+ *               modules of one call, sum rows*cols/C, must number below 2^32
+ *               (tile indices are 32-bit), else AWSRC_ERR_UNSUPPORTED.
  *   W, W0       device, rows*cols elements of w_dtype / w0_dtype (F32 or BF16).
  *               The encoder reads both; the decoder reads W0 only (W may be NULL).
  *   act         device, cols floats: activation second moments a_j = E[x_j^2].
@@ -221,7 +223,8 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod,
  *   sdq_codes   device, G int8 c_g (SDQ), or NULL.
  *   sdq_consts  device, 2*ceil(G/256) floats (mu, step) per block (SDQ), or NULL.
  *   W0          device, rows*cols elements of w0_dtype (16-byte aligned), or NULL.
- * Errors: INVALID_ARG, SHAPE (cols % 128), CUDA.
+ * Errors: INVALID_ARG, SHAPE (cols % 128), UNSUPPORTED (rows*cols > 2^46),
+ * CUDA.
  */
 awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32_t w_dtype, int32_t sdq,
                                 uint8_t* codes, uint16_t* scales, int8_t* sdq_codes, float* sdq_consts,
@@ -232,7 +235,8 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
  * backbone: 2 bytes per group of 128, or with SDQ 1 per group plus 8 per block
  * of 256 groups. Under a fixed total budget the bytes SDQ saves can go to the
  * residual records (Sec. 3.3): raise the rate given to awsrc_select_records by
- * 8 * saved / N_scope bits/weight. Returns -1 for a bad shape.
+ * 8 * saved / N_scope bits/weight. Returns -1 for a bad shape or rows*cols
+ * above 2^46.
  */
 int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq);
 

@@ -17,6 +17,9 @@ thread_local char g_err[512] = "";
 thread_local cudaEvent_t g_ev_before = nullptr, g_ev_after = nullptr;
 std::atomic<uint64_t> g_launches{0};
 constexpr int64_t kTargetBlocks = 1216;  // enough blocks to fill a GB300 (152 SMs) several times
+// one RTN launch has a block per 256 groups of 128 weights: 2^46 weights keep
+// its grid far inside gridDim.x and every size product inside int64
+constexpr int64_t kMaxBackboneWeights = 1ll << 46;
 
 int ceil_log2_host(uint64_t x) {
   int n = 0;
@@ -56,9 +59,11 @@ awsrc_status check_modules(const Prm& pr, int32_t n_mod, const awsrc_module* mod
           !aligned(md.act, 4) || !aligned(md.fisher, 4))
         return AWSRC_ERR_INVALID_ARG;
     }
-    T += md.rows * (md.cols / pr.C);
+    // tile indices are 32-bit: refuse before rows * n_cb can overflow
+    const int64_t n_cb = md.cols / pr.C;
+    if (md.rows > ((1ll << 32) - 1 - T) / n_cb) return AWSRC_ERR_UNSUPPORTED;
+    T += md.rows * n_cb;
   }
-  if (T >= (1ll << 32)) return AWSRC_ERR_UNSUPPORTED;
   *T_out = T;
   return AWSRC_OK;
 }
@@ -229,6 +234,7 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
                                 uint8_t* codes, uint16_t* scales, int8_t* sdq_codes, float* sdq_consts,
                                 void* W0, int32_t w0_dtype, void* stream) {
   if (rows < 1 || cols < 1 || cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
+  if (rows > kMaxBackboneWeights / cols) return AWSRC_ERR_UNSUPPORTED;
   if (w_dtype != AWSRC_DTYPE_F32 && w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
   if (w0_dtype != AWSRC_DTYPE_F32 && w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
   if (sdq != 0 && sdq != 1) return AWSRC_ERR_INVALID_ARG;
@@ -241,7 +247,7 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
 }
 
 int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq) {
-  if (rows < 1 || cols < 1 || cols % rtn_group() != 0) return -1;
+  if (rows < 1 || cols < 1 || cols % rtn_group() != 0 || rows > kMaxBackboneWeights / cols) return -1;
   const int64_t G = rows * cols / rtn_group();
   return sdq ? G + 8 * ((G + sdq_block() - 1) / sdq_block()) : 2 * G;
 }

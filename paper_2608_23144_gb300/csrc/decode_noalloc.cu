@@ -100,9 +100,10 @@ extern "C" awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* p
     dm[m].w0_dtype = md.w0_dtype;
     dm[m].pad_ = 0;
     if (m > 0 && md.w0_dtype != mods[0].w0_dtype) return AWSRC_ERR_INVALID_ARG;
-    T += md.rows * (md.cols / pr.C);
+    const int64_t n_cb = md.cols / pr.C;
+    if (md.rows > ((1ll << 32) - 1 - T) / n_cb) return AWSRC_ERR_UNSUPPORTED;  // 32-bit tile indices
+    T += md.rows * n_cb;
   }
-  if (T >= (1ll << 32)) return AWSRC_ERR_UNSUPPORTED;
   const int64_t L = awsrc_record_bytes(prm, T), h = awsrc_header_bytes(n_mod);
   if (stream_len < (size_t)h) return AWSRC_ERR_INVALID_ARG;
   const int64_t kmax = std::min<int64_t>(((int64_t)stream_len - h) / L, T);

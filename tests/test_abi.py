@@ -173,3 +173,33 @@ def test_serving_and_diagnostic_arguments_are_refused_on_the_host(libpath):
     assert lib.awsrc_verify_reciprocal(0, 1, None, None) == 1
     assert lib.awsrc_verify_reciprocal(0, 1, 0x50004, None) == 1
     assert lib.awsrc_verify_reciprocal(2, 1, 0x50000, None) == 1
+
+
+def test_size_limits_are_refused_before_any_product_overflows(libpath):
+    """Tile indices are 32-bit and one RTN launch covers at most 2^46 weights:
+    shapes past either limit return UNSUPPORTED (or -1) on the host, including
+    shapes whose rows * cols would overflow int64."""
+    import paper_2608_23144_gb300 as aw
+    from paper_2608_23144_gb300._binding import shape_modules
+    lib = aw.lib
+    p = aw.params(C=64, S=64)
+    n = ct.c_size_t()
+    ws = lambda shapes: lib.awsrc_encode_workspace_bytes(ct.byref(p), len(shapes), shape_modules(shapes),
+                                                         ct.byref(n))
+    assert ws([((1 << 32) - 1, 64)]) == 0                  # 2^32 - 1 tiles: the largest call
+    assert ws([(1 << 32, 64)]) == 3                        # 2^32 tiles
+    assert ws([((1 << 31), 64), ((1 << 31), 64)]) == 3     # the limit is over the whole call
+    assert ws([(1 << 40, 1 << 40)]) == 3                   # rows * cols / C overflows int64
+    assert lib.awsrc_backbone_metadata_bytes(1 << 18, 1 << 28, 0) == 2 * (1 << 39)
+    assert lib.awsrc_backbone_metadata_bytes(1 << 19, 1 << 28, 0) == -1
+    assert lib.awsrc_backbone_metadata_bytes(1 << 40, 1 << 40, 1) == -1
+    bf16 = aw.DTYPE_BF16
+    assert lib.awsrc_rtn_quantize(1 << 40, 1 << 40, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40000,
+                                  bf16, None) == 3
+    # the decoder that allocates nothing applies the same 32-bit tile limit
+    outs = (ct.c_void_p * 2)(0x20000, 0x30000)
+    nd = lambda shapes: lib.awsrc_decode_apply_inplace_noalloc(ct.byref(p), len(shapes), shape_modules(shapes),
+                                                               0x10000, 1 << 20, 0, outs, None)
+    assert nd([(1 << 32, 64)]) == 3
+    assert nd([(1 << 31, 64), (1 << 31, 64)]) == 3
+    assert nd([(1 << 40, 1 << 40)]) == 3
