@@ -157,13 +157,50 @@ def _dev_ptr(t: Optional[torch.Tensor]) -> Optional[int]:
     return t.data_ptr()
 
 
+def _require(t, name: str, dtype=None, shape=None, numel: Optional[int] = None, device=None):
+    """Check a tensor argument on the host before its pointer crosses the ABI.
+    The kernels index every array by the module shapes they are given, so a
+    tensor that is smaller, of another element type or on another device than
+    those shapes imply would be read or written out of bounds on the device."""
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor, not {type(t).__name__}")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, not {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, at least {numel} are needed")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+def _shape(m: Dict[str, object], i: int):
+    """(rows, cols) of module i, from its W0."""
+    W0 = m["W0"]
+    _require(W0, f"modules[{i}]['W0']")
+    if W0.dim() != 2:
+        raise ValueError(f"modules[{i}]['W0'] must be 2-D (rows x cols), not {W0.dim()}-D")
+    return int(W0.shape[0]), int(W0.shape[1])
+
+
 def module_array(modules: Sequence[Dict[str, object]], decoder: bool = False):
-    """awsrc_module[] from dicts with W, W0, act (and fisher, w_act, w_fisher)."""
+    """awsrc_module[] from dicts with W, W0, act (and fisher, w_act, w_fisher).
+    W must have W0's shape, act is float32 with cols entries and fisher float32
+    rows x cols, all on W0's device."""
     arr = (Module * len(modules))()
     for i, m in enumerate(modules):
         W0 = m["W0"]
         W = m.get("W")
-        rows, cols = W0.shape
+        rows, cols = _shape(m, i)
+        dev = W0.device
+        if not decoder:
+            if W is not None:
+                _require(W, f"modules[{i}]['W']", shape=(rows, cols), device=dev)
+            if m.get("act") is not None:
+                _require(m["act"], f"modules[{i}]['act']", dtype=torch.float32, numel=cols, device=dev)
+            if m.get("fisher") is not None:
+                _require(m["fisher"], f"modules[{i}]['fisher']", dtype=torch.float32, shape=(rows, cols),
+                         device=dev)
         arr[i].rows, arr[i].cols = rows, cols
         arr[i].w0_dtype = _dtype_code(W0)
         arr[i].W0 = _dev_ptr(W0)
@@ -180,7 +217,7 @@ def module_array(modules: Sequence[Dict[str, object]], decoder: bool = False):
 
 
 def _tiles(prm: Params, modules) -> int:
-    return sum(int(m["W0"].shape[0]) * int(m["W0"].shape[1]) // prm.C for m in modules)
+    return sum(r * c // prm.C for r, c in (_shape(m, i) for i, m in enumerate(modules)))
 
 
 def awsrc_record_bytes(prm: Params, T: int) -> int:
@@ -201,11 +238,12 @@ def awsrc_encode_workspace_bytes(prm: Params, modules) -> int:
 def awsrc_encode_tiles(prm: Params, modules, out: Optional[torch.Tensor] = None,
                        workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
     """Seed search (Sec. 3.2): one best candidate per tile, uint8 [T, 16] on the device."""
-    mods = module_array(modules)
     T = _tiles(prm, modules)
     dev = modules[0]["W0"].device
     if out is None:
         out = torch.empty((T, 16), dtype=torch.uint8, device=dev)
+    _require(out, "out", dtype=torch.uint8, numel=16 * T, device=dev)
+    mods = module_array(modules)
     need = awsrc_encode_workspace_bytes(prm, modules)
     if workspace is None or workspace.numel() < need:
         workspace = torch.empty(need, dtype=torch.uint8, device=dev)
@@ -222,9 +260,20 @@ def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream
     sdq_codes (int8) and sdq_consts (float32 mean, step per 256 groups) when
     sdq, and W0 (in w0_dtype, default W's dtype). `out` reuses the buffers of
     an earlier call on the same shape."""
+    _require(W, "W")
+    if W.dim() != 2:
+        raise ValueError(f"W must be 2-D (rows x cols), not {W.dim()}-D")
     rows, cols = W.shape
     dev = W.device
     G = rows * cols // 128
+    if out is not None:  # buffers of an earlier call: the same shape and SDQ setting
+        _require(out["codes"], "out['codes']", dtype=torch.uint8, numel=rows * cols // 2, device=dev)
+        _require(out["scales"], "out['scales']", dtype=torch.int16, numel=G, device=dev)
+        _require(out["W0"], "out['W0']", shape=(rows, cols), device=dev)
+        if sdq:
+            _require(out["sdq_codes"], "out['sdq_codes']", dtype=torch.int8, numel=G, device=dev)
+            _require(out["sdq_consts"], "out['sdq_consts']", dtype=torch.float32, numel=2 * ((G + 255) // 256),
+                     device=dev)
     if out is None:
         out = {"codes": torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev),
                "scales": torch.empty(G, dtype=torch.int16, device=dev)}
@@ -273,10 +322,25 @@ def awsrc_packed_gemv(prm: Params, shapes, m: int, backbone: Dict[str, torch.Ten
     awsrc_rtn_quantize's codes and scales (or SDQ codes and constants)."""
     mods = shape_modules(shapes)
     rows, cols = shapes[m]
+    _require(x, "x", dtype=torch.float32)
+    if x.numel() % cols != 0:
+        raise ValueError(f"x holds {x.numel()} elements, not a whole number of rows of {cols}")
     x = x.reshape(-1, cols)
+    dev = x.device
     if y is None:
-        y = torch.empty(x.shape[0], rows, dtype=torch.float32, device=x.device)
+        y = torch.empty(x.shape[0], rows, dtype=torch.float32, device=dev)
+    _require(y, "y", dtype=torch.float32, shape=(x.shape[0], rows), device=dev)
     sdq = "sdq_codes" in backbone
+    G = rows * cols // 128
+    _require(backbone["codes"], "backbone['codes']", dtype=torch.uint8, numel=rows * cols // 2, device=dev)
+    if sdq:
+        _require(backbone["sdq_codes"], "backbone['sdq_codes']", dtype=torch.int8, numel=G, device=dev)
+        _require(backbone["sdq_consts"], "backbone['sdq_consts']", dtype=torch.float32,
+                 numel=2 * ((G + 255) // 256), device=dev)
+    else:
+        _require(backbone["scales"], "backbone['scales']", dtype=torch.int16, numel=G, device=dev)
+    if sidecar is not None:
+        _require(sidecar, "sidecar", dtype=torch.uint8, device=dev)
     pw = PackedWeights(_dev_ptr(backbone["codes"]), None if sdq else _dev_ptr(backbone["scales"]),
                        _dev_ptr(backbone.get("sdq_codes")), _dev_ptr(backbone.get("sdq_consts")), int(sdq), 0)
     _check(lib.awsrc_packed_gemv(ct.byref(prm), len(shapes), mods, m, ct.byref(pw), _dev_ptr(sidecar),
@@ -307,8 +371,13 @@ def awsrc_select_records(prm: Params, modules, cands: torch.Tensor, rates: Seque
     """Sec. 3.3 allocation + Eq. 5 serialisation. Returns (stream bytes [capacity] uint8,
     counts int64 (U: per module, PF: per rate), bytes int64 (per rate)), all on the device.
     Only the first bytes[r] bytes of the stream are written."""
-    mods = module_array(modules, decoder=True)
+    _require(cands, "cands", dtype=torch.uint8, numel=16 * _tiles(prm, modules))
     dev = cands.device
+    # caller buffers: the stream is bytes, counts and bytes are written as int64
+    for name, t, dt in (("out", out, torch.uint8), ("counts", counts, torch.int64), ("nbytes", nbytes, torch.int64)):
+        if t is not None:
+            _require(t, name, dtype=dt, device=dev)
+    mods = module_array(modules, decoder=True)
     r = (ct.c_double * len(rates))(*rates)
     cap = awsrc_stream_capacity(prm, modules, rates)
     n = ct.c_size_t()
@@ -329,18 +398,30 @@ def awsrc_select_records(prm: Params, modules, cands: torch.Tensor, rates: Seque
     return out, counts, nbytes
 
 
+def _check_outs(modules, outs, dtype):
+    """One output per module, of the module's shape, in `dtype`, on its device:
+    the decoder writes rows*cols elements through each pointer."""
+    if len(outs) != len(modules):
+        raise ValueError(f"{len(outs)} outputs for {len(modules)} modules")
+    for i, (m, o) in enumerate(zip(modules, outs)):
+        _require(o, f"outs[{i}]", dtype=dtype, shape=tuple(m["W0"].shape), device=m["W0"].device)
+
+
 def awsrc_decode_apply(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
                        outs: Optional[List[torch.Tensor]] = None, out_dtype=None,
                        mode: int = DECODE_DENSE, workspace: Optional[torch.Tensor] = None,
                        stream=None) -> List[torch.Tensor]:
     """Decoder (Sec. 3.2): W_hat = W0 + B_s alpha_hat for the first K records (K < 0: all)."""
-    mods = module_array(modules, decoder=True)
     dev = stream_bytes.device
     if out_dtype is None:
-        out_dtype = modules[0]["W0"].dtype
+        out_dtype = outs[0].dtype if outs else modules[0]["W0"].dtype
+    if out_dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError(f"out_dtype must be torch.float32 or torch.bfloat16, not {out_dtype}")
     code = DTYPE_F32 if out_dtype == torch.float32 else DTYPE_BF16
     if outs is None:
         outs = [torch.empty_like(m["W0"], dtype=out_dtype) for m in modules]
+    _check_outs(modules, outs, out_dtype)
+    mods = module_array(modules, decoder=True)
     ptrs = (ct.c_void_p * len(outs))(*[_dev_ptr(o) for o in outs])
     n = ct.c_size_t()
     _check(lib.awsrc_decode_workspace_bytes(ct.byref(prm), len(modules), mods, mode, ct.byref(n)), "decode_workspace_bytes")
@@ -358,6 +439,7 @@ def awsrc_decode_apply_inplace_noalloc(prm: Params, modules, stream_bytes: torch
                                        outs: List[torch.Tensor], stream=None) -> List[torch.Tensor]:
     """In-place decode that allocates nothing on either side of the ABI: `outs`
     must already hold W0; their tiles named by the first K records get W0 + r_hat."""
+    _check_outs(modules, outs, modules[0]["W0"].dtype)
     mods = module_array(modules, decoder=True)
     ptrs = (ct.c_void_p * len(outs))(*[_dev_ptr(o) for o in outs])
     _check(lib.awsrc_decode_apply_inplace_noalloc(ct.byref(prm), len(modules), mods, _dev_ptr(stream_bytes),
