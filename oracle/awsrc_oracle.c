@@ -395,10 +395,18 @@ static void orc_tile_inputs(const orc_params* prm, int64_t cols, const float* W,
   const int C = prm->C;
   for (int j = 0; j < C; ++j) {
     int64_t idx = row * cols + cb * C + j;
+#if ORC_MUTANT == 22
+    r[j] = W0[idx] - W[idx];
+#else
     r[j] = W[idx] - W0[idx];
+#endif
     float a = act[cb * C + j];
     if (prm->variant == 0) d[j] = a;
+#if ORC_MUTANT == 21
+    else d[j] = w_act * a + w_fisher * fisher[row * cols + j];
+#else
     else d[j] = w_act * a + w_fisher * fisher[idx];
+#endif
   }
 }
 

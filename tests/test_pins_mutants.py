@@ -33,6 +33,8 @@ MUTANTS = {
     18: "record fields packed seed before tile",
     19: "packed GEMV subtracting the sidecar correction",
     20: "sign word bits read most-significant first",
+    21: "P_F Fisher term read without the column block offset",
+    22: "residual taken as W0 - W",
 }
 
 
