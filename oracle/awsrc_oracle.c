@@ -350,13 +350,21 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     for (int p = 0; p < P; ++p) {
       float q = rintf(alpha[p] * inv);
       if (q > (float)qmax) q = (float)qmax;
+#if ORC_MUTANT == 23
+      if (q < (float)(-qmax - 1)) q = (float)(-qmax - 1);
+#else
       if (q < (float)-qmax) q = (float)-qmax;
+#endif
       codes[p] = (int)q;
     }
     sc = ldexpf(1.0f, e);
     scale_field = (int16_t)e;
   } else {
+#if ORC_MUTANT == 25
+    uint16_t h = orc_f32_to_f16(amax / (float)(qmax + 1));
+#else
     uint16_t h = orc_f32_to_f16(amax / (float)qmax);
+#endif
     sc = orc_f16_to_f32(h);
     if (!(sc > 0.0f && sc <= FLT_MAX)) return 0;
     for (int p = 0; p < P; ++p) {
@@ -646,7 +654,11 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
       int64_t kend = kbeg;
       while (kend < npos && keys[kend].tile < off + mod_tiles[m]) ++kend;
       qsort(keys + kbeg, (size_t)(kend - kbeg), sizeof(orc_key), orc_key_cmp);
+#if ORC_MUTANT == 24
+      unsigned __int128 q = (unsigned __int128)(uint64_t)B * (uint64_t)mod_weights[m];
+#else
       unsigned __int128 q = (unsigned __int128)(uint64_t)(B - h) * (uint64_t)mod_weights[m];
+#endif
       int64_t quota = (int64_t)(q / (uint64_t)Nscope);
       int64_t K = quota / L;
       if (K > kend - kbeg) K = kend - kbeg;
@@ -807,7 +819,11 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
       const int64_t n = G - b0 < block ? G - b0 : block;
       double sum = 0.0;
       for (int64_t g = b0; g < b0 + n; ++g) sum += (double)s_eff[g];
+#if ORC_MUTANT == 26
+      const float mu = (float)(sum / (double)block);
+#else
       const float mu = (float)(sum / (double)n);
+#endif
       float a = 0.0f;
       for (int64_t g = b0; g < b0 + n; ++g) {
         const float d = fabsf(s_eff[g] - mu);

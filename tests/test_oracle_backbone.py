@@ -82,6 +82,25 @@ def test_sdq_error_bound_and_constant_block(orc):
     assert np.array_equal(dq["q"], plain["q"])
 
 
+def test_sdq_short_last_block(orc):
+    """A last block with fewer than 256 groups: its constant is the mean of its
+    own n scales (numpy's mean, rounded once), and a short block of equal
+    scales is reproduced exactly (their mean is that scale, the step is 0)."""
+    rng = np.random.default_rng(6)
+    W = _weights(rng, 64, 2176)                       # 17 groups a row: G = 1088 = 4 * 256 + 64
+    plain, dq = orc.rtn_quantize(W), orc.rtn_quantize(W, sdq=True, block=256)
+    s = plain["s_eff"].astype(np.float64)
+    mu = dq["consts"][0::2].astype(np.float64)
+    assert len(s) == 1088 and len(mu) == 5
+    m = s[1024:].mean()
+    assert abs(mu[4] - m) <= np.spacing(np.float32(m))
+    # 3 groups a row, blocks of 16 over 8 rows: G = 24 = 16 + 8, every scale equal
+    Wc = np.tile(np.concatenate([np.full(127, 0.01, np.float32), [0.07]]), (8, 3)).astype(np.float32)
+    r = orc.rtn_quantize(Wc, sdq=True, block=16)
+    assert len(r["consts"]) == 4 and not r["c8"].any() and r["consts"][3] == 0.0
+    assert np.array_equal(r["s_eff"], orc.rtn_quantize(Wc)["s_eff"])
+
+
 def test_backbone_metadata_bytes():
     """FP16 group scales cost 16 bits per 128 weights (0.125 bpw, Sec. 3.3);
     SDQ with 8-bit codes and a binary32 (mean, step) pair per 256 groups costs

@@ -91,6 +91,30 @@ def test_exponent_and_codes_pow2(orc):
             assert np.array_equal(out["codes"], expect.astype(np.int64))
 
 
+def test_exponent_field_clips_and_codes_stay_symmetric(orc):
+    """A 2-bit exponent field holds e in [-2, 1]: an exponent outside it is
+    clamped to the field and the codes to [-qmax, qmax], so a coefficient
+    beyond the range gets +-qmax with its own sign, never -qmax - 1."""
+    rng = np.random.default_rng(9)
+    qmax = 7
+    prm = orc.params(C=32, P=3, b=4, b_e=2, ridge_rel=1e-4)
+    clipped_neg = clipped_low = 0
+    for s in range(60):
+        r, d = _tile(rng, 32, scale_r=10 ** rng.uniform(-4, 2))
+        neg = orc.gen_basis(0, s, 32, 3, 1)[3]
+        out = orc.score_candidate(prm, r, d, neg)
+        a = out["alpha"].astype(np.float64)
+        smallest = next(k for k in range(-200, 200) if np.abs(a).max() <= qmax * 2.0 ** k)
+        e = min(max(smallest, -2), 1)
+        assert out["scale"] == e
+        x = a * 2.0 ** -e
+        assert np.array_equal(out["codes"], np.clip(np.rint(x), -qmax, qmax).astype(np.int64))
+        assert np.abs(out["codes"]).max() <= qmax
+        clipped_neg += int((x < -qmax - 0.5).sum())
+        clipped_low += int(smallest < -2)
+    assert clipped_neg > 0 and clipped_low > 0     # both ends of the field were exercised
+
+
 def test_codes_fp16_scale(orc):
     rng = np.random.default_rng(5)
     prm = orc.params(C=64, P=4, b=4, scale_mode=1, b_e=16, ridge_rel=1e-4)

@@ -35,6 +35,10 @@ MUTANTS = {
     20: "sign word bits read most-significant first",
     21: "P_F Fisher term read without the column block offset",
     22: "residual taken as W0 - W",
+    23: "codes clamped to [-qmax - 1, qmax] when the exponent field clips",
+    24: "U quotas shared out of B instead of B - h",
+    25: "binary16 scale max|alpha| / (qmax + 1)",
+    26: "SDQ mean of a short last block divided by the full block size",
 }
 
 
