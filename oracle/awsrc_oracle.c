@@ -219,7 +219,11 @@ int orc_fixed_point(int C, const float* x, int32_t* X) {
 #else
   int q = ilogbf(m) - 20;
 #endif
+#if ORC_MUTANT == 27
+  for (int j = 0; j < C; ++j) X[j] = (int32_t)ldexpf(x[j], -q);
+#else
   for (int j = 0; j < C; ++j) X[j] = (int32_t)rintf(ldexpf(x[j], -q));
+#endif
   return q;
 }
 
@@ -380,7 +384,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
   for (int p = 0; p < P; ++p) Aq = fmaf((float)codes[p], bvec[p], Aq);
   float Qq = 0.0f;
   for (int p = 0; p < P; ++p) {
+#if ORC_MUTANT == 29
+    Qq = fmaf((float)(codes[p] * codes[p]), A[p][p], Qq);
+#else
     Qq = fmaf((float)(codes[p] * codes[p]), G[p][p], Qq);
+#endif
     for (int q = p + 1; q < P; ++q) Qq = fmaf((float)(2 * codes[p] * codes[q]), G[p][q], Qq);
   }
   float t = sc * Qq;
@@ -583,7 +591,11 @@ void orc_pack_record(const orc_params* prm, int64_t T, int64_t tile, const orc_c
   orc_put_bits(rec, &pos, cd->seed, orc_ceil_log2((uint64_t)prm->S));
 #endif
   uint64_t sf;
+#if ORC_MUTANT == 31
+  if (prm->scale_mode == 0) sf = (uint64_t)(int64_t)(cd->scale + prm->e_bias);
+#else
   if (prm->scale_mode == 0) sf = (uint64_t)(int64_t)(cd->scale - prm->e_bias);
+#endif
   else sf = (uint16_t)cd->scale;
   orc_put_bits(rec, &pos, sf & ((prm->b_e >= 64) ? ~0ULL : ((1ULL << prm->b_e) - 1)), prm->b_e);
   for (int p = 0; p < prm->P; ++p)
@@ -676,6 +688,8 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
       if (B < h) { rc = 4; goto done; }
 #if ORC_MUTANT == 9
       int64_t K = (B - h) / L + 1;
+#elif ORC_MUTANT == 28
+      int64_t K = B / L;
 #else
       int64_t K = (B - h) / L;
 #endif
@@ -736,7 +750,11 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
   int64_t T = 0;
   for (int m = 0; m < n_mod; ++m) T += mod_rows[m] * mod_cols[m] / C;
   const int64_t h = orc_header_bytes(n_mod), L = orc_record_bytes(prm, T);
+#if ORC_MUTANT == 30
+  const float c = (float)(1.0 / (double)C);
+#else
   const float c = (float)(1.0 / sqrt((double)C));
+#endif
   uint8_t sign[256], neg[8 * 256];
   int32_t perm[256], cols[8];
   int bad = 0;

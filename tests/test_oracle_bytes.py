@@ -58,6 +58,12 @@ def test_record_bytes_by_hand(orc):
     tile, back = orc.unpack_record(prm, 2048, rec)
     assert tile == 5 and back["seed"] == 3 and back["scale"] == -13
     assert list(back["code"][:4]) == [-1, -6, -5, 6]
+    # the same record with e_bias = -20: the field holds e - e_bias = 7 (11100000)
+    prm = orc.params(C=64, P=4, b=4, S=256, b_e=8, e_bias=-20)
+    rec = orc.pack_record(prm, 2048, 5, cand)
+    assert rec == bytes([0x05, 0x18, 0x38, 0x78, 0x5D, 0x03])
+    tile, back = orc.unpack_record(prm, 2048, rec)
+    assert tile == 5 and back["scale"] == -13
 
 
 def test_record_round_trip_extremes(orc):

@@ -2,6 +2,7 @@
 -DORC_MUTANT=k carries one plausible mistake (below), and the pin files
 (tests/test_oracle_*.py) run against that build in a subprocess must fail.
 A mistake that no pin catches means the oracle is not pinned there."""
+import concurrent.futures as cf
 import glob
 import os
 import subprocess
@@ -39,13 +40,30 @@ MUTANTS = {
     24: "U quotas shared out of B instead of B - h",
     25: "binary16 scale max|alpha| / (qmax + 1)",
     26: "SDQ mean of a short last block divided by the full block size",
+    27: "fixed-point grid values truncated instead of rounded",
+    28: "P_F prefixes taken out of B instead of B - h",
+    29: "Eq. 4 gain with the ridge in G",
+    30: "decoder normalising by 1/C instead of C^-1/2",
+    31: "scale field holding e + e_bias",
 }
 
 
+def _run_pins(k):
+    env = dict(os.environ, AWSRC_ORACLE_MUTANT=str(k), OMP_NUM_THREADS="1")
+    return subprocess.run([sys.executable, "-m", "pytest", *PIN_FILES, "-x", "-q", "-m", "not gpu",
+                           "-p", "no:cacheprovider"], env=env, cwd=ROOT, capture_output=True, text=True,
+                          timeout=900)
+
+
+@pytest.fixture(scope="module")
+def outcomes():
+    """Every mutant's pin run, the runs side by side (one OpenMP thread each)."""
+    ks = sorted(MUTANTS)
+    with cf.ThreadPoolExecutor(max(1, min(len(ks), os.cpu_count() or 1))) as ex:
+        return dict(zip(ks, ex.map(_run_pins, ks)))
+
+
 @pytest.mark.parametrize("k", sorted(MUTANTS))
-def test_pins_catch_planted_mistake(k):
-    env = dict(os.environ, AWSRC_ORACLE_MUTANT=str(k))
-    r = subprocess.run([sys.executable, "-m", "pytest", *PIN_FILES, "-x", "-q", "-m", "not gpu",
-                        "-p", "no:cacheprovider"], env=env, cwd=ROOT, capture_output=True, text=True,
-                       timeout=900)
+def test_pins_catch_planted_mistake(outcomes, k):
+    r = outcomes[k]
     assert r.returncode == 1, f"mistake {k} ({MUTANTS[k]}) not caught by any pin:\n{r.stdout[-3000:]}"
