@@ -558,7 +558,11 @@ int64_t orc_record_bytes(const orc_params* prm, int64_t T) {
 }
 
 int64_t orc_budget_bytes(double rate_bpw, int64_t n_scope) {
+#if ORC_MUTANT == 33
+  return (int64_t)ceil(rate_bpw * (double)n_scope / 8.0);
+#else
   return (int64_t)floor(rate_bpw * (double)n_scope / 8.0);
+#endif
 }
 
 static void orc_put_bits(uint8_t* rec, int* pos, uint64_t value, int nbits) {
@@ -766,7 +770,11 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
     int64_t m = 0, off = 0;
     while (tile >= off + mod_rows[m] * mod_cols[m] / C) { off += mod_rows[m] * mod_cols[m] / C; ++m; }
     int64_t lt = tile - off, n_cb = mod_cols[m] / C;
+#if ORC_MUTANT == 32
+    int64_t base = (lt / n_cb) * mod_cols[m] + ((lt + 1) % n_cb) * C;
+#else
     int64_t base = (lt / n_cb) * mod_cols[m] + (lt % n_cb) * C;
+#endif
     orc_gen_basis(prm->gen_seed, cd.seed, C, P, prm->permute, sign, perm, cols, neg);
     float sc = prm->scale_mode == 0 ? ldexpf(1.0f, cd.scale) : orc_f16_to_f32((uint16_t)cd.scale);
     for (int j = 0; j < C; ++j) {
@@ -844,7 +852,11 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
 #endif
       float a = 0.0f;
       for (int64_t g = b0; g < b0 + n; ++g) {
+#if ORC_MUTANT == 34
+        const float d = s_eff[g] - mu;
+#else
         const float d = fabsf(s_eff[g] - mu);
+#endif
         if (d > a) a = d;
       }
 #if ORC_MUTANT == 15

@@ -82,6 +82,20 @@ def test_sdq_error_bound_and_constant_block(orc):
     assert np.array_equal(dq["q"], plain["q"])
 
 
+def test_sdq_extreme_deviation_below_the_mean(orc):
+    """One block where the scale farthest from the mean lies below it (a group
+    of tiny weights among ordinary ones): its step still covers that deviation,
+    so every reconstructed scale is within half a step of its own."""
+    rng = np.random.default_rng(7)
+    W = rng.normal(0, 0.02, (16, 2048)).astype(np.float32)    # 256 groups, one block
+    W[5, 640:768] *= 1e-3
+    plain, dq = orc.rtn_quantize(W), orc.rtn_quantize(W, sdq=True, block=256)
+    s, st = plain["s_eff"].astype(np.float64), dq["s_eff"].astype(np.float64)
+    mu, step = float(dq["consts"][0]), float(dq["consts"][1])
+    assert np.argmax(np.abs(s - mu)) == 5 * 16 + 5 and s[5 * 16 + 5] < mu
+    assert (np.abs(st - s) <= 0.5 * step + 4 * np.spacing(np.float32(s.max()))).all()
+
+
 def test_sdq_short_last_block(orc):
     """A last block with fewer than 256 groups: its constant is the mean of its
     own n scales (numpy's mean, rounded once), and a short block of equal

@@ -112,6 +112,26 @@ def test_pf_progressive_prefixes_nest(orc):
     assert sum(m[1] for m in mods) == K
 
 
+def test_stream_never_exceeds_the_rate_budget(orc):
+    """Eq. 5: the whole stream, header included, fits rate * N / 8 bytes. At
+    211/512 bit/weight on 2048 weights the budget is 105.5 bytes: after the
+    56-byte header nine 5-byte records (101 bytes) fit and a tenth (106) does
+    not, for the progressive prefixes and for one module's quota alike."""
+    rng = np.random.default_rng(23)
+    shapes = [(16, 64), (32, 32)]
+    rate = 211 / 512
+    for variant in (1, 0):
+        prm = orc.params(C=16, P=4, b=4, S=8, variant=variant)
+        sh = shapes if variant == 1 else [(32, 64)]      # U: one module takes the whole budget
+        cands = _cands(orc, rng, prm, sh)
+        assert (cands["gain"] > 0).sum() >= 10
+        assert orc.record_bytes(prm, 128) == 5 and orc.header_bytes(len(sh)) == 40 + 8 * len(sh)
+        stream, counts, nbytes = orc.select_records(prm, sh, cands, [rate])
+        h = 40 + 8 * len(sh)
+        k = (105 - h) // 5                                # records that fit in 105.5 bytes
+        assert int(counts.sum()) == k and int(nbytes[0]) == h + 5 * k <= 105.5 < h + 5 * (k + 1)
+
+
 def test_budget_below_header_is_an_error(orc):
     prm = orc.params(C=16, P=2, b=4, S=4)
     cands = np.zeros(4, orc.CANDIDATE_DTYPE)

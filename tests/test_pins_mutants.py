@@ -45,6 +45,9 @@ MUTANTS = {
     29: "Eq. 4 gain with the ridge in G",
     30: "decoder normalising by 1/C instead of C^-1/2",
     31: "scale field holding e + e_bias",
+    32: "decoder adding a record to the next column block",
+    33: "byte budget rounded up",
+    34: "SDQ step from the largest deviation above the mean only",
 }
 
 
