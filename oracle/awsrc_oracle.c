@@ -98,7 +98,11 @@ static int orc_popcount(uint32_t v) {
 
 void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
                    uint8_t* sign, int32_t* perm, int32_t* cols, uint8_t* negmask) {
+#if ORC_MUTANT == 35
+  uint64_t key = orc_splitmix64_output(gen_seed, (uint64_t)s);
+#else
   uint64_t key = orc_splitmix64_output(gen_seed, (uint64_t)s + 1);
+#endif
   uint64_t n = 1;
   /* sign pattern: one 64-bit draw per 64 coordinates */
   for (int w = 0; w * 64 < C; ++w) {
@@ -127,11 +131,23 @@ void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
   for (int j = 0; j < C; ++j) pool[j] = j;
   for (int p = 0; p < P; ++p) {
     uint64_t x = orc_splitmix64_output(key, n++) >> 32;
+#if ORC_MUTANT == 37
+    cols[p] = (int)((x * (uint64_t)C) >> 32);
+    (void)pool;
+#else
     int k = p + (int)((x * (uint64_t)(C - p)) >> 32);
     int32_t t = pool[p]; pool[p] = pool[k]; pool[k] = t;
     cols[p] = pool[p];
+#endif
   }
   /* B_s[j][p] = C^-1/2 * sigma_j * H[pi(j), c_p],  H[i][k] = (-1)^popcount(i & k) */
+#if ORC_MUTANT == 36
+  {
+    int32_t inv[256];
+    for (int j = 0; j < C; ++j) inv[perm[j]] = j;
+    for (int j = 0; j < C; ++j) perm[j] = inv[j];
+  }
+#endif
   for (int p = 0; p < P; ++p)
     for (int j = 0; j < C; ++j)
 #if ORC_MUTANT == 13

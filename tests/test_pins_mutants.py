@@ -48,6 +48,9 @@ MUTANTS = {
     32: "decoder adding a record to the next column block",
     33: "byte budget rounded up",
     34: "SDQ step from the largest deviation above the mean only",
+    35: "seed key taken from stream output s instead of s + 1",
+    36: "coordinate permutation applied inverted",
+    37: "Hadamard columns drawn with replacement",
 }
 
 
