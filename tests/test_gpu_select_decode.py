@@ -174,3 +174,28 @@ def test_decode_dense_many_modules_small_tiles(aw, orc, C, P):
     for g, o in zip(outs, oouts):
         assert np.array_equal(g.float().cpu().numpy(), o)
     assert aw.awsrc_workspace_status(outs[0]._awsrc_workspace) == 0
+
+
+def test_clipping_exponent_field_with_bias(aw, orc):
+    """A 3-bit exponent field with e_bias = -10 holds e in [-14, -7]: tiles whose
+    coefficients need a larger exponent get -7 with their codes clamped to
+    [-qmax, qmax] (the tcgen05 search without pruning), and the stream stores
+    e - e_bias in 3 bits (2 e_bias is not a multiple of 8, so a bias applied
+    with the wrong sign would change the bytes). Candidates, stream bytes and
+    decoded weights match the oracle bit for bit."""
+    shapes = [(100, 256), (64, 128)]
+    mods, dmods, prm, oprm, cands, ocands = _setup(aw, orc, shapes, dict(C=64, P=4, b=4, S=64, b_e=3, e_bias=-10))
+    assert (ocands["scale"][ocands["gain"] > -np.inf] == -7).sum() > 0    # the top of the field is reached
+    stream, counts, nbytes = aw.awsrc_select_records(prm, dmods, cands, [1.0])
+    ostream, ocounts, obytes = orc.select_records(oprm, shapes, ocands, [1.0])
+    assert list(counts.cpu().numpy()) == list(ocounts)
+    assert list(nbytes.cpu().numpy()) == list(obytes)
+    assert bytes(stream.cpu().numpy()[: int(nbytes[0])]) == ostream
+    K = int(ocounts.sum())
+    W0s = [m["W0"].float().numpy() for m in mods]
+    outs = aw.awsrc_decode_apply(prm, dmods, stream, K)
+    torch.cuda.synchronize()
+    oouts, _ = orc.decode_apply(oprm, W0s, ostream, K, out_bf16=True)
+    for g, o in zip(outs, oouts):
+        assert np.array_equal(g.float().cpu().numpy(), o)
+    assert aw.awsrc_workspace_status(outs[0]._awsrc_workspace) == 0
