@@ -319,7 +319,8 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  *   stream_len  bytes readable at `stream`; records beyond it are never read.
  *   K        records to apply (0 <= K <= header's K). K < 0 applies all the
  *            header's records (read on the device; no synchronisation). Either
- *            way at most (stream_len - h) / L records are applied.
+ *            way at most (stream_len - h) / L records are applied; an explicit
+ *            K above that returns AWSRC_ERR_INVALID_ARG.
  *   W_hat    host array of n_mod device pointers, rows*cols elements of out_dtype.
  *   mode     DENSE: every element of W_hat is written (W0 copied, corrected where
  *            a record exists). INPLACE: only the tiles named by records are
