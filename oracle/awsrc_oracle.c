@@ -675,7 +675,11 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
   /* eligibility: non-positive (or non-finite) records are discarded (Sec. 3.3) */
   int64_t npos = 0;
   for (int64_t t = 0; t < T; ++t)
+#if ORC_MUTANT == 38
+    if (cands[t].gain >= 0.0f && cands[t].gain <= FLT_MAX) { keys[npos].gain = cands[t].gain; keys[npos].tile = t; ++npos; }
+#else
     if (cands[t].gain > 0.0f && cands[t].gain <= FLT_MAX) { keys[npos].gain = cands[t].gain; keys[npos].tile = t; ++npos; }
+#endif
   int64_t* order = (int64_t*)malloc(sizeof(int64_t) * (size_t)(T > 0 ? T : 1));
   if (prm->variant == 0) {
     /* U: within each module, the best records that fit its quota */
@@ -778,7 +782,11 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
   uint8_t sign[256], neg[8 * 256];
   int32_t perm[256], cols[8];
   int bad = 0;
+#if ORC_MUTANT == 39
+  for (int64_t k = 0; k < K - 1; ++k) {
+#else
   for (int64_t k = 0; k < K; ++k) {
+#endif
     int64_t tile;
     orc_candidate cd;
     orc_unpack_record(prm, T, stream + h + k * L, &tile, &cd);

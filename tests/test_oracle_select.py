@@ -132,6 +132,24 @@ def test_stream_never_exceeds_the_rate_budget(orc):
         assert int(counts.sum()) == k and int(nbytes[0]) == h + 5 * k <= 105.5 < h + 5 * (k + 1)
 
 
+def test_zero_gains_never_make_records(orc):
+    """Sec. 3.3: only a positive weighted error reduction earns a record, so
+    candidates with a gain of exactly +0 or -0 are dropped even when the
+    budget (16 bits/weight here) would hold every tile."""
+    rng = np.random.default_rng(24)
+    shapes = [(16, 64), (32, 32)]
+    for variant in (0, 1):
+        prm = orc.params(C=16, P=4, b=4, S=8, variant=variant)
+        cands = _cands(orc, rng, prm, shapes)
+        cands["gain"][::4] = 0.0
+        cands["gain"][1::9] = -0.0
+        npos = int((cands["gain"] > 0).sum())
+        stream, counts, nbytes = orc.select_records(prm, shapes, cands, [16.0])
+        K, mods, recs = _parse(orc, prm, stream, shapes)
+        assert K == npos == int(counts.sum())
+        assert all(cands[t]["gain"] > 0 for t, _ in recs)
+
+
 def test_budget_below_header_is_an_error(orc):
     prm = orc.params(C=16, P=2, b=4, S=4)
     cands = np.zeros(4, orc.CANDIDATE_DTYPE)

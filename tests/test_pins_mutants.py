@@ -51,6 +51,8 @@ MUTANTS = {
     35: "seed key taken from stream output s instead of s + 1",
     36: "coordinate permutation applied inverted",
     37: "Hadamard columns drawn with replacement",
+    38: "candidates with a zero gain kept",
+    39: "decoder dropping the last of its K records",
 }
 
 
