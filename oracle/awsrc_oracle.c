@@ -24,6 +24,12 @@
  * a relative ridge eps = ridge_rel * mean(d) (Sec. 3.2 gives no value), the
  * symmetric code range [-qmax, qmax], the smallest non-clipping power-of-two
  * exponent, the 40 + 8*n_mod byte header (Sec. 4 gives 904 B for 108 modules).
+ *
+ * Parity unpinned by the paper: the generator (orc_gen_basis). The paper
+ * prints no generator values, so it is pinned only to SplitMix64's published
+ * outputs, to an independent restatement of the draw schedule in the tests,
+ * and to the basis structure (bijective permutation, distinct columns, exact
+ * orthonormality).
  */
 #include <float.h>
 #include <math.h>
