@@ -204,8 +204,12 @@ float orc_f16_to_f32(uint16_t h) {
 uint16_t orc_f32_to_bf16(float f) {
   uint32_t x = orc_f2u(f);
   if ((x & 0x7fffffffu) > 0x7f800000u) return (uint16_t)((x >> 16) | 0x40u);
+#if ORC_MUTANT == 40
+  return (uint16_t)(x >> 16);
+#else
   uint32_t lsb = (x >> 16) & 1u;
   return (uint16_t)((x + 0x7fffu + lsb) >> 16);
+#endif
 }
 
 /* ------------------------------------------------------------------------ */
@@ -701,7 +705,11 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
 #else
       unsigned __int128 q = (unsigned __int128)(uint64_t)(B - h) * (uint64_t)mod_weights[m];
 #endif
+#if ORC_MUTANT == 41
+      int64_t quota = (int64_t)((q + (uint64_t)Nscope - 1) / (uint64_t)Nscope);
+#else
       int64_t quota = (int64_t)(q / (uint64_t)Nscope);
+#endif
       int64_t K = quota / L;
       if (K > kend - kbeg) K = kend - kbeg;
       for (int64_t k = 0; k < K; ++k) order[K_stream++] = keys[kbeg + k].tile;
@@ -862,7 +870,11 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
     for (int j = 0; j < group; ++j) {
       float v = 0.0f;
       if (s > 0.0f) {
+#if ORC_MUTANT == 42
+        v = rintf(w[j] * (1.0f / s));
+#else
         v = rintf(w[j] / s);
+#endif
         if (v < -8.0f) v = -8.0f;
         if (v > 7.0f) v = 7.0f;
       }

@@ -82,6 +82,21 @@ def test_sdq_error_bound_and_constant_block(orc):
     assert np.array_equal(dq["q"], plain["q"])
 
 
+def test_rtn_divides_by_the_scale(orc):
+    """The codes are rint(w / s_g) with the correctly rounded binary32 quotient
+    (numpy's division), ties to even. With s_g = 7 * 2^-10 (a group whose
+    largest weight is 7 s_g) the weights +-6.5 s_g are exact ties and give +-6,
+    where a product with the rounded reciprocal 1/s_g would give +-7."""
+    s = np.float32(0.0068359375)
+    w = np.zeros((1, 128), np.float32)
+    w[0, :4] = [7 * s, 0.04443359375, -0.04443359375, 0.02392577938735485]
+    out = orc.rtn_quantize(w)
+    assert out["s_eff"][0] == s
+    expect = np.rint(w[0, :4] / s)
+    assert list(expect) == [7, 6, -6, 3]
+    assert list(out["q"].reshape(-1)[:4]) == list(expect)
+
+
 def test_sdq_extreme_deviation_below_the_mean(orc):
     """One block where the scale farthest from the mean lies below it (a group
     of tiny weights among ordinary ones): its step still covers that deviation,

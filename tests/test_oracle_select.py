@@ -130,6 +130,12 @@ def test_stream_never_exceeds_the_rate_budget(orc):
         h = 40 + 8 * len(sh)
         k = (105 - h) // 5                                # records that fit in 105.5 bytes
         assert int(counts.sum()) == k and int(nbytes[0]) == h + 5 * k <= 105.5 < h + 5 * (k + 1)
+    # U over two equal modules at 105/256 bit/weight: B - h = 49 bytes, so each
+    # module's quota is 24 bytes (4 records) and the stream 96 of 105 bytes
+    prm = orc.params(C=16, P=4, b=4, S=8, variant=0)
+    cands = _cands(orc, rng, prm, shapes)
+    stream, counts, nbytes = orc.select_records(prm, shapes, cands, [105 / 256])
+    assert list(counts) == [4, 4] and int(nbytes[0]) == 96
 
 
 def test_zero_gains_never_make_records(orc):

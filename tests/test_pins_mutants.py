@@ -53,6 +53,9 @@ MUTANTS = {
     37: "Hadamard columns drawn with replacement",
     38: "candidates with a zero gain kept",
     39: "decoder dropping the last of its K records",
+    40: "BF16 output truncated instead of rounded to nearest even",
+    41: "U quotas rounded up",
+    42: "RTN codes from the product with the rounded reciprocal of the scale",
 }
 
 
