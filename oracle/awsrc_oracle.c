@@ -43,12 +43,6 @@
 #define ORC_MAXP 8
 #define ORC_GAMMA 0x9E3779B97F4A7C15ULL
 
-/* Planted mistakes for the mutation test of the pins: a build with
- * -DORC_MUTANT=k carries mistake k (listed in the test), and the pins must
- * catch every one. The default, 0, is the oracle itself. */
-#ifndef ORC_MUTANT
-#define ORC_MUTANT 0
-#endif
 
 /* Candidate record layout mirrors the ABI's 16-byte struct (an interface, not code). */
 typedef struct {
@@ -104,31 +98,19 @@ static int orc_popcount(uint32_t v) {
 
 void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
                    uint8_t* sign, int32_t* perm, int32_t* cols, uint8_t* negmask) {
-#if ORC_MUTANT == 35
-  uint64_t key = orc_splitmix64_output(gen_seed, (uint64_t)s);
-#else
   uint64_t key = orc_splitmix64_output(gen_seed, (uint64_t)s + 1);
-#endif
   uint64_t n = 1;
   /* sign pattern: one 64-bit draw per 64 coordinates */
   for (int w = 0; w * 64 < C; ++w) {
     uint64_t word = orc_splitmix64_output(key, n++);
-#if ORC_MUTANT == 20
-    for (int j = w * 64; j < C && j < w * 64 + 64; ++j) sign[j] = (uint8_t)((word >> (63 - (j - w * 64))) & 1u);
-#else
     for (int j = w * 64; j < C && j < w * 64 + 64; ++j) sign[j] = (uint8_t)((word >> (j - w * 64)) & 1u);
-#endif
   }
   /* coordinate permutation: Fisher-Yates (Durstenfeld), index by multiply-shift */
   for (int j = 0; j < C; ++j) perm[j] = j;
   if (permute) {
     for (int i = C - 1; i >= 1; --i) {
       uint64_t x = orc_splitmix64_output(key, n++) >> 32;
-#if ORC_MUTANT == 12
-      int k = (int)((x * (uint64_t)i) >> 32);
-#else
       int k = (int)((x * (uint64_t)(i + 1)) >> 32);
-#endif
       int32_t t = perm[i]; perm[i] = perm[k]; perm[k] = t;
     }
   }
@@ -137,30 +119,14 @@ void orc_gen_basis(uint64_t gen_seed, uint32_t s, int C, int P, int permute,
   for (int j = 0; j < C; ++j) pool[j] = j;
   for (int p = 0; p < P; ++p) {
     uint64_t x = orc_splitmix64_output(key, n++) >> 32;
-#if ORC_MUTANT == 37
-    cols[p] = (int)((x * (uint64_t)C) >> 32);
-    (void)pool;
-#else
     int k = p + (int)((x * (uint64_t)(C - p)) >> 32);
     int32_t t = pool[p]; pool[p] = pool[k]; pool[k] = t;
     cols[p] = pool[p];
-#endif
   }
   /* B_s[j][p] = C^-1/2 * sigma_j * H[pi(j), c_p],  H[i][k] = (-1)^popcount(i & k) */
-#if ORC_MUTANT == 36
-  {
-    int32_t inv[256];
-    for (int j = 0; j < C; ++j) inv[perm[j]] = j;
-    for (int j = 0; j < C; ++j) perm[j] = inv[j];
-  }
-#endif
   for (int p = 0; p < P; ++p)
     for (int j = 0; j < C; ++j)
-#if ORC_MUTANT == 13
-      negmask[p * C + j] = (uint8_t)((sign[j] + orc_popcount((uint32_t)(perm[j] | cols[p]))) & 1);
-#else
       negmask[p * C + j] = (uint8_t)((sign[j] + orc_popcount((uint32_t)(perm[j] & cols[p]))) & 1);
-#endif
 }
 
 /* ------------------------------------------------------------------------ */
@@ -204,12 +170,8 @@ float orc_f16_to_f32(uint16_t h) {
 uint16_t orc_f32_to_bf16(float f) {
   uint32_t x = orc_f2u(f);
   if ((x & 0x7fffffffu) > 0x7f800000u) return (uint16_t)((x >> 16) | 0x40u);
-#if ORC_MUTANT == 40
-  return (uint16_t)(x >> 16);
-#else
   uint32_t lsb = (x >> 16) & 1u;
   return (uint16_t)((x + 0x7fffu + lsb) >> 16);
-#endif
 }
 
 /* ------------------------------------------------------------------------ */
@@ -240,16 +202,8 @@ int orc_fixed_point(int C, const float* x, int32_t* X) {
     for (int j = 0; j < C; ++j) X[j] = 0;
     return 0;
   }
-#if ORC_MUTANT == 17
-  int q = ilogbf(m) - 19;
-#else
   int q = ilogbf(m) - 20;
-#endif
-#if ORC_MUTANT == 27
-  for (int j = 0; j < C; ++j) X[j] = (int32_t)ldexpf(x[j], -q);
-#else
   for (int j = 0; j < C; ++j) X[j] = (int32_t)rintf(ldexpf(x[j], -q));
-#endif
   return q;
 }
 
@@ -284,11 +238,7 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     int64_t su = 0;
     for (int j = 0; j < C; ++j) su += negmask[p * C + j] ? -(int64_t)Y[j] : (int64_t)Y[j];
     float u = ldexpf((float)su, qy);
-#if ORC_MUTANT == 3
-    bvec[p] = u;
-#else
     bvec[p] = c * u;
-#endif
   }
   /* Gram G = B_s^T D B_s */
   float G[ORC_MAXP][ORC_MAXP];
@@ -300,22 +250,12 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     for (int q = p + 1; q < P; ++q) {
       int64_t sv = 0;
       for (int j = 0; j < C; ++j)
-#if ORC_MUTANT == 1
-        sv += (negmask[p * C + j] ^ negmask[q * C + j]) ? (int64_t)Dq[j] : -(int64_t)Dq[j];
-#elif ORC_MUTANT == 2
-        sv += (negmask[p * C + j] ^ negmask[p * C + (j ^ 1)]) ? -(int64_t)Dq[j] : (int64_t)Dq[j];
-#else
         sv += (negmask[p * C + j] ^ negmask[q * C + j]) ? -(int64_t)Dq[j] : (int64_t)Dq[j];
-#endif
       G[p][q] = G[q][p] = c2 * ldexpf((float)sv, qd);
     }
   }
   /* ridge (Eq. 3): A = G + eps I */
-#if ORC_MUTANT == 5
-  float eps = prm->ridge_rel;
-#else
   float eps = prm->ridge_rel * gd;
-#endif
   float A[ORC_MAXP][ORC_MAXP];
   for (int p = 0; p < P; ++p)
     for (int q = 0; q < P; ++q) A[p][q] = G[p][q];
@@ -339,11 +279,7 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
   float z[ORC_MAXP], alpha[ORC_MAXP];
   for (int k = 0; k < P; ++k) {
     float v = bvec[k];
-#if ORC_MUTANT == 16
-    for (int i = 0; i < k - 1; ++i) v = fmaf(-L[k][i], z[i], v);
-#else
     for (int i = 0; i < k; ++i) v = fmaf(-L[k][i], z[i], v);
-#endif
     z[k] = v;
   }
   for (int k = P - 1; k >= 0; --k) {
@@ -369,32 +305,20 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
     int lo, hi;
     orc_exp_range(prm, &lo, &hi);
     int e0 = ilogbf(amax) - (prm->b - 2);   /* ilogb(qmax) = b - 2 */
-#if ORC_MUTANT == 4
-    int e = e0 + (amax > ldexpf((float)qmax, e0) ? 1 : 0) + 1;
-#else
     int e = e0 + (amax > ldexpf((float)qmax, e0) ? 1 : 0);
-#endif
     if (e < lo) e = lo;
     if (e > hi) e = hi;
     float inv = ldexpf(1.0f, -e);
     for (int p = 0; p < P; ++p) {
       float q = rintf(alpha[p] * inv);
       if (q > (float)qmax) q = (float)qmax;
-#if ORC_MUTANT == 23
-      if (q < (float)(-qmax - 1)) q = (float)(-qmax - 1);
-#else
       if (q < (float)-qmax) q = (float)-qmax;
-#endif
       codes[p] = (int)q;
     }
     sc = ldexpf(1.0f, e);
     scale_field = (int16_t)e;
   } else {
-#if ORC_MUTANT == 25
-    uint16_t h = orc_f32_to_f16(amax / (float)(qmax + 1));
-#else
     uint16_t h = orc_f32_to_f16(amax / (float)qmax);
-#endif
     sc = orc_f16_to_f32(h);
     if (!(sc > 0.0f && sc <= FLT_MAX)) return 0;
     for (int p = 0; p < P; ++p) {
@@ -410,19 +334,11 @@ int orc_score_candidate(const orc_params* prm, const float* r, const float* d,
   for (int p = 0; p < P; ++p) Aq = fmaf((float)codes[p], bvec[p], Aq);
   float Qq = 0.0f;
   for (int p = 0; p < P; ++p) {
-#if ORC_MUTANT == 29
-    Qq = fmaf((float)(codes[p] * codes[p]), A[p][p], Qq);
-#else
     Qq = fmaf((float)(codes[p] * codes[p]), G[p][p], Qq);
-#endif
     for (int q = p + 1; q < P; ++q) Qq = fmaf((float)(2 * codes[p] * codes[q]), G[p][q], Qq);
   }
   float t = sc * Qq;
-#if ORC_MUTANT == 6
-  float g = sc * (Aq - t);
-#else
   float g = sc * (2.0f * Aq - t);
-#endif
   *gain_out = g;
   *scale_out = scale_field;
   for (int p = 0; p < ORC_MAXP; ++p) codes_out[p] = (int8_t)(p < P ? codes[p] : 0);
@@ -437,18 +353,10 @@ static void orc_tile_inputs(const orc_params* prm, int64_t cols, const float* W,
   const int C = prm->C;
   for (int j = 0; j < C; ++j) {
     int64_t idx = row * cols + cb * C + j;
-#if ORC_MUTANT == 22
-    r[j] = W0[idx] - W[idx];
-#else
     r[j] = W[idx] - W0[idx];
-#endif
     float a = act[cb * C + j];
     if (prm->variant == 0) d[j] = a;
-#if ORC_MUTANT == 21
-    else d[j] = w_act * a + w_fisher * fisher[row * cols + j];
-#else
     else d[j] = w_act * a + w_fisher * fisher[idx];
-#endif
   }
 }
 
@@ -473,11 +381,7 @@ void orc_encode_tiles(const orc_params* prm, int64_t rows, int64_t cols, const f
       for (int s = 0; s < prm->S; ++s) {
         float g; int16_t sf; int8_t codes[8];
         if (!orc_score_candidate(prm, r, d, masks + (size_t)s * P * C, &g, &sf, codes, NULL)) continue;
-#if ORC_MUTANT == 7
-        if (g >= best.gain) {
-#else
         if (g > best.gain) {
-#endif
           best.gain = g;
           best.seed = (uint16_t)s;
           best.scale = sf;
@@ -576,19 +480,11 @@ int64_t orc_header_bytes(int32_t n_mod) { return 40 + 8 * (int64_t)n_mod; }
 int64_t orc_record_bytes(const orc_params* prm, int64_t T) {
   int64_t bits = orc_ceil_log2((uint64_t)T) + orc_ceil_log2((uint64_t)prm->S) + prm->b_e +
                  (int64_t)prm->P * prm->b;
-#if ORC_MUTANT == 10
-  return (bits + 8) / 8;
-#else
   return (bits + 7) / 8;
-#endif
 }
 
 int64_t orc_budget_bytes(double rate_bpw, int64_t n_scope) {
-#if ORC_MUTANT == 33
-  return (int64_t)ceil(rate_bpw * (double)n_scope / 8.0);
-#else
   return (int64_t)floor(rate_bpw * (double)n_scope / 8.0);
-#endif
 }
 
 static void orc_put_bits(uint8_t* rec, int* pos, uint64_t value, int nbits) {
@@ -613,19 +509,10 @@ void orc_pack_record(const orc_params* prm, int64_t T, int64_t tile, const orc_c
   int64_t L = orc_record_bytes(prm, T);
   memset(rec, 0, (size_t)L);
   int pos = 0;
-#if ORC_MUTANT == 18
-  orc_put_bits(rec, &pos, cd->seed, orc_ceil_log2((uint64_t)prm->S));
-  orc_put_bits(rec, &pos, (uint64_t)tile, orc_ceil_log2((uint64_t)T));
-#else
   orc_put_bits(rec, &pos, (uint64_t)tile, orc_ceil_log2((uint64_t)T));
   orc_put_bits(rec, &pos, cd->seed, orc_ceil_log2((uint64_t)prm->S));
-#endif
   uint64_t sf;
-#if ORC_MUTANT == 31
-  if (prm->scale_mode == 0) sf = (uint64_t)(int64_t)(cd->scale + prm->e_bias);
-#else
   if (prm->scale_mode == 0) sf = (uint64_t)(int64_t)(cd->scale - prm->e_bias);
-#endif
   else sf = (uint16_t)cd->scale;
   orc_put_bits(rec, &pos, sf & ((prm->b_e >= 64) ? ~0ULL : ((1ULL << prm->b_e) - 1)), prm->b_e);
   for (int p = 0; p < prm->P; ++p)
@@ -657,11 +544,7 @@ static int orc_key_cmp(const void* a, const void* b) {
   const orc_key* y = (const orc_key*)b;
   if (x->gain > y->gain) return -1;   /* rho = gain / L with one L: gain descending */
   if (x->gain < y->gain) return 1;
-#if ORC_MUTANT == 8
-  return (x->tile < y->tile) - (x->tile > y->tile);
-#else
   return (x->tile > y->tile) - (x->tile < y->tile);  /* ties: tile ascending */
-#endif
 }
 
 /*
@@ -685,11 +568,7 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
   /* eligibility: non-positive (or non-finite) records are discarded (Sec. 3.3) */
   int64_t npos = 0;
   for (int64_t t = 0; t < T; ++t)
-#if ORC_MUTANT == 38
-    if (cands[t].gain >= 0.0f && cands[t].gain <= FLT_MAX) { keys[npos].gain = cands[t].gain; keys[npos].tile = t; ++npos; }
-#else
     if (cands[t].gain > 0.0f && cands[t].gain <= FLT_MAX) { keys[npos].gain = cands[t].gain; keys[npos].tile = t; ++npos; }
-#endif
   int64_t* order = (int64_t*)malloc(sizeof(int64_t) * (size_t)(T > 0 ? T : 1));
   if (prm->variant == 0) {
     /* U: within each module, the best records that fit its quota */
@@ -700,16 +579,8 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
       int64_t kend = kbeg;
       while (kend < npos && keys[kend].tile < off + mod_tiles[m]) ++kend;
       qsort(keys + kbeg, (size_t)(kend - kbeg), sizeof(orc_key), orc_key_cmp);
-#if ORC_MUTANT == 24
-      unsigned __int128 q = (unsigned __int128)(uint64_t)B * (uint64_t)mod_weights[m];
-#else
       unsigned __int128 q = (unsigned __int128)(uint64_t)(B - h) * (uint64_t)mod_weights[m];
-#endif
-#if ORC_MUTANT == 41
-      int64_t quota = (int64_t)((q + (uint64_t)Nscope - 1) / (uint64_t)Nscope);
-#else
       int64_t quota = (int64_t)(q / (uint64_t)Nscope);
-#endif
       int64_t K = quota / L;
       if (K > kend - kbeg) K = kend - kbeg;
       for (int64_t k = 0; k < K; ++k) order[K_stream++] = keys[kbeg + k].tile;
@@ -724,13 +595,7 @@ int orc_select_records(const orc_params* prm, int32_t n_mod, const int64_t* mod_
     for (int r = 0; r < n_rates; ++r) {
       int64_t B = orc_budget_bytes(rates[r], Nscope);
       if (B < h) { rc = 4; goto done; }
-#if ORC_MUTANT == 9
-      int64_t K = (B - h) / L + 1;
-#elif ORC_MUTANT == 28
-      int64_t K = B / L;
-#else
       int64_t K = (B - h) / L;
-#endif
       if (K > npos) K = npos;
       counts[r] = K;
       bytes_out[r] = h + K * L;
@@ -788,19 +653,11 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
   int64_t T = 0;
   for (int m = 0; m < n_mod; ++m) T += mod_rows[m] * mod_cols[m] / C;
   const int64_t h = orc_header_bytes(n_mod), L = orc_record_bytes(prm, T);
-#if ORC_MUTANT == 30
-  const float c = (float)(1.0 / (double)C);
-#else
   const float c = (float)(1.0 / sqrt((double)C));
-#endif
   uint8_t sign[256], neg[8 * 256];
   int32_t perm[256], cols[8];
   int bad = 0;
-#if ORC_MUTANT == 39
-  for (int64_t k = 0; k < K - 1; ++k) {
-#else
   for (int64_t k = 0; k < K; ++k) {
-#endif
     int64_t tile;
     orc_candidate cd;
     orc_unpack_record(prm, T, stream + h + k * L, &tile, &cd);
@@ -808,21 +665,13 @@ int orc_decode_apply(const orc_params* prm, int32_t n_mod, const int64_t* mod_ro
     int64_t m = 0, off = 0;
     while (tile >= off + mod_rows[m] * mod_cols[m] / C) { off += mod_rows[m] * mod_cols[m] / C; ++m; }
     int64_t lt = tile - off, n_cb = mod_cols[m] / C;
-#if ORC_MUTANT == 32
-    int64_t base = (lt / n_cb) * mod_cols[m] + ((lt + 1) % n_cb) * C;
-#else
     int64_t base = (lt / n_cb) * mod_cols[m] + (lt % n_cb) * C;
-#endif
     orc_gen_basis(prm->gen_seed, cd.seed, C, P, prm->permute, sign, perm, cols, neg);
     float sc = prm->scale_mode == 0 ? ldexpf(1.0f, cd.scale) : orc_f16_to_f32((uint16_t)cd.scale);
     for (int j = 0; j < C; ++j) {
       int kj = 0;
       for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
-#if ORC_MUTANT == 11
-      float rh = ((float)kj * c) * (0.5f * sc);
-#else
       float rh = ((float)kj * c) * sc;
-#endif
       out[m][base + j] = out[m][base + j] + rh;
     }
   }
@@ -860,21 +709,13 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
       const float a = fabsf(w[j]);
       if (a > amax) amax = a;
     }
-#if ORC_MUTANT == 14
-    const uint16_t h = orc_f32_to_f16(amax / 8.0f);
-#else
     const uint16_t h = orc_f32_to_f16(amax / 7.0f);
-#endif
     s16[g] = h;
     const float s = orc_f16_to_f32(h);
     for (int j = 0; j < group; ++j) {
       float v = 0.0f;
       if (s > 0.0f) {
-#if ORC_MUTANT == 42
-        v = rintf(w[j] * (1.0f / s));
-#else
         v = rintf(w[j] / s);
-#endif
         if (v < -8.0f) v = -8.0f;
         if (v > 7.0f) v = 7.0f;
       }
@@ -887,25 +728,13 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
       const int64_t n = G - b0 < block ? G - b0 : block;
       double sum = 0.0;
       for (int64_t g = b0; g < b0 + n; ++g) sum += (double)s_eff[g];
-#if ORC_MUTANT == 26
-      const float mu = (float)(sum / (double)block);
-#else
       const float mu = (float)(sum / (double)n);
-#endif
       float a = 0.0f;
       for (int64_t g = b0; g < b0 + n; ++g) {
-#if ORC_MUTANT == 34
-        const float d = s_eff[g] - mu;
-#else
         const float d = fabsf(s_eff[g] - mu);
-#endif
         if (d > a) a = d;
       }
-#if ORC_MUTANT == 15
-      const float step = a / 128.0f;
-#else
       const float step = a / 127.0f;
-#endif
       consts[2 * (b0 / block)] = mu;
       consts[2 * (b0 / block) + 1] = step;
       for (int64_t g = b0; g < b0 + n; ++g) {
@@ -963,11 +792,7 @@ int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_row
     for (int j = 0; j < C; ++j) {
       int kj = 0;
       for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
-#if ORC_MUTANT == 19
-      Wt[base + j] -= (double)kj * c * sc;
-#else
       Wt[base + j] += (double)kj * c * sc;
-#endif
     }
   }
   for (int v = 0; v < M; ++v)

@@ -44,21 +44,26 @@ class Params(ct.Structure):
     ]
 
 
-def _mutant() -> int:
-    """Planted-mistake build selected by AWSRC_ORACLE_MUTANT (the mutation test
-    of the pins only; 0 or unset is the oracle itself)."""
-    return int(os.environ.get("AWSRC_ORACLE_MUTANT", "0") or 0)
+def _source() -> str:
+    """The oracle's C source. AWSRC_ORACLE_SRC names another file only for the
+    mutation test of the pins, which builds copies of this source with one
+    planted mistake each; unset, it is the oracle itself."""
+    return os.environ.get("AWSRC_ORACLE_SRC") or _SRC
 
 
-def build(force: bool = False, mutant: int = 0) -> str:
+def build(force: bool = False, src: str = None) -> str:
     """Compile the oracle with gcc (-ffp-contract=off: no implicit fusion)."""
-    os.makedirs(_BUILD, exist_ok=True)
-    path = _LIB_PATH if mutant == 0 else os.path.join(_BUILD, f"liboracle_mutant{mutant}.so")
-    if not force and os.path.exists(path) and os.path.getmtime(path) >= os.path.getmtime(_SRC):
+    src = src or _source()
+    if src == _SRC:
+        os.makedirs(_BUILD, exist_ok=True)
+        path = _LIB_PATH
+    else:  # a copy built by the mutation test, next to its source
+        path = os.path.splitext(src)[0] + ".so"
+    if not force and os.path.exists(path) and os.path.getmtime(path) >= os.path.getmtime(src):
         return path
     tmp = path + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=gnu11", "-ffp-contract=off", "-fno-fast-math", "-fopenmp",
-           "-fPIC", "-shared", f"-DORC_MUTANT={mutant}", "-o", tmp, _SRC, "-lm"]
+           "-fPIC", "-shared", "-o", tmp, src, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, path)
     return path
@@ -68,7 +73,7 @@ def lib():
     global _lib
     with _lock:
         if _lib is None:
-            L = ct.CDLL(build(mutant=_mutant()))
+            L = ct.CDLL(build())
             P = ct.POINTER
             vp = ct.c_void_p
             L.orc_num_threads.restype = ct.c_int

@@ -138,3 +138,39 @@ def test_pf_weights_blend_activation_and_fisher(orc):
     f1 = orc.encode_tiles(pf, W, W0, act, fisher=Frow, w_act=0.5, w_fisher=0.25)
     u1 = orc.encode_tiles(pu, W, W0, blend)
     assert np.array_equal(f1, u1)
+
+
+@pytest.mark.parametrize("seed", [21, 23])
+def test_wide_dynamic_range_tiles(orc, seed):
+    """Activation moments spread over twelve decades: the per-tile fixed-point
+    grid of the correlations (21 bits below the tile's largest |d_j r_j|)
+    rounds many low-weight coordinates to zero. The binary32 search must still
+    pick a seed that is optimal by the double-precision definition of Eq. 4
+    (each seed scored from its own quantised codes, near-ties of 1e-6 relative
+    allowed), and its gain must be within 1e-5 of the tile's weighted energy of
+    the direct definition."""
+    rng = np.random.default_rng(seed)
+    C, P, b, S = 64, 4, 4, 256
+    prm = orc.params(C=C, P=P, b=b, S=S)
+    rows, cols = 16, 256
+    W0 = rng.normal(0, 0.02, (rows, cols)).astype(np.float32)
+    W = (W0 + rng.normal(0, 1e-3, (rows, cols))).astype(np.float32)
+    act = (10.0 ** rng.uniform(-6, 6, cols)).astype(np.float32)
+    masks = orc.basis_masks(prm)
+    cand = orc.encode_tiles(prm, W, W0, act, masks=masks)
+    zeroed = 0
+    for t in range(len(cand)):
+        r, d = _tile_rd(W, W0, act, C, t)
+        y = d * r
+        _, Y = orc.fixed_point(y)
+        zeroed += int(((Y == 0) & (y != 0)).sum())
+        energy = float(np.sum(d.astype(np.float64) * r.astype(np.float64) ** 2))
+        g = np.full(S, -np.inf)
+        for s in range(S):
+            out = orc.score_candidate(prm, r, d, masks[s])
+            if out is not None:
+                g[s] = orc.def_gain(C, P, r, d, masks[s], out["codes"], orc.scale_value(prm, out["scale"]))
+        s_star = int(cand[t]["seed"])
+        assert g[s_star] >= g.max() - 1e-6 * abs(g.max()), t
+        assert abs(cand[t]["gain"] - g[s_star]) <= 1e-5 * energy, t
+    assert zeroed > rows * cols // 4   # the case exercises the grid's lower end
