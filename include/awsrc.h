@@ -330,11 +330,12 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  * integer k_j = sum_p sign_{j,p} * code_p, rounded once more to BF16 when
  * out_dtype is BF16. Records naming a tile >= T or a seed >= S are skipped and
  * reported through awsrc_workspace_status(). A stream names each tile at most
- * once (the encoder never repeats one); DENSE decoding of a stream that does
- * applies only the tile's later record and reports it the same way, INPLACE
- * leaves such a tile unspecified. Requires the same params as the encoder.
+ * once (the encoder never repeats one); decoding a stream that does, in either
+ * mode, applies only the tile's later record and reports it the same way.
+ * Requires the same params as the encoder.
  * Workspace (awsrc_decode_workspace_bytes): the basis masks, plus for DENSE a
- * tile -> record map and the unpacked records, 16 bytes per tile.
+ * tile -> record map and the unpacked records, 16 bytes per tile; for INPLACE
+ * one claim word per tile (4 bytes).
  */
 awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 const awsrc_module* mods, const uint8_t* stream,
@@ -361,9 +362,12 @@ awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
  * numbers in awsrc_last_error_message()); at most 16 modules per call.
  * All calls share the one array per device and leave their contents in it;
  * calls whose kernels overlap on the GPU race on it, so the caller serialises
- * them. The first call on a device looks up the array's address with that
- * device current and should come before any stream capture. Records naming a
- * tile or seed out of range are skipped; this entry point does not report them.
+ * them. Every call looks up the array's address on the current device (the
+ * device that holds W_hat and the stream must be current); the first call on a
+ * device should come before any stream capture. Records naming a tile or seed
+ * out of range are skipped; this entry point does not report them. The stream
+ * must name each tile at most once, as the encoder's streams do: there is no
+ * room for per-tile claims here, so a tile named twice is left unspecified.
  */
 awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t n_mod,
                                                 const awsrc_module* mods, const uint8_t* stream,
@@ -444,6 +448,18 @@ void awsrc_set_timing_events(void* before_search, void* after_search);
 
 /* Number of kernels this library has launched in the process so far. */
 uint64_t awsrc_kernel_launches(void);
+
+/*
+ * awsrc_set_search_pruning — for the calling host thread, enabled = 0 makes
+ * every later awsrc_encode_tiles score every (tile, seed) candidate; 1 (the
+ * default) restores the exact pruning of the C = 64, P = 4, AWSRC-U search.
+ * That search skips a candidate whose upper bound on the Eq. 4 gain (the
+ * maximum b^T G^-1 b of the unquantised fit, inflated by a per-seed margin for
+ * binary32 rounding) lies below the best gain its row has already reached, so
+ * its candidates are by design identical either way; this switch exists to
+ * check that on real inputs. The other searches never prune.
+ */
+void awsrc_set_search_pruning(int32_t enabled);
 
 /*
  * awsrc_verify_reciprocal — a check of the library's own arithmetic (no

@@ -42,6 +42,7 @@ from ._binding import (  # noqa: F401
     awsrc_verify_reciprocal,
     awsrc_record_bytes,
     awsrc_select_records,
+    awsrc_set_search_pruning,
     awsrc_set_timing_events,
     awsrc_stream_capacity,
     awsrc_workspace_status,

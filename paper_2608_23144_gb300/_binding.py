@@ -108,6 +108,8 @@ def _load():
     L.awsrc_set_timing_events.argtypes = [vp, vp]
     L.awsrc_kernel_launches.restype = ct.c_uint64
     L.awsrc_kernel_launches.argtypes = []
+    L.awsrc_set_search_pruning.restype = None
+    L.awsrc_set_search_pruning.argtypes = [ct.c_int32]
     L.awsrc_verify_reciprocal.restype = st
     L.awsrc_verify_reciprocal.argtypes = [ct.c_uint32, ct.c_uint32, vp, vp]
     L.awsrc_workspace_status.restype = st
@@ -438,13 +440,25 @@ def awsrc_decode_apply(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
 def awsrc_decode_apply_inplace_noalloc(prm: Params, modules, stream_bytes: torch.Tensor, K: int,
                                        outs: List[torch.Tensor], stream=None) -> List[torch.Tensor]:
     """In-place decode that allocates nothing on either side of the ABI: `outs`
-    must already hold W0; their tiles named by the first K records get W0 + r_hat."""
+    must already hold W0; their tiles named by the first K records get W0 + r_hat.
+    The library keeps one scratch array per device and uses the current
+    device's, so the call runs with the device of `outs` current; the stream
+    bytes and every output must live on that device."""
+    if not outs:
+        raise ValueError("outs must hold one tensor per module")
+    dev = outs[0].device
+    _require(stream_bytes, "stream_bytes", dtype=torch.uint8, device=dev)
+    for i, o in enumerate(outs):
+        _require(o, f"outs[{i}]", device=dev)
     _check_outs(modules, outs, modules[0]["W0"].dtype)
     mods = module_array(modules, decoder=True)
     ptrs = (ct.c_void_p * len(outs))(*[_dev_ptr(o) for o in outs])
-    _check(lib.awsrc_decode_apply_inplace_noalloc(ct.byref(prm), len(modules), mods, _dev_ptr(stream_bytes),
-                                                  stream_bytes.numel(), int(K), ptrs, _stream(stream)),
-           "decode_apply_inplace_noalloc")
+    with torch.cuda.device(dev):
+        _check(lib.awsrc_decode_apply_inplace_noalloc(ct.byref(prm), len(modules), mods, _dev_ptr(stream_bytes),
+                                                      stream_bytes.numel(), int(K), ptrs,
+                                                      _stream(stream if stream is not None
+                                                              else torch.cuda.current_stream(dev))),
+               "decode_apply_inplace_noalloc")
     return outs
 
 
@@ -466,6 +480,12 @@ def awsrc_set_timing_events(before: Optional[torch.cuda.Event], after: Optional[
 
 def awsrc_kernel_launches() -> int:
     return int(lib.awsrc_kernel_launches())
+
+
+def awsrc_set_search_pruning(enabled: bool):
+    """For this host thread: False makes later encode calls score every
+    candidate (results identical by design; a check of the pruning bound)."""
+    lib.awsrc_set_search_pruning(1 if enabled else 0)
 
 
 def awsrc_verify_reciprocal(first: int, last: int, stream=None, device="cuda") -> int:

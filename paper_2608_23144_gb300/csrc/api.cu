@@ -15,6 +15,7 @@ namespace awsrc {
 namespace {
 thread_local char g_err[512] = "";
 thread_local cudaEvent_t g_ev_before = nullptr, g_ev_after = nullptr;
+thread_local int g_prune = 1;
 std::atomic<uint64_t> g_launches{0};
 constexpr int64_t kTargetBlocks = 1216;  // enough blocks to fill a GB300 (152 SMs) several times
 // one RTN launch has a block per 256 groups of 128 weights: 2^46 weights keep
@@ -174,6 +175,7 @@ awsrc_status make_prm(const awsrc_params* p, Prm* out) {
   // [-100 - (b-2), 33 - (b-2)]; if the range covers that, it never binds
   r.fast_pow2 = (p->scale_mode == AWSRC_SCALE_POW2) && r.e_lo <= -100 - (p->b - 2) &&
                 r.e_hi >= 33 - (p->b - 2);
+  r.prune = 1;
   *out = r;
   return AWSRC_OK;
 }
@@ -207,6 +209,8 @@ void awsrc_set_timing_events(void* before_search, void* after_search) {
 }
 
 uint64_t awsrc_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+void awsrc_set_search_pruning(int32_t enabled) { g_prune = enabled ? 1 : 0; }
 
 int64_t awsrc_header_bytes(int32_t n_mod) { return n_mod < 0 ? -1 : 40 + 8 * (int64_t)n_mod; }
 
@@ -267,6 +271,7 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   Prm pr;
   awsrc_status s = make_prm(prm, &pr);
   if (s != AWSRC_OK) return s;
+  pr.prune = g_prune;
   int64_t T;
   if ((s = check_modules(pr, n_mod, mods, true, &T)) != AWSRC_OK) return s;
   if (!out || !aligned(out, 4)) return AWSRC_ERR_INVALID_ARG;

@@ -42,6 +42,7 @@ struct Prm {
   int logC;       // log2(C)
   int fast_pow2;  // POW2 scale whose exponent range can never bind for a valid candidate
   uint32_t mant_q;  // mantissa field of (float)qmax
+  int prune;        // 1: the C = 64, P = 4 U search skips candidates its bound rules out
 };
 
 // ---------------------------------------------------------------- generator --

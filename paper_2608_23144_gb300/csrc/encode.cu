@@ -172,7 +172,8 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     float* po = reinterpret_cast<float*>(pairs) +
                 (size_t)((md.gram_off + cb * pr.S_pad + s) >> 1) * pair_stride(P) * 2 + (s & 1);
     constexpr int nl = P * (P - 1) / 2;
-    const float m = ok ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
+    // pr.prune == 0 scores every candidate (the same results, for tests of the bound)
+    const float m = ok && pr.prune ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
 #pragma unroll
     for (int i = 0; i < nl; ++i) po[2 * i] = -L[i];
     // invD * m rounded up: the bound's terms z_k (z_k invD_k m) are then never

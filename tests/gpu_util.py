@@ -38,3 +38,13 @@ def assert_candidates_equal(got, want, label=""):
         i = bad[0]
         raise AssertionError(f"{label}: {len(bad)} of {len(got)} tiles differ; first tile {i}: "
                              f"gpu {got[i]} oracle {want[i]}")
+
+
+def block_tiles(rng, rows, n_cb, block_rows=128):
+    """Tile indices of one whole block of the C = 64 search (block_rows
+    consecutive rows of one column block, chosen at random), plus every tile of
+    the module's first row."""
+    nb = (rows + block_rows - 1) // block_rows
+    rb, cb = int(rng.integers(nb)), int(rng.integers(n_cb))
+    r = np.arange(rb * block_rows, min(rows, (rb + 1) * block_rows))
+    return np.concatenate([r * n_cb + cb, np.arange(n_cb)])

@@ -3,14 +3,15 @@ weights, 1,204,224 tiles, S = 4096 seeds, AWSRC-U at 0.162 bits/weight) in the
 launch configuration the benchmark times:
 
 * encode: sampled tiles of every module re-searched by the oracle over all
-  4096 seeds, every field bit for bit;
+  4096 seeds, every field bit for bit (one whole 128-row block of the search
+  kernel, the module's first row, its corner tiles and random tiles);
 * select: the oracle re-selects from the GPU's candidates; stream identical;
 * decode: the oracle decodes the GPU's stream; every weight identical."""
 import numpy as np
 import pytest
 import torch
 
-from gpu_util import assert_candidates_equal, host_f32
+from gpu_util import assert_candidates_equal, block_tiles, host_f32
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
@@ -39,7 +40,8 @@ def test_fullsize_encode_sampled_tiles(layer, orc):
         T_m = m["rows"] * m["cols"] // wl.C
         n_cb = m["cols"] // wl.C
         tiles = np.unique(np.concatenate([[0, n_cb - 1, T_m - n_cb, T_m - 1],
-                                          rng.choice(T_m, 20, replace=False)]))
+                                          rng.choice(T_m, 20, replace=False),
+                                          block_tiles(rng, m["rows"], n_cb)]))
         want = orc.encode_tiles(oprm, host_f32(m["W"]), host_f32(m["W0"]), host_f32(m["act"]),
                                 tiles=tiles, masks=masks)
         assert_candidates_equal(got[off + tiles], want, m["name"])
