@@ -16,9 +16,13 @@
 //            k_j = sum_p sign * code_p exact in integers.
 //  in-place mode, and dense mode with tiles shorter than one vector (after a
 //  plain copy of W0):
+//   claim    one thread per record raises its tile's claim word to k + 1
+//            (atomicMax), so a tile named twice is flagged and only its later
+//            record is applied;
 //   patch    one thread per vector of a recorded tile: unpack tile, seed, scale,
 //            codes; bounds-check tile < T and seed < S (a bad record is skipped
-//            and flagged); rewrite the tile from W0, which may be W_hat itself.
+//            and flagged); skip a record whose tile a later record claims;
+//            rewrite the tile from W0, which may be W_hat itself.
 #include <algorithm>
 #include <utility>
 
@@ -50,6 +54,7 @@ struct DecArgs {
   int n_mod;
   int64_t T, L, h, K;  // K < 0: read from the header
   int64_t kmax;        // records that fit in the stream buffer (<= T)
+  const uint32_t* claim;  // record-by-record patch: per tile, 1 + the last record naming it (or null)
   DecodeMod m[kMaxModsPerLaunch];
 };
 
@@ -328,6 +333,7 @@ __global__ void __launch_bounds__(256) patch_kernel(Prm pr, const __grid_constan
     int mi = 0;
     for (int i = 1; i < a.n_mod; ++i)
       if (tile >= a.m[i].tile_off) mi = i;
+    if (a.claim && a.claim[tile] != (uint32_t)(k + 1)) continue;  // a later record names this tile
     const DecodeMod& md = a.m[mi];
     const int j0 = gj * G;
     const int64_t e0 = (tile - md.tile_off) * pr.C + j0;
@@ -362,6 +368,7 @@ __global__ void __launch_bounds__(256) patch_small_kernel(Prm pr, const __grid_c
     int mi = 0;
     for (int i = 1; i < a.n_mod; ++i)
       if (tile >= a.m[i].tile_off) mi = i;
+    if (a.claim && a.claim[tile] != (uint32_t)(k + 1)) continue;  // a later record names this tile
     const DecodeMod& md = a.m[mi];
     const int64_t e = (tile - md.tile_off) * pr.C + j;
     const uint64_t* mk = masks + (size_t)d.seed * pr.P * pr.W;
@@ -369,6 +376,23 @@ __global__ void __launch_bounds__(256) patch_small_kernel(Prm pr, const __grid_c
     for (int p = 0; p < pr.P; ++p) kj += ((mk[(size_t)p * pr.W + (j >> 6)] >> (j & 63)) & 1ull) ? -code_of(d, p) : code_of(d, p);
     const float w = Io<TI>::ld(static_cast<const TI*>(md.W0) + e, 0);
     static_cast<TO*>(md.out)[e] = Io<TO>::cvt(__fadd_rn(w, __fmul_rn(__fmul_rn((float)kj, pr.c), scale_of(pr, d.scale))));
+  }
+}
+
+// Claims for the record-by-record patch: claim[tile] = 1 + the largest record
+// index naming the tile, so that exactly one record (the later one) rewrites
+// a tile named twice, whatever the order the patch threads run in; the second
+// naming is reported. One thread per record; claim holds T zeroed words.
+__global__ void __launch_bounds__(256) claim_kernel(Prm pr, const __grid_constant__ DecArgs a,
+                                                    const uint8_t* __restrict__ stream,
+                                                    uint32_t* __restrict__ claim, uint32_t* __restrict__ status) {
+  const int64_t Kd = stream_K(stream, a.K, a.kmax);
+  const int64_t end = a.h + a.kmax * a.L;
+  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < Kd; k += (int64_t)gridDim.x * blockDim.x) {
+    DecRec d;
+    const int64_t tile = unpack(pr, stream, a.T, a.L, a.h, k, &d, end);
+    if (tile < 0) continue;  // flagged by the patch pass
+    if (atomicMax(claim + tile, (uint32_t)(k + 1)) != 0u) atomicOr(status, kFaultRecord);
   }
 }
 
@@ -608,6 +632,7 @@ cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, co
   DecArgs a;
   a.n_mod = 0;
   a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
+  a.claim = nullptr;
   const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
   int dev = 0, nsm = 148;
   cudaGetDevice(&dev);
@@ -639,11 +664,30 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
   const bool fused = decode_clears_status(pr, mode) && scratch != nullptr;
   unsigned long long* map = nullptr;
   uint2* codes = nullptr;
+  // the record-by-record patch with a workspace claims tiles first (without
+  // one, as for the no-allocation entry point, the stream must name each tile
+  // at most once)
+  uint32_t* claim = (!fused && scratch != nullptr) ? static_cast<uint32_t*>(scratch) : nullptr;
   if (fused) {
     map = static_cast<unsigned long long*>(scratch);
     codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
     const cudaError_t e = launch_dense_prep(pr, T, L, h, stream, K, kmax, masks, scratch, status, st);
     if (e != cudaSuccess) return e;
+  }
+  if (claim) {
+    const int64_t work = K >= 0 ? std::min(K, kmax) : kmax;
+    cudaError_t e = cudaMemsetAsync(claim, 0, (size_t)T * sizeof(uint32_t), st);
+    if (e != cudaSuccess) return e;
+    if (work > 0) {
+      DecArgs a;
+      a.n_mod = 0;
+      a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
+      a.claim = nullptr;
+      const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, 1 << 20));
+      claim_kernel<<<gx, 256, 0, st>>>(pr, a, stream, claim, status);
+      note_launches(1);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
   }
   int i0 = 0;
   while (i0 < n_mod) {
@@ -652,6 +696,7 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     DecArgs a;
     a.n_mod = i1 - i0;
     a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
+    a.claim = claim;
     for (int i = 0; i < a.n_mod; ++i) a.m[i] = mods[i0 + i];
     const cudaError_t e =
         fused ? launch_fused(pr, a, mods[i0].w0_dtype, out_dtype, map, codes, masks, st)
@@ -667,8 +712,8 @@ bool decode_clears_status(const Prm& pr, int mode) { return mode == AWSRC_DECODE
 
 size_t decode_scratch_bytes(int64_t T, int mode) {
   // dense: tile -> record map (8 B per tile) and each record's codes (8 B, at
-  // most one record per tile)
-  if (mode != AWSRC_DECODE_DENSE) return 0;
+  // most one record per tile); in-place: one claim word per tile
+  if (mode != AWSRC_DECODE_DENSE) return align_up((size_t)T * 4, 256);
   return align_up((size_t)T * 8, 256) + align_up((size_t)T * 8, 256);
 }
 

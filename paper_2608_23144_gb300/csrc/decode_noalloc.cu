@@ -20,10 +20,14 @@
 //  * every call shares the one array per device and leaves its contents there;
 //    calls whose work overlaps on the GPU (other streams, other host threads)
 //    race on it and must be serialised by the caller;
-//  * the first call on a device looks up the array's device address with that
-//    device current; make that first call before any stream capture.
+//  * every call looks up the array's device address on the current device
+//    (cudaGetSymbolAddress, which allocates nothing), so the address is never
+//    stale after a device reset; make the first call on a device before any
+//    stream capture, since that lookup may load the library's module there;
+//  * the stream must name each tile at most once (the encoder never repeats
+//    one); this entry point has no room for per-tile claims, so a tile named
+//    twice is left unspecified.
 #include <algorithm>
-#include <mutex>
 
 #include "internal.h"
 
@@ -34,31 +38,23 @@ namespace {
 constexpr int kStatusWords = (int)(kStatusBytes / sizeof(uint64_t));  // 32 words = 256 B
 constexpr int kMaxMaskWords = 131072;                                   // 1 MiB of masks
 constexpr int kScratchWords = kStatusWords + kMaxMaskWords;
-constexpr int kMaxDevices = 64;
 
 // The scratch: [fault word + padding (256 B)] [basis masks (up to 1 MiB)].
 static __device__ __align__(256) uint64_t g_noalloc_scratch[kScratchWords];
 
-std::mutex g_setup_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array for the current device (set-up once per
-// device). Host code must not use the array's name as an address: on the host
-// it is only a stand-in symbol.
+// Device address of the scratch array on the current device, looked up on
+// every call: a cached address would outlive a device reset or a recreated
+// primary context. Host code must not use the array's name as an address: on
+// the host it is only a stand-in symbol.
 awsrc_status scratch_for_current_device(uint64_t** out) {
-  int dev = -1;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, "decode_noalloc: cudaGetDevice");
-  if (dev < 0 || dev >= kMaxDevices) return AWSRC_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lk(g_setup_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "decode_noalloc: cudaGetSymbolAddress");
-    if (!p) return AWSRC_ERR_CUDA;
-    g_scratch_ptr[dev] = p;
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "decode_noalloc: cudaGetSymbolAddress");
+  if (!p) {
+    set_error_message("decode_noalloc: no device address for the scratch array");
+    return AWSRC_ERR_CUDA;
   }
-  *out = static_cast<uint64_t*>(g_scratch_ptr[dev]);
+  *out = static_cast<uint64_t*>(p);
   return AWSRC_OK;
 }
 

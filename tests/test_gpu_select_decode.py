@@ -134,8 +134,8 @@ def test_decode_rejects_K_beyond_stream(aw, orc):
 
 def test_decode_repeated_tile_takes_later_record(aw, orc):
     """A stream that names a tile twice (never written by the encoder) is reported;
-    dense decoding applies the later record, i.e. it equals decoding the stream
-    without the earlier one."""
+    dense and in-place decoding apply the later record, i.e. they equal decoding
+    the stream without the earlier one."""
     shapes = [(100, 256)]
     mods, dmods, prm, oprm, cands, ocands = _setup(aw, orc, shapes, dict(C=64, P=4, b=4, S=64))
     stream, counts, nbytes = aw.awsrc_select_records(prm, dmods, cands, [1.0])
@@ -156,6 +156,15 @@ def test_decode_repeated_tile_takes_later_record(aw, orc):
     oouts, obad = orc.decode_apply(oprm, [mods[0]["W0"].float().numpy()], fixed.tobytes(), K - 1, out_bf16=True)
     assert obad == 0
     assert np.array_equal(outs[0].float().cpu().numpy(), oouts[0])
+    # in place (W_hat is W0 itself): the same result and the same report, on
+    # every repetition (the later record claims the tile before any patch runs)
+    for _ in range(3):
+        w = dmods[0]["W0"].clone()
+        out = aw.awsrc_decode_apply(prm, [{**dmods[0], "W0": w}], torch.from_numpy(dup).cuda(), K, outs=[w],
+                                    mode=aw.DECODE_INPLACE)
+        flags = aw.awsrc_workspace_status(out[0]._awsrc_workspace)
+        assert flags & 1, "a repeated tile must be reported in place too"
+        assert np.array_equal(w.float().cpu().numpy(), oouts[0])
 
 
 @pytest.mark.parametrize("C,P", [(16, 4), (8, 2), (4, 1)])

@@ -14,13 +14,16 @@ import torch
 pytestmark = pytest.mark.gpu
 
 
-def _case(aw, shapes, seed, **kw):
+def _case(aw, shapes, seed, w_dtype="bf16", rates=(1.0,), **kw):
     from synth import make_module
-    mods = [make_module(r, c, seed=seed + 11 * i, device="cuda", w_dtype="bf16") for i, (r, c) in enumerate(shapes)]
+    pf = kw.get("variant", 0) == 1
+    mods = [make_module(r, c, seed=seed + 11 * i, device="cuda", w_dtype=w_dtype, fisher=pf, blend=(0.5, 0.5))
+            for i, (r, c) in enumerate(shapes)]
     prm = aw.params(**kw)
     cands = aw.awsrc_encode_tiles(prm, mods)
-    stream, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, [1.0])
-    return mods, prm, stream[: int(nbytes[0])].clone(), int(counts.sum())
+    stream, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, list(rates))
+    K = int(counts.sum()) if not pf else int(counts.max())
+    return mods, prm, stream[: int(nbytes.max())].clone(), K
 
 
 def test_noalloc_decode_matches_regular_decode_twice():
@@ -56,3 +59,24 @@ def test_noalloc_decode_rejects_tables_beyond_its_limit():
         aw.awsrc_decode_apply_inplace_noalloc(prm, mods, stream, 0, [mods[0]["W0"]])
     assert ei.value.status == 3
     assert b"131072" in aw.lib.awsrc_last_error_message()
+
+
+def test_noalloc_decode_f32_and_header_count_pf_stream():
+    """F32 weights decoded in place, and a progressive AWSRC-P_F stream decoded
+    with K = -1 (the header's record count, read on the device), each against
+    the regular dense decoder, twice in a row."""
+    import paper_2608_23144_gb300 as aw
+    cases = [
+        (_case(aw, [(72, 256), (40, 64)], 3, w_dtype="f32", C=64, P=4, b=4, S=128), None),
+        (_case(aw, [(90, 128), (33, 192)], 4, rates=(0.25, 1.0), C=64, P=4, b=4, S=96, variant=1), -1),
+    ]
+    for _ in range(2):
+        for (mods, prm, stream, K), k_arg in cases:
+            k_call = K if k_arg is None else k_arg
+            ref = aw.awsrc_decode_apply(prm, mods, stream, k_call, mode=aw.DECODE_DENSE)
+            outs = [m["W0"].clone() for m in mods]
+            aw.awsrc_decode_apply_inplace_noalloc(prm, mods, stream, k_call, outs)
+            torch.cuda.synchronize()
+            for a, b in zip(ref, outs):
+                assert a.dtype == b.dtype and torch.equal(a, b)
+            assert any(not torch.equal(o, m["W0"]) for o, m in zip(outs, mods))
