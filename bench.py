@@ -9,12 +9,16 @@ decode-apply of every module. Inputs are resident in HBM (308 MB of W and W0,
 larger than the 129 MB L2) when the timed region starts.
 
 Reported: (tile, seed) candidates/s for the whole step (`value`), layers/s,
-decode-apply GB/s, the search kernel against the FP32 pipe (`roofline`: the
-FP32 work every candidate needs before pruning), the
-end-to-end figure through the public API with host buffers (`e2e`), and the
-CPU oracle on a bounded sample (`cpu_baseline`). `--impl reference` times the
-oracle alone (the baseline arm). Under torchrun each rank encodes its own layer
-(weak scaling, no collective on the data path).
+decode-apply GB/s, the search kernel against the pipe its contraction runs on
+(`roofline`: the method's 2*C*P flop of correlation per candidate against the
+measured dense bf16 tensor peak, fp16 having the same rate; the FP32 epilogue,
+the executed tensor work and the DRAM traffic beside it), the end-to-end
+figure through the public API with host buffers (`e2e`), the whole
+Qwen2.5-3B, Qwen2.5-7B (AWSRC-P_F) and Qwen2.5-32B (AWSRC-U and AWSRC-P_F)
+synthetic models (`model_stack`, `full_models`), and the CPU oracle on a
+bounded sample (`cpu_baseline`). `--impl reference` times the oracle alone
+(the baseline arm). Under torchrun each rank encodes its own layer (weak
+scaling, no collective on the data path).
 """
 from __future__ import annotations
 
@@ -35,16 +39,24 @@ WORKLOAD = "qwen2.5-3b_layer"
 RATE = 0.162
 METRIC = "AWSRC encode (tile,seed) candidates/s + layers/s; decode-apply HBM GB/s"
 UNIT = "candidates/s"
-# FP32-pipe operations every (tile, seed) candidate of the C=64, P=4, U search
-# needs before it can be pruned: forming the rounded correlation from its two
-# halves (1 per atom), the forward substitution (6), z * (D^-1 m) (4) and the
-# bound z^T (z D^-1 m) (4); the bound is taken on the unscaled correlations, so
-# no scaling is needed before the decision. The ~0.5% of candidates that
-# survive the bound add about 50 more each (scaling, the forward substitution
-# in the recipe's units, back substitution, quantiser, gain), not counted here.
-# The correlation itself is tensor-core work: 2 halves x C x P x 2 FLOP.
+# The method's own work per (tile, seed) candidate of the C = 64, P = 4 search:
+# the correlation b = B_s^T (D r) of Eq. 3, C*P multiply-adds = 2*C*P flop. It
+# is a dense contraction (128 tiles x 64 inputs by 64 inputs x 4 atoms per
+# seed) and runs on the tensor cores, so it is the roofline's work, against
+# the dense fp16/bf16 tensor peak.
+METHOD_FLOP_PER_CANDIDATE = 2 * 64 * 4
+# What the kernel executes on the tensor cores: the exact fixed-point
+# correlation takes two fp16 halves of Y, so twice the method's flop.
+TENSOR_FLOP_PER_CANDIDATE = 2 * METHOD_FLOP_PER_CANDIDATE
+# FP32-pipe operations every candidate needs before it can be pruned: forming
+# the rounded correlation from its two halves (1 per atom), the forward
+# substitution (6), z * (D^-1 m) (4) and the bound z^T (z D^-1 m) (4). The ~0.5%
+# of candidates that survive the bound add about 50 more each, not counted.
 OPS_PER_CANDIDATE = 4 + 6 + 4 + 4
-TENSOR_FLOP_PER_CANDIDATE = 2 * 64 * 4 * 2
+# Bytes the search must move per launch at the least: W and W0 of the layer
+# (BF16, read once) and the 16-byte candidates written.
+def search_algorithmic_bytes(weights: int, tiles: int) -> int:
+    return 4 * weights + 16 * tiles
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
 SEARCH_TRAFFIC = {"source_sha256": "6d1079712f4600ea47f9057a1375d6b7b73847b96f7a4fb1e394b59ed11273ca",
@@ -81,9 +93,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pf", action="store_true", help="skip the P_F encode measurement")
-    ap.add_argument("--full-models", action="store_true",
-                    help="also encode, select and decode the whole 28-layer Qwen2.5-7B (P_F) and 64-layer "
-                         "Qwen2.5-32B (U and P_F) synthetic models (about a minute of GPU time)")
+    ap.add_argument("--no-full-models", action="store_true",
+                    help="skip the whole 28-layer Qwen2.5-7B (P_F) and 64-layer Qwen2.5-32B (U and P_F) "
+                         "synthetic models (encode, select, decode; about a minute of GPU time)")
     ap.add_argument("--no-model", action="store_true",
                     help="skip the whole 36-layer Qwen2.5-3B stack (encode, select, decode)")
     ap.add_argument("--modules", default="",
@@ -652,15 +664,30 @@ def run_ours(args):
     peaks, peak_kind = measured_peaks()
     nsm = torch.cuda.get_device_properties(dev).multi_processor_count
     fp32_peak = nsm * 128 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
-    achieved = cands_per_step * OPS_PER_CANDIDATE / (search_ms * 1e-3)
+    tensor_peak = float(peaks.get("bf16_tflops", 1900.0)) * 1e12
+    method_flops = cands_per_step * METHOD_FLOP_PER_CANDIDATE / (search_ms * 1e-3)
+    executed_flops = cands_per_step * TENSOR_FLOP_PER_CANDIDATE / (search_ms * 1e-3)
+    fp32_ops = cands_per_step * OPS_PER_CANDIDATE / (search_ms * 1e-3)
     counters_valid = SEARCH_TRAFFIC["source_sha256"] == search_source_sha()
     traffic = SEARCH_TRAFFIC["bytes_per_launch"] if counters_valid else None
-    roofline = {"bound": "alu", "kernel": "search_c64p4", "achieved": achieved / 1e9,
-                "peak": fp32_peak / 1e9, "unit": "Gop/s", "frac": achieved / fp32_peak,
-                "traffic": traffic, "peak_kind": f"{peak_kind}: {nsm} SMs x 128 FP32 lanes x "
-                f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
-                "ops_per_candidate": OPS_PER_CANDIDATE, "search_ms": search_ms,
-                "tensor_tflops": cands_per_step * TENSOR_FLOP_PER_CANDIDATE / (search_ms * 1e-3) / 1e12,
+    weights = sum(m["rows"] * m["cols"] for m in mods)
+    alg_bytes = search_algorithmic_bytes(weights, T)
+    roofline = {"bound": "tensor", "kernel": "search_c64p4", "achieved": method_flops / 1e12,
+                "peak": tensor_peak / 1e12, "unit": "TFLOP/s", "frac": method_flops / tensor_peak,
+                "traffic": traffic,
+                "peak_kind": f"{peak_kind} dense bf16 burst (fp16, the operands' type, has the same rate)",
+                "work": f"{METHOD_FLOP_PER_CANDIDATE} flop per (tile, seed) candidate (2*C*P, the Eq. 3 "
+                        f"correlation) x {cands_per_step:,} candidates per launch",
+                "search_ms": search_ms,
+                "executed_tensor": {"flop_per_candidate": TENSOR_FLOP_PER_CANDIDATE,
+                                    "tflops": executed_flops / 1e12, "frac": executed_flops / tensor_peak},
+                "fp32_epilogue": {"ops_per_candidate_before_pruning": OPS_PER_CANDIDATE,
+                                  "gops": fp32_ops / 1e9, "peak_gops": fp32_peak / 1e9,
+                                  "frac": fp32_ops / fp32_peak,
+                                  "peak_kind": f"{nsm} SMs x 128 FP32 lanes x "
+                                               f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz"},
+                "dram": {"algorithmic_bytes": alg_bytes, "traffic_bytes": traffic,
+                         "traffic_over_algorithmic": traffic / alg_bytes if traffic else None},
                 "ncu": ({k: SEARCH_TRAFFIC[k] for k in ("ncu_fma_pipe_pct", "ncu_issue_active_pct",
                                                          "ncu_tensor_pipe_pct")} if counters_valid else None)}
     decode = {"gbs": dec_gbs, "ms": dec_ms, "frac_of_hbm": dec_gbs / float(peaks.get("hbm_gbs", 6800.0)),
@@ -765,7 +792,7 @@ def run_ours(args):
     if rank == 0 and world == 1 and not args.no_model and not args.modules:
         model = model_stack(dev, float(peaks.get("hbm_gbs", 6800.0)))
     models = None
-    if rank == 0 and world == 1 and args.full_models:
+    if rank == 0 and world == 1 and not args.no_full_models and not args.modules:
         models = {n: full_model(dev, float(peaks.get("hbm_gbs", 6800.0)), n)
                   for n in ("qwen2.5-7b_stack_pf", "qwen2.5-32b_stack")}
 
