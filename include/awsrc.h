@@ -215,7 +215,7 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod,
  *   W0 = q * s_eff with s_eff = s_g, or s~_g under SDQ (codes stay those of s_g).
  * Metadata: binary16 scales cost 2 bytes per group (0.125 bits/weight); SDQ
  * 1 byte per group plus 8 per block (0.0645 bits/weight on whole blocks), see
- * awsrc_backbone_metadata_bytes. W must be finite.
+ * awsrc_backbone_metadata_bytes and awsrc_rate_with_sdq_savings. W must be finite.
  *   W           device, rows*cols elements of w_dtype, 16-byte aligned.
  *   codes       device, rows*cols/2 bytes (4-byte aligned): element 2i in the
  *               low nibble of byte i, 4-bit two's complement.
@@ -234,11 +234,30 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
  * awsrc_backbone_metadata_bytes — scale metadata of a rows x cols RTN-INT4
  * backbone: 2 bytes per group of 128, or with SDQ 1 per group plus 8 per block
  * of 256 groups. Under a fixed total budget the bytes SDQ saves can go to the
- * residual records (Sec. 3.3): raise the rate given to awsrc_select_records by
- * 8 * saved / N_scope bits/weight. Returns -1 for a bad shape or rows*cols
- * above 2^46.
+ * residual records (Sec. 3.3): awsrc_rate_with_sdq_savings gives the rate for
+ * awsrc_select_records that does so exactly. Returns -1 for a bad shape or
+ * rows*cols above 2^46.
  */
 int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq);
+
+/*
+ * awsrc_rate_with_sdq_savings — the rate to give awsrc_select_records when the
+ * backbone's scales are double quantised and the metadata bytes SDQ saves go
+ * to the residual records (Sec. 3.3) under an unchanged total budget. With
+ * binary16 scales the scope holds meta_fp16 + B bytes, B = floor(rate_bpw *
+ * N_scope / 8) (Eq. 5, header included); with SDQ the sidecar may then take
+ * B + saved bytes, saved = sum_m (awsrc_backbone_metadata_bytes(m, 0) -
+ * awsrc_backbone_metadata_bytes(m, 1)). *rate_out is a rate whose budget
+ * floor(rate_out * N_scope / 8) is exactly B + saved, so that backbone
+ * metadata plus stream never exceed meta_fp16 + B; *saved_bytes (may be NULL)
+ * receives saved. On modules of a few groups SDQ's 8-byte block constants
+ * cost more than it saves: saved is then negative and the budget shrinks.
+ * Reads rows and cols of each module (cols % 128 == 0). Host-only.
+ * Errors: INVALID_ARG, SHAPE, BUDGET (B + saved < 0), UNSUPPORTED
+ * (N_scope >= 2^52).
+ */
+awsrc_status awsrc_rate_with_sdq_savings(int32_t n_mod, const awsrc_module* mods, double rate_bpw,
+                                         double* rate_out, int64_t* saved_bytes);
 
 /*
  * awsrc_gen_basis — writes the sign masks of GenBasis (Eq. 2) for seeds [0, S):
@@ -460,6 +479,25 @@ uint64_t awsrc_kernel_launches(void);
  * check that on real inputs. The other searches never prune.
  */
 void awsrc_set_search_pruning(int32_t enabled);
+
+/*
+ * awsrc_set_wait_test — a test of the kernels' failure handling, for the
+ * calling host thread (no counterpart in the paper). Every wait inside the
+ * tcgen05 search kernels (for bulk copies, tensor-core results and the release
+ * of shared buffers) gives up after a time limit, 2 s by default; the block
+ * then records bit 2 of the workspace's fault word, waits (with the same
+ * limit) for its own copies and tensor-core work still in flight, frees its
+ * tensor memory and exits, so the GPU context stays usable.
+ *   wait_ns      the limit of every such wait in later awsrc_encode_tiles
+ *                calls (0: the default 2 s).
+ *   stall_chunk  >= 0: the C = 64, P = 4, AWSRC-U search issues no copies of
+ *                its seed chunks from this one (counted within each block's
+ *                range of 32-seed chunks) on, so its waits for that chunk run
+ *                out; -1: normal operation.
+ * The call's candidates are then undefined and awsrc_workspace_status reports
+ * bit 2. awsrc_set_wait_test(0, -1) restores normal operation.
+ */
+void awsrc_set_wait_test(uint64_t wait_ns, int32_t stall_chunk);
 
 /*
  * awsrc_verify_reciprocal — a check of the library's own arithmetic (no

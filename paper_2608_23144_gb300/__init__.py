@@ -34,6 +34,7 @@ from ._binding import (  # noqa: F401
     awsrc_gen_basis,
     awsrc_rtn_quantize,
     awsrc_backbone_metadata_bytes,
+    awsrc_rate_with_sdq_savings,
     awsrc_sidecar_prepare,
     awsrc_packed_gemv,
     shape_modules,
@@ -44,6 +45,7 @@ from ._binding import (  # noqa: F401
     awsrc_select_records,
     awsrc_set_search_pruning,
     awsrc_set_timing_events,
+    awsrc_set_wait_test,
     awsrc_stream_capacity,
     awsrc_workspace_status,
     candidates_to_numpy,

@@ -110,6 +110,8 @@ def _load():
     L.awsrc_kernel_launches.argtypes = []
     L.awsrc_set_search_pruning.restype = None
     L.awsrc_set_search_pruning.argtypes = [ct.c_int32]
+    L.awsrc_set_wait_test.restype = None
+    L.awsrc_set_wait_test.argtypes = [ct.c_uint64, ct.c_int32]
     L.awsrc_verify_reciprocal.restype = st
     L.awsrc_verify_reciprocal.argtypes = [ct.c_uint32, ct.c_uint32, vp, vp]
     L.awsrc_workspace_status.restype = st
@@ -119,6 +121,9 @@ def _load():
                                      ct.c_int32, vp]
     L.awsrc_backbone_metadata_bytes.restype = ct.c_int64
     L.awsrc_backbone_metadata_bytes.argtypes = [ct.c_int64, ct.c_int64, ct.c_int32]
+    L.awsrc_rate_with_sdq_savings.restype = st
+    L.awsrc_rate_with_sdq_savings.argtypes = [ct.c_int32, P(Module), ct.c_double, P(ct.c_double),
+                                              P(ct.c_int64)]
     L.awsrc_sidecar_workspace_bytes.restype = st
     L.awsrc_sidecar_workspace_bytes.argtypes = [P(Params), ct.c_int32, P(Module), P(sz)]
     L.awsrc_sidecar_prepare.restype = st
@@ -293,6 +298,17 @@ def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream
 
 def awsrc_backbone_metadata_bytes(rows: int, cols: int, sdq: bool) -> int:
     return int(lib.awsrc_backbone_metadata_bytes(rows, cols, int(sdq)))
+
+
+def awsrc_rate_with_sdq_savings(shapes, rate: float):
+    """(rate for awsrc_select_records, saved bytes): the sidecar budget grows by
+    the metadata bytes SDQ saves on these (rows, cols) modules (Sec. 3.3)."""
+    mods = shape_modules(shapes)
+    out = ct.c_double()
+    saved = ct.c_int64()
+    _check(lib.awsrc_rate_with_sdq_savings(len(shapes), mods, float(rate), ct.byref(out), ct.byref(saved)),
+           "rate_with_sdq_savings")
+    return out.value, saved.value
 
 
 def shape_modules(shapes):
@@ -486,6 +502,14 @@ def awsrc_set_search_pruning(enabled: bool):
     """For this host thread: False makes later encode calls score every
     candidate (results identical by design; a check of the pruning bound)."""
     lib.awsrc_set_search_pruning(1 if enabled else 0)
+
+
+def awsrc_set_wait_test(wait_ns: int = 0, stall_chunk: int = -1):
+    """For this host thread: the limit of the kernels' bounded waits (0 = 2 s)
+    and, for stall_chunk >= 0, the seed chunk from which the C = 64, P = 4 U
+    search issues no copies, so that its waits run out (a test of the timeout
+    path). awsrc_set_wait_test() restores normal operation."""
+    lib.awsrc_set_wait_test(int(wait_ns), int(stall_chunk))
 
 
 def awsrc_verify_reciprocal(first: int, last: int, stream=None, device="cuda") -> int:

@@ -16,6 +16,8 @@ namespace {
 thread_local char g_err[512] = "";
 thread_local cudaEvent_t g_ev_before = nullptr, g_ev_after = nullptr;
 thread_local int g_prune = 1;
+thread_local uint64_t g_wait_ns = 0;  // 0: the default limit
+thread_local int g_stall_chunk = -1;
 std::atomic<uint64_t> g_launches{0};
 constexpr int64_t kTargetBlocks = 1216;  // enough blocks to fill a GB300 (152 SMs) several times
 // one RTN launch has a block per 256 groups of 128 weights: 2^46 weights keep
@@ -176,6 +178,8 @@ awsrc_status make_prm(const awsrc_params* p, Prm* out) {
   r.fast_pow2 = (p->scale_mode == AWSRC_SCALE_POW2) && r.e_lo <= -100 - (p->b - 2) &&
                 r.e_hi >= 33 - (p->b - 2);
   r.prune = 1;
+  r.stall_chunk = -1;
+  r.wait_ns = kWaitLimitNs;
   *out = r;
   return AWSRC_OK;
 }
@@ -211,6 +215,11 @@ void awsrc_set_timing_events(void* before_search, void* after_search) {
 uint64_t awsrc_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
 void awsrc_set_search_pruning(int32_t enabled) { g_prune = enabled ? 1 : 0; }
+
+void awsrc_set_wait_test(uint64_t wait_ns, int32_t stall_chunk) {
+  g_wait_ns = wait_ns;
+  g_stall_chunk = stall_chunk < 0 ? -1 : stall_chunk;
+}
 
 int64_t awsrc_header_bytes(int32_t n_mod) { return n_mod < 0 ? -1 : 40 + 8 * (int64_t)n_mod; }
 
@@ -256,6 +265,32 @@ int64_t awsrc_backbone_metadata_bytes(int64_t rows, int64_t cols, int32_t sdq) {
   return sdq ? G + 8 * ((G + sdq_block() - 1) / sdq_block()) : 2 * G;
 }
 
+awsrc_status awsrc_rate_with_sdq_savings(int32_t n_mod, const awsrc_module* mods, double rate_bpw,
+                                         double* rate_out, int64_t* saved_bytes) {
+  if (n_mod < 1 || !mods || !rate_out) return AWSRC_ERR_INVALID_ARG;
+  if (!(rate_bpw >= 0.0) || !std::isfinite(rate_bpw)) return AWSRC_ERR_INVALID_ARG;
+  int64_t N = 0, saved = 0;
+  for (int m = 0; m < n_mod; ++m) {
+    const int64_t fp16 = awsrc_backbone_metadata_bytes(mods[m].rows, mods[m].cols, 0);
+    const int64_t sdq = awsrc_backbone_metadata_bytes(mods[m].rows, mods[m].cols, 1);
+    if (fp16 < 0 || sdq < 0) return AWSRC_ERR_SHAPE;
+    if (N > (1ll << 52) - mods[m].rows * mods[m].cols) return AWSRC_ERR_UNSUPPORTED;
+    N += mods[m].rows * mods[m].cols;
+    saved += fp16 - sdq;
+  }
+  // the budget awsrc_select_records derives from a rate, B = floor(rate N / 8)
+  auto budget = [N](double r) { return (int64_t)std::floor(r * (double)N / 8.0); };
+  const int64_t target = budget(rate_bpw) + saved;
+  if (target < 0) return AWSRC_ERR_BUDGET;  // SDQ's block constants cost more than it saves
+  double r = 8.0 * (double)target / (double)N;
+  for (int i = 0; i < 64 && budget(r) < target; ++i) r = std::nextafter(r, INFINITY);
+  for (int i = 0; i < 64 && budget(r) > target; ++i) r = std::nextafter(r, 0.0);
+  if (budget(r) != target) return AWSRC_ERR_UNSUPPORTED;
+  *rate_out = r;
+  if (saved_bytes) *saved_bytes = saved;
+  return AWSRC_OK;
+}
+
 awsrc_status awsrc_gen_basis(const awsrc_params* prm, uint64_t* masks, void* stream) {
   Prm pr;
   awsrc_status s = make_prm(prm, &pr);
@@ -272,6 +307,8 @@ awsrc_status awsrc_encode_tiles(const awsrc_params* prm, int32_t n_mod, const aw
   awsrc_status s = make_prm(prm, &pr);
   if (s != AWSRC_OK) return s;
   pr.prune = g_prune;
+  if (g_wait_ns) pr.wait_ns = g_wait_ns;
+  pr.stall_chunk = g_stall_chunk;
   int64_t T;
   if ((s = check_modules(pr, n_mod, mods, true, &T)) != AWSRC_OK) return s;
   if (!out || !aligned(out, 4)) return AWSRC_ERR_INVALID_ARG;

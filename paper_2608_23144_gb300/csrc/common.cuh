@@ -43,7 +43,12 @@ struct Prm {
   int fast_pow2;  // POW2 scale whose exponent range can never bind for a valid candidate
   uint32_t mant_q;  // mantissa field of (float)qmax
   int prune;        // 1: the C = 64, P = 4 U search skips candidates its bound rules out
+  int stall_chunk;  // test of the bounded waits: the U search's producer issues no copies from
+                    // this chunk of its block's range on (-1: never)
+  uint64_t wait_ns; // limit of every bounded wait inside a kernel (2 s)
 };
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 // ---------------------------------------------------------------- generator --
 // SplitMix64 (Steele, Lea & Flood 2014): n-th output of the stream at state x.

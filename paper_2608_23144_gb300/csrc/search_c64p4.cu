@@ -32,7 +32,10 @@
 // flight while a pair is scored.
 // Every mbarrier wait is bounded in time; on expiry the block records a timeout
 // fault, waits (bounded) for its own copies and MMAs in flight, frees its TMEM
-// and returns.
+// and returns. A test of that path (Prm::stall_chunk >= 0) makes the producer
+// issue no copies from that chunk of its range on, with a short limit, so
+// that the producer's wait for the chunk's copies and the epilogue's wait for
+// its MMAs both run out.
 #include "internal.h"
 #include "tc05.cuh"
 
@@ -309,7 +312,7 @@ __global__ void __launch_bounds__(NT, 1)
 
   int issued = 0;  // chunks whose copies the producer issued
   if (warp == EW && lane == 0) {
-    for (; issued < STAGES && issued < nck; ++issued) {
+    for (; issued < STAGES && issued < nck && issued != pr.stall_chunk; ++issued) {
       mbar_expect_tx(&sm.full[issued], kBBytes + kPBytes);
       bulk_g2s(&sm.stage[issued][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[issued]);
       bulk_g2s(&sm.stage[issued][kBBytes], pf_src + (size_t)issued * kPBytes, kPBytes, &sm.full[issued]);
@@ -371,9 +374,9 @@ __global__ void __launch_bounds__(NT, 1)
       int k = 0;
       for (; k < nck; ++k) {
         const int st = k % STAGES, tb = k & 1;
-        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
+        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1), pr.wait_ns)) { timed_out = true; break; }
         // every epilogue warp has loaded chunk k-2 from its accumulator
-        if (k >= 2 && !mbar_wait(&sm.aempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
+        if (k >= 2 && !mbar_wait(&sm.aempty[tb], (uint32_t)(((k - 2) >> 1) & 1), pr.wait_ns)) { timed_out = true; break; }
         tc_fence_after();
         const uint32_t bsm = smem_addr(&sm.stage[st][0]);
 #pragma unroll
@@ -385,10 +388,10 @@ __global__ void __launch_bounds__(NT, 1)
           }
         }
         umma_commit(&sm.afull[tb]);
-        if (k >= 2 && issued < nck) {
+        if (k >= 2 && issued < nck && issued != pr.stall_chunk) {
           // chunk k-2's factors are no longer read: its stage takes chunk k+2
           const int ps = (k - 2) % STAGES;
-          if (!mbar_wait(&sm.sempty[ps], (uint32_t)(((k - 2) / STAGES) & 1))) { timed_out = true; ++k; break; }
+          if (!mbar_wait(&sm.sempty[ps], (uint32_t)(((k - 2) / STAGES) & 1), pr.wait_ns)) { timed_out = true; ++k; break; }
           const int ns = issued % STAGES;
           mbar_expect_tx(&sm.full[ns], kBBytes + kPBytes);
           bulk_g2s(&sm.stage[ns][0], at_src + (size_t)issued * kBBytes, kBBytes, &sm.full[ns]);
@@ -399,8 +402,8 @@ __global__ void __launch_bounds__(NT, 1)
       if (timed_out) {
         // wait (bounded) for this block's copies and MMAs still in flight
         for (int j = max(0, issued - STAGES); j < issued; ++j)
-          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
-        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1));
+          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1), pr.wait_ns);
+        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1), pr.wait_ns);
       }
     }
   } else {
@@ -426,10 +429,10 @@ __global__ void __launch_bounds__(NT, 1)
     // the whole tie rule within a thread.
     for (int k = 0; k < nck; ++k) {
       const int st = k % STAGES, tb = k & 1;
-      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1))) { timed_out = true; break; }
+      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1), pr.wait_ns)) { timed_out = true; break; }
       // the stage's factors landed before the chunk's MMAs were issued; this
       // wait (already complete) makes the copy visible to this warp's reads
-      if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
+      if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1), pr.wait_ns)) { timed_out = true; break; }
       tc_fence_after();
       // Pruning threshold: the best gain any of the row's SUBS warps has found
       // so far. Each of them is a gain some candidate of this row reaches, so

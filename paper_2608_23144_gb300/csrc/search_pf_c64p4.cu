@@ -344,8 +344,8 @@ __global__ void __launch_bounds__(NT, 1)
       int k = 0;
       for (; k < nck; ++k) {
         const int st = k % STAGES, tb = k & 1;
-        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1))) { timed_out = true; break; }
-        if (k >= 2 && !mbar_wait(&sm.tempty[tb], (uint32_t)(((k - 2) >> 1) & 1))) { timed_out = true; break; }
+        if (!mbar_wait(&sm.full[st], (uint32_t)((k / STAGES) & 1), pr.wait_ns)) { timed_out = true; break; }
+        if (k >= 2 && !mbar_wait(&sm.tempty[tb], (uint32_t)(((k - 2) >> 1) & 1), pr.wait_ns)) { timed_out = true; break; }
         tc_fence_after();
         const uint32_t sa = smem_addr(&sm.stage[st][0]), sq = sa + kABytes;
         const uint32_t acc = tmem + (uint32_t)(tb * 256);
@@ -370,8 +370,8 @@ __global__ void __launch_bounds__(NT, 1)
       }
       if (timed_out) {
         for (int j = max(0, issued - STAGES); j < issued; ++j)
-          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
-        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1));
+          (void)mbar_wait(&sm.full[j % STAGES], (uint32_t)((j / STAGES) & 1), pr.wait_ns);
+        if (k > 0) (void)mbar_wait(&sm.afull[(k - 1) & 1], (uint32_t)(((k - 1) >> 1) & 1), pr.wait_ns);
       }
     }
   } else {
@@ -384,7 +384,7 @@ __global__ void __launch_bounds__(NT, 1)
     uint32_t bsd = 0xffffffffu;
     for (int k = 0; k < nck; ++k) {
       const int tb = k & 1;
-      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1))) { timed_out = true; break; }
+      if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1), pr.wait_ns)) { timed_out = true; break; }
       tc_fence_after();
       const uint32_t base = tmem + lane_base + (uint32_t)(tb * 256);
       float ah[8], al[8], qh[12], ql[12];

@@ -8,7 +8,6 @@
 namespace awsrc {
 namespace tc05 {
 
-constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per bounded wait
 
 // MMA instruction descriptor (kind::f16): D FP32 (bits 4-5 = 1), A and B FP16
 // (bits 7-9, 10-12 = 0), both K-major (bits 15, 16 = 0), N >> 3 at bit 17,
@@ -55,12 +54,13 @@ __device__ __forceinline__ bool mbar_try_wait(unsigned long long* mb, uint32_t p
   return ok != 0;
 }
 
-// Bounded wait: true when the phase with `parity` completed within kWaitNs.
-__device__ __forceinline__ bool mbar_wait(unsigned long long* mb, uint32_t parity) {
+// Bounded wait: true when the phase with `parity` completed within limit_ns
+// (Prm::wait_ns, 2 s unless a test shortens it).
+__device__ __forceinline__ bool mbar_wait(unsigned long long* mb, uint32_t parity, uint64_t limit_ns) {
   if (mbar_try_wait(mb, parity)) return true;
   const uint64_t t0 = globaltimer();
   while (!mbar_try_wait(mb, parity)) {
-    if (globaltimer() - t0 > kWaitNs) return false;
+    if (globaltimer() - t0 > limit_ns) return false;
   }
   return true;
 }
