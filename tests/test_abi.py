@@ -146,6 +146,37 @@ def test_backbone_metadata_bytes(libpath):
     assert aw.awsrc_backbone_metadata_bytes(1, 128, True) == 1 + 8
 
 
+@pytest.mark.parametrize("rate", [0.0, 0.05, 0.162, 0.25, 1.0])
+def test_rate_with_sdq_savings_gives_the_saved_bytes_to_the_sidecar(libpath, orc, rate):
+    """Sec. 3.3: the metadata bytes SDQ saves against binary16 scales go to the
+    residual records under an unchanged total. The returned rate's budget
+    (Eq. 5, floor(rate N / 8)) must be exactly the old budget plus the saving,
+    counted here from the two metadata layouts (2 bytes per group of 128, or 1
+    per group plus 8 per 256 groups)."""
+    import math
+    import paper_2608_23144_gb300 as aw
+    from synth.workloads import _QWEN3B, _QWEN32B
+    for shapes in ([(r, c) for _, r, c in _QWEN3B], [(r, c) for _, r, c in _QWEN32B], [(3, 128), (1, 384)]):
+        N = sum(r * c for r, c in shapes)
+        saved = 0
+        for r, c in shapes:
+            G = r * c // 128
+            saved += 2 * G - (G + 8 * math.ceil(G / 256))
+        if orc.budget_bytes(rate, N) + saved < 0:     # SDQ's block constants cost more than it saves
+            with pytest.raises(aw.AwsrcError) as ei:
+                aw.awsrc_rate_with_sdq_savings(shapes, rate)
+            assert ei.value.status == 4
+            continue
+        r2, got_saved = aw.awsrc_rate_with_sdq_savings(shapes, rate)
+        assert got_saved == saved
+        assert orc.budget_bytes(r2, N) == orc.budget_bytes(rate, N) + saved
+        assert (r2 >= rate) == (saved >= 0)
+    with pytest.raises(aw.AwsrcError):
+        aw.awsrc_rate_with_sdq_savings([(4, 100)], 0.1)       # cols not a multiple of 128
+    with pytest.raises(aw.AwsrcError):
+        aw.awsrc_rate_with_sdq_savings([(4, 128)], -1.0)
+
+
 def test_serving_and_diagnostic_arguments_are_refused_on_the_host(libpath):
     """Pointer values are only compared (no device memory exists): the backbone
     quantiser, the packed GEMV and the reciprocal check return INVALID_ARG or

@@ -50,3 +50,35 @@ def test_backbone_matches_oracle(aw, orc, rows, cols, w_dtype, w0_dtype, sdq):
     assert torch.equal(got["W0"].cpu().view(torch.int16 if w0_dtype == torch.bfloat16 else torch.int32),
                        W0.view(torch.int16 if w0_dtype == torch.bfloat16 else torch.int32))
 
+
+
+def test_sdq_savings_returned_to_the_sidecar_budget(aw, orc):
+    """Sec. 3.3 end to end on one Qwen2.5-3B-shaped layer: the RTN-INT4 backbone
+    with SDQ scales (W0 from the double-quantised scales), the encoder against
+    that W0, and AWSRC-U selection at the rate that gives the metadata bytes SDQ
+    saves to the records. Backbone metadata plus stream must fit the budget of
+    binary16 scales plus a 0.162 bits/weight sidecar, the stream must hold more
+    records than at 0.162 bits/weight, and the oracle must write the same stream."""
+    from synth import WORKLOADS, make_layer
+    wl = WORKLOADS["qwen2.5-3b_layer"]
+    mods = make_layer(wl, layer=1, device="cuda")
+    for m in mods:
+        m["W0"] = aw.awsrc_rtn_quantize(m["W"], sdq=True)["W0"]
+    shapes = [(m["rows"], m["cols"]) for m in mods]
+    N = sum(r * c for r, c in shapes)
+    kw = dict(C=wl.C, P=wl.P, b=wl.b, S=wl.S)
+    prm, oprm = aw.params(**kw), orc.params(**kw)
+    cands = aw.awsrc_encode_tiles(prm, mods)
+    assert aw.awsrc_workspace_status(cands._awsrc_workspace) == 0
+    rate2, saved = aw.awsrc_rate_with_sdq_savings(shapes, 0.162)
+    meta_fp16 = sum(aw.awsrc_backbone_metadata_bytes(r, c, False) for r, c in shapes)
+    meta_sdq = sum(aw.awsrc_backbone_metadata_bytes(r, c, True) for r, c in shapes)
+    assert saved == meta_fp16 - meta_sdq > 0
+    stream, counts, nbytes = aw.awsrc_select_records(prm, mods, cands, [rate2])
+    _, counts0, _ = aw.awsrc_select_records(prm, mods, cands, [0.162])
+    assert meta_sdq + int(nbytes[0]) <= meta_fp16 + orc.budget_bytes(0.162, N)
+    assert int(counts.sum()) > int(counts0.sum())
+    got = aw.candidates_to_numpy(cands)
+    ostream, ocounts, _ = orc.select_records(oprm, shapes, got, [rate2])
+    assert list(counts.cpu().numpy()) == list(ocounts)
+    assert bytes(stream.cpu().numpy()[: int(nbytes[0])]) == ostream
