@@ -59,11 +59,11 @@ def search_algorithmic_bytes(weights: int, tiles: int) -> int:
     return 4 * weights + 16 * tiles
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "6d1079712f4600ea47f9057a1375d6b7b73847b96f7a4fb1e394b59ed11273ca",
-                  "bytes_per_launch": 443179008 + 16896512,
+SEARCH_TRAFFIC = {"source_sha256": "e61d64bbea72a01eaeb5c93cf58021cee233ae96659755503b3a4161f4186609",
+                  "bytes_per_launch": 442491648 + 16684288,
                   # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
-                  "ncu_fma_pipe_pct": 38.26, "ncu_issue_active_pct": 45.31,
-                  "ncu_tensor_pipe_pct": 23.66}
+                  "ncu_fma_pipe_pct": 38.24, "ncu_issue_active_pct": 45.31,
+                  "ncu_tensor_pipe_pct": 23.65}
 
 
 def search_source_sha() -> str:
