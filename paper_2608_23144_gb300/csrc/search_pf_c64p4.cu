@@ -78,6 +78,27 @@ __device__ __forceinline__ float2 neg2(float2 v) { return make_float2(-v.x, -v.y
 
 __device__ __forceinline__ bool pivot_ok(float d) { return d > 0.0f && d <= 3.402823466e38f; }
 
+// rcp_rn on both components: the hardware approximations, then Markstein's
+// fused correction y + y (1 - x y) as two packed fmas (each component rounds
+// as the scalar form does). A component outside [2^-125, 2^125) takes
+// __frcp_rn instead, in a branch the active lanes take together only when
+// one of them needs it.
+__device__ __forceinline__ float2 rcp2_rn(float2 x) {
+  float yx, yy;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yx) : "f"(x.x));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yy) : "f"(x.y));
+  const float2 y = make_float2(yx, yy);
+  const float2 e = __ffma2_rn(make_float2(-x.x, -x.y), y, make_float2(1.0f, 1.0f));
+  float2 r = __ffma2_rn(y, e, y);
+  const bool fx = __float_as_uint(x.x) - 0x01000000u < 0x7D000000u - 0x01000000u;
+  const bool fy = __float_as_uint(x.y) - 0x01000000u < 0x7D000000u - 0x01000000u;
+  if (__any_sync(__activemask(), !(fx && fy))) {
+    if (!fx) r.x = __frcp_rn(x.x);
+    if (!fy) r.y = __frcp_rn(x.y);
+  }
+  return r;
+}
+
 // Fit of one seed pair of this thread's row; ah/al: atom p of the two seeds
 // at [2p], [2p+1]; qh/ql: product q (tri order) at [2q], [2q+1]. Returns b, the
 // off-diagonal G, alpha and whether each candidate's pivots are valid.
@@ -110,7 +131,7 @@ __device__ __forceinline__ void pf_pair_fit(const float* ah, const float* al, co
     for (int i = 0; i < k; ++i) dk = __ffma2_rn(nL[tri(k, i)], E[tri(k, i)], dk);
     *okx = *okx && pivot_ok(dk.x);
     *oky = *oky && pivot_ok(dk.y);
-    invD[k] = make_float2(rcp_rn(dk.x), rcp_rn(dk.y));
+    invD[k] = rcp2_rn(dk);
   }
   ldl_solve2<4>(nL, invD, bv, alpha);
 }
@@ -388,17 +409,23 @@ __global__ void __launch_bounds__(NT, 1)
       tc_fence_after();
       const uint32_t base = tmem + lane_base + (uint32_t)(tb * 256);
       float ah[8], al[8], qh[12], ql[12];
-      tmem_ld4(base + kYH + 8 * pi, ah);
-      tmem_ld4(base + kYH + 8 * pi + 4, ah + 4);
-      tmem_ld4(base + kYL + 8 * pi, al);
-      tmem_ld4(base + kYL + 8 * pi + 4, al + 4);
-#pragma unroll
-      for (int i = 0; i < 3; ++i) {
-        tmem_ld4(base + kDH + 12 * pi + 4 * i, qh + 4 * i);
-        tmem_ld4(base + kDL + 12 * pi + 4 * i, ql + 4 * i);
+      tmem_ld8(base + kYH + 8 * pi, ah);
+      tmem_ld8(base + kYL + 8 * pi, al);
+      // the pair's 12 product columns start at 12 pi: the 8-column load goes
+      // where it is 8-aligned (warp-uniform branch on pi)
+      if ((pi & 1) == 0) {
+        tmem_ld8(base + kDH + 12 * pi, qh);
+        tmem_ld4(base + kDH + 12 * pi + 8, qh + 8);
+        tmem_ld8(base + kDL + 12 * pi, ql);
+        tmem_ld4(base + kDL + 12 * pi + 8, ql + 8);
+      } else {
+        tmem_ld4(base + kDH + 12 * pi, qh);
+        tmem_ld8(base + kDH + 12 * pi + 4, qh + 4);
+        tmem_ld4(base + kDL + 12 * pi, ql);
+        tmem_ld8(base + kDL + 12 * pi + 4, ql + 4);
       }
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      tmem_tie4(ah); tmem_tie4(ah + 4); tmem_tie4(al); tmem_tie4(al + 4);
+      tmem_tie8(ah); tmem_tie8(al);
 #pragma unroll
       for (int i = 0; i < 3; ++i) { tmem_tie4(qh + 4 * i); tmem_tie4(ql + 4 * i); }
       tc_fence_before();
