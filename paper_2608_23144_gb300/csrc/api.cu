@@ -509,7 +509,7 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
   if (mode != AWSRC_DECODE_DENSE && mode != AWSRC_DECODE_INPLACE) return AWSRC_ERR_INVALID_ARG;
   int64_t T;
   if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
-  *bytes = kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256) + decode_scratch_bytes(T, mode);
+  *bytes = kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256) + decode_scratch_bytes(pr, T, mode);
   return AWSRC_OK;
 }
 
@@ -628,7 +628,7 @@ awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const aws
     a.masks = reinterpret_cast<const uint64_t*>(ws + kStatusBytes);
     const uint8_t* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
     a.map = reinterpret_cast<const unsigned long long*>(scratch);
-    a.rcodes = reinterpret_cast<const uint2*>(scratch + align_up((size_t)T * 8, 256));
+    a.rcodes = reinterpret_cast<const uint4*>(scratch + dense_scratch(pr, T).slots_off);
   }
   const cudaError_t e = launch_gemv(pr, a, M, (cudaStream_t)stream);
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "packed_gemv");

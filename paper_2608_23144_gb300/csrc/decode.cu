@@ -239,12 +239,92 @@ __device__ __forceinline__ void patch_vec(const Prm& pr, const Vec<TI, G>& w, ui
   }
 }
 
-// Dense-mode record pass: record k's codes go to codes[k] and map[tile] is
-// raised to (k + 1) << 32 | seed << 16 | scale field (map cleared to 0
+// Code tables of the dense decoder for P = 4 and C in {8, 16, 32, 64}
+// (code_tables()). With n_j = sum_p bit_p(j) 2^p the sign pattern of the four
+// atoms at element j (bit set: -1), k_j = sum_p code_p (1 - 2 bit_p(j)) is
+// T[n_j & 7] - 2 code_3 [n_j >= 8], with T[m] = code_3 + sum_{p<3} code_p
+// (1 - 2 bit_p(m)): eight signed bytes per record. Per seed and
+// window of 8 elements, nib holds (n_j & 7) in nibble j of x and, for elements
+// 0..3 and 4..7, a byte mask (0xFF where n_j >= 8) in y and z. A vector's k_j
+// then come from two byte permutes and two byte-wise subtractions, exactly.
+// With codes of at most 6 bits |k_j| <= 128, so T and k fit in signed bytes.
+__host__ __device__ __forceinline__ bool code_tables(const Prm& pr) {
+  return pr.P == 4 && pr.b <= 6 && pr.C <= 64 && (pr.C & 7) == 0;
+}
+
+// The record slot of the dense decoder: the codes (x, y; code p in byte p)
+// and, in table mode, T[0..7] (z, w).
+__device__ __forceinline__ uint4 record_slot(const Prm& pr, const DecRec& d) {
+  uint32_t t0 = 0u, t1 = 0u;
+  if (code_tables(pr)) {
+    const int c0 = code_of(d, 0), c1 = code_of(d, 1), c2 = code_of(d, 2), c3 = code_of(d, 3);
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+      const int v = c3 + ((m & 1) ? -c0 : c0) + ((m & 2) ? -c1 : c1) + ((m & 4) ? -c2 : c2);
+      const uint32_t b = (uint32_t)(v & 0xFF) << (8 * (m & 3));
+      if (m < 4) t0 |= b;
+      else t1 |= b;
+    }
+  }
+  return make_uint4(d.cw[0], d.cw[1], t0, t1);
+}
+
+// The nibble-major table of seed s from its four mask words (C <= 64, one
+// word per atom): window w of C / 8, lanes 0 .. C/8 - 1 of a warp.
+__device__ __forceinline__ void nib_window(const uint64_t* __restrict__ mk, int w, uint4* __restrict__ out) {
+  uint32_t lo = 0u, h0 = 0u, h1 = 0u;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int j = 8 * w + e;
+    uint32_t n = 0u;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) n |= (uint32_t)((mk[p] >> j) & 1ull) << p;
+    lo |= (n & 7u) << (4 * e);
+    if (n & 8u) {
+      if (e < 4) h0 |= 0xFFu << (8 * e);
+      else h1 |= 0xFFu << (8 * (e - 4));
+    }
+  }
+  *out = make_uint4(lo, h0, h1, 0u);
+}
+
+// Four consecutive k_j from the record slot's table: sel holds (n_j & 7) in
+// its four low nibbles, hm the byte mask of n_j >= 8.
+__device__ __forceinline__ void table_k4(const uint4& slot, uint32_t sel, uint32_t hm, float* k) {
+  const uint32_t c3x2 = ((slot.x >> 24) * 2u & 0xFFu) * 0x01010101u;  // 2 code_3, each byte
+  const uint32_t kb = __vsub4(__byte_perm(slot.z, slot.w, sel & 0xFFFFu), hm & c3x2);
+  const uint32_t ub = __vadd4(kb, 0x80808080u);  // k + 128 in [0, 255]
+#pragma unroll
+  for (int e = 0; e < 4; ++e)
+    k[e] = __fsub_rn(__uint_as_float(__byte_perm(ub, 0x4B000000u, 0x7650u + e)), 8388736.0f);  // 2^23 + 128
+}
+
+// patch_vec in table mode: the same k_j, hence the same results bit for bit.
+template <typename TI, typename TO, int G>
+__device__ __forceinline__ void patch_vec_tab(const Prm& pr, const Vec<TI, G>& w, const uint4& slot, uint4 nb,
+                                              int j0, float sc, Vec<TO, G>& o) {
+  float k[G];
+  if constexpr (G == 8) {
+    table_k4(slot, nb.x, nb.y, k);
+    table_k4(slot, nb.x >> 16, nb.z, k + 4);
+  } else {
+    const bool hi = (j0 & 4) != 0;
+    table_k4(slot, hi ? nb.x >> 16 : nb.x, hi ? nb.z : nb.y, k);
+  }
+  const float2 c2 = make_float2(pr.c, pr.c), s2 = make_float2(sc, sc);
+#pragma unroll
+  for (int e = 0; e < G; e += 2) {
+    const float2 r = __fmul2_rn(__fmul2_rn(make_float2(k[e], k[e + 1]), c2), s2);
+    Io2<TO>::st(o.v + e, __fadd2_rn(Io2<TI>::ld(w.v + e), r));
+  }
+}
+
+// Dense-mode record pass: record k's slot (record_slot) goes to codes[k] and
+// map[tile] is raised to (k + 1) << 32 | seed << 16 | scale field (map cleared to 0
 // beforehand). Records naming a tile or seed out of range, and tiles named
 // twice, raise kFaultRecord. Threads [i0, i0 + n) of a grid-stride range.
 __device__ __forceinline__ void map_records(const Prm& pr, const DecArgs& a, const uint8_t* __restrict__ stream,
-                                            unsigned long long* __restrict__ map, uint2* __restrict__ codes,
+                                            unsigned long long* __restrict__ map, uint4* __restrict__ codes,
                                             uint32_t* __restrict__ status, int64_t i0, int64_t n) {
   const int64_t Kd = stream_K(stream, a.K, a.kmax);
   const int64_t end = a.h + a.kmax * a.L;
@@ -256,7 +336,7 @@ __device__ __forceinline__ void map_records(const Prm& pr, const DecArgs& a, con
       atomicOr(status, kFaultRecord);
       continue;
     }
-    codes[k] = make_uint2(d.cw[0], d.cw[1]);
+    codes[k] = record_slot(pr, d);
     const unsigned long long e = ((unsigned long long)(k + 1) << 32) | ((unsigned long long)d.seed << 16) |
                                  (unsigned long long)(uint16_t)d.scale;
     if (atomicMax(map + tile, e) != 0ull) atomicOr(status, kFaultRecord);
@@ -414,8 +494,9 @@ struct FusedQ {
 template <typename TI, typename TO, int G, int PT>
 __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const __grid_constant__ DecArgs a,
                                                                  const unsigned long long* __restrict__ map,
-                                                                 const uint2* __restrict__ codes,
-                                                                 const uint64_t* __restrict__ masks) {
+                                                                 const uint4* __restrict__ codes,
+                                                                 const uint64_t* __restrict__ masks,
+                                                                 const uint4* __restrict__ nib) {
   static_assert(sizeof(Vec<TI, G>) == 16, "16-byte vectors");
   __shared__ FusedQ q[kFusedChunk];
   __shared__ int qn;
@@ -475,8 +556,14 @@ __global__ void __launch_bounds__(kFusedThreads, 4) fused_kernel(Prm pr, const _
       const uint32_t seed = (uint32_t)(x.e >> 16) & 0xFFFFu;
       const int j0 = (int)(x.g & ((1 << vshift) - 1)) * G;
       Vec<TO, G> o;
-      patch_vec<TI, TO, G, PT>(pr, w, __ldg(codes + k), masks + (size_t)seed * pr.P * pr.W + (j0 >> 6), j0,
-                               scale_of(pr, (int16_t)(uint16_t)(x.e & 0xFFFFull)), o);
+      const uint4 slot = __ldg(codes + k);
+      const float sc = scale_of(pr, (int16_t)(uint16_t)(x.e & 0xFFFFull));
+      if (PT == 4 && nib) {
+        patch_vec_tab<TI, TO, G>(pr, w, slot, __ldg(nib + (size_t)seed * (pr.C >> 3) + (j0 >> 3)), j0, sc, o);
+      } else {
+        patch_vec<TI, TO, G, PT>(pr, w, make_uint2(slot.x, slot.y), masks + (size_t)seed * pr.P * pr.W + (j0 >> 6),
+                                 j0, sc, o);
+      }
       st_stream(dst + x.g, o);
     }
     __syncthreads();
@@ -516,13 +603,20 @@ __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant
                                                    const uint8_t* __restrict__ stream,
                                                    uint64_t* __restrict__ masks,
                                                    unsigned long long* __restrict__ map,
-                                                   uint2* __restrict__ codes, uint32_t* __restrict__ status,
-                                                   int nb) {
+                                                   uint4* __restrict__ codes, uint32_t* __restrict__ status,
+                                                   uint4* __restrict__ nib, int nb) {
   pdl_trigger();  // the fused pass may launch now; it waits for this grid
   if ((int)blockIdx.x < nb) {
     __shared__ __align__(16) uint8_t bsm[8][kBasisSmem];
     const int warp = threadIdx.x >> 5;
-    basis_warp(pr, masks, (int64_t)blockIdx.x * 8 + warp, pr.S, bsm[warp]);
+    const int64_t w = (int64_t)blockIdx.x * 8 + warp;
+    basis_warp(pr, masks, w, pr.S, bsm[warp]);
+    if (nib && w < pr.S) {  // table mode: one selector per warp (C <= 64), one mask word per atom
+      __syncwarp();  // the masks this warp just wrote
+      const int lane = threadIdx.x & 31;
+      if (lane < (pr.C >> 3))
+        nib_window(masks + (size_t)w * 4, lane, nib + (size_t)w * (pr.C >> 3) + lane);
+    }
     return;
   }
   map_records(pr, a, stream, map, codes, status, (int64_t)(blockIdx.x - nb) * blockDim.x + threadIdx.x,
@@ -531,7 +625,7 @@ __global__ void __launch_bounds__(256) prep_kernel(Prm pr, const __grid_constant
 
 template <typename TI, typename TO, int G>
 cudaError_t launch_fused_t(const Prm& pr, const DecArgs& a, const unsigned long long* map,
-                           const uint2* codes, const uint64_t* masks, cudaStream_t st) {
+                           const uint4* codes, const uint64_t* masks, const uint4* nib, cudaStream_t st) {
   int64_t maxg = 0;
   for (int i = 0; i < a.n_mod; ++i) maxg = std::max<int64_t>(maxg, a.m[i].rows * a.m[i].cols / G);
   int dev = 0, nsm = 148;
@@ -541,21 +635,21 @@ cudaError_t launch_fused_t(const Prm& pr, const DecArgs& a, const unsigned long 
   const int64_t gx = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)nsm * 8));
   const dim3 grid((unsigned)gx, (unsigned)a.n_mod);
   cudaError_t e = pr.P == 4 ? launch_pdl(fused_kernel<TI, TO, G, 4>, grid, dim3(kFusedThreads), st, pr, a, map,
-                                         codes, masks)
+                                         codes, masks, nib)
                             : launch_pdl(fused_kernel<TI, TO, G, 0>, grid, dim3(kFusedThreads), st, pr, a, map,
-                                         codes, masks);
+                                         codes, masks, nib);
   note_launches(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_fused(const Prm& pr, const DecArgs& a, int w0_dtype, int out_dtype,
-                         const unsigned long long* map, const uint2* codes, const uint64_t* masks,
-                         cudaStream_t st) {
+                         const unsigned long long* map, const uint4* codes, const uint64_t* masks,
+                         const uint4* nib, cudaStream_t st) {
   const bool f32in = (w0_dtype == AWSRC_DTYPE_F32), f32out = (out_dtype == AWSRC_DTYPE_F32);
-  if (f32in && f32out) return launch_fused_t<float, float, 4>(pr, a, map, codes, masks, st);
-  if (f32in) return launch_fused_t<float, __nv_bfloat16, 4>(pr, a, map, codes, masks, st);
-  if (f32out) return launch_fused_t<__nv_bfloat16, float, 8>(pr, a, map, codes, masks, st);
-  return launch_fused_t<__nv_bfloat16, __nv_bfloat16, 8>(pr, a, map, codes, masks, st);
+  if (f32in && f32out) return launch_fused_t<float, float, 4>(pr, a, map, codes, masks, nib, st);
+  if (f32in) return launch_fused_t<float, __nv_bfloat16, 4>(pr, a, map, codes, masks, nib, st);
+  if (f32out) return launch_fused_t<__nv_bfloat16, float, 8>(pr, a, map, codes, masks, nib, st);
+  return launch_fused_t<__nv_bfloat16, __nv_bfloat16, 8>(pr, a, map, codes, masks, nib, st);
 }
 
 // copy: stream the modules of `a`; basis: also generate the masks (an extra
@@ -622,13 +716,23 @@ cudaError_t launch_group(const Prm& pr, const DecArgs& a, int w0_dtype, int out_
 
 }  // namespace
 
+DenseScratch dense_scratch(const Prm& pr, int64_t T) {
+  DenseScratch d;
+  d.slots_off = align_up((size_t)T * 8, 256);
+  d.nib_off = d.slots_off + align_up((size_t)T * 16, 256);
+  d.bytes = d.nib_off + (code_tables(pr) ? align_up((size_t)pr.S * (pr.C / 8) * 16, 256) : 0);
+  return d;
+}
+
 // Dense preparation: clear the tile map (and the fault word), then generate
-// the masks and unpack the records into the map and the code array of
-// `scratch` (map: align_up(T * 8, 256) bytes, then 8 bytes per record).
+// the masks (and, in table mode, the nibble tables) and unpack the records
+// into the map and the record slots of `scratch` (layout: dense_scratch()).
 cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, const uint8_t* stream, int64_t K,
                               int64_t kmax, uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
+  const DenseScratch ds = dense_scratch(pr, T);
   unsigned long long* map = static_cast<unsigned long long*>(scratch);
-  uint2* codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
+  uint4* codes = reinterpret_cast<uint4*>(static_cast<uint8_t*>(scratch) + ds.slots_off);
+  uint4* nib = code_tables(pr) ? reinterpret_cast<uint4*>(static_cast<uint8_t*>(scratch) + ds.nib_off) : nullptr;
   DecArgs a;
   a.n_mod = 0;
   a.T = T; a.L = L; a.h = h; a.K = K; a.kmax = kmax;
@@ -648,7 +752,7 @@ cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, co
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   e = launch_pdl(prep_kernel, dim3((unsigned)(nb + nr)), dim3(256), st, pr, a, stream, masks, map, codes, status,
-                 nb);
+                 nib, nb);
   note_launches(1);
   if (e == cudaSuccess) e = cudaGetLastError();
   return e;
@@ -663,14 +767,17 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st) {
   const bool fused = decode_clears_status(pr, mode) && scratch != nullptr;
   unsigned long long* map = nullptr;
-  uint2* codes = nullptr;
+  uint4* codes = nullptr;
+  uint4* nib = nullptr;
   // the record-by-record patch with a workspace claims tiles first (without
   // one, as for the no-allocation entry point, the stream must name each tile
   // at most once)
   uint32_t* claim = (!fused && scratch != nullptr) ? static_cast<uint32_t*>(scratch) : nullptr;
   if (fused) {
+    const DenseScratch ds = dense_scratch(pr, T);
     map = static_cast<unsigned long long*>(scratch);
-    codes = reinterpret_cast<uint2*>(static_cast<uint8_t*>(scratch) + align_up((size_t)T * 8, 256));
+    codes = reinterpret_cast<uint4*>(static_cast<uint8_t*>(scratch) + ds.slots_off);
+    if (code_tables(pr)) nib = reinterpret_cast<uint4*>(static_cast<uint8_t*>(scratch) + ds.nib_off);
     const cudaError_t e = launch_dense_prep(pr, T, L, h, stream, K, kmax, masks, scratch, status, st);
     if (e != cudaSuccess) return e;
   }
@@ -699,7 +806,7 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
     a.claim = claim;
     for (int i = 0; i < a.n_mod; ++i) a.m[i] = mods[i0 + i];
     const cudaError_t e =
-        fused ? launch_fused(pr, a, mods[i0].w0_dtype, out_dtype, map, codes, masks, st)
+        fused ? launch_fused(pr, a, mods[i0].w0_dtype, out_dtype, map, codes, masks, nib, st)
               : launch_group(pr, a, mods[i0].w0_dtype, out_dtype, mode == AWSRC_DECODE_DENSE, i0 == 0, stream,
                              masks, status, st);
     if (e != cudaSuccess) return e;
@@ -710,11 +817,10 @@ cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64
 
 bool decode_clears_status(const Prm& pr, int mode) { return mode == AWSRC_DECODE_DENSE && pr.C >= 8; }
 
-size_t decode_scratch_bytes(int64_t T, int mode) {
-  // dense: tile -> record map (8 B per tile) and each record's codes (8 B, at
-  // most one record per tile); in-place: one claim word per tile
+size_t decode_scratch_bytes(const Prm& pr, int64_t T, int mode) {
+  // dense: dense_scratch(); in-place: one claim word per tile
   if (mode != AWSRC_DECODE_DENSE) return align_up((size_t)T * 4, 256);
-  return align_up((size_t)T * 8, 256) + align_up((size_t)T * 8, 256);
+  return dense_scratch(pr, T).bytes;
 }
 
 }  // namespace awsrc

@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(32 * kGemvWarps) gemv_kernel(Prm pr, GemvArgs 
         const int64_t k = (int64_t)(en >> 32) - 1;
         const uint32_t seed = (uint32_t)(en >> 16) & 0xFFFFu;
         const float sc = sidecar_scale(pr, (int16_t)(uint16_t)(en & 0xFFFFull));
-        const uint2 cw = __ldg(a.rcodes + k);
+        const uint2 cw = __ldg(reinterpret_cast<const uint2*>(a.rcodes + k));  // the slot's codes
         const int jt = (int)(((gb + u) * 128 + 4 * lane) & (pr.C - 1));  // position in the tile
         const uint64_t* mk = a.masks + (size_t)seed * pr.P * pr.W + (jt >> 6);
         int kj[4] = {0, 0, 0, 0};
@@ -275,7 +275,7 @@ __global__ void __launch_bounds__(32 * kGemvWarps) gemv_warp_kernel(Prm pr, Gemv
 #pragma unroll
         for (int i = 0; i < kPrefetchWords; ++i) mw[i] = 0ull;
         if (ent != 0ull) {
-          cw = __ldg(a.rcodes + ((int64_t)(ent >> 32) - 1));
+          cw = __ldg(reinterpret_cast<const uint2*>(a.rcodes + ((int64_t)(ent >> 32) - 1)));
           if (pre) {
             const uint64_t* mk = a.masks + (size_t)((uint32_t)(ent >> 16) & 0xFFFFu) * pr.P * pr.W;
 #pragma unroll

@@ -89,7 +89,14 @@ struct DecodeMod {
 cudaError_t launch_decode(const Prm& pr, int n_mod, const DecodeMod* mods, int64_t T, int64_t L,
                           int64_t h, const uint8_t* stream, int64_t K, int64_t kmax, int out_dtype, int mode,
                           uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
-size_t decode_scratch_bytes(int64_t T, int mode);
+size_t decode_scratch_bytes(const Prm& pr, int64_t T, int mode);
+// Dense scratch: the tile map (8 B per tile, from offset 0), then one 16-byte
+// slot per record (codes x, y; code tables z, w) at slots_off, then (P = 4,
+// C <= 64) the nibble tables at nib_off.
+struct DenseScratch {
+  size_t slots_off, nib_off, bytes;
+};
+DenseScratch dense_scratch(const Prm& pr, int64_t T);
 cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, const uint8_t* stream, int64_t K,
                               int64_t kmax, uint64_t* masks, void* scratch, uint32_t* status, cudaStream_t st);
 // The dense fused decoder clears the fault word itself (no separate memset).
@@ -104,7 +111,7 @@ struct GemvArgs {
   const int8_t* sdq_codes;       // per group (sdq)
   const float* sdq_consts;       // (mean, step) per 256 groups (sdq)
   const unsigned long long* map; // tile map of the prepared sidecar, or null (no residual)
-  const uint2* rcodes;           // per-record codes of the prepared sidecar
+  const uint4* rcodes;           // per-record slots of the prepared sidecar (codes in x, y)
   const uint64_t* masks;         // basis masks of the prepared sidecar
   const float* x;                // M x cols
   float* y;                      // M x rows
