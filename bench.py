@@ -296,9 +296,10 @@ def backbone_and_serving(dev, prm, mods, outs, stream, records, hbm_gbs):
     of each call. Algorithmic bytes: the backbone reads W (2 B/weight) and
     writes the 4-bit codes, the SDQ scale codes and constants and W0 (BF16);
     the GEMV (one vector) reads the codes, the SDQ scale codes and constants,
-    the prepared sidecar's tile map (8 B per tile), record codes (8 B per
-    record) and masks, x and writes y. cuBLAS's BF16 GEMV of the decoded
-    weights (2 B/weight) is timed the same way for context."""
+    the prepared sidecar's tile map (8 B per tile), record slots (16 B per
+    record) and nibble tables, x and writes y; it is timed as seven calls and
+    as one batched call. cuBLAS's BF16 GEMV of the decoded weights (2 B/weight)
+    is timed the same way for context."""
     import torch
     import paper_2608_23144_gb300 as aw
     reps = 10
@@ -320,6 +321,11 @@ def backbone_and_serving(dev, prm, mods, outs, stream, records, hbm_gbs):
     def gemv():
         for i in range(len(mods)):
             aw.awsrc_packed_gemv(prm, shapes, i, bb[i], xs[i], sidecar=side, y=ys[i])
+
+    batch = [(i, bb[i], xs[i], ys[i]) for i in range(len(mods))]
+
+    def gemv_batch():
+        aw.awsrc_packed_gemv_batch(prm, shapes, batch, sidecar=side)
 
     def dense():
         for o, x, y in zip(outs, xb, yb):
@@ -347,16 +353,22 @@ def backbone_and_serving(dev, prm, mods, outs, stream, records, hbm_gbs):
 
     q_ms = graph_ms(quantise)
     g_ms = graph_ms(gemv)
+    b_ms = graph_ms(gemv_batch)
     d_ms = graph_ms(dense)
     q_bytes = N * 2 + N // 2 + G + 8 * ((G + 255) // 256) + N * 2
-    g_bytes = (N // 2 + G + 8 * ((G + 255) // 256) + 8 * T + 8 * records + 8 * prm.S * prm.P
+    # codes, SDQ codes and constants, tile map (8 B per tile), record slots
+    # (16 B per record), the seeds' nibble tables (16 B per 8 elements), x, y
+    g_bytes = (N // 2 + G + 8 * ((G + 255) // 256) + 8 * T + 16 * records + 16 * prm.S * (prm.C // 8)
                + 4 * sum(m["cols"] + m["rows"] for m in mods))
     return {"workload": "the 7 modules of the benchmark layer (77,070,336 weights), 0.162-bpw stream; "
-                        "7 calls per figure, captured in a CUDA graph",
+                        "7 calls per figure (or one batched call), captured in a CUDA graph",
             "rtn_sdq": {"ms": q_ms, "gbs": q_bytes / (q_ms * 1e-3) / 1e9,
                         "frac_of_hbm": q_bytes / (q_ms * 1e-3) / 1e9 / hbm_gbs, "bytes": q_bytes},
-            "packed_gemv_m1": {"ms": g_ms, "gbs": g_bytes / (g_ms * 1e-3) / 1e9,
-                               "frac_of_hbm": g_bytes / (g_ms * 1e-3) / 1e9 / hbm_gbs, "bytes": g_bytes},
+            "packed_gemv_m1": {"ms": b_ms, "gbs": g_bytes / (b_ms * 1e-3) / 1e9,
+                               "frac_of_hbm": g_bytes / (b_ms * 1e-3) / 1e9 / hbm_gbs, "bytes": g_bytes,
+                               "call": "awsrc_packed_gemv_batch, the 7 modules in one launch"},
+            "packed_gemv_m1_per_module_calls": {"ms": g_ms, "gbs": g_bytes / (g_ms * 1e-3) / 1e9,
+                                                "frac_of_hbm": g_bytes / (g_ms * 1e-3) / 1e9 / hbm_gbs},
             "cublas_bf16_gemv_of_decoded_m1_ms": d_ms}
 
 

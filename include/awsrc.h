@@ -413,9 +413,10 @@ awsrc_status awsrc_decode_apply_inplace_noalloc(const awsrc_params* prm, int32_t
  *   aligned; y is M x rows): W0_ij = fl(q_ij * s_eff) from the packed backbone
  *   (awsrc_rtn_quantize's outputs; binary16 scales or SDQ), r_ij =
  *   fl(fl(k_j * C^-1/2) * scale) on the tiles the sidecar names (none when
- *   `sidecar` is NULL), both accumulated in binary32 with fma. The result
- *   equals the double-precision product of those values within binary32
- *   summation error (bounded by (2*cols/32 + 8) * 2^-24 * sum_j |(W0 + r) x|).
+ *   `sidecar` is NULL), both accumulated in binary32 with fma (the residual
+ *   terms in their own sums). The result equals the double-precision product
+ *   sum_j (W0_ij + r_ij) x_j, r_ij = k_j C^-1/2 scale, within
+ *   (cols / min(C, 32) + 32) * 2^-24 * sum_j (|W0_ij x_j| + |r_ij x_j|).
  *   The module needs cols % 128 == 0.
  * Errors: INVALID_ARG, SHAPE, UNSUPPORTED, WORKSPACE, CUDA.
  */
@@ -436,6 +437,28 @@ awsrc_status awsrc_sidecar_prepare(const awsrc_params* prm, int32_t n_mod, const
 awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods, int32_t m,
                                const awsrc_packed_weights* pw, const void* sidecar, size_t sidecar_bytes,
                                int32_t M, const float* x, float* y, void* stream);
+
+/*
+ * awsrc_packed_gemv_batch — awsrc_packed_gemv for 1 <= n_task <= 16 tasks in
+ * one launch (tasks whose M x cols inputs exceed 96 KB take one more launch
+ * each): task i computes y_i = (W0 + r_hat) x_i for module tasks[i].m with
+ * its packed backbone tasks[i].pw, all with the same sidecar and M. Tasks may
+ * name the same module and share x (the q/k/v or gate/up projections of one
+ * input); y arrays must not overlap each other or any input. Each y_i is
+ * bit-identical to the single call's. Errors: as awsrc_packed_gemv;
+ * UNSUPPORTED for n_task > 16.
+ */
+typedef struct awsrc_gemv_task {
+  int32_t m;                 /* module index in the list */
+  int32_t pad_;
+  awsrc_packed_weights pw;   /* module m's packed backbone */
+  const float* x;            /* M x cols, 16-byte aligned */
+  float* y;                  /* M x rows */
+} awsrc_gemv_task;
+
+awsrc_status awsrc_packed_gemv_batch(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                     int32_t n_task, const awsrc_gemv_task* tasks, const void* sidecar,
+                                     size_t sidecar_bytes, int32_t M, void* stream);
 
 /*
  * awsrc_workspace_status — synchronises `stream`, then reads and clears the

@@ -758,8 +758,10 @@ void orc_rtn_quantize(int64_t rows, int64_t cols, int group, int sdq, int block,
 /* y[v][i] = sum_j (W0_ij + r_ij) x[v][j] in double, W0_ij = q_ij * s_eff    */
 /* (the backbone's binary32 value), r the decoder's residual (Sec. 3.2) on    */
 /* the module's tiles named by the first K records, in double:                */
-/* k_j * C^-1/2 * scale. yabs = sum_j |(W0_ij + r_ij) x[v][j]| bounds the    */
-/* rounding of any binary32 evaluation. x: M x cols, y and yabs: M x rows.   */
+/* k_j * C^-1/2 * scale. yabs = sum_j (|W0_ij x[v][j]| + |r_ij x[v][j]|),    */
+/* the magnitude a binary32 evaluation that sums the backbone's and the      */
+/* residual's terms separately is rounded against. x: M x cols, y and yabs:  */
+/* M x rows.                                                                  */
 /* ------------------------------------------------------------------------ */
 int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_rows, const int64_t* mod_cols,
                     int32_t m, int group, const int8_t* q, const float* s_eff, const uint8_t* stream, int64_t K,
@@ -773,7 +775,12 @@ int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_row
   const int64_t rows = mod_rows[m], cols = mod_cols[m], Tm = rows * cols / C, n_cb = cols / C;
   const int64_t h = orc_header_bytes(n_mod), L = orc_record_bytes(prm, T);
   double* Wt = (double*)malloc(sizeof(double) * (size_t)(rows * cols));
-  if (!Wt) return -1;
+  double* Rt = (double*)calloc((size_t)(rows * cols), sizeof(double));
+  if (!Wt || !Rt) {
+    free(Wt);
+    free(Rt);
+    return -1;
+  }
   for (int64_t i = 0; i < rows * cols; ++i) Wt[i] = (double)((float)q[i] * s_eff[i / group]);
   const double c = 1.0 / sqrt((double)C);
   uint8_t sign[256], neg[8 * 256];
@@ -792,20 +799,21 @@ int orc_packed_gemv(const orc_params* prm, int32_t n_mod, const int64_t* mod_row
     for (int j = 0; j < C; ++j) {
       int kj = 0;
       for (int p = 0; p < P; ++p) kj += neg[p * C + j] ? -cd.code[p] : cd.code[p];
-      Wt[base + j] += (double)kj * c * sc;
+      Rt[base + j] = (double)kj * c * sc;  /* a later record of the tile replaces it */
     }
   }
   for (int v = 0; v < M; ++v)
     for (int64_t i = 0; i < rows; ++i) {
       double acc = 0.0, aabs = 0.0;
       for (int64_t j = 0; j < cols; ++j) {
-        const double t = Wt[i * cols + j] * (double)x[(int64_t)v * cols + j];
-        acc += t;
-        aabs += fabs(t);
+        const double xj = (double)x[(int64_t)v * cols + j];
+        acc += (Wt[i * cols + j] + Rt[i * cols + j]) * xj;
+        aabs += fabs(Wt[i * cols + j] * xj) + fabs(Rt[i * cols + j] * xj);
       }
       y[(int64_t)v * rows + i] = acc;
       yabs[(int64_t)v * rows + i] = aabs;
     }
   free(Wt);
+  free(Rt);
   return bad;
 }

@@ -10,8 +10,8 @@ binding with the same entry-point names:
 * ``awsrc_decode_apply``   decoder, W_hat = W0 + B_s alpha_hat (Eq. 1)
 * ``awsrc_rtn_quantize``   the RTN-INT4 backbone W0 = Q(W) with optional scale
   double quantisation (Sec. 3.3)
-* ``awsrc_sidecar_prepare`` / ``awsrc_packed_gemv``  the sidecar applied inside a
-  packed INT4 product, W_hat never formed
+* ``awsrc_sidecar_prepare`` / ``awsrc_packed_gemv`` / ``awsrc_packed_gemv_batch``  the
+  sidecar applied inside a packed INT4 product, W_hat never formed
 """
 from ._binding import (  # noqa: F401
     CANDIDATE_DTYPE,
@@ -37,6 +37,7 @@ from ._binding import (  # noqa: F401
     awsrc_rate_with_sdq_savings,
     awsrc_sidecar_prepare,
     awsrc_packed_gemv,
+    awsrc_packed_gemv_batch,
     shape_modules,
     awsrc_header_bytes,
     awsrc_kernel_launches,

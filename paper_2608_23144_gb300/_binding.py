@@ -60,6 +60,11 @@ class PackedWeights(ct.Structure):
                 ("sdq_consts", ct.c_void_p), ("sdq", ct.c_int32), ("pad_", ct.c_int32)]
 
 
+class GemvTask(ct.Structure):
+    _fields_ = [("m", ct.c_int32), ("pad_", ct.c_int32), ("pw", PackedWeights), ("x", ct.c_void_p),
+                ("y", ct.c_void_p)]
+
+
 def params(C=64, P=4, b=4, S=4096, b_e=8, e_bias=0, scale_mode=SCALE_POW2, permute=1,
            variant=VARIANT_U, ridge_rel=1e-6, gen_seed=0) -> Params:
     return Params(C, P, b, S, b_e, e_bias, scale_mode, permute, variant,
@@ -131,6 +136,9 @@ def _load():
     L.awsrc_packed_gemv.restype = st
     L.awsrc_packed_gemv.argtypes = [P(Params), ct.c_int32, P(Module), ct.c_int32, P(PackedWeights), vp, sz,
                                     ct.c_int32, vp, vp, vp]
+    L.awsrc_packed_gemv_batch.restype = st
+    L.awsrc_packed_gemv_batch.argtypes = [P(Params), ct.c_int32, P(Module), ct.c_int32, P(GemvTask), vp, sz,
+                                          ct.c_int32, vp]
     return L
 
 
@@ -333,12 +341,9 @@ def awsrc_sidecar_prepare(prm: Params, shapes, stream_bytes: torch.Tensor, K: in
     return workspace
 
 
-def awsrc_packed_gemv(prm: Params, shapes, m: int, backbone: Dict[str, torch.Tensor], x: torch.Tensor,
-                      sidecar: Optional[torch.Tensor] = None, y: Optional[torch.Tensor] = None,
-                      stream=None) -> torch.Tensor:
-    """y = (W0 + r_hat) x for module m (x: M x cols float32); backbone holds
-    awsrc_rtn_quantize's codes and scales (or SDQ codes and constants)."""
-    mods = shape_modules(shapes)
+def _gemv_operands(shapes, m: int, backbone: Dict[str, torch.Tensor], x: torch.Tensor,
+                   y: Optional[torch.Tensor]):
+    """Checks one product's operands; returns (x as M x cols, y, PackedWeights)."""
     rows, cols = shapes[m]
     _require(x, "x", dtype=torch.float32)
     if x.numel() % cols != 0:
@@ -357,14 +362,52 @@ def awsrc_packed_gemv(prm: Params, shapes, m: int, backbone: Dict[str, torch.Ten
                  numel=2 * ((G + 255) // 256), device=dev)
     else:
         _require(backbone["scales"], "backbone['scales']", dtype=torch.int16, numel=G, device=dev)
-    if sidecar is not None:
-        _require(sidecar, "sidecar", dtype=torch.uint8, device=dev)
     pw = PackedWeights(_dev_ptr(backbone["codes"]), None if sdq else _dev_ptr(backbone["scales"]),
                        _dev_ptr(backbone.get("sdq_codes")), _dev_ptr(backbone.get("sdq_consts")), int(sdq), 0)
+    return x, y, pw
+
+
+def awsrc_packed_gemv(prm: Params, shapes, m: int, backbone: Dict[str, torch.Tensor], x: torch.Tensor,
+                      sidecar: Optional[torch.Tensor] = None, y: Optional[torch.Tensor] = None,
+                      stream=None) -> torch.Tensor:
+    """y = (W0 + r_hat) x for module m (x: M x cols float32); backbone holds
+    awsrc_rtn_quantize's codes and scales (or SDQ codes and constants)."""
+    mods = shape_modules(shapes)
+    _require(x, "x", dtype=torch.float32)
+    if sidecar is not None:
+        _require(sidecar, "sidecar", dtype=torch.uint8, device=x.device)
+    x, y, pw = _gemv_operands(shapes, m, backbone, x, y)
     _check(lib.awsrc_packed_gemv(ct.byref(prm), len(shapes), mods, m, ct.byref(pw), _dev_ptr(sidecar),
                                  0 if sidecar is None else sidecar.numel(), x.shape[0], _dev_ptr(x), _dev_ptr(y),
                                  _stream(stream)), "packed_gemv")
     return y
+
+
+def awsrc_packed_gemv_batch(prm: Params, shapes, tasks, sidecar: Optional[torch.Tensor] = None,
+                            stream=None) -> List[torch.Tensor]:
+    """Several products in one launch: tasks is a list of (m, backbone, x) or
+    (m, backbone, x, y) with the same number M of vectors; returns the y's."""
+    mods = shape_modules(shapes)
+    if sidecar is not None and tasks:
+        _require(tasks[0][2], "x", dtype=torch.float32)
+        _require(sidecar, "sidecar", dtype=torch.uint8, device=tasks[0][2].device)
+    arr = (GemvTask * len(tasks))()
+    ys, Ms, dev = [], set(), None
+    for i, t in enumerate(tasks):
+        m, backbone, x = t[0], t[1], t[2]
+        x, y, pw = _gemv_operands(shapes, m, backbone, x, t[3] if len(t) > 3 else None)
+        if dev is not None and x.device != dev:
+            raise ValueError("every task's tensors must be on one device")
+        dev = x.device
+        Ms.add(x.shape[0])
+        arr[i] = GemvTask(m, 0, pw, _dev_ptr(x), _dev_ptr(y))
+        ys.append((x, y))  # x kept alive with y until the call returns
+    if len(Ms) != 1:
+        raise ValueError(f"tasks must share M, got {sorted(Ms)}")
+    _check(lib.awsrc_packed_gemv_batch(ct.byref(prm), len(shapes), mods, len(tasks), arr, _dev_ptr(sidecar),
+                                       0 if sidecar is None else sidecar.numel(), Ms.pop(), _stream(stream)),
+           "packed_gemv_batch")
+    return [y for _, y in ys]
 
 
 def awsrc_gen_basis(prm: Params, stream=None, device="cuda") -> torch.Tensor:

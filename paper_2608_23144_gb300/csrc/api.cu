@@ -184,6 +184,57 @@ awsrc_status make_prm(const awsrc_params* p, Prm* out) {
   return AWSRC_OK;
 }
 
+namespace {
+
+// One GEMV task: module m of the list with its packed backbone, x and y.
+awsrc_status gemv_task(const Prm& pr, int32_t n_mod, const awsrc_module* mods, int32_t m,
+                       const awsrc_packed_weights* pw, const float* x, float* y, GemvTask* t) {
+  if (m < 0 || m >= n_mod || !pw || !x || !y) return AWSRC_ERR_INVALID_ARG;
+  if (mods[m].cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
+  if (pw->sdq != 0 && pw->sdq != 1) return AWSRC_ERR_INVALID_ARG;
+  if (!pw->codes || (pw->sdq ? (!pw->sdq_codes || !pw->sdq_consts) : !pw->scales)) return AWSRC_ERR_INVALID_ARG;
+  if (!aligned(pw->codes, 4) || !aligned(pw->scales, 2) || !aligned(pw->sdq_consts, 8) || !aligned(x, 16) ||
+      !aligned(y, 4))
+    return AWSRC_ERR_INVALID_ARG;
+  *t = GemvTask{};
+  t->rows = mods[m].rows;
+  t->cols = mods[m].cols;
+  for (int i = 0; i < m; ++i) t->tile_off += mods[i].rows * (mods[i].cols / pr.C);
+  t->sdq = pw->sdq;
+  t->codes = reinterpret_cast<const uint16_t*>(pw->codes);
+  t->scales = pw->scales;
+  t->sdq_codes = pw->sdq_codes;
+  t->sdq_consts = pw->sdq_consts;
+  t->x = x;
+  t->y = y;
+  return AWSRC_OK;
+}
+
+// The sidecar's arrays (none when `sidecar` is null).
+awsrc_status gemv_sidecar(const awsrc_params* prm, const Prm& pr, int32_t n_mod, const awsrc_module* mods,
+                          int64_t T, const void* sidecar, size_t sidecar_bytes, GemvArgs* a) {
+  a->map = nullptr;
+  a->slots = nullptr;
+  a->masks = nullptr;
+  a->nib = nullptr;
+  if (!sidecar) return AWSRC_OK;
+  size_t need;
+  const awsrc_status s = awsrc_sidecar_workspace_bytes(prm, n_mod, mods, &need);
+  if (s != AWSRC_OK) return s;
+  if (sidecar_bytes < need) return AWSRC_ERR_WORKSPACE;
+  if (!aligned(sidecar, 256)) return AWSRC_ERR_INVALID_ARG;
+  const uint8_t* ws = static_cast<const uint8_t*>(sidecar);
+  const uint8_t* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
+  const DenseScratch ds = dense_scratch(pr, T);
+  a->masks = reinterpret_cast<const uint64_t*>(ws + kStatusBytes);
+  a->map = reinterpret_cast<const unsigned long long*>(scratch);
+  a->slots = reinterpret_cast<const uint4*>(scratch + ds.slots_off);
+  if (gemv_tables(pr)) a->nib = reinterpret_cast<const uint4*>(scratch + ds.nib_off);
+  return AWSRC_OK;
+}
+
+}  // namespace
+
 }  // namespace awsrc
 
 using namespace awsrc;
@@ -596,40 +647,31 @@ awsrc_status awsrc_sidecar_prepare(const awsrc_params* prm, int32_t n_mod, const
 awsrc_status awsrc_packed_gemv(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods, int32_t m,
                                const awsrc_packed_weights* pw, const void* sidecar, size_t sidecar_bytes,
                                int32_t M, const float* x, float* y, void* stream) {
+  awsrc_gemv_task task{};
+  task.m = m;
+  if (pw) task.pw = *pw;
+  task.x = x;
+  task.y = y;
+  if (!pw) return AWSRC_ERR_INVALID_ARG;
+  return awsrc_packed_gemv_batch(prm, n_mod, mods, 1, &task, sidecar, sidecar_bytes, M, stream);
+}
+
+awsrc_status awsrc_packed_gemv_batch(const awsrc_params* prm, int32_t n_mod, const awsrc_module* mods,
+                                     int32_t n_task, const awsrc_gemv_task* tasks, const void* sidecar,
+                                     size_t sidecar_bytes, int32_t M, void* stream) {
   Prm pr;
   awsrc_status s = make_prm(prm, &pr);
   if (s != AWSRC_OK) return s;
   int64_t T;
   if ((s = check_modules(pr, n_mod, mods, false, &T)) != AWSRC_OK) return s;
-  if (m < 0 || m >= n_mod || !pw || !x || !y || M < 1 || M > 8) return AWSRC_ERR_INVALID_ARG;
-  if (mods[m].cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
-  if (pw->sdq != 0 && pw->sdq != 1) return AWSRC_ERR_INVALID_ARG;
-  if (!pw->codes || (pw->sdq ? (!pw->sdq_codes || !pw->sdq_consts) : !pw->scales)) return AWSRC_ERR_INVALID_ARG;
-  if (!aligned(pw->codes, 4) || !aligned(pw->scales, 2) || !aligned(pw->sdq_consts, 8) || !aligned(x, 16) ||
-      !aligned(y, 4))
-    return AWSRC_ERR_INVALID_ARG;
+  if (!tasks || n_task < 1 || M < 1 || M > 8) return AWSRC_ERR_INVALID_ARG;
+  if (n_task > kMaxGemvTasks) return AWSRC_ERR_UNSUPPORTED;
   GemvArgs a{};
-  a.rows = mods[m].rows;
-  a.cols = mods[m].cols;
-  for (int i = 0; i < m; ++i) a.tile_off += mods[i].rows * (mods[i].cols / pr.C);
-  a.sdq = pw->sdq;
-  a.codes = reinterpret_cast<const uint16_t*>(pw->codes);
-  a.scales = pw->scales;
-  a.sdq_codes = pw->sdq_codes;
-  a.sdq_consts = pw->sdq_consts;
-  a.x = x;
-  a.y = y;
-  if (sidecar) {
-    size_t need;
-    if ((s = awsrc_sidecar_workspace_bytes(prm, n_mod, mods, &need)) != AWSRC_OK) return s;
-    if (sidecar_bytes < need) return AWSRC_ERR_WORKSPACE;
-    if (!aligned(sidecar, 256)) return AWSRC_ERR_INVALID_ARG;
-    const uint8_t* ws = static_cast<const uint8_t*>(sidecar);
-    a.masks = reinterpret_cast<const uint64_t*>(ws + kStatusBytes);
-    const uint8_t* scratch = ws + kStatusBytes + align_up((size_t)pr.S * pr.P * pr.W * 8, 256);
-    a.map = reinterpret_cast<const unsigned long long*>(scratch);
-    a.rcodes = reinterpret_cast<const uint4*>(scratch + dense_scratch(pr, T).slots_off);
-  }
+  a.n_task = n_task;
+  for (int i = 0; i < n_task; ++i)
+    if ((s = gemv_task(pr, n_mod, mods, tasks[i].m, &tasks[i].pw, tasks[i].x, tasks[i].y, &a.t[i])) != AWSRC_OK)
+      return s;
+  if ((s = gemv_sidecar(prm, pr, n_mod, mods, T, sidecar, sidecar_bytes, &a)) != AWSRC_OK) return s;
   const cudaError_t e = launch_gemv(pr, a, M, (cudaStream_t)stream);
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "packed_gemv");
 }

@@ -102,20 +102,29 @@ cudaError_t launch_dense_prep(const Prm& pr, int64_t T, int64_t L, int64_t h, co
 // The dense fused decoder clears the fault word itself (no separate memset).
 bool decode_clears_status(const Prm& pr, int mode);
 
-// gemv.cu: y[m] = (W0 + r_hat) x[m] for one module of a prepared sidecar.
-struct GemvArgs {
+// gemv.cu: y[m] = (W0 + r_hat) x[m] for a batch of (module, x, y) tasks of a
+// prepared sidecar, one launch for the tasks whose x fits in shared memory.
+struct GemvTask {
   int64_t rows, cols, tile_off;  // tile_off: the module's first global tile
-  int32_t sdq, pad_;
+  int32_t sdq, block0;           // block0: the task's first block (set by launch_gemv)
   const uint16_t* codes;         // 4 codes per uint16, element 2i in the low nibble of byte i
   const uint16_t* scales;        // binary16 per group (sdq == 0)
   const int8_t* sdq_codes;       // per group (sdq)
   const float* sdq_consts;       // (mean, step) per 256 groups (sdq)
-  const unsigned long long* map; // tile map of the prepared sidecar, or null (no residual)
-  const uint4* rcodes;           // per-record slots of the prepared sidecar (codes in x, y)
-  const uint64_t* masks;         // basis masks of the prepared sidecar
   const float* x;                // M x cols
   float* y;                      // M x rows
 };
+constexpr int kMaxGemvTasks = 16;
+struct GemvArgs {
+  int n_task;
+  const unsigned long long* map; // tile map of the prepared sidecar, or null (no residual)
+  const uint4* slots;            // per-record slots of the prepared sidecar (codes in x, y)
+  const uint64_t* masks;         // basis masks of the prepared sidecar
+  const uint4* nib;              // nibble tables of the prepared sidecar when gemv_tables(), else null
+  GemvTask t[kMaxGemvTasks];
+};
+// Whether the GEMV walks recorded tiles with the decoder's code tables.
+bool gemv_tables(const Prm& pr);
 cudaError_t launch_gemv(const Prm& pr, const GemvArgs& a, int M, cudaStream_t st);
 
 // backbone.cu: RTN-INT4 groups of rtn_group() inputs, SDQ blocks of sdq_block() groups.

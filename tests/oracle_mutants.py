@@ -119,9 +119,9 @@ MUTANTS = {
 """),
     ]),
     19: ('packed GEMV subtracting the sidecar correction', [
-        ("""      Wt[base + j] += (double)kj * c * sc;
+        ("""      Rt[base + j] = (double)kj * c * sc;  /* a later record of the tile replaces it */
 """,
-         """      Wt[base + j] -= (double)kj * c * sc;
+         """      Rt[base + j] = -(double)kj * c * sc;  /* a later record of the tile replaces it */
 """),
     ]),
     20: ('sign word bits read most-significant first', [
@@ -277,6 +277,18 @@ MUTANTS = {
         ("""        v = rintf(w[j] / s);
 """,
          """        v = rintf(w[j] * (1.0f / s));
+"""),
+    ]),
+    43: ('packed GEMV adding both records of a tile named twice', [
+        ("""      Rt[base + j] = (double)kj * c * sc;  /* a later record of the tile replaces it */
+""",
+         """      Rt[base + j] += (double)kj * c * sc;  /* a later record of the tile replaces it */
+"""),
+    ]),
+    44: ('packed GEMV magnitude of the summed weight instead of its two terms', [
+        ("""        aabs += fabs(Wt[i * cols + j] * xj) + fabs(Rt[i * cols + j] * xj);
+""",
+         """        aabs += fabs((Wt[i * cols + j] + Rt[i * cols + j]) * xj);
 """),
     ]),
 }

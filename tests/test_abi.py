@@ -200,6 +200,18 @@ def test_serving_and_diagnostic_arguments_are_refused_on_the_host(libpath):
     assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 0, ct.byref(pw), None, 0, 1, 0x30008, 0x40000, None) == 1
     pw.codes = 0x10002
     assert lib.awsrc_packed_gemv(ct.byref(p), 1, mods, 0, ct.byref(pw), None, 0, 1, 0x30000, 0x40000, None) == 1
+    # awsrc_packed_gemv_batch: 1 <= n_task <= 16 (more: UNSUPPORTED), each task checked like a single call
+    from paper_2608_23144_gb300._binding import GemvTask
+    pw.codes = 0x10000
+    tasks = (GemvTask * 17)(*[GemvTask(0, 0, pw, 0x30000, 0x40000 + 0x100 * i) for i in range(17)])
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 0, tasks, None, 0, 1, None) == 1
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 17, tasks, None, 0, 1, None) == 3
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 2, None, None, 0, 1, None) == 1
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 2, tasks, None, 0, 0, None) == 1
+    tasks[1].m = 1
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 2, tasks, None, 0, 1, None) == 1
+    tasks[1].m, tasks[1].x = 0, 0x30004
+    assert lib.awsrc_packed_gemv_batch(ct.byref(p), 1, mods, 2, tasks, None, 0, 1, None) == 1
     # awsrc_verify_reciprocal: null, misaligned counter, empty-range order
     assert lib.awsrc_verify_reciprocal(0, 1, None, None) == 1
     assert lib.awsrc_verify_reciprocal(0, 1, 0x50004, None) == 1

@@ -168,6 +168,45 @@ def test_packed_product_definition(orc):
     ref = x.astype(np.float64) @ dec[0].astype(np.float64).T
     assert (np.abs(y - ref) <= 2.0 ** -22 * yabs + 1e-30).all()
     assert (yabs >= np.abs(y)).all() and not np.allclose(y, y0)
+    # yabs sums the backbone's and the residual's magnitudes separately; the
+    # residual is the decoded weights less W0 (both binary32, so within one
+    # rounding of the decoded weight)
+    W0d = bb["W0"].astype(np.float64)
+    R = dec[0].astype(np.float64) - W0d
+    xa = np.abs(x.astype(np.float64))
+    want = xa @ np.abs(W0d).T + xa @ np.abs(R).T
+    assert (np.abs(yabs - want) <= 2.0 ** -22 * (xa @ np.abs(dec[0].astype(np.float64)).T) + 1e-30).all()
+    assert (want - xa @ np.abs(W0d + R).T > 2.0 ** -18 * want).any()  # the two magnitudes differ here
+
+
+def test_packed_product_repeated_tile_takes_later_record(orc):
+    """A stream that names a tile twice (never written by the encoder): the
+    product applies only the later record, as the decoder does, i.e. it equals
+    the product of the stream without the earlier record."""
+    rng = np.random.default_rng(7)
+    rows, cols = 40, 256
+    W = _weights(rng, rows, cols, zero_groups=False)
+    bb = orc.rtn_quantize(W)
+    prm = orc.params(C=64, P=4, b=4, S=64)
+    cands = orc.encode_tiles(prm, W, bb["W0"], (rng.lognormal(0, 1, cols) ** 2).astype(np.float32))
+    stream, counts, _ = orc.select_records(prm, [(rows, cols)], cands, [2.0])
+    K = int(counts.sum())
+    raw = np.frombuffer(stream, np.uint8).copy()
+    h, T = orc.header_bytes(1), rows * cols // 64
+    L = orc.record_bytes(prm, T)
+    tb = int(np.ceil(np.log2(T)))
+    rec = lambda k: int.from_bytes(raw[h + k * L: h + (k + 1) * L].tobytes(), "little")
+    mask = (1 << tb) - 1
+    dup = raw.copy()
+    dup[h + L: h + 2 * L] = np.frombuffer(((rec(1) & ~mask) | (rec(0) & mask)).to_bytes(L, "little"), np.uint8)
+    fixed = np.concatenate([raw[:h], dup[h + L:]])
+    x = rng.normal(0, 1, (2, cols)).astype(np.float32)
+    y, yabs, bad = orc.packed_gemv(prm, bb["q"], bb["s_eff"], 128, dup.tobytes(), K, x)
+    yf, yabsf, badf = orc.packed_gemv(prm, bb["q"], bb["s_eff"], 128, fixed.tobytes(), K - 1, x)
+    assert bad == 0 and badf == 0
+    assert np.array_equal(y, yf) and np.array_equal(yabs, yabsf)
+    y2, _, _ = orc.packed_gemv(prm, bb["q"], bb["s_eff"], 128, raw.tobytes(), K, x)
+    assert not np.allclose(y, y2)
 
 
 def test_packed_product_second_module_of_a_stream(orc):
