@@ -231,6 +231,28 @@ awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32
                                 void* W0, int32_t w0_dtype, void* stream);
 
 /*
+ * awsrc_rtn_quantize_batch — awsrc_rtn_quantize for n_task >= 1 modules in as
+ * few launches as their dtypes allow (one when all share w_dtype and
+ * w0_dtype and there are at most 16): every output is bit-identical to the
+ * single call's. Arguments per task as for awsrc_rtn_quantize; the output
+ * arrays of different tasks must not overlap. Errors: as awsrc_rtn_quantize
+ * (the first failing task decides; nothing is launched then).
+ */
+typedef struct awsrc_rtn_task {
+  int64_t rows, cols;
+  const void* W;
+  int32_t w_dtype, sdq;
+  uint8_t* codes;
+  uint16_t* scales;
+  int8_t* sdq_codes;
+  float* sdq_consts;
+  void* W0;
+  int32_t w0_dtype, pad_;
+} awsrc_rtn_task;
+
+awsrc_status awsrc_rtn_quantize_batch(int32_t n_task, const awsrc_rtn_task* tasks, void* stream);
+
+/*
  * awsrc_backbone_metadata_bytes — scale metadata of a rows x cols RTN-INT4
  * backbone: 2 bytes per group of 128, or with SDQ 1 per group plus 8 per block
  * of 256 groups. Under a fixed total budget the bytes SDQ saves can go to the

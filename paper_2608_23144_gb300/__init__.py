@@ -33,6 +33,7 @@ from ._binding import (  # noqa: F401
     awsrc_encode_workspace_bytes,
     awsrc_gen_basis,
     awsrc_rtn_quantize,
+    awsrc_rtn_quantize_batch,
     awsrc_backbone_metadata_bytes,
     awsrc_rate_with_sdq_savings,
     awsrc_sidecar_prepare,

@@ -60,6 +60,12 @@ class PackedWeights(ct.Structure):
                 ("sdq_consts", ct.c_void_p), ("sdq", ct.c_int32), ("pad_", ct.c_int32)]
 
 
+class RtnTask(ct.Structure):
+    _fields_ = [("rows", ct.c_int64), ("cols", ct.c_int64), ("W", ct.c_void_p), ("w_dtype", ct.c_int32),
+                ("sdq", ct.c_int32), ("codes", ct.c_void_p), ("scales", ct.c_void_p), ("sdq_codes", ct.c_void_p),
+                ("sdq_consts", ct.c_void_p), ("W0", ct.c_void_p), ("w0_dtype", ct.c_int32), ("pad_", ct.c_int32)]
+
+
 class GemvTask(ct.Structure):
     _fields_ = [("m", ct.c_int32), ("pad_", ct.c_int32), ("pw", PackedWeights), ("x", ct.c_void_p),
                 ("y", ct.c_void_p)]
@@ -124,6 +130,8 @@ def _load():
     L.awsrc_rtn_quantize.restype = st
     L.awsrc_rtn_quantize.argtypes = [ct.c_int64, ct.c_int64, vp, ct.c_int32, ct.c_int32, vp, vp, vp, vp, vp,
                                      ct.c_int32, vp]
+    L.awsrc_rtn_quantize_batch.restype = st
+    L.awsrc_rtn_quantize_batch.argtypes = [ct.c_int32, P(RtnTask), vp]
     L.awsrc_backbone_metadata_bytes.restype = ct.c_int64
     L.awsrc_backbone_metadata_bytes.argtypes = [ct.c_int64, ct.c_int64, ct.c_int32]
     L.awsrc_rate_with_sdq_savings.restype = st
@@ -268,13 +276,8 @@ def awsrc_encode_tiles(prm: Params, modules, out: Optional[torch.Tensor] = None,
     return out
 
 
-def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream=None,
-                       out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
-    """RTN-INT4 backbone of one module (groups of 128 inputs), optional SDQ.
-    Returns codes (uint8, two per byte), scales (binary16 bits as int16),
-    sdq_codes (int8) and sdq_consts (float32 mean, step per 256 groups) when
-    sdq, and W0 (in w0_dtype, default W's dtype). `out` reuses the buffers of
-    an earlier call on the same shape."""
+def _rtn_buffers(W: torch.Tensor, sdq: bool, w0_dtype, out: Optional[Dict[str, torch.Tensor]]):
+    """Checks W (and `out`, when given) or allocates the outputs of one module."""
     _require(W, "W")
     if W.dim() != 2:
         raise ValueError(f"W must be 2-D (rows x cols), not {W.dim()}-D")
@@ -289,19 +292,47 @@ def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream
             _require(out["sdq_codes"], "out['sdq_codes']", dtype=torch.int8, numel=G, device=dev)
             _require(out["sdq_consts"], "out['sdq_consts']", dtype=torch.float32, numel=2 * ((G + 255) // 256),
                      device=dev)
-    if out is None:
-        out = {"codes": torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev),
-               "scales": torch.empty(G, dtype=torch.int16, device=dev)}
-        if sdq:
-            out["sdq_codes"] = torch.empty(G, dtype=torch.int8, device=dev)
-            out["sdq_consts"] = torch.empty(2 * ((G + 255) // 256), dtype=torch.float32, device=dev)
-        w0t = W.dtype if w0_dtype is None else w0_dtype
-        out["W0"] = torch.empty(rows, cols, dtype=w0t, device=dev)
+        return out
+    out = {"codes": torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev),
+           "scales": torch.empty(G, dtype=torch.int16, device=dev)}
+    if sdq:
+        out["sdq_codes"] = torch.empty(G, dtype=torch.int8, device=dev)
+        out["sdq_consts"] = torch.empty(2 * ((G + 255) // 256), dtype=torch.float32, device=dev)
+    w0t = W.dtype if w0_dtype is None else w0_dtype
+    out["W0"] = torch.empty(rows, cols, dtype=w0t, device=dev)
+    return out
+
+
+def awsrc_rtn_quantize(W: torch.Tensor, sdq: bool = False, w0_dtype=None, stream=None,
+                       out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
+    """RTN-INT4 backbone of one module (groups of 128 inputs), optional SDQ.
+    Returns codes (uint8, two per byte), scales (binary16 bits as int16),
+    sdq_codes (int8) and sdq_consts (float32 mean, step per 256 groups) when
+    sdq, and W0 (in w0_dtype, default W's dtype). `out` reuses the buffers of
+    an earlier call on the same shape."""
+    out = _rtn_buffers(W, sdq, w0_dtype, out)
+    rows, cols = W.shape
     _check(lib.awsrc_rtn_quantize(rows, cols, _dev_ptr(W), _dtype_code(W), int(sdq), _dev_ptr(out["codes"]),
                                   _dev_ptr(out["scales"]), _dev_ptr(out.get("sdq_codes")),
                                   _dev_ptr(out.get("sdq_consts")), _dev_ptr(out["W0"]), _dtype_code(out["W0"]),
                                   _stream(stream)), "rtn_quantize")
     return out
+
+
+def awsrc_rtn_quantize_batch(Ws: Sequence[torch.Tensor], sdq: bool = False, w0_dtype=None, stream=None,
+                             outs: Optional[List[Dict[str, torch.Tensor]]] = None) -> List[Dict[str, torch.Tensor]]:
+    """awsrc_rtn_quantize of several modules in one launch (per run of equal
+    dtypes); returns one output dict per module, as the single call does."""
+    if outs is not None and len(outs) != len(Ws):
+        raise ValueError(f"{len(outs)} output sets for {len(Ws)} modules")
+    res = [_rtn_buffers(W, sdq, w0_dtype, None if outs is None else outs[i]) for i, W in enumerate(Ws)]
+    arr = (RtnTask * len(Ws))()
+    for i, (W, o) in enumerate(zip(Ws, res)):
+        arr[i] = RtnTask(W.shape[0], W.shape[1], _dev_ptr(W), _dtype_code(W), int(sdq), _dev_ptr(o["codes"]),
+                         _dev_ptr(o["scales"]), _dev_ptr(o.get("sdq_codes")), _dev_ptr(o.get("sdq_consts")),
+                         _dev_ptr(o["W0"]), _dtype_code(o["W0"]), 0)
+    _check(lib.awsrc_rtn_quantize_batch(len(Ws), arr, _stream(stream)), "rtn_quantize_batch")
+    return res
 
 
 def awsrc_backbone_metadata_bytes(rows: int, cols: int, sdq: bool) -> int:

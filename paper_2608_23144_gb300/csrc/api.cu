@@ -297,16 +297,64 @@ awsrc_status awsrc_encode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
 awsrc_status awsrc_rtn_quantize(int64_t rows, int64_t cols, const void* W, int32_t w_dtype, int32_t sdq,
                                 uint8_t* codes, uint16_t* scales, int8_t* sdq_codes, float* sdq_consts,
                                 void* W0, int32_t w0_dtype, void* stream) {
-  if (rows < 1 || cols < 1 || cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
-  if (rows > kMaxBackboneWeights / cols) return AWSRC_ERR_UNSUPPORTED;
-  if (w_dtype != AWSRC_DTYPE_F32 && w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
-  if (w0_dtype != AWSRC_DTYPE_F32 && w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
-  if (sdq != 0 && sdq != 1) return AWSRC_ERR_INVALID_ARG;
-  if (!W || !codes || !aligned(W, 16) || !aligned(codes, 4) || !aligned(scales, 2) || !aligned(sdq_consts, 4) ||
-      !aligned(W0, 16))
-    return AWSRC_ERR_INVALID_ARG;
-  const cudaError_t e = launch_rtn(W, w_dtype, rows, cols, sdq, codes, scales, sdq_codes, sdq_consts, W0,
-                                   w0_dtype, (cudaStream_t)stream);
+  const awsrc_rtn_task t{rows, cols, W, w_dtype, sdq, codes, scales, sdq_codes, sdq_consts, W0, w0_dtype, 0};
+  return awsrc_rtn_quantize_batch(1, &t, stream);
+}
+
+awsrc_status awsrc_rtn_quantize_batch(int32_t n_task, const awsrc_rtn_task* tasks, void* stream) {
+  if (n_task < 1 || !tasks) return AWSRC_ERR_INVALID_ARG;
+  for (int i = 0; i < n_task; ++i) {
+    const awsrc_rtn_task& t = tasks[i];
+    if (t.rows < 1 || t.cols < 1 || t.cols % rtn_group() != 0) return AWSRC_ERR_SHAPE;
+    if (t.rows > kMaxBackboneWeights / t.cols) return AWSRC_ERR_UNSUPPORTED;
+    if (t.w_dtype != AWSRC_DTYPE_F32 && t.w_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+    if (t.w0_dtype != AWSRC_DTYPE_F32 && t.w0_dtype != AWSRC_DTYPE_BF16) return AWSRC_ERR_INVALID_ARG;
+    if (t.sdq != 0 && t.sdq != 1) return AWSRC_ERR_INVALID_ARG;
+    if (!t.W || !t.codes || !aligned(t.W, 16) || !aligned(t.codes, 4) || !aligned(t.scales, 2) ||
+        !aligned(t.sdq_consts, 4) || !aligned(t.W0, 16))
+      return AWSRC_ERR_INVALID_ARG;
+  }
+  // one launch per run of tasks with the same dtypes, at most kMaxRtnTasks
+  // pieces and rtn_max_blocks() blocks of 256 groups each; a module larger than
+  // that is cut into pieces on block boundaries (the blocks are independent)
+  const int64_t gpb = sdq_block(), maxg = rtn_max_blocks() * gpb, grp = rtn_group();
+  RtnArgs a{};
+  int64_t blocks = 0;
+  int dt_in = -1, dt_out = -1;
+  auto flush = [&]() -> cudaError_t {
+    cudaError_t e = cudaSuccess;
+    if (a.n > 0) e = launch_rtn(a, dt_in, dt_out, (cudaStream_t)stream);
+    a.n = 0;
+    blocks = 0;
+    return e;
+  };
+  for (int i = 0; i < n_task; ++i) {
+    const awsrc_rtn_task& t = tasks[i];
+    const int64_t G = t.rows * t.cols / grp;
+    for (int64_t off = 0; off < G;) {
+      const int64_t len = std::min(G - off, maxg);
+      const int64_t nb = (len + gpb - 1) / gpb;
+      if (a.n == kMaxRtnTasks || blocks + nb > rtn_max_blocks() || t.w_dtype != dt_in || t.w0_dtype != dt_out) {
+        const cudaError_t e = flush();
+        if (e != cudaSuccess) return cuda_fail(e, "rtn_quantize");
+        dt_in = t.w_dtype;
+        dt_out = t.w0_dtype;
+      }
+      const size_t wi = t.w_dtype == AWSRC_DTYPE_F32 ? 4 : 2, wo = t.w0_dtype == AWSRC_DTYPE_F32 ? 4 : 2;
+      RtnTask& r = a.t[a.n++];
+      r.W = static_cast<const uint8_t*>(t.W) + (size_t)(off * grp) * wi;
+      r.G = len;
+      r.sdq = t.sdq;
+      r.codes = reinterpret_cast<uint32_t*>(t.codes) + off * (grp / 8);
+      r.scales = t.scales ? t.scales + off : nullptr;
+      r.sdq_codes = t.sdq_codes ? t.sdq_codes + off : nullptr;
+      r.sdq_consts = t.sdq_consts ? t.sdq_consts + 2 * (off / gpb) : nullptr;
+      r.W0 = t.W0 ? static_cast<uint8_t*>(t.W0) + (size_t)(off * grp) * wo : nullptr;
+      blocks += nb;
+      off += len;
+    }
+  }
+  const cudaError_t e = flush();
   return e == cudaSuccess ? AWSRC_OK : cuda_fail(e, "rtn_quantize");
 }
 

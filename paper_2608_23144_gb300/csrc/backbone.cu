@@ -13,8 +13,12 @@
 // (rtn_fast), and needs no clamp when s is a normal binary16 (|w / s| <= 7.004);
 // a warp iteration with any such element takes the division for all of its
 // elements. With SDQ the block then forms the mean of its scales (their sum
-// is exact in double), the largest deviation, the step and the 8-bit codes,
-// and writes W0 = q * s~ from the codes it kept in registers.
+// is exact as an integer count of 2^-24), the largest deviation, the step and
+// the 8-bit codes,
+// and writes W0 = q * s~ from the codes it kept in registers (nibbles turned
+// into floats by a byte permute into 2^23 + (q + 8) and one subtraction).
+// One launch serves a batch of modules: block b takes SDQ block b - block0 of
+// the module whose block range holds b.
 #include "internal.h"
 
 namespace awsrc {
@@ -72,13 +76,40 @@ constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: x + kMagic rounds x to an 
 // 2^-20 of a half-integer; `tie` is set when |t - rint(t)| > 1/2 - 2^-16 (the
 // caller then divides). |t| < 7.5 needs no clamp. The integer sits in the low
 // mantissa bits of t + kMagic (two's complement, so its low nibble is the code).
-__device__ __forceinline__ uint32_t rtn_fast2(float2 w, float rs, bool& tie) {
+// The pair's codes as floats go to q; the returned word holds t + kMagic of
+// each (its low byte carries the code's nibble).
+__device__ __forceinline__ float2 rtn_fast2(float2 w, float rs, bool& tie, float2& q) {
   const float2 t = __fmul2_rn(w, make_float2(rs, rs));
   const float2 u = __fadd2_rn(t, make_float2(kMagic, kMagic));
-  const float2 q = __fadd2_rn(u, make_float2(-kMagic, -kMagic));
+  q = __fadd2_rn(u, make_float2(-kMagic, -kMagic));
   const float2 d = __fadd2_rn(t, make_float2(-q.x, -q.y));
-  tie |= fabsf(d.x) > 0.5f - 0x1p-16f || fabsf(d.y) > 0.5f - 0x1p-16f;
-  return (__float_as_uint(u.x) & 15u) | ((__float_as_uint(u.y) & 15u) << 4);
+  tie |= fmaxf(fabsf(d.x), fabsf(d.y)) > 0.5f - 0x1p-16f;
+  return u;
+}
+
+// The 8 codes (element 2i in the low nibble of byte i) from the low bytes of
+// t + kMagic of elements 0 .. 7.
+__device__ __forceinline__ uint32_t pack_codes(const float2* u) {
+  const uint32_t e01 = __byte_perm(__float_as_uint(u[0].x), __float_as_uint(u[1].x), 0x0040u);  // 0, 2
+  const uint32_t e23 = __byte_perm(__float_as_uint(u[2].x), __float_as_uint(u[3].x), 0x0040u);  // 4, 6
+  const uint32_t o01 = __byte_perm(__float_as_uint(u[0].y), __float_as_uint(u[1].y), 0x0040u);  // 1, 3
+  const uint32_t o23 = __byte_perm(__float_as_uint(u[2].y), __float_as_uint(u[3].y), 0x0040u);  // 5, 7
+  const uint32_t ev = __byte_perm(e01, e23, 0x5410u), od = __byte_perm(o01, o23, 0x5410u);
+  return (ev & 0x0F0F0F0Fu) | ((od << 4) & 0xF0F0F0F0u);
+}
+
+// Codes i of a packed word as floats (two's complement nibbles): q + 8 is put
+// in the low byte of 2^23 and 2^23 + 8 subtracted, exactly.
+__device__ __forceinline__ void unpack_codes(uint32_t pk, float* q) {
+  const uint32_t lo = (pk & 0x0F0F0F0Fu) ^ 0x08080808u, hi = ((pk >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    const float2 v = __fadd2_rn(make_float2(__uint_as_float(__byte_perm(lo, 0x4B000000u, 0x7540u + b)),
+                                            __uint_as_float(__byte_perm(hi, 0x4B000000u, 0x7540u + b))),
+                                make_float2(-8388616.0f, -8388616.0f));
+    q[2 * b] = v.x;
+    q[2 * b + 1] = v.y;
+  }
 }
 
 // Exact code of one input: clamp(rint(RN(w / s)), -8, 7), 0 when s == 0.
@@ -88,22 +119,25 @@ __device__ __forceinline__ uint32_t rtn_exact(float w, float s) {
   return (uint32_t)(int)q & 15u;
 }
 
-__device__ __forceinline__ int code_at(uint32_t packed, int i) {  // 4-bit two's complement
-  return (int)((int32_t)(packed << (28 - 4 * i)) >> 28);
-}
-
 template <typename TI, typename TO>
-__global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restrict__ W, int64_t G, int sdq,
-                                                             uint32_t* __restrict__ codes,
-                                                             uint16_t* __restrict__ scales,
-                                                             int8_t* __restrict__ sdq_codes,
-                                                             float* __restrict__ sdq_consts, TO* __restrict__ W0) {
+__global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const __grid_constant__ RtnArgs a) {
   __shared__ float sv[kSdqBlock];
-  __shared__ double red_d[kRtnWarps];
+  __shared__ long long red_i[kRtnWarps];
   __shared__ float red_f[kRtnWarps];
   __shared__ float mu_step[2];
+  int ti = 0;
+  for (int i = 1; i < a.n; ++i)
+    if ((int)blockIdx.x >= a.t[i].block0) ti = i;
+  const RtnTask& tk = a.t[ti];
+  const TI* __restrict__ W = static_cast<const TI*>(tk.W);
+  TO* __restrict__ W0 = static_cast<TO*>(tk.W0);
+  uint32_t* __restrict__ codes = tk.codes;
+  uint16_t* __restrict__ scales = tk.scales;
+  const int64_t G = tk.G;
+  const int sdq = tk.sdq;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, h = lane >> 4, hl = lane & 15;
-  const int64_t g0 = (int64_t)blockIdx.x * kSdqBlock;
+  const int64_t blk = (int64_t)blockIdx.x - tk.block0;
+  const int64_t g0 = blk * kSdqBlock;
   const int n = G - g0 < kSdqBlock ? (int)(G - g0) : kSdqBlock;
   uint32_t qs[kIters];  // this lane's 8 codes of each iteration
 #pragma unroll
@@ -132,12 +166,16 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
       const float s = __half2float(hs);
       bool slow = !(s >= 0x1p-14f);  // zero or subnormal binary16 scale
       uint32_t pk = 0u;
+      float2 qf[4];
       if (!slow) {
-        const float rs = __frcp_rn(s);
+        const float rs = rcp_rn(s);
+        float2 u[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) pk |= rtn_fast2(make_float2(w[2 * i], w[2 * i + 1]), rs, slow) << (8 * i);
+        for (int i = 0; i < 4; ++i) u[i] = rtn_fast2(make_float2(w[2 * i], w[2 * i + 1]), rs, slow, qf[i]);
+        pk = pack_codes(u);
       }
-      if (__any_sync(0xffffffffu, slow)) {
+      const bool exact = __any_sync(0xffffffffu, slow);
+      if (exact) {
         pk = 0u;
 #pragma unroll
         for (int i = 0; i < 8; ++i) pk |= rtn_exact(w[i], s) << (4 * i);
@@ -150,10 +188,24 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
           sv[lg] = s;
           if (scales) scales[g] = __half_as_ushort(hs);
         }
-        if (!sdq && W0) {
+        if (!sdq && W0) {  // the integer codes (no -0) times s
+          float q[8];
+          if (exact) {
+            unpack_codes(pk, q);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              q[2 * i] = qf[i].x;
+              q[2 * i + 1] = qf[i].y;
+            }
+          }
           float o[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) o[i] = __fmul_rn((float)code_at(pk, i), s);  // the integer code: no -0
+          for (int i = 0; i < 8; i += 2) {
+            const float2 v = __fmul2_rn(make_float2(q[i], q[i + 1]), make_float2(s, s));
+            o[i] = v.x;
+            o[i + 1] = v.y;
+          }
           Elt<TO>::st8(W0 + g * kRtnGroup + 8 * hl, o);
         }
       }
@@ -161,17 +213,21 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
   }
   if (!sdq) return;
   __syncthreads();
-  // second level: mean (exact sum in double), largest deviation, step, codes
+  // second level: mean, largest deviation, step, codes. Every s_g is a
+  // binary16 value, an integer multiple of 2^-24 below 2^16, so the block's sum
+  // is exact as an integer count of 2^-24 (below 2^48, exact in double too);
+  // for a whole block (n = 256) the mean is RN(sum * 2^-32), one rounding.
   const int t = threadIdx.x;
-  double sum = t < n ? (double)sv[t] : 0.0;
+  long long sum = t < n ? __float2ll_rn(__fmul_rn(sv[t], 0x1p24f)) : 0ll;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-  if (lane == 0) red_d[warp] = sum;
+  if (lane == 0) red_i[warp] = sum;
   __syncthreads();
   if (t == 0) {
-    double tot = 0.0;
-    for (int i = 0; i < kRtnWarps; ++i) tot += red_d[i];
-    mu_step[0] = __double2float_rn(__ddiv_rn(tot, (double)n));
+    long long tot = 0;
+    for (int i = 0; i < kRtnWarps; ++i) tot += red_i[i];
+    mu_step[0] = n == kSdqBlock ? __fmul_rn(__ll2float_rn(tot), 0x1p-32f)
+                                : __double2float_rn(__ddiv_rn(__dmul_rn((double)tot, 0x1p-24), (double)n));
   }
   __syncthreads();
   const float mu = mu_step[0];
@@ -184,9 +240,9 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
     float a = 0.0f;
     for (int i = 0; i < kRtnWarps; ++i) a = fmaxf(a, red_f[i]);
     mu_step[1] = __fdiv_rn(a, 127.0f);
-    if (sdq_consts) {
-      sdq_consts[2 * blockIdx.x] = mu;
-      sdq_consts[2 * blockIdx.x + 1] = mu_step[1];
+    if (tk.sdq_consts) {
+      tk.sdq_consts[2 * blk] = mu;
+      tk.sdq_consts[2 * blk + 1] = mu_step[1];
     }
   }
   __syncthreads();
@@ -194,7 +250,7 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
   if (t < n) {
     const float c = step > 0.0f ? fminf(fmaxf(rintf(__fdiv_rn(__fsub_rn(sv[t], mu), step)), -127.0f), 127.0f)
                                 : 0.0f;
-    if (sdq_codes) sdq_codes[g0 + t] = (int8_t)(int)c;
+    if (tk.sdq_codes) tk.sdq_codes[g0 + t] = (int8_t)(int)c;
     sv[t] = __fadd_rn(mu, __fmul_rn(c, step));  // s~ replaces s (each thread its own entry)
   }
   __syncthreads();
@@ -204,24 +260,26 @@ __global__ void __launch_bounds__(32 * kRtnWarps) rtn_kernel(const TI* __restric
     const int lg = 2 * warp + h + 2 * kRtnWarps * k;
     if (lg >= n) continue;
     const float st = sv[lg];
-    float o[8];
+    float q[8], o[8];
+    unpack_codes(qs[k], q);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) o[i] = __fmul_rn((float)code_at(qs[k], i), st);
+    for (int i = 0; i < 8; i += 2) {
+      const float2 v = __fmul2_rn(make_float2(q[i], q[i + 1]), make_float2(st, st));
+      o[i] = v.x;
+      o[i + 1] = v.y;
+    }
     Elt<TO>::st8(W0 + (g0 + lg) * kRtnGroup + 8 * hl, o);
   }
 }
 
-template <typename TI>
-cudaError_t launch_rtn_ti(const void* W, int64_t G, int sdq, uint32_t* codes, uint16_t* scales, int8_t* sc8,
-                          float* consts, void* W0, int w0_dtype, cudaStream_t st) {
-  const unsigned nb = (unsigned)((G + kSdqBlock - 1) / kSdqBlock);
-  const TI* w = static_cast<const TI*>(W);
-  if (w0_dtype == AWSRC_DTYPE_F32)
-    rtn_kernel<TI, float><<<nb, 32 * kRtnWarps, 0, st>>>(w, G, sdq, codes, scales, sc8, consts,
-                                                          static_cast<float*>(W0));
-  else
-    rtn_kernel<TI, __nv_bfloat16><<<nb, 32 * kRtnWarps, 0, st>>>(w, G, sdq, codes, scales, sc8, consts,
-                                                                  static_cast<__nv_bfloat16*>(W0));
+template <typename TI, typename TO>
+cudaError_t launch_rtn_t(RtnArgs a, cudaStream_t st) {
+  int blocks = 0;
+  for (int i = 0; i < a.n; ++i) {
+    a.t[i].block0 = blocks;
+    blocks += (int)((a.t[i].G + kSdqBlock - 1) / kSdqBlock);
+  }
+  rtn_kernel<TI, TO><<<(unsigned)blocks, 32 * kRtnWarps, 0, st>>>(a);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -231,14 +289,14 @@ cudaError_t launch_rtn_ti(const void* W, int64_t G, int sdq, uint32_t* codes, ui
 int rtn_group() { return kRtnGroup; }
 int sdq_block() { return kSdqBlock; }
 
-cudaError_t launch_rtn(const void* W, int w_dtype, int64_t rows, int64_t cols, int sdq, uint8_t* codes,
-                       uint16_t* scales, int8_t* sdq_codes, float* sdq_consts, void* W0, int w0_dtype,
-                       cudaStream_t st) {
-  const int64_t G = rows * cols / kRtnGroup;
-  uint32_t* c16 = reinterpret_cast<uint32_t*>(codes);
-  return w_dtype == AWSRC_DTYPE_F32
-             ? launch_rtn_ti<float>(W, G, sdq, c16, scales, sdq_codes, sdq_consts, W0, w0_dtype, st)
-             : launch_rtn_ti<__nv_bfloat16>(W, G, sdq, c16, scales, sdq_codes, sdq_consts, W0, w0_dtype, st);
+int64_t rtn_max_blocks() { return 1ll << 30; }
+
+cudaError_t launch_rtn(const RtnArgs& a, int w_dtype, int w0_dtype, cudaStream_t st) {
+  const bool f32in = w_dtype == AWSRC_DTYPE_F32, f32out = w0_dtype == AWSRC_DTYPE_F32;
+  if (f32in && f32out) return launch_rtn_t<float, float>(a, st);
+  if (f32in) return launch_rtn_t<float, __nv_bfloat16>(a, st);
+  if (f32out) return launch_rtn_t<__nv_bfloat16, float>(a, st);
+  return launch_rtn_t<__nv_bfloat16, __nv_bfloat16>(a, st);
 }
 
 }  // namespace awsrc

@@ -130,9 +130,24 @@ cudaError_t launch_gemv(const Prm& pr, const GemvArgs& a, int M, cudaStream_t st
 // backbone.cu: RTN-INT4 groups of rtn_group() inputs, SDQ blocks of sdq_block() groups.
 int rtn_group();
 int sdq_block();
-cudaError_t launch_rtn(const void* W, int w_dtype, int64_t rows, int64_t cols, int sdq, uint8_t* codes,
-                       uint16_t* scales, int8_t* sdq_codes, float* sdq_consts, void* W0, int w0_dtype,
-                       cudaStream_t st);
+// One launch for a batch of modules sharing (w_dtype, w0_dtype).
+struct RtnTask {
+  const void* W;
+  int64_t G;            // groups of 128
+  int32_t sdq, block0;  // block0: the task's first block (set by launch_rtn)
+  uint32_t* codes;
+  uint16_t* scales;
+  int8_t* sdq_codes;
+  float* sdq_consts;
+  void* W0;
+};
+constexpr int kMaxRtnTasks = 16;
+struct RtnArgs {
+  int n;
+  RtnTask t[kMaxRtnTasks];
+};
+cudaError_t launch_rtn(const RtnArgs& a, int w_dtype, int w0_dtype, cudaStream_t st);
+int64_t rtn_max_blocks();  // blocks one launch may take
 
 // numerics.cu: bit patterns in [first, last) where rcp_rn differs from __frcp_rn
 // are added to *bad (device).

@@ -190,6 +190,14 @@ def test_serving_and_diagnostic_arguments_are_refused_on_the_host(libpath):
     assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 0, 0x20002, 0x30000, None, None, 0x40000, bf16, None) == 1
     assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40004, bf16, None) == 1
     assert lib.awsrc_rtn_quantize(8, 128, 0x10000, bf16, 2, 0x20000, 0x30000, None, None, 0x40000, bf16, None) == 1
+    # awsrc_rtn_quantize_batch: every task is checked before anything runs
+    from paper_2608_23144_gb300._binding import RtnTask
+    ok = RtnTask(8, 128, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40000, bf16, 0)
+    bad = RtnTask(8, 100, 0x10000, bf16, 0, 0x20000, 0x30000, None, None, 0x40000, bf16, 0)
+    assert lib.awsrc_rtn_quantize_batch(0, (RtnTask * 1)(ok), None) == 1
+    assert lib.awsrc_rtn_quantize_batch(2, (RtnTask * 2)(ok, bad), None) == 2
+    ok2 = RtnTask(8, 128, 0x10000, bf16, 0, 0x20002, 0x30000, None, None, 0x40000, bf16, 0)
+    assert lib.awsrc_rtn_quantize_batch(2, (RtnTask * 2)(ok, ok2), None) == 1
     # awsrc_packed_gemv: M in [1, 8], module index, 16-byte x, 4-byte codes
     from paper_2608_23144_gb300._binding import PackedWeights, shape_modules
     p = aw.params(C=64, S=64)

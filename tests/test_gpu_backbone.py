@@ -51,6 +51,30 @@ def test_backbone_matches_oracle(aw, orc, rows, cols, w_dtype, w0_dtype, sdq):
                        W0.view(torch.int16 if w0_dtype == torch.bfloat16 else torch.int32))
 
 
+@pytest.mark.parametrize("sdq", [False, True])
+def test_backbone_batch_matches_oracle(aw, orc, sdq):
+    """Several modules in one call (two dtype runs, so two launches; shapes
+    with a partial SDQ block and a zero group): every output equals the oracle's
+    and the single call's bit for bit."""
+    shapes = [(40, 512), (300, 1024), (7, 384), (256, 2048)]
+    dts = [torch.bfloat16, torch.bfloat16, torch.float32, torch.float32]
+    Ws = [torch.from_numpy(_weights(7 * i + r, r, c)).to(dt).cuda() for i, ((r, c), dt) in enumerate(zip(shapes, dts))]
+    got = aw.awsrc_rtn_quantize_batch(Ws, sdq=sdq)
+    torch.cuda.synchronize()
+    for W, g in zip(Ws, got):
+        single = aw.awsrc_rtn_quantize(W, sdq=sdq)
+        for key in single:
+            assert torch.equal(single[key].view(torch.uint8), g[key].view(torch.uint8)), key
+        want = orc.rtn_quantize(W.float().cpu().numpy(), sdq=sdq)
+        assert np.array_equal(g["codes"].cpu().numpy(), _pack(want["q"]))
+        assert np.array_equal(g["scales"].cpu().numpy().view(np.uint16), want["s16"])
+        if sdq:
+            assert np.array_equal(g["sdq_codes"].cpu().numpy(), want["c8"])
+            assert np.array_equal(g["sdq_consts"].cpu().numpy().view(np.uint32), want["consts"].view(np.uint32))
+        W0 = torch.from_numpy(want["W0"]).to(W.dtype)
+        itype = torch.int16 if W.dtype == torch.bfloat16 else torch.int32
+        assert torch.equal(g["W0"].cpu().view(itype), W0.view(itype))
+
 
 def test_sdq_savings_returned_to_the_sidecar_budget(aw, orc):
     """Sec. 3.3 end to end on one Qwen2.5-3B-shaped layer: the RTN-INT4 backbone
