@@ -165,7 +165,11 @@ awsrc_status make_prm(const awsrc_params* p, Prm* out) {
   r.c = (float)(1.0 / std::sqrt((double)p->C));
   r.c2 = 1.0f / (float)p->C;
   r.W = (p->C + 63) / 64;
+  // selectors padded to whole search chunks: 32 seeds (U, C = 64, P = 4) or 12
+  // (P_F, C = 64, P = 4; then a multiple of 96, which keeps the atom table of
+  // 32-seed chunks whole), padding selectors having all-zero masks
   r.S_pad = (p->S + 31) / 32 * 32;
+  if (p->variant == AWSRC_VARIANT_PF && p->C == 64 && p->P == 4) r.S_pad = (p->S + 95) / 96 * 96;
   r.logC = ceil_log2_host((uint64_t)p->C);
   {
     const float qf = r.qmaxf;

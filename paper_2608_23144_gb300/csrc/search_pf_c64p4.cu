@@ -11,13 +11,16 @@
 // epilogue, which then factors G + eps I (LDL^T), solves, quantises and scores
 // every candidate exactly as the binary32 recipe does.
 //
-// Block: 128 tiles of one column block (row m = TMEM lane m), 17 warps. The
-// producer warp streams 8-seed chunks (FP16 atoms 4 KB, a slice of the U
-// search's atom table, and FP16 atom products 6 KB) through a 4-stage
+// Block: 128 tiles of one column block (row m = TMEM lane m), 13 warps. The
+// producer warp streams 12-seed chunks (FP16 atoms 6 KB, a slice of the U
+// search's atom table, and FP16 atom products 10 KB) through a 4-stage
 // bulk-copy ring and issues per chunk 16 MMAs into one of two TMEM
-// accumulators: Y_hi, Y_lo x atoms (N = 32) and D_hi, D_lo x products (N = 48).
-// Epilogue warp w takes TMEM lanes 32(w%4).. and seed pair w/4 of each chunk,
-// as a float2 stream over the pair's two seeds. Every mbarrier wait is bounded.
+// accumulators: Y_hi, Y_lo x atoms (N = 48) and D_hi, D_lo x products (N = 80,
+// the last 8 columns zero). The search is bound by this MMA chain, so a chunk
+// is as many seeds as two accumulators of 256 columns hold. Epilogue warp w
+// takes TMEM lanes 32(w%4).. and seed pairs 2(w/4), 2(w/4) + 1 of each chunk,
+// each as a float2 stream over the pair's two seeds. Every mbarrier wait is
+// bounded.
 #include "internal.h"
 #include "tc05.cuh"
 
@@ -28,20 +31,24 @@ namespace {
 using namespace tc05;
 
 constexpr int BM = 128;             // rows (tiles) per block = TMEM lanes
-constexpr int CH = 8;               // seeds per chunk
-constexpr int NA = 4 * CH;          // atom columns per chunk
+constexpr int CH = 12;              // seeds per chunk
+constexpr int NA = 4 * CH;          // atom columns per chunk (MMA N = 48)
 constexpr int NQ = 6 * CH;          // product columns per chunk
-constexpr int EW = 16;              // epilogue warps: 4 lane quarters x 4 seed pairs
+constexpr int NQP = 80;             // product columns padded to a multiple of 16 (MMA N)
+constexpr int EW = 12;              // epilogue warps: 4 lane quarters x 3 groups of 2 seed pairs
+constexpr int PPW = CH / 2 / (EW / 4);  // seed pairs per epilogue warp and chunk
 constexpr int NT = 32 * (EW + 1);
 constexpr int STAGES = 4;
-constexpr uint32_t kABytes = NA * 64 * 2;      // 4 KB
-constexpr uint32_t kQBytes = NQ * 64 * 2;      // 6 KB
+constexpr uint32_t kABytes = NA * 64 * 2;      // 6 KB
+constexpr uint32_t kQBytes = NQP * 64 * 2;     // 10 KB (the last 8 columns zero)
 constexpr uint32_t kStageBytes = kABytes + kQBytes;
 constexpr uint32_t kTmemCols = 512;            // 2 accumulators of 256 columns
-constexpr int kYH = 0, kYL = 32, kDH = 64, kDL = 112;  // columns within an accumulator
+constexpr int kYH = 0, kYL = NA, kDH = 2 * NA, kDL = 2 * NA + NQP;  // columns within an accumulator
+static_assert(kDL + NQP <= 256, "accumulator of 256 columns");
 constexpr uint32_t kIdA = idesc_f16(BM, NA);
-constexpr uint32_t kIdQ = idesc_f16(BM, NQ);
-static_assert(EW / 4 == CH / 2, "one seed pair per epilogue warp and chunk");
+constexpr uint32_t kIdQ = idesc_f16(BM, NQP);
+static_assert(PPW == 2 && (EW / 4) * PPW * 2 == CH, "two seed pairs per epilogue warp and chunk");
+static_assert(kStageBytes % 1024 == 0 && kABytes % 1024 == 0, "stage layout");
 
 struct Smem {
   __half A[4][BM * 64];  // Y_hi, Y_lo, D_hi, D_lo: canonical K-major, no swizzle
@@ -55,8 +62,8 @@ struct Smem {
   float invd0[BM];    // 1 / D_0 = 1 / diag
   float inv_qy[BM], inv_qd[BM];
   int rowok[BM];
-  float red_g[4][BM];
-  uint32_t red_s[4][BM];
+  float red_g[EW / 4][BM];
+  uint32_t red_s[EW / 4][BM];
   unsigned long long full[STAGES], afull[2], tempty[2];
   uint32_t tmem_base;
 };
@@ -398,7 +405,7 @@ __global__ void __launch_bounds__(NT, 1)
   } else {
     // ------------------------------------------------------------ epilogue --
     const int m = 32 * (warp & 3) + lane;
-    const int pi = warp >> 2;  // seed pair of each chunk
+    const int grp = warp >> 2;  // seed pairs 2 grp and 2 grp + 1 of each chunk
     const uint32_t lane_base = (uint32_t)(32 * (warp & 3)) << 16;
     const float tqc = sm.tqc[m], tqdc = sm.tqdc[m], gd = sm.gd[m], diag = sm.diag[m], invd0 = sm.invd0[m];
     float bg = neg_inf();
@@ -408,44 +415,52 @@ __global__ void __launch_bounds__(NT, 1)
       if (!mbar_wait(&sm.afull[tb], (uint32_t)((k >> 1) & 1), pr.wait_ns)) { timed_out = true; break; }
       tc_fence_after();
       const uint32_t base = tmem + lane_base + (uint32_t)(tb * 256);
-      float ah[8], al[8], qh[12], ql[12];
-      tmem_ld8(base + kYH + 8 * pi, ah);
-      tmem_ld8(base + kYL + 8 * pi, al);
-      // the pair's 12 product columns start at 12 pi: the 8-column load goes
-      // where it is 8-aligned (warp-uniform branch on pi)
-      if ((pi & 1) == 0) {
-        tmem_ld8(base + kDH + 12 * pi, qh);
-        tmem_ld4(base + kDH + 12 * pi + 8, qh + 8);
-        tmem_ld8(base + kDL + 12 * pi, ql);
-        tmem_ld4(base + kDL + 12 * pi + 8, ql + 8);
-      } else {
-        tmem_ld4(base + kDH + 12 * pi, qh);
-        tmem_ld8(base + kDH + 12 * pi + 4, qh + 4);
-        tmem_ld4(base + kDL + 12 * pi, ql);
-        tmem_ld8(base + kDL + 12 * pi + 4, ql + 4);
-      }
+      // both pairs' columns are loaded before the accumulator is released, so
+      // the next MMAs into it wait for no scoring; a pair's 12 product columns
+      // start at 12 pi, 8-aligned for the even pair, 4 past for the odd one
+      float ah[2][8], al[2][8], qh[2][12], ql[2][12];
+      const int p0 = 2 * grp, p1 = p0 + 1;
+      tmem_ld8(base + kYH + 8 * p0, ah[0]);
+      tmem_ld8(base + kYL + 8 * p0, al[0]);
+      tmem_ld8(base + kDH + 12 * p0, qh[0]);
+      tmem_ld4(base + kDH + 12 * p0 + 8, qh[0] + 8);
+      tmem_ld8(base + kDL + 12 * p0, ql[0]);
+      tmem_ld4(base + kDL + 12 * p0 + 8, ql[0] + 8);
+      tmem_ld8(base + kYH + 8 * p1, ah[1]);
+      tmem_ld8(base + kYL + 8 * p1, al[1]);
+      tmem_ld4(base + kDH + 12 * p1, qh[1]);
+      tmem_ld8(base + kDH + 12 * p1 + 4, qh[1] + 4);
+      tmem_ld4(base + kDL + 12 * p1, ql[1]);
+      tmem_ld8(base + kDL + 12 * p1 + 4, ql[1] + 4);
       asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      tmem_tie8(ah); tmem_tie8(al);
 #pragma unroll
-      for (int i = 0; i < 3; ++i) { tmem_tie4(qh + 4 * i); tmem_tie4(ql + 4 * i); }
+      for (int j = 0; j < 2; ++j) {
+        tmem_tie8(ah[j]);
+        tmem_tie8(al[j]);
+#pragma unroll
+        for (int i = 0; i < 3; ++i) { tmem_tie4(qh[j] + 4 * i); tmem_tie4(ql[j] + 4 * i); }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.tempty[tb]);
-      float2 g = pf_pair_gain<FAST>(pr, ah, al, qh, ql, tqc, tqdc, gd, diag, invd0);
-      const int sx = (c0 + k) * CH + 2 * pi;
-      if (sx + 1 >= pr.S) {  // padding selectors (all-zero masks) are not candidates
-        if (sx >= pr.S) g.x = neg_inf();
-        g.y = neg_inf();
-      }
-      // seeds reach a thread in increasing order: a strictly greater gain wins
-      const float cm = fmaxf(g.x, g.y);
-      if (cm > bg) {
-        bg = cm;
-        bsd = (uint32_t)(sx + (g.x == cm ? 0 : 1));
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        float2 g = pf_pair_gain<FAST>(pr, ah[j], al[j], qh[j], ql[j], tqc, tqdc, gd, diag, invd0);
+        const int sx = (c0 + k) * CH + 2 * (p0 + j);
+        if (sx + 1 >= pr.S) {  // padding selectors (all-zero masks) are not candidates
+          if (sx >= pr.S) g.x = neg_inf();
+          g.y = neg_inf();
+        }
+        // seeds reach a thread in increasing order: a strictly greater gain wins
+        const float cm = fmaxf(g.x, g.y);
+        if (cm > bg) {
+          bg = cm;
+          bsd = (uint32_t)(sx + (g.x == cm ? 0 : 1));
+        }
       }
     }
-    sm.red_g[pi][m] = bg;
-    sm.red_s[pi][m] = bsd;
+    sm.red_g[grp][m] = bg;
+    sm.red_s[grp][m] = bsd;
   }
   tc_fence_before();
   if (__syncthreads_or(timed_out)) {
@@ -454,7 +469,7 @@ __global__ void __launch_bounds__(NT, 1)
     float g = sm.red_g[0][tid];
     uint32_t s = sm.red_s[0][tid];
 #pragma unroll
-    for (int i = 1; i < 4; ++i) {
+    for (int i = 1; i < EW / 4; ++i) {
       if (better(sm.red_g[i][tid], sm.red_s[i][tid], g, s)) { g = sm.red_g[i][tid]; s = sm.red_s[i][tid]; }
     }
     const int64_t row = rb * BM + tid;
@@ -486,18 +501,25 @@ __global__ void __launch_bounds__(NT, 1)
 }
 
 // FP16 products of atom pairs in the order the MMAs read them: chunk c
-// (8 seeds) is a 48 x 64 K-major operand in 6 KB; item i (16 bytes, one
-// core-matrix row) is chunk i / 384, column group n8 = (i >> 6) % 6, k group
-// (i >> 3) & 7, row i & 7; column n = 8*n8 + r carries product q = (n % 12) / 2
-// (pairs (1,0), (2,0), (2,1), (3,0), (3,1), (3,2)) of seed 8c + 2*(n / 12) + n % 2.
+// (12 seeds) is an 80 x 64 K-major operand in 10 KB; item i (16 bytes, one
+// core-matrix row) is chunk i / 640, column group n8 = (i >> 6) % 10, k group
+// (i >> 3) & 7, row i & 7; column n = 8*n8 + r < 72 carries product q =
+// (n % 12) / 2 (pairs (1,0), (2,0), (2,1), (3,0), (3,1), (3,2)) of seed
+// 12c + 2*(n / 12) + n % 2, and columns 72 .. 79 are zero.
+constexpr int kQItems = NQP * 8;  // 16-byte items per chunk
+
 __global__ void products_kernel(const uint64_t* __restrict__ masks, uint4* __restrict__ out, int S_pad) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t n_items = (int64_t)(S_pad / CH) * 384;
+  const int64_t n_items = (int64_t)(S_pad / CH) * kQItems;
   if (i >= n_items) return;
-  const int64_t chunk = i / 384;
-  const int w = (int)(i % 384);
+  const int64_t chunk = i / kQItems;
+  const int w = (int)(i % kQItems);
   const int r = w & 7, kg = (w >> 3) & 7, n8 = w >> 6;
   const int n = 8 * n8 + r;
+  if (n >= NQ) {
+    out[i] = make_uint4(0u, 0u, 0u, 0u);
+    return;
+  }
   const int q = (n % 12) >> 1;
   const int64_t seed = chunk * CH + 2 * (n / 12) + (n & 1);
   const int pa = q < 1 ? 1 : (q < 3 ? 2 : 3);
@@ -520,7 +542,7 @@ int search_pf_c64p4_chunk() { return CH; }
 size_t search_pf_c64p4_table_bytes(int S_pad) { return (size_t)(S_pad / CH) * kQBytes; }
 
 cudaError_t launch_products_pf_c64p4(const Prm& pr, const uint64_t* masks, void* out, cudaStream_t st) {
-  const int64_t n = (int64_t)(pr.S_pad / CH) * 384;
+  const int64_t n = (int64_t)(pr.S_pad / CH) * kQItems;
   products_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(masks, static_cast<uint4*>(out), pr.S_pad);
   note_launches(1);
   return cudaGetLastError();
