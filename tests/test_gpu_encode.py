@@ -40,6 +40,9 @@ CASES = [
     ("c64p3_u_generic", dict(C=64, P=3, b=4, S=70), [(90, 192), (5, 64)], "bf16", False),
     ("c64p2_pf_generic", dict(C=64, P=2, b=3, S=21, variant=1), [(77, 128)], "bf16", True),
     ("c32p4_pf_s3", dict(C=32, P=4, b=4, S=3, variant=1), [(50, 96)], "f32", True),
+    # the tcgen05 P_F search takes 12-seed chunks: selectors padded to 96
+    ("c64p4_pf_s100", dict(C=64, P=4, b=4, S=100, variant=1), [(140, 192), (3, 64)], "bf16", True),
+    ("c64p4_pf_s13_b5", dict(C=64, P=4, b=5, S=13, variant=1), [(33, 128)], "f32", True),
 ]
 
 
@@ -123,15 +126,19 @@ def test_degenerate_tiles(aw, orc):
         assert got["gain"][t] == -np.inf and got["seed"][t] == 0 and not got["code"][t].any()
 
 
-def test_seed_splits_do_not_change_the_result(aw, orc):
+@pytest.mark.parametrize("variant", [0, 1])
+def test_seed_splits_do_not_change_the_result(aw, orc, variant):
     """A small module is split over many blocks along the seed axis; a large one is
     not. The same rows embedded in both must give identical candidates."""
-    mods = _mods([(8, 64)], "bf16")
-    big = _mods([(1500, 64)], "bf16", seed=5)
+    mods = _mods([(8, 64)], "bf16", fisher=bool(variant))
+    big = _mods([(1500, 64)], "bf16", seed=5, fisher=bool(variant))
     big[0]["W"][:8] = mods[0]["W"]
     big[0]["W0"][:8] = mods[0]["W0"]
     big[0]["act"] = mods[0]["act"].clone()
-    prm = aw.params(C=64, P=4, S=512)
+    if variant:
+        big[0]["fisher"][:8] = mods[0]["fisher"]
+        big[0]["w_act"], big[0]["w_fisher"] = mods[0]["w_act"], mods[0]["w_fisher"]
+    prm = aw.params(C=64, P=4, S=512, variant=variant)
     a = aw.candidates_to_numpy(aw.awsrc_encode_tiles(prm, to_dev(mods)))
     b = aw.candidates_to_numpy(aw.awsrc_encode_tiles(prm, to_dev(big)))[:8]
     assert_candidates_equal(a, b, "split vs unsplit")
