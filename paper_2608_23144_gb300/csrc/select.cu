@@ -7,7 +7,9 @@
 // one sort yields each module's ranking in its own contiguous segment; PF keeps
 // one global ranking whose prefixes are the rate cuts.
 //
-// The sort is a stable LSD radix sort with 8-bit digits: per pass a block
+// The sort is a stable LSD radix sort with 8-bit digits over the module and
+// gain fields (the keys are made in tile order, which the stable passes keep
+// among equal fields, so the tile field needs no pass): per pass a block
 // histogram, a per-digit scan over blocks, and a scatter whose in-block ranks
 // come from __match_any_sync over each warp plus per-warp digit counters.
 // Counts, cuts, packing and the header are device kernels, so the whole step
@@ -370,9 +372,12 @@ awsrc_status select_run(const Prm& pr, const SelectPlan& sp, const int64_t* tile
     make_keys_kernel<<<(unsigned)((sp.T + 255) / 256), 256, 0, st>>>(cands, ka, a);
     note_launches(1);
     if (cudaGetLastError() != cudaSuccess) return check_launch("select: keys");
-    const int passes = (sp.key_bits + 7) / 8;
+    // the tile field (the low bits) needs no pass: the keys start in tile
+    // order and every pass is stable, so equal (module, gain) keys keep it
+    const int low = sp.tile_bits_local;
+    const int passes = (sp.key_bits - low + 7) / 8;
     for (int ps = 0; ps < passes; ++ps) {
-      const int shift = 8 * ps;
+      const int shift = low + 8 * ps;
       radix_hist_kernel<<<(unsigned)sp.nblocks, RT, 0, st>>>(ka, sp.T, shift, hist, sp.nblocks);
       radix_scan_rows_kernel<<<256, 1024, 0, st>>>(hist, sp.nblocks, totals);
       radix_scatter_kernel<<<(unsigned)sp.nblocks, RT, 0, st>>>(ka, kb, sp.T, shift, hist,
