@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   __shared__ int dok;
   __shared__ float dmax;
   __shared__ float two_qd;
+  __shared__ int sdq;  // sum of the fixed-point weights (exact)
   if (threadIdx.x == 0) dok = 1;
   __syncthreads();
   for (int j = threadIdx.x; j < C; j += blockDim.x) {
@@ -109,10 +110,12 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     if (!(v >= 0.0f && v <= 4294967296.0f)) dok = 0;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {  // the column block's largest |d|, one warp
     float m = 0.0f;
-    for (int j = 0; j < C; ++j) m = fmaxf(m, fabsf(d[j]));
-    dmax = m;
+    for (int j = threadIdx.x; j < C; j += 32) m = fmaxf(m, fabsf(d[j]));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    if (threadIdx.x == 0) dmax = m;
   }
   __syncthreads();
   int qd;
@@ -120,6 +123,13 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
   for (int j = threadIdx.x; j < C; j += blockDim.x) Dq[j] = inv == 0.0f ? 0 : fixed_point_int(d[j], inv);
   if (threadIdx.x == 0) two_qd = pow2f(qd);
   __syncthreads();
+  if (threadIdx.x < 32) {  // integer sum, so the order does not matter
+    int t = 0;
+    for (int j = threadIdx.x; j < C; j += 32) t += Dq[j];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+    if (threadIdx.x == 0) sdq = t;
+  }
   for (int i = threadIdx.x; i < (C / 4) * 16; i += blockDim.x) {
     const int g = i >> 4, nb = i & 15;
     int v = 0;
@@ -129,11 +139,13 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     Dt[g][nb] = v;
   }
   __syncthreads();
-  const int s = blockIdx.x * blockDim.x + threadIdx.x;
-  if (s >= pr.S_pad) return;
+  // threads past S_pad (the last block of a small S_pad) score a dummy seed
+  // whose entries are never written; every thread reaches the barrier below
+  const int s_raw = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s_raw >= pr.S_pad && !pairs) return;
+  const int s = min(s_raw, pr.S_pad - 1);
   constexpr int NL = P * (P - 1) / 2 > 0 ? P * (P - 1) / 2 : 1;
-  int sd = 0;
-  for (int j = 0; j < C; ++j) sd += Dq[j];
+  const int sd = sdq;
   const float gd = __fmul_rn(pr.c2, __fmul_rn(__int2float_rn(sd), two_qd));
   float Goff[NL], L[NL], invD[P];
   const uint64_t* mk = masks + (size_t)s * P * pr.W;
@@ -168,9 +180,12 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     out[P * (P - 1) + P] = gd;
   }
   if (pairs) {
-    // seed s is component s & 1 of seed pair s >> 1 (entries start on even seeds)
-    float* po = reinterpret_cast<float*>(pairs) +
-                (size_t)((md.gram_off + cb * pr.S_pad + s) >> 1) * pair_stride(P) * 2 + (s & 1);
+    // seed s is component s & 1 of seed pair s >> 1 (entries start on even
+    // seeds); the block's 64 pairs are one contiguous run of the table, built
+    // in shared memory and written out in 16-byte stores
+    constexpr int ps = pair_stride(P);
+    __shared__ __align__(16) float stage[128 / 2 * ps * 2];
+    float* po = stage + (threadIdx.x >> 1) * ps * 2 + (threadIdx.x & 1);
     constexpr int nl = P * (P - 1) / 2;
     // pr.prune == 0 scores every candidate (the same results, for tests of the bound)
     const float m = ok && pr.prune ? bound_multiplier<P>(gd, Goff, eps) : __int_as_float(0x7f800000);
@@ -179,13 +194,21 @@ __global__ void __launch_bounds__(128) gram_u_kernel(Prm pr, LaunchDesc ld,
     // invD * m rounded up: the bound's terms z_k (z_k invD_k m) are then never
     // below the exact z_k^2 invD_k m (m = +inf disables pruning)
 #pragma unroll
-    for (int k = 0; k < P; ++k) po[2 * (nl + k)] = ok ? __double2float_ru((double)invD[k] * (double)m) : qnan;
+    for (int k = 0; k < P; ++k) po[2 * (nl + k)] = ok ? __fmul_ru(invD[k], m) : qnan;
 #pragma unroll
     for (int k = 0; k < P; ++k) po[2 * (nl + P + k)] = ok ? invD[k] : qnan;
 #pragma unroll
     for (int i = 0; i < nl; ++i) po[2 * (nl + 2 * P + i)] = pr.fast_pow2 ? __fmul_rn(2.0f, Goff[i]) : Goff[i];
     po[2 * (2 * nl + 2 * P)] = gd;
-    for (int i = 2 * nl + 2 * P + 1; i < pair_stride(P); ++i) po[2 * i] = 0.0f;
+    for (int i = 2 * nl + 2 * P + 1; i < ps; ++i) po[2 * i] = 0.0f;
+    __syncthreads();
+    // seeds s0 .. s0 + 127 of this column block (s0 even, S_pad a multiple of 32)
+    const int s0 = blockIdx.x * blockDim.x;
+    const int npairs = min((int)blockDim.x, pr.S_pad - s0) / 2;
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(pairs) +
+                                            (size_t)((md.gram_off + cb * pr.S_pad + s0) >> 1) * ps * 2);
+    const float4* src = reinterpret_cast<const float4*>(stage);
+    for (int i = threadIdx.x; i < npairs * ps / 2; i += blockDim.x) dst[i] = src[i];
   }
 }
 
