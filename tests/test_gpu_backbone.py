@@ -76,6 +76,19 @@ def test_backbone_batch_matches_oracle(aw, orc, sdq):
         assert torch.equal(g["W0"].cpu().view(itype), W0.view(itype))
 
 
+def test_backbone_batch_of_many_modules(aw):
+    """More modules than one launch takes (20 > 16): the call splits into
+    launches and every output still equals the single call's."""
+    Ws = [torch.from_numpy(_weights(100 + i, 3 + i % 5, 128 * (1 + i % 3))).to(torch.bfloat16).cuda()
+          for i in range(20)]
+    for sdq in (False, True):
+        got = aw.awsrc_rtn_quantize_batch(Ws, sdq=sdq)
+        for W, g in zip(Ws, got):
+            single = aw.awsrc_rtn_quantize(W, sdq=sdq)
+            for key in single:
+                assert torch.equal(single[key].view(torch.uint8), g[key].view(torch.uint8)), key
+
+
 def test_sdq_savings_returned_to_the_sidecar_budget(aw, orc):
     """Sec. 3.3 end to end on one Qwen2.5-3B-shaped layer: the RTN-INT4 backbone
     with SDQ scales (W0 from the double-quantised scales), the encoder against
