@@ -261,18 +261,24 @@ __device__ __forceinline__ uint4 record_slot(const Prm& pr, const DecRec& d) {
 template <typename TI, typename TO, int G>
 __device__ __forceinline__ void patch_vec_tab(const Prm& pr, const Vec<TI, G>& w, const uint4& slot, uint4 nb,
                                               int j0, float sc, Vec<TO, G>& o) {
-  float k[G];
+  const KTab kt = k_tables(slot);
+  const KMagic km = k_magic(pr);
+  float k[G];  // k_j c when c is a power of two, else k_j
   if constexpr (G == 8) {
-    table_k4(slot, nb.x, nb.y, k);
-    table_k4(slot, nb.x >> 16, nb.z, k + 4);
+    table_k4(kt, nb.x, nb.y, km, k);
+    table_k4(kt, nb.x >> 16, nb.z, km, k + 4);
   } else {
     const bool hi = (j0 & 4) != 0;
-    table_k4(slot, hi ? nb.x >> 16 : nb.x, hi ? nb.z : nb.y, k);
+    table_k4(kt, hi ? nb.x >> 16 : nb.x, hi ? nb.z : nb.y, km, k);
   }
-  const float2 c2 = make_float2(pr.c, pr.c), s2 = make_float2(sc, sc);
+  if (!km.folded) {
+#pragma unroll
+    for (int e = 0; e < G; ++e) k[e] = __fmul_rn(k[e], pr.c);
+  }
+  const float2 s2 = make_float2(sc, sc);
 #pragma unroll
   for (int e = 0; e < G; e += 2) {
-    const float2 r = __fmul2_rn(__fmul2_rn(make_float2(k[e], k[e + 1]), c2), s2);
+    const float2 r = __fmul2_rn(make_float2(k[e], k[e + 1]), s2);
     Io2<TO>::st(o.v + e, __fadd2_rn(Io2<TI>::ld(w.v + e), r));
   }
 }

@@ -234,25 +234,25 @@ struct WalkList {
   uint16_t tile[32 * kWalkRound];
 };
 
-template <int M>
+template <int M, int NB>
 __device__ __forceinline__ void walk_tables(const Prm& pr, const GemvArgs& a, const unsigned long long* mrow,
                                             int n_cb, unsigned long long ent0, const float* xsm, int xs_stride,
                                             int lane, WalkList& wl, float2* racc) {
   const int lshift = pr.logC - 4;  // log2 of the lanes per tile
   const int tp = 32 >> lshift;     // tiles per pass
   const int q = lane >> lshift, sub = lane & ((1 << lshift) - 1);
-  const float2 c2 = make_float2(pr.c, pr.c);
-  for (int r0 = 0; r0 < n_cb; r0 += 32 * kWalkRound) {
-    const int nb = min(kWalkRound, (n_cb - r0 + 31) >> 5);
-    unsigned long long e[kWalkRound];
+  const KMagic km = k_magic(pr);
+  for (int r0 = 0; r0 < n_cb; r0 += 32 * NB) {
+    const int nb = min(NB, (n_cb - r0 + 31) >> 5);
+    unsigned long long e[NB];
 #pragma unroll
-    for (int i = 0; i < kWalkRound; ++i) {
+    for (int i = 0; i < NB; ++i) {
       const int t = r0 + 32 * i + lane;
       e[i] = (r0 == 0 && i == 0) ? ent0 : ((i < nb && t < n_cb) ? __ldg(mrow + t) : 0ull);
     }
     int n = 0;
 #pragma unroll
-    for (int i = 0; i < kWalkRound; ++i) {
+    for (int i = 0; i < NB; ++i) {
       if (i < nb) {
         const unsigned rec = __ballot_sync(0xffffffffu, e[i] != 0ull);
         if (e[i] != 0ull) {
@@ -272,15 +272,20 @@ __device__ __forceinline__ void walk_tables(const Prm& pr, const GemvArgs& a, co
         const uint4* nbp = a.nib + (size_t)((uint32_t)(en >> 16) & 0xFFFFu) * (pr.C >> 3) + 2 * sub;
         const uint4 n0 = __ldg(nbp), n1 = __ldg(nbp + 1);
         const float sc = sidecar_scale(pr, (int16_t)(uint16_t)(en & 0xFFFFull));
-        float k[16];
-        table_k4(slot, n0.x, n0.y, k);
-        table_k4(slot, n0.x >> 16, n0.z, k + 4);
-        table_k4(slot, n1.x, n1.y, k + 8);
-        table_k4(slot, n1.x >> 16, n1.z, k + 12);
+        const KTab kt = k_tables(slot);
+        float k[16];  // k_j c when c is a power of two, else k_j
+        table_k4(kt, n0.x, n0.y, km, k);
+        table_k4(kt, n0.x >> 16, n0.z, km, k + 4);
+        table_k4(kt, n1.x, n1.y, km, k + 8);
+        table_k4(kt, n1.x >> 16, n1.z, km, k + 12);
+        if (!km.folded) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) k[i] = __fmul_rn(k[i], pr.c);
+        }
         const float2 s2 = make_float2(sc, sc);
         float2 r[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) r[i] = __fmul2_rn(__fmul2_rn(make_float2(k[2 * i], k[2 * i + 1]), c2), s2);
+        for (int i = 0; i < 8; ++i) r[i] = __fmul2_rn(make_float2(k[2 * i], k[2 * i + 1]), s2);
         // inputs col0 .. col0 + 15 (col0 a multiple of 16): four float4 128 floats apart
         const float* xq = xsm + xs_index(tile * pr.C + 16 * sub);
 #pragma unroll
@@ -424,7 +429,10 @@ __global__ void __launch_bounds__(32 * kGemvWarps, M <= 2 ? 3 : 1) gemv_warp_ker
     if (a.map) {
       const unsigned long long* mrow = a.map + tk.tile_off + row * n_cb;
       if (tables) {
-        walk_tables<M>(pr, a, mrow, n_cb, cur.ent, xsm, xs_stride, lane, wlist[warp], racc);
+        if (n_cb <= 32)  // one batch of map entries, already loaded with the row head
+          walk_tables<M, 1>(pr, a, mrow, n_cb, cur.ent, xsm, xs_stride, lane, wlist[warp], racc);
+        else
+          walk_tables<M, kWalkRound>(pr, a, mrow, n_cb, cur.ent, xsm, xs_stride, lane, wlist[warp], racc);
       } else {
         for (int tb = 0; tb < n_cb; tb += 32) {
           const unsigned long long ent =

@@ -19,8 +19,9 @@
 // the last 8 columns zero). The search is bound by this MMA chain, so a chunk
 // is as many seeds as two accumulators of 256 columns hold. Epilogue warp w
 // takes TMEM lanes 32(w%4).. and seed pairs 2(w/4), 2(w/4) + 1 of each chunk,
-// each as a float2 stream over the pair's two seeds. Every mbarrier wait is
-// bounded.
+// each as a float2 stream over the pair's two seeds, the two pairs factored
+// side by side so that their dependency chains interleave. Every mbarrier
+// wait is bounded.
 #include "internal.h"
 #include "tc05.cuh"
 
@@ -85,100 +86,161 @@ __device__ __forceinline__ float2 neg2(float2 v) { return make_float2(-v.x, -v.y
 
 __device__ __forceinline__ bool pivot_ok(float d) { return d > 0.0f && d <= 3.402823466e38f; }
 
-// rcp_rn on both components: the hardware approximations, then Markstein's
-// fused correction y + y (1 - x y) as two packed fmas (each component rounds
-// as the scalar form does). A component outside [2^-125, 2^125) takes
-// __frcp_rn instead, in a branch the active lanes take together only when
-// one of them needs it.
-__device__ __forceinline__ float2 rcp2_rn(float2 x) {
-  float yx, yy;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yx) : "f"(x.x));
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yy) : "f"(x.y));
-  const float2 y = make_float2(yx, yy);
-  const float2 e = __ffma2_rn(make_float2(-x.x, -x.y), y, make_float2(1.0f, 1.0f));
-  float2 r = __ffma2_rn(y, e, y);
-  const bool fx = __float_as_uint(x.x) - 0x01000000u < 0x7D000000u - 0x01000000u;
-  const bool fy = __float_as_uint(x.y) - 0x01000000u < 0x7D000000u - 0x01000000u;
-  if (__any_sync(__activemask(), !(fx && fy))) {
-    if (!fx) r.x = __frcp_rn(x.x);
-    if (!fy) r.y = __frcp_rn(x.y);
+// rcp_rn on both components of NP pairs: the hardware approximations, then
+// Markstein's fused correction y + y (1 - x y) as two packed fmas (each
+// component rounds as the scalar form does). A component outside
+// [2^-125, 2^125) takes __frcp_rn instead, in a branch the active lanes take
+// together only when one of them needs it.
+template <int NP>
+__device__ __forceinline__ void rcp2_rn(const float2* x, float2* r) {
+  bool fx[NP], fy[NP], ok = true;
+#pragma unroll
+  for (int j = 0; j < NP; ++j) {
+    float yx, yy;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yx) : "f"(x[j].x));
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(yy) : "f"(x[j].y));
+    const float2 y = make_float2(yx, yy);
+    const float2 e = __ffma2_rn(make_float2(-x[j].x, -x[j].y), y, make_float2(1.0f, 1.0f));
+    r[j] = __ffma2_rn(y, e, y);
+    fx[j] = __float_as_uint(x[j].x) - 0x01000000u < 0x7D000000u - 0x01000000u;
+    fy[j] = __float_as_uint(x[j].y) - 0x01000000u < 0x7D000000u - 0x01000000u;
+    ok = ok && fx[j] && fy[j];
   }
-  return r;
+  if (__any_sync(__activemask(), !ok)) {
+#pragma unroll
+    for (int j = 0; j < NP; ++j) {
+      if (!fx[j]) r[j].x = __frcp_rn(x[j].x);
+      if (!fy[j]) r[j].y = __frcp_rn(x[j].y);
+    }
+  }
 }
 
-// Fit of one seed pair of this thread's row; ah/al: atom p of the two seeds
-// at [2p], [2p+1]; qh/ql: product q (tri order) at [2q], [2q+1]. Returns b, the
+// quant_gain_fast2 with the off-diagonal G as it is rather than doubled: each
+// off-diagonal term takes q_p * (2 q_r), the exact double of q_p q_r (codes
+// are small integers), so that fma(q_p (2 q_r), G, Qq) rounds the same exact
+// value as fma(q_p q_r, 2 G, Qq) (|G| <= 2^38 on the tile domain: 2 G is exact).
+template <int P>
+__device__ __forceinline__ float2 quant_gain_fast2_g(const Prm& pr, const float2* alpha, const float2* bv,
+                                                     float2 gd, const float2* Goff) {
+  float m0 = fabsf(alpha[0].x), m1 = fabsf(alpha[0].y);
+#pragma unroll
+  for (int p = 1; p < P; ++p) {
+    m0 = fmaxf(m0, fabsf(alpha[p].x));
+    m1 = fmaxf(m1, fabsf(alpha[p].y));
+  }
+  const uint32_t s0 = fast_scale_bits(pr, m0), s1 = fast_scale_bits(pr, m1);
+  const float2 sc = make_float2(__uint_as_float(s0), __uint_as_float(s1));
+  const float2 nsc = make_float2(__uint_as_float(s0 | 0x80000000u), __uint_as_float(s1 | 0x80000000u));
+  const float2 inv = make_float2(__uint_as_float(0x7F000000u - s0), __uint_as_float(0x7F000000u - s1));
+  const float2 magic = make_float2(12582912.0f, 12582912.0f);
+  const float2 nmagic = make_float2(-12582912.0f, -12582912.0f);
+  float2 q[P], q2[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    q[p] = __fadd2_rn(__ffma2_rn(alpha[p], inv, magic), nmagic);
+    q2[p] = __fadd2_rn(q[p], q[p]);
+  }
+  float2 Aq = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int p = 0; p < P; ++p) Aq = __ffma2_rn(q[p], bv[p], Aq);
+  float2 Qq = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    Qq = __ffma2_rn(__fmul2_rn(q[p], q[p]), gd, Qq);
+#pragma unroll
+    for (int r = p + 1; r < P; ++r) Qq = __ffma2_rn(__fmul2_rn(q[p], q2[r]), Goff[tri(r, p)], Qq);
+  }
+  const float2 tn = __fmul2_rn(nsc, Qq);
+  float2 g = __fmul2_rn(sc, __ffma2_rn(make_float2(2.0f, 2.0f), Aq, tn));
+  if (s0 == 0u) g.x = -__int_as_float(0x7f800000);
+  if (s1 == 0u) g.y = -__int_as_float(0x7f800000);
+  return g;
+}
+
+// Fits of NP seed pairs of this thread's row, factored side by side so that
+// their chains interleave; ah/al[j]: atom p of pair j's two seeds at [2p],
+// [2p+1]; qh/ql[j]: product q (tri order) at [2q], [2q+1]. Gives b, the
 // off-diagonal G, alpha and whether each candidate's pivots are valid.
-__device__ __forceinline__ void pf_pair_fit(const float* ah, const float* al, const float* qh, const float* ql,
-                                            float tqc, float tqdc, float diag, float invd0, float2* bv,
-                                            float2* G, float2* alpha, bool* okx, bool* oky) {
+template <int NP>
+__device__ __forceinline__ void pf_fit(const float (*ah)[8], const float (*al)[8], const float (*qh)[12],
+                                       const float (*ql)[12], float tqc, float tqdc, float diag, float invd0,
+                                       float2 (*bv)[4], float2 (*G)[6], float2 (*alpha)[4], bool* okx, bool* oky) {
   const float2 tq2 = make_float2(tqc, tqc), td2 = make_float2(tqdc, tqdc);
-#pragma unroll
-  for (int p = 0; p < 4; ++p) bv[p] = pair_sum(ah, al, 2 * p, tq2);
-#pragma unroll
-  for (int q = 0; q < 6; ++q) G[q] = pair_sum(qh, ql, 2 * q, td2);
-  // LDL^T of G + eps I in the recipe's order; D_0 = diag for every seed
   const float2 dg = make_float2(diag, diag);
-  float2 nL[6], E[6], invD[4];
-  invD[0] = make_float2(invd0, invd0);
-  *okx = true;
-  *oky = true;
+  float2 nL[NP][6], E[NP][6], invD[NP][4];
+#pragma unroll
+  for (int j = 0; j < NP; ++j) {
+#pragma unroll
+    for (int p = 0; p < 4; ++p) bv[j][p] = pair_sum(ah[j], al[j], 2 * p, tq2);
+#pragma unroll
+    for (int q = 0; q < 6; ++q) G[j][q] = pair_sum(qh[j], ql[j], 2 * q, td2);
+    invD[j][0] = make_float2(invd0, invd0);  // D_0 = diag for every seed
+    okx[j] = true;
+    oky[j] = true;
+  }
+  // LDL^T of G + eps I in the recipe's order
 #pragma unroll
   for (int k = 1; k < 4; ++k) {
+    float2 dk[NP], rk[NP];
 #pragma unroll
-    for (int j = 0; j < k; ++j) {
-      float2 v = G[tri(k, j)];
+    for (int jp = 0; jp < NP; ++jp) {
 #pragma unroll
-      for (int i = 0; i < j; ++i) v = __ffma2_rn(nL[tri(k, i)], E[tri(j, i)], v);
-      E[tri(k, j)] = v;
-      nL[tri(k, j)] = __fmul2_rn(v, neg2(invD[j]));  // -(v * invD_j), exact negation
+      for (int j = 0; j < k; ++j) {
+        float2 v = G[jp][tri(k, j)];
+#pragma unroll
+        for (int i = 0; i < j; ++i) v = __ffma2_rn(nL[jp][tri(k, i)], E[jp][tri(j, i)], v);
+        E[jp][tri(k, j)] = v;
+        nL[jp][tri(k, j)] = __fmul2_rn(v, neg2(invD[jp][j]));  // -(v * invD_j), exact negation
+      }
+      dk[jp] = dg;
+#pragma unroll
+      for (int i = 0; i < k; ++i) dk[jp] = __ffma2_rn(nL[jp][tri(k, i)], E[jp][tri(k, i)], dk[jp]);
+      okx[jp] = okx[jp] && pivot_ok(dk[jp].x);
+      oky[jp] = oky[jp] && pivot_ok(dk[jp].y);
     }
-    float2 dk = dg;
+    rcp2_rn<NP>(dk, rk);
 #pragma unroll
-    for (int i = 0; i < k; ++i) dk = __ffma2_rn(nL[tri(k, i)], E[tri(k, i)], dk);
-    *okx = *okx && pivot_ok(dk.x);
-    *oky = *oky && pivot_ok(dk.y);
-    invD[k] = rcp2_rn(dk);
+    for (int jp = 0; jp < NP; ++jp) invD[jp][k] = rk[jp];
   }
-  ldl_solve2<4>(nL, invD, bv, alpha);
+#pragma unroll
+  for (int j = 0; j < NP; ++j) ldl_solve2<4>(nL[j], invD[j], bv[j], alpha[j]);
 }
 
-// Gains of one seed pair (operands as for pf_pair_fit).
-template <bool FAST>
-__device__ __forceinline__ float2 pf_pair_gain(const Prm& pr, const float* ah, const float* al, const float* qh,
-                                               const float* ql, float tqc, float tqdc, float gd, float diag,
-                                               float invd0, float2* alpha_out = nullptr) {
-  float2 bv[4], G[6], alpha[4];
-  bool okx, oky;
-  pf_pair_fit(ah, al, qh, ql, tqc, tqdc, diag, invd0, bv, G, alpha, &okx, &oky);
-  if (alpha_out) {
+// Gains of NP seed pairs (operands as for pf_fit).
+template <bool FAST, int NP>
+__device__ __forceinline__ void pf_gain(const Prm& pr, const float (*ah)[8], const float (*al)[8],
+                                        const float (*qh)[12], const float (*ql)[12], float tqc, float tqdc,
+                                        float gd, float diag, float invd0, float2* g,
+                                        float2 (*alpha_out)[4] = nullptr) {
+  float2 bv[NP][4], G[NP][6], alpha[NP][4];
+  bool okx[NP], oky[NP];
+  pf_fit<NP>(ah, al, qh, ql, tqc, tqdc, diag, invd0, bv, G, alpha, okx, oky);
 #pragma unroll
-    for (int p = 0; p < 4; ++p) alpha_out[p] = alpha[p];
+  for (int j = 0; j < NP; ++j) {
+    if (alpha_out) {
+#pragma unroll
+      for (int p = 0; p < 4; ++p) alpha_out[j][p] = alpha[j][p];
+    }
+    if constexpr (FAST) {
+      g[j] = quant_gain_fast2_g<4>(pr, alpha[j], bv[j], make_float2(gd, gd), G[j]);
+    } else {
+      float q4[4];
+      int sf;
+      float Gx[6], a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 6; ++i) Gx[i] = G[j][i].x;
+#pragma unroll
+      for (int p = 0; p < 4; ++p) { a[p] = alpha[j][p].x; b[p] = bv[j][p].x; }
+      g[j].x = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
+#pragma unroll
+      for (int i = 0; i < 6; ++i) Gx[i] = G[j][i].y;
+#pragma unroll
+      for (int p = 0; p < 4; ++p) { a[p] = alpha[j][p].y; b[p] = bv[j][p].y; }
+      g[j].y = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
+    }
+    if (!okx[j]) g[j].x = neg_inf();
+    if (!oky[j]) g[j].y = neg_inf();
   }
-  float2 g;
-  if constexpr (FAST) {
-    float2 G2[6];
-#pragma unroll
-    for (int q = 0; q < 6; ++q) G2[q] = __fmul2_rn(G[q], make_float2(2.0f, 2.0f));  // exact
-    g = quant_gain_fast2<4>(pr, alpha, bv, make_float2(gd, gd), G2);
-  } else {
-    float q4[4];
-    int sf;
-    float Gx[6], a[4], b[4];
-#pragma unroll
-    for (int i = 0; i < 6; ++i) Gx[i] = G[i].x;
-#pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].x; b[p] = bv[p].x; }
-    g.x = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
-#pragma unroll
-    for (int i = 0; i < 6; ++i) Gx[i] = G[i].y;
-#pragma unroll
-    for (int p = 0; p < 4; ++p) { a[p] = alpha[p].y; b[p] = bv[p].y; }
-    g.y = quant_gain<4>(pr, a, b, gd, Gx, q4, &sf);
-  }
-  if (!okx) g.x = neg_inf();
-  if (!oky) g.y = neg_inf();
-  return g;
 }
 
 // Codes and scale field of the winning seed of row m. The search keeps only
@@ -211,25 +273,24 @@ __device__ __forceinline__ float pf_winner(const Prm& pr, const Smem& sm, int m,
 #pragma unroll
     for (int q = 0; q < 6; ++q) nd[q] += ((wq[q] >> j) & 1ull) ? d : 0;
   }
-  float ah[8], al[8], qh[12], ql[12];
+  float ah[1][8], al[1][8], qh[1][12], ql[1][12];
 #pragma unroll
   for (int p = 0; p < 4; ++p) {
     const int u = ty - 2 * ny[p];  // |u| <= 64 * 2^21
-    ah[2 * p] = ah[2 * p + 1] = (float)(u >> 11);
-    al[2 * p] = al[2 * p + 1] = (float)(u & 2047);
+    ah[0][2 * p] = ah[0][2 * p + 1] = (float)(u >> 11);
+    al[0][2 * p] = al[0][2 * p + 1] = (float)(u & 2047);
   }
 #pragma unroll
   for (int q = 0; q < 6; ++q) {
     const int u = td - 2 * nd[q];
-    qh[2 * q] = qh[2 * q + 1] = (float)(u >> 11);
-    ql[2 * q] = ql[2 * q + 1] = (float)(u & 2047);
+    qh[0][2 * q] = qh[0][2 * q + 1] = (float)(u >> 11);
+    ql[0][2 * q] = ql[0][2 * q + 1] = (float)(u & 2047);
   }
-  float2 alpha[4];
-  const float2 g = pf_pair_gain<FAST>(pr, ah, al, qh, ql, sm.tqc[m], sm.tqdc[m], sm.gd[m], sm.diag[m],
-                                      sm.invd0[m], alpha);
+  float2 alpha[1][4], g;
+  pf_gain<FAST, 1>(pr, ah, al, qh, ql, sm.tqc[m], sm.tqdc[m], sm.gd[m], sm.diag[m], sm.invd0[m], &g, alpha);
   float a[4], q4[4], zero[6] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-  for (int p = 0; p < 4; ++p) a[p] = odd ? alpha[p].y : alpha[p].x;
+  for (int p = 0; p < 4; ++p) a[p] = odd ? alpha[0][p].y : alpha[0][p].x;
   if constexpr (FAST) (void)quant_gain_fast<4>(pr, a, zero, 0.0f, zero, q4, sf);
   else (void)quant_gain<4>(pr, a, zero, 0.0f, zero, q4, sf);
   uint32_t c = 0u;
@@ -443,9 +504,11 @@ __global__ void __launch_bounds__(NT, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.tempty[tb]);
+      float2 g2[2];
+      pf_gain<FAST, 2>(pr, ah, al, qh, ql, tqc, tqdc, gd, diag, invd0, g2);
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
-        float2 g = pf_pair_gain<FAST>(pr, ah[j], al[j], qh[j], ql[j], tqc, tqdc, gd, diag, invd0);
+        float2 g = g2[j];
         const int sx = (c0 + k) * CH + 2 * (p0 + j);
         if (sx + 1 >= pr.S) {  // padding selectors (all-zero masks) are not candidates
           if (sx >= pr.S) g.x = neg_inf();

@@ -30,7 +30,8 @@ def _bound(cols, C, yabs):
 
 @pytest.mark.parametrize("sdq", [False, True])
 @pytest.mark.parametrize("kw", [dict(C=64, P=4, b=4, S=64), dict(C=16, P=4, b=4, S=16, scale_mode=1, b_e=16),
-                                dict(C=32, P=4, b=6, S=32), dict(C=8, P=4, b=3, S=16),
+                                dict(C=32, P=4, b=5, S=32), dict(C=64, P=4, b=6, S=32),
+                                dict(C=8, P=4, b=3, S=16),
                                 dict(C=128, P=2, b=4, S=8)])
 def test_packed_gemv_matches_definition(aw, orc, sdq, kw):
     rng = np.random.default_rng(11)

@@ -167,7 +167,7 @@ def test_decode_repeated_tile_takes_later_record(aw, orc):
         assert np.array_equal(w.float().cpu().numpy(), oouts[0])
 
 
-@pytest.mark.parametrize("C,P", [(16, 4), (8, 2), (4, 1)])
+@pytest.mark.parametrize("C,P", [(16, 4), (32, 4), (8, 2), (4, 1)])
 def test_decode_dense_many_modules_small_tiles(aw, orc, C, P):
     """20 modules (two launch runs of at most 16) and tiles of one or two 16-byte
     vectors (and a 4-element tile, below one BF16 vector)."""
