@@ -307,16 +307,16 @@ __device__ __forceinline__ void ldl_solve2(const float2* nL, const float2* invD,
   }
 }
 
-// Scale bits 2^e of one candidate for quant_gain_fast2, or 0 when amax is
-// outside [2^-100, 2^32] (inf and NaN patterns included). Adding
-// 0x7FFFFF - mant_q carries into the exponent field exactly when the mantissa
-// field of amax exceeds that of qmax, which is the [f_a > f_qmax] step of
-// quant_gain_fast.
-__device__ __forceinline__ uint32_t fast_scale_bits(const Prm& pr, float amax) {
-  const uint32_t ab = __float_as_uint(amax);
-  const bool ok = (ab - 0x0D800000u) <= (0x4F800000u - 0x0D800000u);
-  const uint32_t sc_bits = ((ab + (0x007FFFFFu - pr.mant_q)) & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23);
-  return ok ? sc_bits : 0u;
+// Scale bits 2^e of a candidate for quant_gain_fast2 from amax's bits ab,
+// valid when ab is in range (amax in [2^-100, 2^32]; inf and NaN patterns are
+// not): adding 0x7FFFFF - mant_q carries into the exponent field exactly when
+// the mantissa field of amax exceeds that of qmax, which is the
+// [f_a > f_qmax] step of quant_gain_fast.
+__device__ __forceinline__ bool fast_scale_in_range(uint32_t ab) {
+  return (ab - 0x0D800000u) <= (0x4F800000u - 0x0D800000u);
+}
+__device__ __forceinline__ uint32_t fast_scale_bits(const Prm& pr, uint32_t ab) {
+  return ((ab + (0x007FFFFFu - pr.mant_q)) & 0x7F800000u) - ((uint32_t)(pr.b - 2) << 23);
 }
 
 // quant_gain_fast on two candidates. Each code is RN(alpha*2^-e + 1.5*2^23) -
@@ -334,7 +334,10 @@ __device__ __forceinline__ float2 quant_gain_fast2(const Prm& pr, const float2* 
     m0 = fmaxf(m0, fabsf(alpha[p].x));
     m1 = fmaxf(m1, fabsf(alpha[p].y));
   }
-  const uint32_t s0 = fast_scale_bits(pr, m0), s1 = fast_scale_bits(pr, m1);
+  // an amax out of range gets a gain of -inf below, whatever its bits give
+  const uint32_t ab0 = __float_as_uint(m0), ab1 = __float_as_uint(m1);
+  const bool in0 = fast_scale_in_range(ab0), in1 = fast_scale_in_range(ab1);
+  const uint32_t s0 = fast_scale_bits(pr, ab0), s1 = fast_scale_bits(pr, ab1);
   const float2 sc = make_float2(__uint_as_float(s0), __uint_as_float(s1));
   const float2 nsc = make_float2(__uint_as_float(s0 | 0x80000000u), __uint_as_float(s1 | 0x80000000u));
   const float2 inv = make_float2(__uint_as_float(0x7F000000u - s0), __uint_as_float(0x7F000000u - s1));
@@ -355,8 +358,8 @@ __device__ __forceinline__ float2 quant_gain_fast2(const Prm& pr, const float2* 
   }
   const float2 tn = __fmul2_rn(nsc, Qq);
   float2 g = __fmul2_rn(sc, __ffma2_rn(make_float2(2.0f, 2.0f), Aq, tn));
-  if (s0 == 0u) g.x = -__int_as_float(0x7f800000);
-  if (s1 == 0u) g.y = -__int_as_float(0x7f800000);
+  if (!in0) g.x = -__int_as_float(0x7f800000);
+  if (!in1) g.y = -__int_as_float(0x7f800000);
   return g;
 }
 

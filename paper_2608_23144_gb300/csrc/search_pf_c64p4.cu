@@ -86,14 +86,15 @@ __device__ __forceinline__ float2 neg2(float2 v) { return make_float2(-v.x, -v.y
 
 __device__ __forceinline__ bool pivot_ok(float d) { return d > 0.0f && d <= 3.402823466e38f; }
 
-// rcp_rn on both components of NP pairs: the hardware approximations, then
+// Pivots k of NP pairs: the validity of each (pivot_ok) and rcp_rn of each
+// component. When every component of the warp's pairs is in [2^-125, 2^125)
+// (positive, normal, finite: hence valid), the hardware approximation and
 // Markstein's fused correction y + y (1 - x y) as two packed fmas (each
-// component rounds as the scalar form does). A component outside
-// [2^-125, 2^125) takes __frcp_rn instead, in a branch the active lanes take
-// together only when one of them needs it.
+// component rounds as the scalar form does); otherwise, in a branch the lanes
+// take together, the exact checks and __frcp_rn for the components outside.
 template <int NP>
-__device__ __forceinline__ void rcp2_rn(const float2* x, float2* r) {
-  bool fx[NP], fy[NP], ok = true;
+__device__ __forceinline__ void pivots_rcp(const float2* x, float2* r, bool* okx, bool* oky) {
+  bool fx[NP], fy[NP], in = true;
 #pragma unroll
   for (int j = 0; j < NP; ++j) {
     float yx, yy;
@@ -104,11 +105,13 @@ __device__ __forceinline__ void rcp2_rn(const float2* x, float2* r) {
     r[j] = __ffma2_rn(y, e, y);
     fx[j] = __float_as_uint(x[j].x) - 0x01000000u < 0x7D000000u - 0x01000000u;
     fy[j] = __float_as_uint(x[j].y) - 0x01000000u < 0x7D000000u - 0x01000000u;
-    ok = ok && fx[j] && fy[j];
+    in = in && fx[j] && fy[j];
   }
-  if (__any_sync(__activemask(), !ok)) {
+  if (__any_sync(__activemask(), !in)) {
 #pragma unroll
     for (int j = 0; j < NP; ++j) {
+      okx[j] = okx[j] && pivot_ok(x[j].x);
+      oky[j] = oky[j] && pivot_ok(x[j].y);
       if (!fx[j]) r[j].x = __frcp_rn(x[j].x);
       if (!fy[j]) r[j].y = __frcp_rn(x[j].y);
     }
@@ -128,7 +131,10 @@ __device__ __forceinline__ float2 quant_gain_fast2_g(const Prm& pr, const float2
     m0 = fmaxf(m0, fabsf(alpha[p].x));
     m1 = fmaxf(m1, fabsf(alpha[p].y));
   }
-  const uint32_t s0 = fast_scale_bits(pr, m0), s1 = fast_scale_bits(pr, m1);
+  // an amax out of range gets a gain of -inf below, whatever its bits give
+  const uint32_t ab0 = __float_as_uint(m0), ab1 = __float_as_uint(m1);
+  const bool in0 = fast_scale_in_range(ab0), in1 = fast_scale_in_range(ab1);
+  const uint32_t s0 = fast_scale_bits(pr, ab0), s1 = fast_scale_bits(pr, ab1);
   const float2 sc = make_float2(__uint_as_float(s0), __uint_as_float(s1));
   const float2 nsc = make_float2(__uint_as_float(s0 | 0x80000000u), __uint_as_float(s1 | 0x80000000u));
   const float2 inv = make_float2(__uint_as_float(0x7F000000u - s0), __uint_as_float(0x7F000000u - s1));
@@ -152,8 +158,8 @@ __device__ __forceinline__ float2 quant_gain_fast2_g(const Prm& pr, const float2
   }
   const float2 tn = __fmul2_rn(nsc, Qq);
   float2 g = __fmul2_rn(sc, __ffma2_rn(make_float2(2.0f, 2.0f), Aq, tn));
-  if (s0 == 0u) g.x = -__int_as_float(0x7f800000);
-  if (s1 == 0u) g.y = -__int_as_float(0x7f800000);
+  if (!in0) g.x = -__int_as_float(0x7f800000);
+  if (!in1) g.y = -__int_as_float(0x7f800000);
   return g;
 }
 
@@ -195,10 +201,8 @@ __device__ __forceinline__ void pf_fit(const float (*ah)[8], const float (*al)[8
       dk[jp] = dg;
 #pragma unroll
       for (int i = 0; i < k; ++i) dk[jp] = __ffma2_rn(nL[jp][tri(k, i)], E[jp][tri(k, i)], dk[jp]);
-      okx[jp] = okx[jp] && pivot_ok(dk[jp].x);
-      oky[jp] = oky[jp] && pivot_ok(dk[jp].y);
     }
-    rcp2_rn<NP>(dk, rk);
+    pivots_rcp<NP>(dk, rk, okx, oky);
 #pragma unroll
     for (int jp = 0; jp < NP; ++jp) invD[jp][k] = rk[jp];
   }
