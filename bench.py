@@ -59,11 +59,11 @@ def search_algorithmic_bytes(weights: int, tiles: int) -> int:
     return 4 * weights + 16 * tiles
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "56bf42dd8c4f33614b6cf6d9b77a88edab601e348d154c4a068a6bb3eef7ae51",
-                  "bytes_per_launch": 442290176 + 16653824,
+SEARCH_TRAFFIC = {"source_sha256": "1cd04d07d4d90c26f3b67e029fc662bf93ad2d481cfa4e122f26502badacc31e",
+                  "bytes_per_launch": 442118144 + 16535808,
                   # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
-                  "ncu_fma_pipe_pct": 38.20, "ncu_issue_active_pct": 45.26,
-                  "ncu_tensor_pipe_pct": 23.63}
+                  "ncu_fma_pipe_pct": 39.22, "ncu_issue_active_pct": 46.81,
+                  "ncu_tensor_pipe_pct": 24.17}
 
 
 def search_source_sha() -> str:

@@ -96,11 +96,11 @@ __device__ __forceinline__ int a_offset(int m, int k) {
 // (-L, then invD m rounded up). Returns U = u^T (G + eps I)^-1 u times the
 // seed's bound multiplier, as z^T (z * invD m) with z = L^-1 u: a sum of
 // non-negative terms.
-__device__ __forceinline__ float2 pair_bound(const float* hi, const float* lo, const float4* pe, float2* u) {
+__device__ __forceinline__ float2 pair_bound(const float* hi, const float* lo, const float4* pf, float2* u) {
   float2 pv[10];
 #pragma unroll
   for (int i = 0; i < 5; ++i) {
-    const float4 v = pe[i];
+    const float4 v = pf[i];
     pv[2 * i] = make_float2(v.x, v.y);
     pv[2 * i + 1] = make_float2(v.z, v.w);
   }
@@ -449,8 +449,11 @@ __global__ void __launch_bounds__(NT, 1)
       // loads are outstanding), issue pair i + 1's, then score pair i.
       const uint32_t cbase = tmem + lane_base + (uint32_t)(tb * 256 + 8 * SUB_PAIRS * sub);
       float hb[2][8], lb[2][8];
+      float4 fb[2][5];  // the bound's factors (-L, invD m) of the pair and of the next one
       tmem_ld8(cbase, hb[0]);
       tmem_ld8(cbase + 128, lb[0]);
+#pragma unroll
+      for (int j = 0; j < 5; ++j) fb[0][j] = pbase[SUB_PAIRS * sub * (PS / 2) + j];
 #pragma unroll
       for (int i = 0; i < SUB_PAIRS; ++i) {
         float* hi = hb[i & 1];
@@ -460,6 +463,8 @@ __global__ void __launch_bounds__(NT, 1)
         if (i + 1 < SUB_PAIRS) {
           tmem_ld8(cbase + 8 * (i + 1), hb[(i + 1) & 1]);
           tmem_ld8(cbase + 128 + 8 * (i + 1), lb[(i + 1) & 1]);
+#pragma unroll
+          for (int j = 0; j < 5; ++j) fb[(i + 1) & 1][j] = pbase[(SUB_PAIRS * sub + i + 1) * (PS / 2) + j];
         } else {
           // the warp's last loads of this accumulator are complete: release it
           // now, so that chunk k+2's MMAs need not wait for the last scores
@@ -471,7 +476,7 @@ __global__ void __launch_bounds__(NT, 1)
         {
           const float4* pe = pbase + pj * (PS / 2);
           float2 u[4];
-          const float2 ub = pair_bound(hi, lo, pe, u);
+          const float2 ub = pair_bound(hi, lo, fb[i & 1], u);
           // prune: a candidate whose gain bound is below the running best
           // cannot win (NaN bounds stay live)
           const bool lx = !FAST || !(ub.x < thr), ly = !FAST || !(ub.y < thr);
