@@ -126,12 +126,12 @@ __device__ __forceinline__ float2 pair_bound(const float* hi, const float* lo, c
 
 // Forward half of the ridge solve in the recipe's units: b = u (2^q c),
 // z = L^-1 b and w = D^-1 z, so that alpha = L^-T w.
-__device__ __forceinline__ void pair_forward(const float2* u, float2 tqc, const float4* pe, float2* bv,
-                                             float2* w) {
+__device__ __forceinline__ void pair_forward(const float2* u, float2 tqc, const float4* pl, const float4* pe,
+                                             float2* bv, float2* w) {
   float2 nL[6], invD[4];
 #pragma unroll
   for (int i = 0; i < 3; ++i) {
-    const float4 v = pe[i];
+    const float4 v = pl[i];
     nL[2 * i] = make_float2(v.x, v.y);
     nL[2 * i + 1] = make_float2(v.z, v.w);
   }
@@ -155,11 +155,11 @@ __device__ __forceinline__ void pair_forward(const float2* u, float2 tqc, const 
 }
 
 // Back half of the solve: alpha = L^-T w, in the order of ldl_solve2.
-__device__ __forceinline__ void pair_back(const float4* pe, const float2* w, float2* alpha) {
+__device__ __forceinline__ void pair_back(const float4* pl, const float2* w, float2* alpha) {
   float2 nL[6];
 #pragma unroll
   for (int i = 0; i < 3; ++i) {
-    const float4 v = pe[i];
+    const float4 v = pl[i];
     nL[2 * i] = make_float2(v.x, v.y);
     nL[2 * i + 1] = make_float2(v.z, v.w);
   }
@@ -239,7 +239,7 @@ __device__ __forceinline__ float winner_codes(const Prm& pr, const Smem& sm, int
   for (int p = 0; p < 4; ++p)
     u[p] = __ffma2_rn(make_float2(2048.0f, 2048.0f), make_float2(hi[2 * p], hi[2 * p + 1]),
                       make_float2(lo[2 * p], lo[2 * p + 1]));
-  pair_forward(u, make_float2(tq, tq), pe, bv, wv);
+  pair_forward(u, make_float2(tq, tq), pe, pe, bv, wv);
   pair_back(pe, wv, al);
   float a[4], q[4], zero[6] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
@@ -482,8 +482,9 @@ __global__ void __launch_bounds__(NT, 1)
           const bool lx = !FAST || !(ub.x < thr), ly = !FAST || !(ub.y < thr);
           if (__any_sync(0xffffffffu, lx || ly)) {
             float2 bv[4], wv[4], al[4];
-            pair_forward(u, tqc, pe, bv, wv);
-            pair_back(pe, wv, al);
+            // -L from the bound's registers, the rest from the stage
+            pair_forward(u, tqc, fb[i & 1], pe, bv, wv);
+            pair_back(fb[i & 1], wv, al);
             const float2 gp = pair_gain<FAST>(pr, bv, al, pe);
             // running argmax in seed order: a strictly greater gain wins
             const uint32_t s = (uint32_t)((c0 + k) * CH + 2 * pj);
