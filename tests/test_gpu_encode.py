@@ -89,6 +89,41 @@ def test_pruned_search_matches_oracle_on_adversarial_tiles(aw, orc, kind):
     assert_candidates_equal(got, want, kind)
 
 
+@pytest.mark.parametrize("kind", ["wide_fisher", "sparse_fisher", "sparse_ridge0", "tiny_sparse_ridge0"])
+def test_pf_search_matches_oracle_on_adversarial_weights(aw, orc, kind):
+    """The tcgen05 P_F search takes the fast reciprocal of a pivot only while
+    every pivot of the warp's two seed pairs is in [2^-125, 2^125); otherwise
+    it takes the exact validity checks and correctly rounded reciprocals.
+    Fisher weights over twelve decades; mostly-zero Fisher weights with no
+    activation part (singular Gram matrices held off by the ridge alone, or,
+    without a ridge, pivots of zero, rounding residue or either sign, which
+    take the exact branch); and the same near the smallest element weights the
+    fixed-point grids take (1e-28): the oracle's candidates bit for bit."""
+    sparse = kind != "wide_fisher"
+    mods = _mods([(130, 192), (7, 64)], "bf16", fisher=True, seed=11, blend=(0.0, 1.0) if sparse else (0.5, 0.5))
+    g = torch.Generator().manual_seed(13)
+    for m in mods:
+        F = m["fisher"]
+        if sparse:
+            F = F * (torch.rand(F.shape, generator=g) < 0.1).float()
+        else:
+            F = F * (10.0 ** (torch.rand(F.shape, generator=g) * 12 - 6)).float()
+        if kind == "tiny_sparse_ridge0":
+            F = F * 1e-29
+        m["fisher"] = F
+    kw = dict(C=64, P=4, b=4, S=48, variant=1)
+    if kind.endswith("ridge0"):
+        kw["ridge_rel"] = 0.0
+    prm, oprm = aw.params(**kw), orc.params(**kw)
+    cands = aw.awsrc_encode_tiles(prm, to_dev(mods))
+    flags = aw.awsrc_workspace_status(cands._awsrc_workspace)
+    got = aw.candidates_to_numpy(cands)
+    want = np.concatenate(oracle_encode(orc, oprm, mods))
+    assert flags == 0, f"device fault flags {flags:#x}"
+    assert_candidates_equal(got, want, kind)
+    assert np.isfinite(want["gain"]).sum() > 0, "no tile with a valid candidate"
+
+
 @pytest.mark.parametrize("variant", [0, 1])
 def test_padding_selectors_never_win(aw, orc, variant):
     """Seeds are searched in chunks padded up to a multiple of 32 with all-zero
