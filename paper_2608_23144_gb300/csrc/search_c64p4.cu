@@ -28,11 +28,15 @@
 //    tile's candidate.
 // Columns of a chunk are seed-pair major: column 8i + 2p + e holds atom p of
 // seed 2i + e, so one 32x32b.x8 TMEM load gives a thread one seed pair with
-// each atom's two seeds in adjacent registers; the next pair's loads are in
-// flight while a pair is scored.
-// Every mbarrier wait is bounded in time; on expiry the block records a timeout
-// fault, waits (bounded) for its own copies and MMAs in flight, frees its TMEM
-// and returns. A test of that path (Prm::stall_chunk >= 0) makes the producer
+// each atom's two seeds in adjacent registers; the next pair's loads (and
+// bound factors) are in flight while a pair is scored.
+// One CTA per SM takes tile blocks blockIdx.x, blockIdx.x + gridDim.x, ...:
+// it holds its TMEM allocation across them, initialises its barriers again
+// for each, and prefetches the next tile block's W and W0 rows into L2 while
+// one is searched.
+// Every mbarrier wait is bounded in time; on expiry the CTA records a timeout
+// fault, waits (bounded) for its own copies and MMAs in flight, takes no
+// further tile block, frees its TMEM and returns. A test of that path (Prm::stall_chunk >= 0) makes the producer
 // issue no copies from that chunk of its range on, with a short limit, so
 // that the producer's wait for the chunk's copies and the epilogue's wait for
 // its MMAs both run out.
@@ -254,20 +258,51 @@ __device__ __forceinline__ float winner_codes(const Prm& pr, const Smem& sm, int
   return odd ? g.y : g.x;
 }
 
+// Tile block blk of the launch: rows 128 rb .. of column block cb of its
+// module, split z of the seeds.
+struct BlockPos {
+  int mi, z;
+  int64_t rb, cb;
+};
+
+__device__ __forceinline__ BlockPos block_pos(const LaunchDesc& ld, int64_t blk) {
+  BlockPos p;
+  p.mi = find_mod(ld, blk);
+  const ModDesc& md = ld.m[p.mi];
+  const int64_t b = blk - md.block_off;
+  p.z = (int)(b % md.nsplit);
+  const int64_t rest = b / md.nsplit;
+  p.rb = rest % md.n_rb;
+  p.cb = rest / md.n_rb;
+  return p;
+}
+
+// Starts the L2 fills of tile block blk's W and W0 rows (one 128-byte row
+// segment per thread and matrix), so that its staging finds them on chip.
+__device__ __forceinline__ void prefetch_block(const LaunchDesc& ld, int64_t blk, int tid) {
+  if (tid >= BM) return;
+  const BlockPos p = block_pos(ld, blk);
+  const ModDesc& md = ld.m[p.mi];
+  const int64_t row = p.rb * BM + tid;
+  if (row >= md.rows) return;
+  const int64_t idx = row * md.cols + p.cb * 64;
+  const char* w = static_cast<const char*>(md.W) + idx * (md.w_dtype == AWSRC_DTYPE_F32 ? 4 : 2);
+  const char* w0 = static_cast<const char*>(md.W0) + idx * (md.w0_dtype == AWSRC_DTYPE_F32 ? 4 : 2);
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(w));
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(w0));
+  if (md.w_dtype == AWSRC_DTYPE_F32) asm volatile("prefetch.global.L2 [%0];" ::"l"(w + 128));
+  if (md.w0_dtype == AWSRC_DTYPE_F32) asm volatile("prefetch.global.L2 [%0];" ::"l"(w0 + 128));
+}
+
 template <bool FAST>
-__global__ void __launch_bounds__(NT, 1)
-    search_c64p4_kernel(Prm pr, LaunchDesc ld, const uint4* __restrict__ atoms,
-                        const float2* __restrict__ pairs, const uint64_t* __restrict__ masks,
-                        awsrc_candidate* __restrict__ cands,
-                        uint32_t* __restrict__ status) {
-  extern __shared__ unsigned char smem_raw[];
-  // 1 KB aligned by pointer arithmetic on the shared array, so that the
-  // compiler keeps the shared address space (LDS/STS, not generic accesses)
-  Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
+__device__ __forceinline__ bool search_block(const Prm& pr, const LaunchDesc& ld, int64_t blk, Smem& sm,
+                                             const uint4* __restrict__ atoms, const float2* __restrict__ pairs,
+                                             const uint64_t* __restrict__ masks, awsrc_candidate* __restrict__ cands,
+                                             uint32_t* __restrict__ status) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int mi = find_mod(ld, blockIdx.x);
+  const int mi = find_mod(ld, blk);
   const ModDesc& md = ld.m[mi];
-  const int64_t b = blockIdx.x - md.block_off;
+  const int64_t b = blk - md.block_off;
   const int z = (int)(b % md.nsplit);
   const int64_t rest = b / md.nsplit;
   const int64_t rb = rest % md.n_rb;
@@ -284,12 +319,7 @@ __global__ void __launch_bounds__(NT, 1)
       reinterpret_cast<const unsigned char*>(pairs) +
       (size_t)((md.gram_off + cb * pr.S_pad + (int64_t)c0 * CH) / 2) * PS * 8;
 
-  if (warp == EW) {  // the producer warp owns the TMEM allocation
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_addr(&sm.tmem_base)),
-                 "r"(kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  if (warp == EW) {
     if (lane == 0) {
       for (int i = 0; i < STAGES; ++i) mbar_init(&sm.full[i], 1);
       for (int i = 0; i < 2; ++i) {
@@ -505,7 +535,8 @@ __global__ void __launch_bounds__(NT, 1)
     sm.red_s[sub][m] = bsd;
   }
   tc_fence_before();
-  if (__syncthreads_or(timed_out)) {
+  const bool any_timeout = __syncthreads_or(timed_out);
+  if (any_timeout) {
     if (tid == 0) atomicOr(status, kFaultTimeout);
   } else if (tid < BM) {
     // merge the SUBS warps of each row (smaller seed on equal gains) and write
@@ -539,9 +570,41 @@ __global__ void __launch_bounds__(NT, 1)
       cands[(size_t)z * ld.T + tt] = cd;
     }
   }
+  return any_timeout;
+}
+
+// One block per SM, taking tile blocks blockIdx.x, blockIdx.x + gridDim.x, ...;
+// the next tile block's W and W0 are prefetched into L2 while one is searched.
+template <bool FAST>
+__global__ void __launch_bounds__(NT, 1)
+    search_c64p4_kernel(Prm pr, const __grid_constant__ LaunchDesc ld, int64_t n_blocks,
+                        const uint4* __restrict__ atoms, const float2* __restrict__ pairs,
+                        const uint64_t* __restrict__ masks, awsrc_candidate* __restrict__ cands,
+                        uint32_t* __restrict__ status) {
+  extern __shared__ unsigned char smem_raw[];
+  // 1 KB aligned by pointer arithmetic on the shared array, so that the
+  // compiler keeps the shared address space (LDS/STS, not generic accesses)
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u));
+  const int warp = threadIdx.x >> 5;
+  if (warp == EW) {  // the producer warp owns the TMEM allocation, held for all tile blocks
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_addr(&sm.tmem_base)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  for (int64_t blk = blockIdx.x; blk < n_blocks; blk += gridDim.x) {
+    if (blk + gridDim.x < n_blocks) prefetch_block(ld, blk + gridDim.x, threadIdx.x);
+    // a tile block whose waits ran out ends the CTA's work: its copies or MMAs
+    // may still be in flight into this shared memory
+    if (search_block<FAST>(pr, ld, blk, sm, atoms, pairs, masks, cands, status)) break;
+    __syncthreads();  // the block's shared memory is reused by the next tile block
+  }
+  tc_fence_before();
+  __syncthreads();
   if (warp == EW) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(sm.tmem_base), "r"(kTmemCols)
                  : "memory");
   }
 }
@@ -612,8 +675,12 @@ cudaError_t launch_search_c64p4(const Prm& pr, const LaunchDesc& ld, const void*
   auto kern = pr.fast_pow2 ? search_c64p4_kernel<true> : search_c64p4_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<(unsigned)n_blocks, NT, smem, st>>>(pr, ld, static_cast<const uint4*>(table), pairs, masks, cands,
-                                            status);
+  int dev = 0, nsm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(n_blocks, nsm));
+  kern<<<(unsigned)grid, NT, smem, st>>>(pr, ld, n_blocks, static_cast<const uint4*>(table), pairs, masks, cands,
+                                         status);
   note_launches(1);
   return cudaGetLastError();
 }
