@@ -59,11 +59,11 @@ def search_algorithmic_bytes(weights: int, tiles: int) -> int:
     return 4 * weights + 16 * tiles
 # DRAM traffic (read + write) of one full-layer search launch, from an ncu launch
 # list of this workload; valid only for the kernel source it was measured on.
-SEARCH_TRAFFIC = {"source_sha256": "5bd51c0bf67fee5b932b37a9fb0303e24d57ae07c0df24c48d6da691f553bcb5",
-                  "bytes_per_launch": 441948160 + 16826624,
+SEARCH_TRAFFIC = {"source_sha256": "1ec4496c84e47a59c8b2fdba2e99964251f41e20adbb67b77e1e7ad911cb1316",
+                  "bytes_per_launch": 443022848 + 16460032,
                   # the same kernel's pipe utilisation in an ncu --set full capture (gate + up)
-                  "ncu_fma_pipe_pct": 39.54, "ncu_issue_active_pct": 47.10,
-                  "ncu_tensor_pipe_pct": 24.45}
+                  "ncu_fma_pipe_pct": 40.23, "ncu_issue_active_pct": 48.50,
+                  "ncu_tensor_pipe_pct": 24.69}
 
 
 def search_source_sha() -> str:
