@@ -376,8 +376,8 @@ awsrc_status awsrc_decode_workspace_bytes(const awsrc_params* prm, int32_t n_mod
  * Requires the same params as the encoder.
  * Workspace (awsrc_decode_workspace_bytes): the basis masks, plus for DENSE a
  * tile -> record map and the unpacked records, 24 bytes per tile (and, for
- * P = 4 with C <= 64, 2*C bytes per seed of code tables); for INPLACE one
- * claim word per tile (4 bytes).
+ * P = 4 with C <= 64 and b <= 5, 2*C bytes per seed of code tables); for
+ * INPLACE one claim word per tile (4 bytes).
  */
 awsrc_status awsrc_decode_apply(const awsrc_params* prm, int32_t n_mod,
                                 const awsrc_module* mods, const uint8_t* stream,
