@@ -36,10 +36,10 @@
 // one is searched.
 // Every mbarrier wait is bounded in time; on expiry the CTA records a timeout
 // fault, waits (bounded) for its own copies and MMAs in flight, takes no
-// further tile block, frees its TMEM and returns. A test of that path (Prm::stall_chunk >= 0) makes the producer
-// issue no copies from that chunk of its range on, with a short limit, so
-// that the producer's wait for the chunk's copies and the epilogue's wait for
-// its MMAs both run out.
+// further tile block, frees its TMEM and returns. A test of that path
+// (Prm::stall_chunk >= 0) makes the producer issue no copies from that chunk
+// of its range on, with a short limit, so that the producer's wait for the
+// chunk's copies and the epilogue's wait for its MMAs both run out.
 #include "internal.h"
 #include "tc05.cuh"
 
